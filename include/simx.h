@@ -1,0 +1,301 @@
+/*
+ * simx.h — C ABI of libsimx.so, the GB300 (sm_103a) batched rollout engine for
+ * "Adaptive Inference Batching using Policy Gradients".
+ *
+ * The library runs thousands of independent copies of the paper's discrete-event
+ * inference-serving simulator (Sec. 3.1, Sec. 3.2) in lockstep on one GPU, evaluates the
+ * policy network of Sec. 4.2 fused into the step, and computes the REINFORCE returns,
+ * GAE advantages and REINFORCE / PPO loss gradients of Sec. 4.3 over the rollout buffer.
+ *
+ * Conventions shared by every entry point
+ *   - Every pointer argument whose name starts with d_ (and every pointer inside
+ *     simx_mlp / simx_rollout) is DEVICE memory owned by the caller; the library
+ *     never frees it.  Host pointers are marked "host".
+ *   - `stream` is a cudaStream_t passed as void*; NULL is the legacy default stream.
+ *     Calls are asynchronous on it; only sim_stats, sim_save, sim_load and
+ *     simx_last_status synchronise.
+ *   - Argument errors are detected on the host before any launch and returned as
+ *     a simx_status; nothing throws across the ABI.  simx_last_error() returns a
+ *     human-readable message for the last failure on the calling thread.
+ *   - Device-side errors (time overflow, event-loop cap, invalid external action)
+ *     never trap: they set a per-env status word, visible through
+ *     simx_last_status() and sim_save().
+ *   - Layouts are time-major: a [H][E] array holds step t of env e at t*ld + e and
+ *     observations are [H][D][E] (feature d of env e at step t at (t*D + d)*ld + e).
+ *   - Time inside the simulator is an unsigned 32-bit count of microseconds; any
+ *     time that would reach 2^31 us sets SIMX_DEV_TIME_OVERFLOW.
+ *
+ * The meaning of every field below is the executable specification the oracle
+ * (a separate single-threaded C program) implements independently.
+ */
+#ifndef SIMX_H
+#define SIMX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SIMX_ABI_VERSION 1u
+#define SIMX_MAX_TYPES 2
+#define SIMX_MAX_SERVERS 8
+#define SIMX_MAX_BSIZES 8
+#define SIMX_MAX_LAYERS 4
+#define SIMX_MAX_WIDTH 256      /* widest hidden layer */
+#define SIMX_MAX_OUT 257        /* widest output layer: actions + value row */
+#define SIMX_MAX_OBS 64
+#define SIMX_DIURNAL_MAX 128
+#define SIMX_STATE_HEADER_WORDS 32
+#define SIMX_TRACE_WIDTH 4
+
+typedef enum {
+  SIMX_OK = 0,
+  SIMX_EINVAL = 1,     /* invalid argument or configuration (host-side check) */
+  SIMX_ENOMEM = 2,     /* device or host allocation failed in sim_create */
+  SIMX_ECUDA = 3,      /* a CUDA runtime call failed (message has the CUDA error) */
+  SIMX_EOVERFLOW = 4,  /* an env raised a device status flag (see SIMX_DEV_*) */
+  SIMX_ESTATE = 5      /* call out of order (e.g. step before reset) */
+} simx_status;
+
+/* Per-env device status bits (OR-ed into the env's status word). */
+#define SIMX_DEV_TIME_OVERFLOW 1u   /* a simulated time reached 2^31 us */
+#define SIMX_DEV_EVENT_CAP 2u       /* more than 2^20 arrival candidates in one decision */
+#define SIMX_DEV_BAD_ACTION 4u      /* external action outside [0, n_actions): action 0 used */
+
+/* Simulator mode (Sec. 3.1 "Multi-GPU Support"; Sec. 4.1 action space). */
+typedef enum {
+  SIMX_MODE_SINGLE = 0,  /* one server; a decision whenever it is free and work is queued;
+                            action = (type to serve, batch size)                          */
+  SIMX_MODE_ROUTE = 1    /* K servers; one decision per arriving request;
+                            action = (target server, that server's batch size)            */
+} simx_mode;
+
+/* Arrival process (Sec. 3.2 workloads). */
+typedef enum {
+  SIMX_ARR_THINNED = 0,  /* Poisson candidate stream thinned by a 1- or 2-state modulating
+                            chain: Poisson when n_mod_states = 1, MMPP when 2            */
+  SIMX_ARR_DIURNAL = 1   /* piecewise-constant rate per epoch: diurnal table x lognormal
+                            burst factor; stands in for the trace replay of Sec. 3.2      */
+} simx_arrival_kind;
+
+/* Action selection (Sec. 4.2 stochastic policy; Sec. 5.1 baselines). */
+typedef enum {
+  SIMX_POLICY_SAMPLE = 0,   /* categorical sample from softmax(logits)                   */
+  SIMX_POLICY_ARGMAX = 1,   /* first index of the largest logit                          */
+  SIMX_POLICY_STATIC = 2,   /* single mode: oldest-head type, batch bsizes[static_bi]     */
+  SIMX_POLICY_RR = 3,       /* route mode: server t mod K, batch bsizes[static_bi]        */
+  SIMX_POLICY_SQ = 4,       /* route mode: server with fewest queued requests             */
+  SIMX_POLICY_RANDOM = 5,   /* uniform action from the POLICY Philox stream              */
+  SIMX_POLICY_EXTERNAL = 6  /* sim_step_batched only: caller-supplied actions            */
+} simx_policy_mode;
+
+/*
+ * Environment configuration (plain data, copied by sim_create).
+ * Every numeric value enters the simulator exactly as given; nothing here is
+ * recomputed by the library, so the same struct fed to the oracle fixes every bit.
+ */
+typedef struct simx_config {
+  uint32_t abi_version;        /* must be SIMX_ABI_VERSION */
+  uint32_t mode;               /* simx_mode */
+  uint32_t n_envs;             /* E, 1 .. 2^24 */
+  uint32_t n_servers;          /* K: 1 in SINGLE mode, 1..SIMX_MAX_SERVERS in ROUTE mode */
+  uint32_t n_types;            /* request types (Sec. 3.1 model type m_i): 1 or 2 */
+  uint32_t queue_cap;          /* FIFO capacity per (server, type); power of two <= 4096;
+                                  arrivals to a full queue are dropped (Sec. 3.1 Queuing) */
+  uint32_t episode_len;        /* done[t] = 1 when (global step + 1) % episode_len == 0 */
+  uint32_t arrival_kind;       /* simx_arrival_kind */
+  /* THINNED: candidates at i.i.d. exponential gaps, accepted with probability
+     accept_thr[state] / 2^24 where state is the modulating chain's state */
+  float    cand_mean_gap_us;   /* mean candidate gap (1e6 / max rate) */
+  uint32_t n_mod_states;       /* 1 (Poisson) or 2 (two-state MMPP) */
+  uint32_t accept_thr[2];      /* acceptance threshold per state, out of 2^24 */
+  float    dwell_mean_us;      /* mean exponential dwell of the modulating chain */
+  /* DIURNAL: rate(epoch) = diurnal_rate[(epoch + offset_env) % diurnal_len] * exp(sigma Z) */
+  uint32_t epoch_us;           /* epoch length */
+  uint32_t diurnal_len;        /* 1 .. SIMX_DIURNAL_MAX */
+  float    diurnal_rate[SIMX_DIURNAL_MAX]; /* base arrival rate per epoch slot, requests/s */
+  float    burst_sigma;        /* lognormal sigma of the per-epoch burst factor */
+  /* request types and the execution model L = alpha + beta * n (Sec. 3.1) */
+  uint32_t type0_thr;          /* P(type 0) * 2^24 */
+  uint32_t alpha_us[SIMX_MAX_TYPES];
+  uint32_t beta_us[SIMX_MAX_TYPES];
+  int32_t  cost_type;          /* type whose batch time is alpha + the sum of per-request
+                                  costs drawn at arrival (-1: none; beta then unused) */
+  uint32_t cost_kind;          /* 0: Pareto(x_m = cost_scale_us, shape 1/pareto_inv_alpha);
+                                  1: exponential with mean cost_scale_us */
+  float    cost_scale_us;
+  float    pareto_inv_alpha;
+  /* reward (Sec. 4.1): r = n_dispatched - sum_type w_wait[type] * queueing_us */
+  float    w_wait[SIMX_MAX_TYPES];
+  /* actions (Sec. 4.1): a = major * n_bsizes + i, major = type (SINGLE) or server (ROUTE) */
+  uint32_t n_bsizes;
+  uint32_t bsizes[SIMX_MAX_BSIZES];
+  uint32_t static_bi;          /* batch-size index of the policy-free baselines and the
+                                  initial per-server batch size in ROUTE mode */
+  /* observation (Sec. 4.1 state) */
+  uint32_t obs_extra;          /* append the extra features (see obs layout below) */
+  uint32_t obs_dim;            /* must equal simx_obs_dim(cfg) */
+  float    t_window_us;        /* time normaliser T_window */
+  float    rate_scale;         /* SINGLE: rate feature = n_arrivals * rate_scale / dt_us */
+  float    rate_ref;           /* ROUTE: EWMA rate normaliser and its initial value */
+  float    busy_norm_us;       /* ROUTE: busy-remaining normaliser */
+  uint32_t phase_period_us;    /* ROUTE extra: diurnal phase period */
+} simx_config;
+
+/*
+ * Policy network (Sec. 4.2): a tanh MLP.  Layer l maps dims[l] -> dims[l+1] with
+ * z_j = (sum_k W_l[j][k] x_k, accumulated in fp32 by fused multiply-adds in k order
+ * from k = 0) + b_l[j]; hidden layers apply tanh.  The last layer has n_actions rows
+ * followed by one value row when has_value (the value head of Sec. 4.2 sharing the
+ * trunk).  W_l is row-major [dims[l+1]][dims[l]] fp32, device memory.
+ */
+typedef struct simx_mlp {
+  int32_t n_layers;                     /* 1 .. SIMX_MAX_LAYERS */
+  int32_t dims[SIMX_MAX_LAYERS + 1];
+  const float* W[SIMX_MAX_LAYERS];
+  const float* b[SIMX_MAX_LAYERS];
+  int32_t has_value;
+} simx_mlp;
+
+/* Rollout buffer (device memory, caller-owned).  ld >= n_envs is the env stride. */
+typedef struct simx_rollout {
+  int64_t  ld;
+  float*   obs;      /* [H][obs_dim][ld] observation at each decision */
+  uint8_t* action;   /* [H][ld] action index */
+  float*   logp;     /* [H][ld] log pi(a|s) (0 for policy-free modes); may be NULL */
+  float*   value;    /* [H][ld] value head output; NULL unless has_value */
+  float*   reward;   /* [H][ld] reward of the step */
+  uint8_t* done;     /* [H][ld] segment end flag */
+  int64_t* trace;    /* [H][SIMX_TRACE_WIDTH][ld] or NULL: decision time (us), requests
+                        dispatched in the step, their summed queueing us, requests queued
+                        after the decision */
+} simx_rollout;
+
+/* Loss selection for ppo_loss_grad (Sec. 4.3). */
+typedef enum { SIMX_ALGO_REINFORCE = 0, SIMX_ALGO_PPO = 1 } simx_algo;
+
+typedef struct simx_loss_params {
+  int32_t algo;        /* simx_algo */
+  float   clip_eps;    /* PPO clip range epsilon */
+  float   c_value;     /* value-loss coefficient (used when the MLP has a value row) */
+  float   c_entropy;   /* entropy bonus coefficient */
+} simx_loss_params;
+
+/* Aggregate counters over all envs (sim_stats). */
+typedef struct simx_counters {
+  uint64_t arrived, dropped, dispatched, batches, queued, sum_wait_us, decisions;
+  uint32_t envs_flagged;     /* envs whose status word is non-zero */
+  uint32_t status_or;        /* OR of all env status words */
+} simx_counters;
+
+typedef struct simx_ctx simx_ctx;
+
+/* Observation width implied by a configuration (0 if the configuration is invalid):
+   SINGLE: 2T + 6 (+6 with obs_extra); ROUTE: 3K + 1 (+3 with obs_extra). */
+uint32_t simx_obs_dim(const simx_config* cfg);
+/* Words of one env's canonical state image (sim_save layout). */
+uint64_t simx_state_words(const simx_config* cfg);
+
+/* Create a simulator context on `device`: validates cfg, allocates the SoA env state
+   and FIFO rings in device memory (owned by the context).  *out is NULL on error. */
+simx_status sim_create(const simx_config* cfg, int device, simx_ctx** out);
+void sim_destroy(simx_ctx* ctx);
+
+/* Reset every env to time 0 with empty queues and idle servers, keyed by `seed`
+   (Philox key), and advance each to its first decision point. */
+simx_status sim_reset(simx_ctx* ctx, uint64_t seed, void* stream);
+
+/* Write the current observation of every env to d_obs [obs_dim][ld]. */
+simx_status sim_observe(simx_ctx* ctx, float* d_obs, int64_t ld, void* stream);
+
+/*
+ * One decision step of every env (the gym-style step of Sec. 4.1).
+ *   policy_mode == SIMX_POLICY_EXTERNAL: d_actions [E] int32 chosen by the caller;
+ *   otherwise the internal policy (pol required for SAMPLE/ARGMAX).
+ * Outputs (any may be NULL): d_obs [obs_dim][ld] next observation, d_reward [E],
+ * d_done [E], d_action [E] u8 action taken, d_logp [E].
+ */
+simx_status sim_step_batched(simx_ctx* ctx, const int32_t* d_actions, const simx_mlp* pol,
+                             int policy_mode, float* d_obs, int64_t ld, float* d_reward,
+                             uint8_t* d_done, uint8_t* d_action, float* d_logp, void* stream);
+
+/*
+ * Collect `horizon` decision steps of every env into `out` in one persistent launch:
+ * observation, fused policy forward, action, reward, done (Sec. 4.1, Sec. 4.2).
+ * Equivalent, bit for bit, to `horizon` calls of sim_step_batched.
+ */
+simx_status rollout_collect(simx_ctx* ctx, const simx_mlp* pol, int policy_mode,
+                            int32_t horizon, const simx_rollout* out, void* stream);
+
+/*
+ * Batched policy forward (Sec. 4.2) for n observation columns d_obs [dims[0]][ld].
+ * Column i is env (env_base + i) at global decision step `step`, which fixes its
+ * POLICY Philox counter, so this reproduces the actions the rollout drew.
+ * Outputs (any may be NULL): d_logits [n_actions][ld], d_value [ld], d_action [ld] u8,
+ * d_logp [ld].  policy_mode: SAMPLE or ARGMAX.
+ */
+simx_status policy_forward(const simx_mlp* pol, const float* d_obs, int64_t ld, int64_t n,
+                           int policy_mode, uint64_t seed, uint32_t step, uint32_t env_base,
+                           float* d_logits, float* d_value, uint8_t* d_action, float* d_logp,
+                           void* stream);
+
+/*
+ * Returns and advantages over a [T][E] buffer (Sec. 4.3):
+ *   lam < 0 : REINFORCE returns G_t = r_t + gamma (1 - d_t) G_{t+1}, G_T = last_value
+ *             (d_ret gets G; d_adv may be NULL);
+ *   lam >= 0: GAE  delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t, V_T = last_value,
+ *             A_t = delta_t + gamma lam (1 - d_t) A_{t+1}, R_t = A_t + V_t.
+ * d_val is required for GAE; d_last_val [E] may be NULL (zeros).  ld >= E.
+ */
+simx_status compute_returns_gae(const float* d_rew, const float* d_val, const uint8_t* d_done,
+                                const float* d_last_val, int64_t T, int64_t E, int64_t ld,
+                                float gamma, float lam, float* d_ret, float* d_adv,
+                                void* stream);
+
+/*
+ * Mean-return baseline (Sec. 4.3 REINFORCE with a baseline): mean = (1/n) sum x_i,
+ * accumulated in fp64; d_adv_out[i] = x_i - mean (fp32); d_mean_out[0] = mean (fp32).
+ * d_workspace must hold returns_baseline_workspace_size(n) bytes.
+ */
+size_t returns_baseline_workspace_size(int64_t n);
+simx_status returns_baseline(const float* d_x, int64_t n, float* d_adv_out, float* d_mean_out,
+                             void* d_workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Loss and gradient over a minibatch (Sec. 4.3).  Row r of the rollout is
+ * (t = r / E, e = r % E) with E = n_rows_per_step; the minibatch is rows d_idx[0..n)
+ * (d_idx == NULL: rows 0..n-1).  With pi = softmax(logits):
+ *   REINFORCE: L = -mean(adv * log pi(a))
+ *   PPO      : rho = exp(log pi(a) - logp_old),
+ *              L = -mean(min(rho adv, clip(rho, 1-eps, 1+eps) adv))
+ *   both     : + c_value mean((V - ret)^2) (value row only) - c_entropy mean(H[pi]).
+ * d_grad [n_params] fp32 is overwritten with dL/dtheta in the order W0,b0,W1,b1,...;
+ * d_stats [5] = {L, policy term, mean (V-ret)^2, mean entropy, clip fraction}.
+ * d_workspace must hold ppo_loss_grad_workspace_size(pol, n) bytes.
+ */
+size_t ppo_loss_grad_workspace_size(const simx_mlp* pol, int64_t n);
+simx_status ppo_loss_grad(const simx_mlp* pol, const simx_rollout* buf, int64_t n_rows_per_step,
+                          const float* d_ret, const float* d_adv, const int64_t* d_idx, int64_t n,
+                          const simx_loss_params* params, float* d_grad, float* d_stats,
+                          void* d_workspace, size_t workspace_bytes, void* stream);
+
+/* Aggregate counters (synchronises the context's last stream). host_out: host. */
+simx_status sim_stats(simx_ctx* ctx, simx_counters* host_out);
+
+/* Canonical state images (synchronising).  host_buf: host, n_envs * simx_state_words
+   u32 words; env e's image starts at word e * simx_state_words(cfg). */
+simx_status sim_save(simx_ctx* ctx, uint32_t* host_buf, uint64_t n_words);
+simx_status sim_load(simx_ctx* ctx, const uint32_t* host_buf, uint64_t n_words);
+
+/* OR of all env status words (synchronising).  Returns SIMX_EOVERFLOW if non-zero. */
+simx_status simx_last_status(simx_ctx* ctx, uint32_t* device_code);
+
+const char* simx_strerror(simx_status s);
+const char* simx_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SIMX_H */

@@ -1,0 +1,136 @@
+"""Returns, GAE, baseline and loss gradients in numpy fp64 (test infrastructure only).
+
+Written from the paper's Sec. 4.3 (REINFORCE: Monte-Carlo policy gradient with
+discounted returns and a baseline; PPO: clipped surrogate with an entropy bonus) and
+the GAE estimator of Schulman et al. (2016).  Each function is the plain definition:
+a reverse loop over time for the recurrences, explicit forward and backward passes
+of the tanh MLP for the gradients.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+REINFORCE, PPO = 0, 1
+
+
+def returns(rew, done, gamma, last_value=None):
+    """REINFORCE returns G_t = r_t + gamma (1 - d_t) G_{t+1}, G_T = last_value."""
+    rew = np.asarray(rew, np.float64)
+    done = np.asarray(done, np.float64)
+    T, E = rew.shape
+    G = np.zeros((T, E))
+    nxt = np.zeros(E) if last_value is None else np.asarray(last_value, np.float64).copy()
+    for t in range(T - 1, -1, -1):
+        nxt = rew[t] + gamma * (1.0 - done[t]) * nxt
+        G[t] = nxt
+    return G
+
+
+def gae(rew, val, done, gamma, lam, last_value=None):
+    """GAE: delta_t = r_t + gamma (1-d_t) V_{t+1} - V_t; A_t = delta_t + gamma lam (1-d_t) A_{t+1};
+    returns (A, R = A + V)."""
+    rew = np.asarray(rew, np.float64)
+    val = np.asarray(val, np.float64)
+    done = np.asarray(done, np.float64)
+    T, E = rew.shape
+    A = np.zeros((T, E))
+    next_v = np.zeros(E) if last_value is None else np.asarray(last_value, np.float64).copy()
+    next_a = np.zeros(E)
+    for t in range(T - 1, -1, -1):
+        mask = 1.0 - done[t]
+        delta = rew[t] + gamma * mask * next_v - val[t]
+        next_a = delta + gamma * lam * mask * next_a
+        A[t] = next_a
+        next_v = val[t]
+    return A, A + val
+
+
+def baseline(x):
+    """Mean-return baseline: (x - mean(x), mean(x)) with the mean in fp64."""
+    x = np.asarray(x, np.float64)
+    m = x.sum() / x.size
+    return x - m, m
+
+
+def forward(Ws, bs, X):
+    """tanh MLP forward in fp64; returns the list of layer inputs and the last layer's output."""
+    h = np.asarray(X, np.float64)
+    inputs = []
+    L = len(Ws)
+    for l in range(L):
+        inputs.append(h)
+        z = h @ np.asarray(Ws[l], np.float64).T + np.asarray(bs[l], np.float64)
+        h = np.tanh(z) if l + 1 < L else z
+    return inputs, h
+
+
+def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=0.2,
+              c_value=0.5, c_entropy=0.01):
+    """Loss, statistics and the gradient with respect to every W_l, b_l (fp64).
+
+    pi = softmax(logits); policy term REINFORCE -mean(adv log pi(a)) or PPO
+    -mean(min(rho adv, clip(rho, 1-eps, 1+eps) adv)) with rho = exp(log pi(a) - logp_old);
+    plus c_value mean((V - ret)^2) when a value row exists, minus c_entropy mean(H[pi]).
+    Returns (grads [(gW, gb) per layer], stats [L, pg, v, H, clipfrac]).
+    """
+    inputs, Z = forward(Ws, bs, X)
+    n = Z.shape[0]
+    A = Z.shape[1] - (1 if has_value else 0)
+    logits = Z[:, :A]
+    m = logits.max(axis=1, keepdims=True)
+    lse = m + np.log(np.exp(logits - m).sum(axis=1, keepdims=True))
+    logpi = logits - lse
+    pi = np.exp(logpi)
+    a = np.asarray(actions, np.int64)
+    rows = np.arange(n)
+    lpa = logpi[rows, a]
+    adv = np.asarray(adv, np.float64)
+    onehot = np.zeros_like(logits)
+    onehot[rows, a] = 1.0
+    if algo == REINFORCE:
+        pg = -np.mean(adv * lpa)
+        coef = adv
+        clipfrac = 0.0
+    else:
+        rho = np.exp(lpa - np.asarray(logp_old, np.float64))
+        s1 = rho * adv
+        s2 = np.clip(rho, 1.0 - clip_eps, 1.0 + clip_eps) * adv
+        pg = -np.mean(np.minimum(s1, s2))
+        coef = np.where(s1 <= s2, adv, 0.0) * rho
+        clipfrac = float(np.mean(np.abs(rho - 1.0) > clip_eps))
+    dlogits = -(coef[:, None] / n) * (onehot - pi)
+    H = -(pi * logpi).sum(axis=1)
+    dlogits += (c_entropy / n) * pi * (logpi + H[:, None])
+    loss = pg - c_entropy * H.mean()
+    vloss = 0.0
+    dZ = np.zeros_like(Z)
+    dZ[:, :A] = dlogits
+    if has_value:
+        v = Z[:, A]
+        r = np.asarray(ret, np.float64)
+        vloss = float(np.mean((v - r) ** 2))
+        loss += c_value * vloss
+        dZ[:, A] = 2.0 * c_value * (v - r) / n
+    grads = [None] * len(Ws)
+    dz = dZ
+    for l in range(len(Ws) - 1, -1, -1):
+        h_in = inputs[l]
+        grads[l] = (dz.T @ h_in, dz.sum(axis=0))
+        if l > 0:
+            dh = dz @ np.asarray(Ws[l], np.float64)
+            dz = dh * (1.0 - h_in ** 2)
+    stats = np.array([loss, pg, vloss, H.mean(), clipfrac])
+    return grads, stats
+
+
+def flat(grads):
+    """Concatenate gradients in the library's order W0, b0, W1, b1, ..."""
+    return np.concatenate([np.concatenate([g.ravel(), b.ravel()]) for g, b in grads])
+
+
+def gather_rows(obs, actions, logp, idx, E):
+    """Minibatch rows of a [T][D][E] rollout: row r is (t = r // E, e = r % E)."""
+    idx = np.asarray(idx, np.int64)
+    t, e = idx // E, idx % E
+    X = obs[t, :, e]
+    return X, np.asarray(actions)[t, e], np.asarray(logp)[t, e]

@@ -1,0 +1,180 @@
+"""Seeded synthetic inputs shared by the CUDA path, the oracle and the benchmark.
+
+This module holds only workload *inputs*: the five environment configurations the
+engine is measured on, policy weights, the diurnal rate table and minibatch
+permutations.  It contains none of the method's arithmetic (no simulation, policy,
+return or loss code), so both sides can take their inputs from here.
+
+The configurations restate the paper's workloads (Sec. 3.2: Poisson, bursty,
+trace-shaped, heterogeneous multi-server) and latency model (Sec. 3.1,
+L = alpha + beta * b) at the sizes of the engine's five benchmark configurations:
+
+* ``c1``  64 envs x 10,000 steps, one server, one type, Poisson 800 req/s,
+  2000 + 100 n us, queue 128, batch sizes {1,2,4,8,16,32}, MLP 8-32-6, REINFORCE.
+* ``c2``  4096 envs x 512, one server, two-state MMPP 300 / 3000 req/s (dwell
+  200 ms), 80/20 short (1000 + 50 n) / long (20,000 + 2000 n), queues 256,
+  action (type, batch), MLP 16-64-64-12, REINFORCE with a mean baseline.
+* ``c3``  16,384 envs x 256, four servers, Poisson 4000 req/s, 70/30 mix,
+  action (server, batch in {1,4,16,32}), MLP 13-128-128-16 + value, PPO/GAE.
+* ``c4``  65,536 envs x 512, eight servers, diurnal 1000-8000 req/s over 60 s x
+  lognormal(0, 1) per 500 ms, long requests with Pareto(1.5, 10 ms) per-request
+  cost, 85/15 mix, MLP 28-256-256-48 + value, PPO/GAE.
+* ``c5``  c3's environment at 1024 ... 1,048,576 envs x 1024, argmax policy.
+
+The public Azure Functions / BurstGPT traces the paper replays are not available
+here; ``c4``'s diurnal x lognormal x Pareto load stands in for them.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+ABI_VERSION = 1
+MODE_SINGLE, MODE_ROUTE = 0, 1
+ARR_THINNED, ARR_DIURNAL = 0, 1
+POLICY = {"sample": 0, "argmax": 1, "static": 2, "rr": 3, "sq": 4, "random": 5, "external": 6}
+TWO24 = 1 << 24
+
+# Field order of the configuration record (same order as the C struct).
+CONFIG_FIELDS = [
+    ("abi_version", "u32"), ("mode", "u32"), ("n_envs", "u32"), ("n_servers", "u32"),
+    ("n_types", "u32"), ("queue_cap", "u32"), ("episode_len", "u32"), ("arrival_kind", "u32"),
+    ("cand_mean_gap_us", "f32"), ("n_mod_states", "u32"), ("accept_thr", "u32[2]"),
+    ("dwell_mean_us", "f32"), ("epoch_us", "u32"), ("diurnal_len", "u32"),
+    ("diurnal_rate", "f32[128]"), ("burst_sigma", "f32"), ("type0_thr", "u32"),
+    ("alpha_us", "u32[2]"), ("beta_us", "u32[2]"), ("cost_type", "i32"), ("cost_kind", "u32"),
+    ("cost_scale_us", "f32"), ("pareto_inv_alpha", "f32"), ("w_wait", "f32[2]"),
+    ("n_bsizes", "u32"), ("bsizes", "u32[8]"), ("static_bi", "u32"), ("obs_extra", "u32"),
+    ("obs_dim", "u32"), ("t_window_us", "f32"), ("rate_scale", "f32"), ("rate_ref", "f32"),
+    ("busy_norm_us", "f32"), ("phase_period_us", "u32"),
+]
+
+
+def _thr(p: float) -> int:
+    """Probability as an integer threshold out of 2^24 (rounded to nearest)."""
+    return int(round(p * TWO24))
+
+
+def diurnal_table(n: int = 120, lo: float = 1000.0, hi: float = 8000.0) -> list:
+    """Base arrival rate per 500 ms slot of a 60 s period: a sinusoid from lo to hi.
+
+    This is workload input, like a trace file: computed once in fp64 and stored as fp32.
+    """
+    mid, amp = 0.5 * (lo + hi), 0.5 * (hi - lo)
+    return [float(np.float32(mid + amp * math.sin(2.0 * math.pi * i / n))) for i in range(n)]
+
+
+def _base(**kw) -> dict:
+    c = dict(
+        abi_version=ABI_VERSION, mode=MODE_SINGLE, n_envs=64, n_servers=1, n_types=1,
+        queue_cap=128, episode_len=1000, arrival_kind=ARR_THINNED,
+        cand_mean_gap_us=1250.0, n_mod_states=1, accept_thr=[TWO24, TWO24],
+        dwell_mean_us=0.0, epoch_us=0, diurnal_len=1, diurnal_rate=[0.0] * 128,
+        burst_sigma=0.0, type0_thr=TWO24, alpha_us=[2000, 0], beta_us=[100, 0],
+        cost_type=-1, cost_kind=0, cost_scale_us=0.0, pareto_inv_alpha=0.0,
+        w_wait=[0.001, 0.0], n_bsizes=6, bsizes=[1, 2, 4, 8, 16, 32, 0, 0], static_bi=3,
+        obs_extra=0, obs_dim=8, t_window_us=10000.0, rate_scale=1250.0, rate_ref=800.0,
+        busy_norm_us=100000.0, phase_period_us=0,
+    )
+    c.update(kw)
+    return c
+
+
+def c1(n_envs: int = 64) -> dict:
+    """Tiny single-server env: Poisson 800 req/s, 2000 + 100 n us, queue 128."""
+    return _base(n_envs=n_envs)
+
+
+def c2(n_envs: int = 4096) -> dict:
+    """Single-server bursty heterogeneous env: MMPP 300/3000 req/s, 80/20 short/long."""
+    return _base(
+        n_envs=n_envs, n_types=2, queue_cap=256, episode_len=512,
+        cand_mean_gap_us=float(np.float32(1e6 / 3000.0)), n_mod_states=2,
+        accept_thr=[_thr(300.0 / 3000.0), TWO24], dwell_mean_us=200000.0,
+        type0_thr=_thr(0.8), alpha_us=[1000, 20000], beta_us=[50, 2000],
+        w_wait=[0.001, 0.0001], obs_extra=1, obs_dim=16,
+        rate_scale=float(np.float32(1e6 / 1650.0)), rate_ref=1650.0,
+    )
+
+
+def c3(n_envs: int = 16384, episode_len: int = 256) -> dict:
+    """Multi-server routing env: 4 servers, Poisson 4000 req/s, 70/30 short/long."""
+    return _base(
+        mode=MODE_ROUTE, n_envs=n_envs, n_servers=4, n_types=2, queue_cap=256,
+        episode_len=episode_len, cand_mean_gap_us=250.0, type0_thr=_thr(0.7),
+        alpha_us=[1000, 20000], beta_us=[50, 2000], w_wait=[0.001, 0.0001],
+        n_bsizes=4, bsizes=[1, 4, 16, 32, 0, 0, 0, 0], static_bi=2, obs_dim=13,
+        rate_scale=0.0, rate_ref=4000.0,
+    )
+
+
+def c4(n_envs: int = 65536) -> dict:
+    """Trace-shaped env: 8 servers, diurnal x lognormal arrivals, Pareto long costs."""
+    tab = diurnal_table()
+    return _base(
+        mode=MODE_ROUTE, n_envs=n_envs, n_servers=8, n_types=2, queue_cap=256,
+        episode_len=512, arrival_kind=ARR_DIURNAL, cand_mean_gap_us=0.0,
+        epoch_us=500000, diurnal_len=len(tab), diurnal_rate=tab + [0.0] * (128 - len(tab)),
+        burst_sigma=1.0, type0_thr=_thr(0.85), alpha_us=[1000, 20000], beta_us=[50, 0],
+        cost_type=1, cost_kind=0, cost_scale_us=10000.0,
+        pareto_inv_alpha=float(np.float32(1.0 / 1.5)), w_wait=[0.001, 0.0001],
+        obs_extra=1, obs_dim=28, rate_scale=0.0, rate_ref=8000.0, phase_period_us=60_000_000,
+    )
+
+
+def c5(n_envs: int = 65536) -> dict:
+    """Scale sweep of c3's env: horizon 1024, one segment per rollout."""
+    return c3(n_envs=n_envs, episode_len=1024)
+
+
+def md1(lam: float, n_envs: int = 64) -> dict:
+    """c1 with fixed batch 1 (M/D/1, D = 2100 us) at arrival rate lam req/s."""
+    return _base(n_envs=n_envs, cand_mean_gap_us=float(np.float32(1e6 / lam)), static_bi=0,
+                 queue_cap=4096, episode_len=1 << 30)
+
+
+def mm1(lam: float, mean_service_us: float = 2100.0, n_envs: int = 64) -> dict:
+    """Single server, batch 1, exponential per-request cost (M/M/1)."""
+    return _base(n_envs=n_envs, cand_mean_gap_us=float(np.float32(1e6 / lam)), static_bi=0,
+                 queue_cap=4096, episode_len=1 << 30, alpha_us=[0, 0], beta_us=[0, 0],
+                 cost_type=0, cost_kind=1, cost_scale_us=float(mean_service_us))
+
+
+CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5}
+
+# Policy network shapes (input, hidden..., actions) and whether a value row follows.
+MLP_SHAPES = {
+    "c1": ([8, 32, 6], False),
+    "c2": ([16, 64, 64, 12], False),
+    "c3": ([13, 128, 128, 16], True),
+    "c4": ([28, 256, 256, 48], True),
+    "c5": ([13, 128, 128, 16], True),
+}
+
+HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024}
+SEED = {name: 0x5EED0000 + i + 1 for i, name in enumerate(["c1", "c2", "c3", "c4", "c5"])}
+
+
+def mlp_dims(name: str) -> tuple:
+    dims, has_value = MLP_SHAPES[name]
+    dims = list(dims)
+    if has_value:
+        dims[-1] += 1
+    return dims, has_value
+
+
+def mlp_weights(dims, seed: int, sigma: float = 0.1):
+    """Gaussian(0, sigma) fp32 weights W_l [dims[l+1], dims[l]] and zero biases."""
+    rng = np.random.default_rng(seed)
+    Ws, bs = [], []
+    for k, n in zip(dims[:-1], dims[1:]):
+        Ws.append((rng.standard_normal((n, k)) * sigma).astype(np.float32))
+        bs.append(np.zeros(n, dtype=np.float32))
+    return Ws, bs
+
+
+def minibatch_perm(n_rows: int, seed: int, epoch: int) -> np.ndarray:
+    """The row permutation of one PPO epoch (int64)."""
+    rng = np.random.default_rng([seed, epoch])
+    return rng.permutation(n_rows).astype(np.int64)
