@@ -292,6 +292,10 @@ simx_status sim_load(simx_ctx* ctx, const uint32_t* host_buf, uint64_t n_words);
 /* OR of all env status words (synchronising).  Returns SIMX_EOVERFLOW if non-zero. */
 simx_status simx_last_status(simx_ctx* ctx, uint32_t* device_code);
 
+/* Number of kernels this library has launched in the process so far (all devices);
+   a tracing aid: the difference across a region counts the region's launches. */
+uint64_t simx_launches(void);
+
 const char* simx_strerror(simx_status s);
 const char* simx_last_error(void);
 

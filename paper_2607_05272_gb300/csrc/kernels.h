@@ -1,0 +1,93 @@
+// kernels.h — launch interfaces between the C ABI (api.cu) and the kernels.
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "../../include/simx.h"
+#include "sim.cuh"
+
+namespace simx {
+
+// Host-side count of kernel launches (every launcher adds its launches).
+void count_launches(int n);
+
+struct RolloutArgs {
+  simx_config cfg;
+  DevState st;
+  DevMlp mlp;
+  uint32_t key0, key1;
+  int policy_mode;
+  uint32_t n_actions;
+  const int32_t* ext;
+  int H;
+  int obs_dim;
+  int64_t ld;
+  float* obs;
+  uint8_t* action;
+  float* logp;
+  float* value;
+  float* reward;
+  uint8_t* done;
+  int64_t* trace;
+  float* next_obs;
+  int64_t next_ld;
+  int act_stride;   // shared floats per env
+  int scratch_off;  // offset of the softmax scratch inside an env's shared block
+};
+
+struct PolicyArgs {
+  DevMlp mlp;
+  const float* obs;
+  int64_t ld, n;
+  int mode;
+  uint32_t key0, key1, step, env_base;
+  float* logits;
+  float* value;
+  uint8_t* action;
+  float* logp;
+  int act_stride, scratch_off;
+};
+
+cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s);
+cudaError_t launch_reset(const RolloutArgs& a, cudaStream_t s);
+cudaError_t launch_observe(const RolloutArgs& a, cudaStream_t s);
+cudaError_t launch_save(const DevState& st, int32_t cost_type, uint64_t words, uint32_t* out, cudaStream_t s);
+cudaError_t launch_load(const DevState& st, int32_t cost_type, uint64_t words, const uint32_t* in, cudaStream_t s);
+cudaError_t launch_stats(const DevState& st, unsigned long long* out, cudaStream_t s);
+cudaError_t launch_repack(const float* W, const float* b, int N, int K, int Npad, float* Wt, float* bias, cudaStream_t s);
+cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s);
+int lanes_per_env();
+int envs_per_block();
+
+// returns.cu
+cudaError_t launch_returns_gae(const float* rew, const float* val, const uint8_t* done,
+                               const float* last_val, int64_t T, int64_t E, int64_t ld,
+                               float gamma, float lam, float* ret, float* adv, cudaStream_t s);
+cudaError_t launch_baseline(const float* x, int64_t n, float* adv, float* mean_out, double* ws,
+                            int nblocks, cudaStream_t s);
+int baseline_blocks(int64_t n);
+
+// loss.cu
+struct LossArgs {
+  int n_layers, has_value, n_actions;
+  int dims[SIMX_MAX_LAYERS + 1];
+  const float* W[SIMX_MAX_LAYERS];
+  const float* b[SIMX_MAX_LAYERS];
+  const float* obs;      // [T][D][E]
+  const uint8_t* action; // [T][E]
+  const float* logp_old; // [T][E]
+  const float* ret;      // [T][E] (value target) or null
+  const float* adv;      // [T][E]
+  int64_t E;             // rows per step
+  const int64_t* idx;    // minibatch rows or null
+  int64_t n;
+  int algo;
+  float clip_eps, c_value, c_entropy;
+  float* grad;           // flat gradient
+  float* stats;          // [5]
+};
+size_t loss_workspace_bytes(const LossArgs& a);
+cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
+
+}  // namespace simx

@@ -1,0 +1,999 @@
+// rollout.cu — the batched discrete-event inference-serving simulator of
+// "Adaptive Inference Batching using Policy Gradients" (Sec. 3.1 dynamics, Sec. 3.2
+// workloads, Sec. 4.1 MDP) with the policy of Sec. 4.2 fused into the step.
+//
+// One lane group (G = 8 lanes) per environment, four environments per warp.  A
+// launch runs H decision steps of every environment with its state in registers:
+// rollout_collect uses H = horizon; sim_step_batched uses H = 1.
+#include <cstdint>
+
+#include "kernels.h"
+#include "sim.cuh"
+
+namespace simx {
+
+constexpr int kG = 8;
+constexpr int kWarpsPerBlock = 8;
+constexpr int kEnvsPerBlock = kWarpsPerBlock * (32 / kG);
+
+struct Scal {
+  uint32_t now, tg, cj, cT, swi, swT, mst, ep, epo, pt, pty, pc;
+  uint32_t narr, ndrop, ndisp, nbat;
+  uint64_t swait;
+  uint32_t tld, prev, nlast, tlast;
+  float lmw, rate;
+  uint32_t na[2], nd[2];
+  uint32_t status, events;
+  uint32_t ep_cached;
+  float ep_factor;
+};
+
+// Per-environment queue state: SINGLE mode keeps it replicated in every lane;
+// ROUTE mode keeps server gl's in lane gl.
+struct Srv {
+  uint32_t busy, bsize, qh[2], qc[2];
+};
+
+__device__ __forceinline__ uint32_t add_time(uint32_t a, uint64_t b, uint32_t& status) {
+  const uint64_t s = (uint64_t)a + b;
+  if (s >= kTimeLimit) {
+    status |= kStTime;
+    return kTimeLimit;
+  }
+  return (uint32_t)s;
+}
+
+__device__ __forceinline__ uint32_t req_cost(const simx_config& c, uint32_t w3) {
+  const float E = expo1(w3);
+  if (c.cost_kind == 0) return duration_us(__fmul_rn(c.cost_scale_us, det_exp(__fmul_rn(c.pareto_inv_alpha, E))));
+  return duration_us(__fmul_rn(c.cost_scale_us, E));
+}
+
+__device__ __forceinline__ uint32_t req_type(const simx_config& c, uint32_t w1) {
+  return (c.n_types > 1 && (w1 >> 8) >= c.type0_thr) ? 1u : 0u;
+}
+
+__device__ __forceinline__ uint64_t service_us(const simx_config& c, uint32_t type, uint32_t n,
+                                               uint64_t csum) {
+  if ((int32_t)type == c.cost_type) return (uint64_t)c.alpha_us[type] + csum;
+  return (uint64_t)c.alpha_us[type] + (uint64_t)c.beta_us[type] * n;
+}
+
+// Time of the modulating chain's switch number i, given switch i-1 at t.
+__device__ __forceinline__ uint32_t switch_time(const RolloutArgs& A, uint32_t env, uint32_t i,
+                                                uint32_t t, uint32_t& status) {
+  const U4 w = philox(i, env, kStreamSwitch, 0u, A.key0, A.key1);
+  return add_time(t, duration_us(__fmul_rn(A.cfg.dwell_mean_us, expo1(w.x))), status);
+}
+
+// G consecutive candidates from (cand_j, cand_T): lane gl holds candidate cj + gl with
+// its Philox block; times are the prefix sums of integer gaps (exact in any order).
+template <int G>
+__device__ __forceinline__ void gen_chunk(const RolloutArgs& A, const Grp<G>& g, uint32_t env,
+                                          const Scal& s, uint32_t& T, bool& over, U4& w) {
+  w = philox(s.cj + g.gl, env, kStreamArrival, 0u, A.key0, A.key1);
+  const uint32_t gap = duration_us(__fmul_rn(A.cfg.cand_mean_gap_us, expo1(w.x)));
+  const uint64_t t64 = (uint64_t)s.cT + g.scan_incl(gap);
+  over = t64 >= kTimeLimit;
+  T = over ? kTimeLimit : (uint32_t)t64;
+}
+
+// SINGLE mode: consume every candidate with time <= target; accepted ones join
+// their type's FIFO (or are dropped when it is full); switches <= target apply.
+template <int G>
+__device__ void advance_single(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
+                               Srv& q, uint32_t* ringb, uint32_t* costb, uint32_t target) {
+  const simx_config& c = A.cfg;
+  const uint32_t cap = c.queue_cap;
+  for (;;) {
+    uint32_t T;
+    bool over;
+    U4 w;
+    gen_chunk<G>(A, g, env, s, T, over, w);
+    const bool cons = T <= target;
+    const int m = __popc(g.ballot(cons));
+    const int peek = m < G ? m : G - 1;
+    if (g.ballot(over && (int)g.gl <= peek)) s.status |= kStTime;
+    if (m == 0) break;
+    const uint32_t Tlast = g.shfl(T, m - 1);
+    uint32_t st = s.mst;
+    if (c.n_mod_states == 2) {
+      while (s.swT <= Tlast) {
+        if (T >= s.swT) st ^= 1u;
+        s.mst ^= 1u;
+        s.swi += 1u;
+        s.swT = switch_time(A, env, s.swi, s.swT, s.status);
+        if (++s.events > kEventCap) {
+          s.status |= kStEvent;
+          return;
+        }
+      }
+    }
+    const bool acc = cons && ((w.z >> 8) < c.accept_thr[st]);
+    const uint32_t type = req_type(c, w.y);
+    const uint32_t cst = (acc && (int32_t)type == c.cost_type) ? req_cost(c, w.w) : 0u;
+    for (uint32_t t = 0; t < c.n_types; ++t) {
+      const bool mine = acc && type == t;
+      const uint32_t bt = g.ballot(mine);
+      const uint32_t cnt = __popc(bt);
+      if (cnt == 0) continue;
+      const uint32_t room = cap - q.qc[t];
+      if (mine) {
+        const uint32_t rank = __popc(bt & ((1u << g.gl) - 1u));
+        if (rank < room) {
+          const uint32_t slot = (q.qh[t] + q.qc[t] + rank) & (cap - 1u);
+          ringb[t * cap + slot] = T;
+          if ((int32_t)t == c.cost_type) costb[slot] = cst;
+        }
+      }
+      const uint32_t adm = cnt < room ? cnt : room;
+      q.qc[t] += adm;
+      s.na[t] += cnt;
+      s.nd[t] += cnt - adm;
+      s.narr += cnt;
+      s.ndrop += cnt - adm;
+    }
+    s.cj += (uint32_t)m;
+    s.cT = Tlast;
+    s.events += (uint32_t)m;
+    if (s.events > kEventCap) {
+      s.status |= kStEvent;
+      return;
+    }
+    if (m < G) break;
+  }
+  if (c.n_mod_states == 2) {
+    while (s.swT <= target) {
+      s.mst ^= 1u;
+      s.swi += 1u;
+      s.swT = switch_time(A, env, s.swi, s.swT, s.status);
+      if (++s.events > kEventCap) {
+        s.status |= kStEvent;
+        return;
+      }
+    }
+  }
+}
+
+// Walk the modulating chain over a chunk without committing: per-lane state at
+// each candidate time, the chain's state after switches <= Tmax and their count.
+template <int G>
+__device__ __forceinline__ void tentative_states(const RolloutArgs& A, uint32_t env, const Scal& s,
+                                                 uint32_t T, uint32_t Tmax, uint32_t& st,
+                                                 uint32_t& ms, uint32_t& si, uint32_t& sT,
+                                                 uint32_t& tflag, uint32_t& nsw) {
+  st = s.mst;
+  ms = s.mst;
+  si = s.swi;
+  sT = s.swT;
+  tflag = 0;
+  nsw = 0;
+  if (A.cfg.n_mod_states != 2) return;
+  while (sT <= Tmax && nsw <= kEventCap) {
+    if (T >= sT) st ^= 1u;
+    ms ^= 1u;
+    si += 1u;
+    sT = switch_time(A, env, si, sT, tflag);
+    nsw += 1u;
+  }
+}
+
+// SINGLE mode: advance to the next accepted arrival and take in all candidates up
+// to its time (the next decision point when nothing is queued).
+template <int G>
+__device__ void jump_single(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
+                            Srv& q, uint32_t* ringb, uint32_t* costb) {
+  const simx_config& c = A.cfg;
+  for (;;) {
+    uint32_t T;
+    bool over;
+    U4 w;
+    gen_chunk<G>(A, g, env, s, T, over, w);
+    const uint32_t Tmax = g.shfl(T, G - 1);
+    uint32_t st, ms, si, sT, tflag, nsw;
+    tentative_states<G>(A, env, s, T, Tmax, st, ms, si, sT, tflag, nsw);
+    const bool acc = (w.z >> 8) < c.accept_thr[st];
+    const uint32_t bm = g.ballot(acc);
+    if (bm) {
+      const uint32_t Tf = g.shfl(T, __ffs(bm) - 1);
+      advance_single<G>(A, g, env, s, q, ringb, costb, Tf);
+      s.now = Tf;
+      return;
+    }
+    if (g.ballot(over)) s.status |= kStTime;
+    s.status |= tflag;
+    s.mst = ms;
+    s.swi = si;
+    s.swT = sT;
+    s.cj += G;
+    s.cT = Tmax;
+    s.events += G + nsw;
+    if (s.events > kEventCap) {
+      s.status |= kStEvent;
+      return;
+    }
+  }
+}
+
+// ROUTE mode: draw the next request arrival into the pending slot.
+template <int G>
+__device__ void next_arrival(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s) {
+  const simx_config& c = A.cfg;
+  if (c.arrival_kind == SIMX_ARR_THINNED) {
+    for (;;) {
+      uint32_t T;
+      bool over;
+      U4 w;
+      gen_chunk<G>(A, g, env, s, T, over, w);
+      const uint32_t Tmax = g.shfl(T, G - 1);
+      uint32_t st, ms, si, sT, tflag, nsw;
+      tentative_states<G>(A, env, s, T, Tmax, st, ms, si, sT, tflag, nsw);
+      const bool acc = (w.z >> 8) < c.accept_thr[st];
+      const uint32_t bm = g.ballot(acc);
+      if (bm) {
+        const int f = __ffs(bm) - 1;
+        const uint32_t Tf = g.shfl(T, f);
+        const uint32_t wy = g.shfl(w.y, f), ww = g.shfl(w.w, f);
+        if (g.ballot(over && (int)g.gl <= f)) s.status |= kStTime;
+        if (c.n_mod_states == 2) {
+          while (s.swT <= Tf) {
+            s.mst ^= 1u;
+            s.swi += 1u;
+            s.swT = switch_time(A, env, s.swi, s.swT, s.status);
+            if (++s.events > kEventCap) {
+              s.status |= kStEvent;
+              return;
+            }
+          }
+        }
+        s.cj += (uint32_t)f + 1u;
+        s.cT = Tf;
+        s.events += (uint32_t)f + 1u;
+        s.pt = Tf;
+        s.pty = req_type(c, wy);
+        s.pc = ((int32_t)s.pty == c.cost_type) ? req_cost(c, ww) : 0u;
+        s.narr += 1u;
+        if (s.events > kEventCap) s.status |= kStEvent;
+        return;
+      }
+      if (g.ballot(over)) s.status |= kStTime;
+      s.status |= tflag;
+      s.mst = ms;
+      s.swi = si;
+      s.swT = sT;
+      s.cj += G;
+      s.cT = Tmax;
+      s.events += G + nsw;
+      if (s.events > kEventCap) {
+        s.status |= kStEvent;
+        return;
+      }
+    }
+  }
+  // DIURNAL: constant rate inside a 500 ms epoch; a gap crossing the epoch end is
+  // discarded and redrawn from the epoch end at the next epoch's rate.  Every lane
+  // of the group computes the same values.
+  for (;;) {
+    if (++s.events > kEventCap) {
+      s.status |= kStEvent;
+      return;
+    }
+    if (s.ep_cached != s.ep) {
+      const U4 we = philox(s.ep, env, kStreamEpoch, 0u, A.key0, A.key1);
+      s.ep_factor = det_exp(__fmul_rn(c.burst_sigma, normal01(we.x, we.y)));
+      s.ep_cached = s.ep;
+    }
+    const float rate = __fmul_rn(c.diurnal_rate[(s.ep + s.epo) % c.diurnal_len], s.ep_factor);
+    const float mean = __fdiv_rn(1.0e6f, rate);
+    const U4 w = philox(s.cj, env, kStreamArrival, 0u, A.key0, A.key1);
+    const uint32_t gap = duration_us(__fmul_rn(mean, expo1(w.x)));
+    s.cj += 1u;
+    const uint64_t end = (uint64_t)(s.ep + 1u) * (uint64_t)c.epoch_us;
+    if ((uint64_t)s.cT + gap < end) {
+      s.cT = add_time(s.cT, gap, s.status);
+      s.pt = s.cT;
+      s.pty = req_type(c, w.y);
+      s.pc = ((int32_t)s.pty == c.cost_type) ? req_cost(c, w.w) : 0u;
+      s.narr += 1u;
+      return;
+    }
+    if (end >= kTimeLimit) {
+      s.status |= kStTime;
+      s.cT = kTimeLimit;
+    } else {
+      s.cT = (uint32_t)end;
+    }
+    s.ep += 1u;
+  }
+}
+
+// ROUTE mode, executed by the lane that owns the server: start a batch at time
+// st from the queue whose head arrived first (tie: type 0).
+__device__ __forceinline__ void try_start(const simx_config& c, uint32_t* ringS, uint32_t* costS,
+                                          Srv& L, uint32_t st, uint32_t& stn, uint64_t& w0,
+                                          uint64_t& w1, uint32_t& nbat, uint32_t& status) {
+  const uint32_t cap = c.queue_cap;
+  uint32_t h;
+  if (L.qc[0] > 0 && L.qc[1] > 0) {
+    const uint32_t h0 = ringS[L.qh[0]], h1 = ringS[cap + L.qh[1]];
+    h = (h1 < h0) ? 1u : 0u;
+  } else if (L.qc[0] > 0) {
+    h = 0;
+  } else if (L.qc[1] > 0) {
+    h = 1;
+  } else {
+    return;
+  }
+  const uint32_t n = L.bsize < L.qc[h] ? L.bsize : L.qc[h];
+  const bool costed = (int32_t)h == c.cost_type;
+  uint64_t W = 0, csum = 0;
+  for (uint32_t i = 0; i < n; ++i) {
+    const uint32_t slot = (L.qh[h] + i) & (cap - 1u);
+    W += (uint64_t)(st - ringS[h * cap + slot]);
+    if (costed) csum += costS[slot];
+  }
+  L.qh[h] = (L.qh[h] + n) & (cap - 1u);
+  L.qc[h] -= n;
+  L.busy = add_time(st, service_us(c, h, n, csum), status);
+  stn += n;
+  if (h) w1 += W; else w0 += W;
+  nbat += 1u;
+}
+
+__device__ __forceinline__ float fdiv_u(uint32_t a, float b) {
+  return __fdiv_rn(__uint2float_rn(a), b);
+}
+
+// Observation (Sec. 4.1 state), written to o[0..D).  SINGLE: lane 0 writes all.
+// ROUTE: lane k writes server k's three features, lane 0 the rest.
+template <int G>
+__device__ void observe_single(const simx_config& c, const Grp<G>& g, const Scal& s,
+                               const Srv& q, const uint32_t* ringb, float* o) {
+  if (g.gl == 0) {
+    const float fcap = __uint2float_rn(c.queue_cap);
+    const uint32_t T = c.n_types;
+    int i = 0;
+    for (uint32_t t = 0; t < T; ++t) o[i++] = fdiv_u(q.qc[t], fcap);
+    o[i++] = fdiv_u(s.now - s.tld, c.t_window_us);
+    uint32_t head[2] = {0u, 0u};
+    uint32_t h = kNone;
+    for (uint32_t t = 0; t < T; ++t) {
+      if (q.qc[t] == 0) continue;
+      head[t] = ringb[t * c.queue_cap + q.qh[t]];
+      if (h == kNone || head[t] < head[h]) h = t;
+    }
+    o[i++] = (h == 0) ? 1.0f : 0.0f;
+    o[i++] = (h == 1) ? 1.0f : 0.0f;
+    o[i++] = 0.0f;
+    uint32_t dt = s.now - s.prev;
+    if (dt < 1u) dt = 1u;
+    const float fdt = __uint2float_rn(dt);
+    o[i++] = __fdiv_rn(__fmul_rn(__uint2float_rn(s.na[0] + s.na[1]), c.rate_scale), fdt);
+    o[i++] = fdiv_u(s.nlast, 32.0f);
+    for (uint32_t t = 0; t < T; ++t) o[i++] = q.qc[t] > 0 ? fdiv_u(s.now - head[t], c.t_window_us) : 0.0f;
+    if (c.obs_extra) {
+      o[i++] = __fdiv_rn(__fmul_rn(__uint2float_rn(s.na[0]), c.rate_scale), fdt);
+      o[i++] = __fdiv_rn(__fmul_rn(__uint2float_rn(s.na[1]), c.rate_scale), fdt);
+      o[i++] = (s.tlast == 0) ? 1.0f : 0.0f;
+      o[i++] = (s.tlast == 1) ? 1.0f : 0.0f;
+      o[i++] = fdiv_u(s.nd[0] + s.nd[1], 32.0f);
+      o[i++] = __fdiv_rn(s.lmw, c.t_window_us);
+    }
+  }
+  g.sync();
+}
+
+template <int G>
+__device__ void observe_route(const simx_config& c, const Grp<G>& g, const Scal& s,
+                              const Srv& L, float* o) {
+  const uint32_t K = c.n_servers;
+  if (g.gl < K) {
+    const float fcap = __uint2float_rn(c.queue_cap);
+    o[3 * g.gl + 0] = fdiv_u(L.qc[0], fcap);
+    o[3 * g.gl + 1] = fdiv_u(c.n_types > 1 ? L.qc[1] : 0u, fcap);
+    const uint32_t rem = L.busy > s.now ? L.busy - s.now : 0u;
+    o[3 * g.gl + 2] = fdiv_u(rem, c.busy_norm_us);
+  }
+  if (g.gl == 0) {
+    o[3 * K] = __fdiv_rn(s.rate, c.rate_ref);
+    if (c.obs_extra) {
+      o[3 * K + 1] = (s.pty == 0) ? 1.0f : 0.0f;
+      o[3 * K + 2] = (s.pty == 1) ? 1.0f : 0.0f;
+      const uint32_t ph = (s.now + s.epo * c.epoch_us) % c.phase_period_us;
+      o[3 * K + 3] = __fdiv_rn(__uint2float_rn(ph), __uint2float_rn(c.phase_period_us));
+    }
+  }
+  g.sync();
+}
+
+__device__ __forceinline__ void load_scal(const DevState& st, uint32_t e, Scal& s) {
+  const uint32_t E = st.E;
+  const uint32_t* h = st.hdr;
+  s.now = h[F_NOW * E + e];
+  s.tg = h[F_TG * E + e];
+  s.cj = h[F_CJ * E + e];
+  s.cT = h[F_CT * E + e];
+  s.swi = h[F_SWI * E + e];
+  s.swT = h[F_SWT * E + e];
+  s.mst = h[F_MST * E + e];
+  s.ep = h[F_EP * E + e];
+  s.epo = h[F_EPO * E + e];
+  s.pt = h[F_PT * E + e];
+  s.pty = h[F_PTY * E + e];
+  s.pc = h[F_PC * E + e];
+  s.narr = h[F_NARR * E + e];
+  s.ndrop = h[F_NDROP * E + e];
+  s.ndisp = h[F_NDISP * E + e];
+  s.nbat = h[F_NBAT * E + e];
+  s.swait = (uint64_t)h[F_SWLO * E + e] | ((uint64_t)h[F_SWHI * E + e] << 32);
+  s.tld = h[F_TLD * E + e];
+  s.prev = h[F_PREV * E + e];
+  s.nlast = h[F_NLAST * E + e];
+  s.tlast = h[F_TLAST * E + e];
+  s.lmw = __uint_as_float(h[F_LMW * E + e]);
+  s.rate = __uint_as_float(h[F_RATE * E + e]);
+  s.na[0] = h[F_NA0 * E + e];
+  s.na[1] = h[F_NA1 * E + e];
+  s.nd[0] = h[F_ND0 * E + e];
+  s.nd[1] = h[F_ND1 * E + e];
+  s.status = h[F_STATUS * E + e];
+  s.events = 0;
+  s.ep_cached = kNone;
+  s.ep_factor = 0.0f;
+}
+
+__device__ __forceinline__ void store_scal(const DevState& st, uint32_t e, const Scal& s) {
+  const uint32_t E = st.E;
+  uint32_t* h = st.hdr;
+  h[F_NOW * E + e] = s.now;
+  h[F_TG * E + e] = s.tg;
+  h[F_CJ * E + e] = s.cj;
+  h[F_CT * E + e] = s.cT;
+  h[F_SWI * E + e] = s.swi;
+  h[F_SWT * E + e] = s.swT;
+  h[F_MST * E + e] = s.mst;
+  h[F_EP * E + e] = s.ep;
+  h[F_EPO * E + e] = s.epo;
+  h[F_PT * E + e] = s.pt;
+  h[F_PTY * E + e] = s.pty;
+  h[F_PC * E + e] = s.pc;
+  h[F_NARR * E + e] = s.narr;
+  h[F_NDROP * E + e] = s.ndrop;
+  h[F_NDISP * E + e] = s.ndisp;
+  h[F_NBAT * E + e] = s.nbat;
+  h[F_SWLO * E + e] = (uint32_t)s.swait;
+  h[F_SWHI * E + e] = (uint32_t)(s.swait >> 32);
+  h[F_TLD * E + e] = s.tld;
+  h[F_PREV * E + e] = s.prev;
+  h[F_NLAST * E + e] = s.nlast;
+  h[F_TLAST * E + e] = s.tlast;
+  h[F_LMW * E + e] = __float_as_uint(s.lmw);
+  h[F_RATE * E + e] = __float_as_uint(s.rate);
+  h[F_NA0 * E + e] = s.na[0];
+  h[F_NA1 * E + e] = s.na[1];
+  h[F_ND0 * E + e] = s.nd[0];
+  h[F_ND1 * E + e] = s.nd[1];
+  h[F_STATUS * E + e] = s.status;
+}
+
+__device__ __forceinline__ void load_srv(const DevState& st, uint32_t e, uint32_t k, Srv& L) {
+  const uint32_t E = st.E, K = st.K, T = st.T;
+  L.busy = st.srv[(0 * K + k) * E + e];
+  L.bsize = st.srv[(1 * K + k) * E + e];
+  for (uint32_t t = 0; t < 2; ++t) {
+    L.qh[t] = t < T ? st.qh[(k * T + t) * E + e] : 0u;
+    L.qc[t] = t < T ? st.qc[(k * T + t) * E + e] : 0u;
+  }
+}
+
+__device__ __forceinline__ void store_srv(const DevState& st, uint32_t e, uint32_t k, const Srv& L) {
+  const uint32_t E = st.E, K = st.K, T = st.T;
+  st.srv[(0 * K + k) * E + e] = L.busy;
+  st.srv[(1 * K + k) * E + e] = L.bsize;
+  for (uint32_t t = 0; t < T; ++t) {
+    st.qh[(k * T + t) * E + e] = L.qh[t];
+    st.qc[(k * T + t) * E + e] = L.qc[t];
+  }
+}
+
+// Action from the policy or a baseline (Sec. 4.2, Sec. 5.1).  Needs the
+// observation in act[0..D).
+template <int G, bool ROUTE>
+__device__ int choose_action(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
+                             const Srv& L, const uint32_t* ringb, float* act, float* scratch,
+                             float& logp, float& value) {
+  const simx_config& c = A.cfg;
+  logp = 0.0f;
+  value = 0.0f;
+  const int mode = A.policy_mode;
+  if (mode == SIMX_POLICY_SAMPLE || mode == SIMX_POLICY_ARGMAX)
+    return policy_eval<G>(A.mlp, act, scratch, mode, A.key0, A.key1, s.tg, env, logp, value, g);
+  if (mode == SIMX_POLICY_EXTERNAL) {
+    const int32_t a = A.ext[env];
+    if (a < 0 || (uint32_t)a >= A.n_actions) {
+      s.status |= kStAction;
+      return 0;
+    }
+    return a;
+  }
+  if (mode == SIMX_POLICY_RANDOM) {
+    const U4 w = philox(s.tg, env, kStreamPolicy, 0u, A.key0, A.key1);
+    return (int)(((uint64_t)(w.y >> 8) * A.n_actions) >> 24);
+  }
+  if (!ROUTE) {  // STATIC: the type whose head arrived first, batch bsizes[static_bi]
+    uint32_t h = 0;
+    if (L.qc[0] > 0 && c.n_types > 1 && L.qc[1] > 0) {
+      h = ringb[c.queue_cap + L.qh[1]] < ringb[L.qh[0]] ? 1u : 0u;
+    } else if (L.qc[0] == 0 && c.n_types > 1 && L.qc[1] > 0) {
+      h = 1u;
+    }
+    return (int)(h * c.n_bsizes + c.static_bi);
+  }
+  if (mode == SIMX_POLICY_RR) return (int)((s.tg % c.n_servers) * c.n_bsizes + c.static_bi);
+  // SQ: server with the fewest queued requests (first such)
+  uint32_t q = g.gl < c.n_servers ? (L.qc[0] + L.qc[1]) : 0xFFFFFFFFu;
+  uint32_t key = (q << 4) | g.gl;  // q <= 2 * 4096 fits in 28 bits
+  if (g.gl >= c.n_servers) key = 0xFFFFFFFFu;
+#pragma unroll
+  for (int d = G / 2; d > 0; d >>= 1) key = min(key, __shfl_xor_sync(g.mask, key, d, G));
+  return (int)((key & 15u) * c.n_bsizes + c.static_bi);
+}
+
+template <int G>
+__device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int D, float* dst,
+                                          int64_t ld, uint32_t e) {
+  if (!dst) return;
+  for (int d = (int)g.gl; d < D; d += G) dst[(int64_t)d * ld + e] = o[d];
+}
+
+// The rollout / step kernel.  Block: kWarpsPerBlock warps; each G-lane group owns
+// one env.  Shared memory: one activation vector of act_stride floats per env.
+template <bool ROUTE>
+__global__ void __launch_bounds__(kWarpsPerBlock * 32)
+k_rollout(const __grid_constant__ RolloutArgs A) {
+  extern __shared__ float smem[];
+  const Grp<kG> g;
+  const uint32_t slot = threadIdx.x / kG;
+  const uint32_t env = blockIdx.x * kEnvsPerBlock + slot;
+  if (env >= A.st.E) return;  // whole groups exit together (E splits at group bounds)
+  float* act = smem + (size_t)slot * A.act_stride;
+  float* scratch = act + A.scratch_off;
+  const simx_config& c = A.cfg;
+  const DevState& st = A.st;
+  const uint32_t K = c.n_servers, T = c.n_types, cap = c.queue_cap;
+  uint32_t* ringb = st.ring + (size_t)env * K * T * cap;
+  uint32_t* costb = st.cost ? st.cost + (size_t)env * K * cap : nullptr;
+
+  Scal s;
+  load_scal(st, env, s);
+  Srv L;
+  if (ROUTE) {
+    if (g.gl < K) load_srv(st, env, g.gl, L);
+    else L = Srv{0u, 0u, {0u, 0u}, {0u, 0u}};
+  } else {
+    load_srv(st, env, 0, L);
+  }
+  uint32_t* ringS = ROUTE ? ringb + (size_t)(g.gl < K ? g.gl : 0) * T * cap : ringb;
+  uint32_t* costS = (ROUTE && costb) ? costb + (size_t)(g.gl < K ? g.gl : 0) * cap : costb;
+  const int D = A.obs_dim;
+
+  for (int t = 0; t < A.H; ++t) {
+    if (ROUTE) observe_route<kG>(c, g, s, L, act);
+    else observe_single<kG>(c, g, s, L, ringb, act);
+    write_obs<kG>(g, act, D, A.obs ? A.obs + (int64_t)t * D * A.ld : nullptr, A.ld, env);
+    g.sync();
+    float logp, value;
+    const int a = choose_action<kG, ROUTE>(A, g, env, s, L, ringb, act, scratch, logp, value);
+    const uint32_t k = (uint32_t)a / c.n_bsizes;
+    const uint32_t b = c.bsizes[(uint32_t)a % c.n_bsizes];
+    const bool frozen = s.status != 0;
+    const uint32_t now = ROUTE ? s.pt : s.now;
+    uint32_t n_step = 0, qafter = 0;
+    uint64_t w_step = 0;
+    float reward;
+    if (!ROUTE) {
+      uint32_t n = 0;
+      uint64_t W = 0, csum = 0;
+      if (!frozen) {
+        n = b < L.qc[k] ? b : L.qc[k];
+        uint64_t wp = 0, cp = 0;
+        for (uint32_t i = g.gl; i < n; i += kG) {
+          const uint32_t sl = (L.qh[k] + i) & (cap - 1u);
+          wp += (uint64_t)(now - ringb[k * cap + sl]);
+          if ((int32_t)k == c.cost_type) cp += costb[sl];
+        }
+        W = g.sum64(wp);
+        csum = g.sum64(cp);
+        L.qh[k] = (L.qh[k] + n) & (cap - 1u);
+        L.qc[k] -= n;
+        if (n > 0) {
+          L.busy = add_time(now, service_us(c, k, n, csum), s.status);
+          s.nlast = n;
+          s.tlast = k;
+          s.tld = now;
+          s.lmw = __fdiv_rn(__ull2float_rn(W), __uint2float_rn(n));
+          s.nbat += 1u;
+        }
+        s.ndisp += n;
+        s.swait += W;
+      }
+      reward = __fsub_rn(__uint2float_rn(n), __fmul_rn(c.w_wait[k], __ull2float_rn(W)));
+      n_step = n;
+      w_step = W;
+      qafter = L.qc[0] + (T > 1 ? L.qc[1] : 0u);
+      s.prev = now;
+      s.na[0] = s.na[1] = 0u;
+      s.nd[0] = s.nd[1] = 0u;
+      s.tg += 1u;
+      if (!frozen) {
+        s.events = 0;
+        if (n > 0) {
+          const uint32_t next = L.busy;
+          advance_single<kG>(A, g, env, s, L, ringb, costb, next);
+          s.now = next;
+          if (L.qc[0] + (T > 1 ? L.qc[1] : 0u) == 0u) jump_single<kG>(A, g, env, s, L, ringb, costb);
+        } else {
+          jump_single<kG>(A, g, env, s, L, ringb, costb);
+        }
+      }
+    } else {
+      const uint32_t mt = s.pty;
+      uint32_t stn = 0, nbat = 0, lstat = 0;
+      uint64_t w0 = 0, w1 = 0;
+      if (!frozen) {
+        s.events = 0;
+        uint32_t dropped = 0;
+        if (g.gl == k) {
+          if (L.qc[mt] < cap) {
+            const uint32_t sl = (L.qh[mt] + L.qc[mt]) & (cap - 1u);
+            ringS[mt * cap + sl] = now;
+            if ((int32_t)mt == c.cost_type) costS[sl] = s.pc;
+            L.qc[mt] += 1u;
+          } else {
+            dropped = 1u;
+          }
+          L.bsize = b;
+          if (L.busy <= now) try_start(c, ringS, costS, L, now, stn, w0, w1, nbat, lstat);
+        }
+        dropped = g.shfl(dropped, (int)k);
+        s.ndrop += dropped;
+        s.nd[mt] += dropped;
+        qafter = g.sum(g.gl < K ? L.qc[0] + L.qc[1] : 0u);
+        next_arrival<kG>(A, g, env, s);
+        uint32_t gap = s.pt - now;
+        if (gap < 1u) gap = 1u;
+        const float inst = __fdiv_rn(1.0e6f, __uint2float_rn(gap));
+        s.rate = __fadd_rn(s.rate, __fmul_rn(0.0625f, __fsub_rn(inst, s.rate)));
+        if (g.gl < K)
+          while (L.busy <= s.pt && (L.qc[0] + L.qc[1]) > 0u)
+            try_start(c, ringS, costS, L, L.busy, stn, w0, w1, nbat, lstat);
+        s.now = s.pt;
+      } else {
+        qafter = g.sum(g.gl < K ? L.qc[0] + L.qc[1] : 0u);
+      }
+      stn = g.sum(stn);
+      w0 = g.sum64(w0);
+      w1 = g.sum64(w1);
+      nbat = g.sum(nbat);
+      s.status |= g.bor(lstat);
+      s.ndisp += stn;
+      s.swait += w0 + w1;
+      s.nbat += nbat;
+      reward = __fsub_rn(__uint2float_rn(stn),
+                         __fadd_rn(__fmul_rn(c.w_wait[0], __ull2float_rn(w0)),
+                                   __fmul_rn(c.w_wait[1], __ull2float_rn(w1))));
+      n_step = stn;
+      w_step = w0 + w1;
+      s.prev = now;
+      s.tg += 1u;
+    }
+    if (g.gl == 0) {
+      const int64_t o = (int64_t)t * A.ld + env;
+      if (A.action) A.action[o] = (uint8_t)a;
+      if (A.logp) A.logp[o] = logp;
+      if (A.value) A.value[o] = value;
+      if (A.reward) A.reward[o] = reward;
+      if (A.done) A.done[o] = (uint8_t)(((s.tg) % c.episode_len) == 0u);
+      if (A.trace) {
+        int64_t* tr = A.trace + (int64_t)t * SIMX_TRACE_WIDTH * A.ld + env;
+        tr[0] = now;
+        tr[A.ld] = n_step;
+        tr[2 * A.ld] = (int64_t)w_step;
+        tr[3 * A.ld] = qafter;
+      }
+    }
+    g.sync();
+  }
+  if (A.next_obs) {
+    if (ROUTE) observe_route<kG>(c, g, s, L, act);
+    else observe_single<kG>(c, g, s, L, ringb, act);
+    write_obs<kG>(g, act, D, A.next_obs, A.next_ld, env);
+  }
+  if (g.gl == 0) store_scal(st, env, s);
+  if (ROUTE) {
+    if (g.gl < K) store_srv(st, env, g.gl, L);
+  } else if (g.gl == 0) {
+    store_srv(st, env, 0, L);
+  }
+}
+
+// Reset: empty queues, idle servers, chain state from the INIT stream, then advance
+// to the first decision point.
+template <bool ROUTE>
+__global__ void __launch_bounds__(kWarpsPerBlock * 32) k_reset(const __grid_constant__ RolloutArgs A) {
+  const Grp<kG> g;
+  const uint32_t slot = threadIdx.x / kG;
+  const uint32_t env = blockIdx.x * kEnvsPerBlock + slot;
+  if (env >= A.st.E) return;
+  const simx_config& c = A.cfg;
+  const DevState& st = A.st;
+  const uint32_t K = c.n_servers, T = c.n_types, cap = c.queue_cap;
+  uint32_t* ringb = st.ring + (size_t)env * K * T * cap;
+  uint32_t* costb = st.cost ? st.cost + (size_t)env * K * cap : nullptr;
+  for (uint32_t i = g.gl; i < K * T * cap; i += kG) ringb[i] = 0u;
+  if (costb)
+    for (uint32_t i = g.gl; i < K * cap; i += kG) costb[i] = 0u;
+  Scal s;
+  s.now = s.tg = s.cj = s.cT = 0u;
+  s.ep = s.epo = s.pt = s.pty = s.pc = 0u;
+  s.narr = s.ndrop = s.ndisp = s.nbat = 0u;
+  s.swait = 0u;
+  s.tld = s.prev = s.nlast = 0u;
+  s.tlast = kNone;
+  s.lmw = 0.0f;
+  s.rate = c.rate_ref;
+  s.na[0] = s.na[1] = s.nd[0] = s.nd[1] = 0u;
+  s.status = 0u;
+  s.events = 0u;
+  s.ep_cached = kNone;
+  s.ep_factor = 0.0f;
+  const U4 w = philox(0u, env, kStreamInit, 0u, A.key0, A.key1);
+  if (c.n_mod_states == 2) {
+    s.mst = w.x >> 31;
+    s.swi = 1u;
+    s.swT = switch_time(A, env, 1u, 0u, s.status);
+  } else {
+    s.mst = 0u;
+    s.swi = 0u;
+    s.swT = kNone;
+  }
+  if (c.arrival_kind == SIMX_ARR_DIURNAL)
+    s.epo = (uint32_t)(((uint64_t)(w.y >> 8) * c.diurnal_len) >> 24);
+  Srv L{0u, c.bsizes[c.static_bi], {0u, 0u}, {0u, 0u}};
+  __syncwarp(g.mask);
+  if (ROUTE) {
+    next_arrival<kG>(A, g, env, s);
+    s.now = s.pt;
+  } else {
+    jump_single<kG>(A, g, env, s, L, ringb, costb);
+  }
+  if (g.gl == 0) store_scal(st, env, s);
+  if (ROUTE) {
+    if (g.gl < K) store_srv(st, env, g.gl, L);
+  } else if (g.gl == 0) {
+    store_srv(st, env, 0, L);
+  }
+}
+
+// Current observation of every env (no state change).
+template <bool ROUTE>
+__global__ void __launch_bounds__(kWarpsPerBlock * 32) k_observe(const __grid_constant__ RolloutArgs A) {
+  extern __shared__ float smem[];
+  const Grp<kG> g;
+  const uint32_t slot = threadIdx.x / kG;
+  const uint32_t env = blockIdx.x * kEnvsPerBlock + slot;
+  if (env >= A.st.E) return;
+  float* act = smem + (size_t)slot * A.act_stride;
+  const simx_config& c = A.cfg;
+  const uint32_t K = c.n_servers, T = c.n_types, cap = c.queue_cap;
+  const uint32_t* ringb = A.st.ring + (size_t)env * K * T * cap;
+  Scal s;
+  load_scal(A.st, env, s);
+  Srv L;
+  if (ROUTE) {
+    if (g.gl < K) load_srv(A.st, env, g.gl, L);
+    else L = Srv{0u, 0u, {0u, 0u}, {0u, 0u}};
+    observe_route<kG>(c, g, s, L, act);
+  } else {
+    load_srv(A.st, env, 0, L);
+    observe_single<kG>(c, g, s, L, ringb, act);
+  }
+  write_obs<kG>(g, act, A.obs_dim, A.next_obs, A.next_ld, env);
+}
+
+// Canonical state image of each env (header, servers, queue lengths, FIFO contents
+// from index 0, costs), one thread per env.
+__global__ void k_save(DevState st, int32_t cost_type, uint64_t words, uint32_t* out) {
+  const uint32_t e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= st.E) return;
+  uint32_t* w = out + (uint64_t)e * words;
+  const uint32_t E = st.E, K = st.K, T = st.T, cap = st.cap;
+  for (int f = 0; f < SIMX_STATE_HEADER_WORDS; ++f) w[f] = f < F_COUNT ? st.hdr[(uint64_t)f * E + e] : 0u;
+  uint32_t* p = w + SIMX_STATE_HEADER_WORDS;
+  for (uint32_t k = 0; k < K; ++k) {
+    *p++ = st.srv[(0 * K + k) * E + e];
+    *p++ = st.srv[(1 * K + k) * E + e];
+  }
+  for (uint32_t k = 0; k < K; ++k)
+    for (uint32_t t = 0; t < T; ++t) *p++ = st.qc[(k * T + t) * E + e];
+  const uint32_t* ringb = st.ring + (size_t)e * K * T * cap;
+  for (uint32_t k = 0; k < K; ++k)
+    for (uint32_t t = 0; t < T; ++t) {
+      const uint32_t h = st.qh[(k * T + t) * E + e], n = st.qc[(k * T + t) * E + e];
+      for (uint32_t i = 0; i < cap; ++i) p[i] = i < n ? ringb[(k * T + t) * cap + ((h + i) & (cap - 1u))] : 0u;
+      p += cap;
+    }
+  if (cost_type >= 0) {
+    const uint32_t* costb = st.cost + (size_t)e * K * cap;
+    for (uint32_t k = 0; k < K; ++k) {
+      const uint32_t h = st.qh[(k * T + cost_type) * E + e], n = st.qc[(k * T + cost_type) * E + e];
+      for (uint32_t i = 0; i < cap; ++i) p[i] = i < n ? costb[k * cap + ((h + i) & (cap - 1u))] : 0u;
+      p += cap;
+    }
+  }
+}
+
+__global__ void k_load(DevState st, int32_t cost_type, uint64_t words, const uint32_t* in) {
+  const uint32_t e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= st.E) return;
+  const uint32_t* w = in + (uint64_t)e * words;
+  const uint32_t E = st.E, K = st.K, T = st.T, cap = st.cap;
+  for (int f = 0; f < F_COUNT; ++f) st.hdr[(uint64_t)f * E + e] = w[f];
+  const uint32_t* p = w + SIMX_STATE_HEADER_WORDS;
+  for (uint32_t k = 0; k < K; ++k) {
+    st.srv[(0 * K + k) * E + e] = *p++;
+    st.srv[(1 * K + k) * E + e] = *p++;
+  }
+  for (uint32_t k = 0; k < K; ++k)
+    for (uint32_t t = 0; t < T; ++t) {
+      st.qc[(k * T + t) * E + e] = *p++;
+      st.qh[(k * T + t) * E + e] = 0u;
+    }
+  uint32_t* ringb = st.ring + (size_t)e * K * T * cap;
+  for (uint32_t i = 0; i < K * T * cap; ++i) ringb[i] = p[i];
+  p += K * T * cap;
+  if (cost_type >= 0) {
+    uint32_t* costb = st.cost + (size_t)e * K * cap;
+    for (uint32_t i = 0; i < K * cap; ++i) costb[i] = p[i];
+  }
+}
+
+// Aggregate counters: out[0..7] (u64) arrived, dropped, dispatched, batches, queued,
+// sum_wait, decisions, flagged; out[8] = OR of status words.
+__global__ void k_stats(DevState st, unsigned long long* out) {
+  const uint32_t e = blockIdx.x * blockDim.x + threadIdx.x;
+  unsigned long long v[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  uint32_t sor = 0;
+  if (e < st.E) {
+    const uint32_t E = st.E;
+    v[0] = st.hdr[F_NARR * E + e];
+    v[1] = st.hdr[F_NDROP * E + e];
+    v[2] = st.hdr[F_NDISP * E + e];
+    v[3] = st.hdr[F_NBAT * E + e];
+    for (uint32_t i = 0; i < st.K * st.T; ++i) v[4] += st.qc[i * E + e];
+    v[5] = (unsigned long long)st.hdr[F_SWLO * E + e] | ((unsigned long long)st.hdr[F_SWHI * E + e] << 32);
+    v[6] = st.hdr[F_TG * E + e];
+    sor = st.hdr[F_STATUS * E + e];
+    v[7] = sor ? 1ull : 0ull;
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    unsigned long long x = v[i];
+    for (int d = 16; d > 0; d >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, d);
+    if ((threadIdx.x & 31u) == 0 && x) atomicAdd(out + i, x);
+  }
+  for (int d = 16; d > 0; d >>= 1) sor |= __shfl_xor_sync(0xFFFFFFFFu, sor, d);
+  if ((threadIdx.x & 31u) == 0 && sor) atomicOr(reinterpret_cast<unsigned int*>(out + 8), sor);
+}
+
+// W [N][K] row-major -> Wt [K][Npad] (zero-padded columns), b [N] -> bias [Npad].
+__global__ void k_repack(const float* __restrict__ W, const float* __restrict__ b, int N, int K,
+                         int Npad, float* __restrict__ Wt, float* __restrict__ bias) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < K * Npad) {
+    const int k = i / Npad, j = i % Npad;
+    Wt[i] = j < N ? W[(size_t)j * K + k] : 0.0f;
+  }
+  if (i < Npad) bias[i] = i < N ? b[i] : 0.0f;
+}
+
+// Batched policy forward (Sec. 4.2) over observation columns [D][ld].
+__global__ void __launch_bounds__(kWarpsPerBlock * 32)
+k_policy_forward(const __grid_constant__ PolicyArgs P) {
+  extern __shared__ float smem[];
+  const Grp<kG> g;
+  const uint32_t slot = threadIdx.x / kG;
+  const int64_t i = (int64_t)blockIdx.x * kEnvsPerBlock + slot;
+  if (i >= P.n) return;
+  float* act = smem + (size_t)slot * P.act_stride;
+  float* scratch = act + P.scratch_off;
+  const int D = P.mlp.dims[0];
+  for (int d = (int)g.gl; d < D; d += kG) act[d] = P.obs[(int64_t)d * P.ld + i];
+  g.sync();
+  float logp, value;
+  const uint32_t env = P.env_base + (uint32_t)i;
+  const int a = policy_eval<kG>(P.mlp, act, scratch, P.mode, P.key0, P.key1, P.step, env, logp,
+                                value, g);
+  if (P.logits)
+    for (int j = (int)g.gl; j < P.mlp.n_actions; j += kG) P.logits[(int64_t)j * P.ld + i] = act[j];
+  if (g.gl == 0) {
+    if (P.value) P.value[i] = value;
+    if (P.action) P.action[i] = (uint8_t)a;
+    if (P.logp) P.logp[i] = logp;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Host launchers
+// ---------------------------------------------------------------------------
+static unsigned grid_for(uint32_t E) { return (E + kEnvsPerBlock - 1) / kEnvsPerBlock; }
+
+cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s) {
+  const size_t sh = (size_t)kEnvsPerBlock * a.act_stride * sizeof(float);
+  if (a.cfg.mode == SIMX_MODE_ROUTE) {
+    cudaFuncSetAttribute(k_rollout<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
+    k_rollout<true><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
+  } else {
+    cudaFuncSetAttribute(k_rollout<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
+    k_rollout<false><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
+  }
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_reset(const RolloutArgs& a, cudaStream_t s) {
+  if (a.cfg.mode == SIMX_MODE_ROUTE) k_reset<true><<<grid_for(a.st.E), kWarpsPerBlock * 32, 0, s>>>(a);
+  else k_reset<false><<<grid_for(a.st.E), kWarpsPerBlock * 32, 0, s>>>(a);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_observe(const RolloutArgs& a, cudaStream_t s) {
+  const size_t sh = (size_t)kEnvsPerBlock * a.act_stride * sizeof(float);
+  if (a.cfg.mode == SIMX_MODE_ROUTE) k_observe<true><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
+  else k_observe<false><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_save(const DevState& st, int32_t cost_type, uint64_t words, uint32_t* out,
+                        cudaStream_t s) {
+  k_save<<<(st.E + 127) / 128, 128, 0, s>>>(st, cost_type, words, out);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_load(const DevState& st, int32_t cost_type, uint64_t words, const uint32_t* in,
+                        cudaStream_t s) {
+  k_load<<<(st.E + 127) / 128, 128, 0, s>>>(st, cost_type, words, in);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stats(const DevState& st, unsigned long long* out, cudaStream_t s) {
+  k_stats<<<(st.E + 255) / 256, 256, 0, s>>>(st, out);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_repack(const float* W, const float* b, int N, int K, int Npad, float* Wt,
+                          float* bias, cudaStream_t s) {
+  const int n = K * Npad > Npad ? K * Npad : Npad;
+  k_repack<<<(n + 255) / 256, 256, 0, s>>>(W, b, N, K, Npad, Wt, bias);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s) {
+  const size_t sh = (size_t)kEnvsPerBlock * p.act_stride * sizeof(float);
+  cudaFuncSetAttribute(k_policy_forward, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
+  const unsigned grid = (unsigned)((p.n + kEnvsPerBlock - 1) / kEnvsPerBlock);
+  k_policy_forward<<<grid, kWarpsPerBlock * 32, sh, s>>>(p);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+int lanes_per_env() { return kG; }
+int envs_per_block() { return kEnvsPerBlock; }
+
+}  // namespace simx

@@ -1,0 +1,161 @@
+"""GPU parity of returns, GAE, the mean baseline and the loss gradients (Sec. 4.3).
+
+The oracle computes in fp64; the CUDA path in fp32 with a different association
+order, so these compare within tolerances derived from the arithmetic:
+* returns / GAE, per element: |x - x_ref| <= 1e-5 * (|x_ref| + s) where s is the
+  same recurrence run on absolute values (the sum of |terms| it adds), and per
+  tensor ||x - x_ref|| <= 1e-5 ||x_ref||;
+* loss gradients, per tensor: ||g - g_ref|| <= 1e-5 ||g_ref||, per element:
+  |g - g_ref| <= 1e-5 (|g_ref| + rms(g_ref)).
+Sizes span several blocks with ragged tails, plus the full c1 returns shape.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import rl
+from paper_2607_05272_gb300 import workloads as W
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+def _simx():
+    from paper_2607_05272_gb300 import build as B
+    B.build()
+    from paper_2607_05272_gb300 import simx
+    return simx
+
+
+def _check_recurrence(x, ref, scale):
+    x = x.astype(np.float64)
+    assert np.all(np.abs(x - ref) <= 1e-5 * (np.abs(ref) + scale) + 1e-30)
+    assert np.linalg.norm(x - ref) <= 1e-5 * np.linalg.norm(ref)
+
+
+@pytest.mark.parametrize("T,E,seg", [(10000, 64, 1000), (512, 4096, 512), (257, 333, 50), (1, 5, 1)])
+def test_reinforce_returns(T, E, seg):
+    simx = _simx()
+    rng = np.random.default_rng(T + E)
+    r = (rng.standard_normal((T, E)) * 3.0 - 1.0).astype(np.float32)
+    d = np.zeros((T, E), np.uint8)
+    d[seg - 1::seg] = 1
+    last = rng.standard_normal(E).astype(np.float32)
+    ret = torch.empty((T, E), device="cuda")
+    simx.compute_returns_gae(torch.from_numpy(r).cuda(), torch.from_numpy(d).cuda(), 0.99, -1.0,
+                             ret, last_val=torch.from_numpy(last).cuda())
+    torch.cuda.synchronize()
+    ref = rl.returns(r, d, 0.99, last)
+    scale = rl.returns(np.abs(r), d, 0.99, np.abs(last))
+    _check_recurrence(ret.cpu().numpy(), ref, scale)
+
+
+@pytest.mark.parametrize("T,E", [(256, 16384), (512, 1000), (1024, 97), (3, 40)])
+def test_gae(T, E):
+    simx = _simx()
+    rng = np.random.default_rng(T * 7 + E)
+    r = rng.standard_normal((T, E)).astype(np.float32)
+    v = rng.standard_normal((T, E)).astype(np.float32)
+    d = (rng.random((T, E)) < 0.02).astype(np.uint8)
+    d[-1] = 1
+    last = rng.standard_normal(E).astype(np.float32)
+    adv = torch.empty((T, E), device="cuda")
+    ret = torch.empty((T, E), device="cuda")
+    simx.compute_returns_gae(torch.from_numpy(r).cuda(), torch.from_numpy(d).cuda(), 0.99, 0.95,
+                             ret, adv=adv, val=torch.from_numpy(v).cuda(),
+                             last_val=torch.from_numpy(last).cuda())
+    torch.cuda.synchronize()
+    A, R = rl.gae(r, v, d, 0.99, 0.95, last)
+    # condition: the GAE recurrence on |delta| terms (|r| + gamma |V'| + |V|)
+    vn = np.vstack([v[1:], last[None]]).astype(np.float64)
+    absd = np.abs(r) + 0.99 * np.abs(vn) + np.abs(v)
+    scale = rl.returns(absd, d, 0.99 * 0.95)
+    _check_recurrence(adv.cpu().numpy(), A, scale)
+    _check_recurrence(ret.cpu().numpy(), R, scale + np.abs(v))
+
+
+@pytest.mark.parametrize("n", [1, 1000, 2_097_152])
+def test_mean_baseline(n):
+    simx = _simx()
+    rng = np.random.default_rng(n)
+    x = (rng.standard_normal(n) * 50.0 - 300.0).astype(np.float32)
+    xt = torch.from_numpy(x).cuda()
+    adv = torch.empty_like(xt)
+    mean = torch.empty(1, device="cuda")
+    ws = torch.empty(simx.returns_baseline_workspace_size(n), dtype=torch.uint8, device="cuda")
+    simx.returns_baseline(xt, adv, mean, ws)
+    torch.cuda.synchronize()
+    a_ref, m_ref = rl.baseline(x)
+    assert abs(mean.item() - m_ref) <= 1e-6 * abs(m_ref)
+    assert np.all(np.abs(adv.cpu().numpy() - a_ref) <= 1e-6 * (np.abs(x) + abs(m_ref)))
+
+
+def _rollout_for_loss(simx, name, E, H):
+    cfg = W.CONFIGS[name](E)
+    dims, hv = W.mlp_dims(name)
+    Ws, bs = W.mlp_weights(dims, 21)
+    bs = [(np.random.default_rng(l).standard_normal(b.shape) * 0.05).astype(np.float32)
+          for l, b in enumerate(bs)]
+    pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws],
+                      [torch.from_numpy(b).cuda() for b in bs], hv)
+    sim = simx.Sim(cfg)
+    sim.reset(W.SEED[name])
+    buf = simx.alloc_rollout(E, sim.D, H, has_value=hv)
+    sim.rollout("sample", H, buf, pol)
+    torch.cuda.synchronize()
+    sim.close()
+    return cfg, pol, (Ws, bs, hv), buf
+
+
+def _check_grad(g, g_ref, layers):
+    off = 0
+    for (W_, b_) in layers:
+        for size in (W_.size, b_.size):
+            gg, rr = g[off:off + size], g_ref[off:off + size]
+            off += size
+            assert np.linalg.norm(gg - rr) <= 1e-5 * np.linalg.norm(rr) + 1e-12
+            rms = np.sqrt(np.mean(rr ** 2))
+            assert np.all(np.abs(gg - rr) <= 1e-5 * (np.abs(rr) + rms) + 1e-12)
+
+
+@pytest.mark.parametrize("name,algo,E,H,nmb", [
+    ("c3", "ppo", 64, 256, 8192),
+    ("c4", "ppo", 33, 128, 3000),
+    ("c2", "reinforce", 40, 512, None),
+    ("c1", "reinforce", 16, 700, 5000),
+])
+def test_loss_gradient_matches_oracle(name, algo, E, H, nmb):
+    simx = _simx()
+    cfg, pol, host, buf = _rollout_for_loss(simx, name, E, H)
+    n_rows = E * H
+    rng = np.random.default_rng(3)
+    adv = (rng.standard_normal((H, E)) * 2.0).astype(np.float32)
+    ret = rng.standard_normal((H, E)).astype(np.float32)
+    logp = buf["logp"].cpu().numpy()
+    if algo == "ppo":
+        # move half the rows' old log-probabilities so clipping is exercised, keeping
+        # rho away from the clip edges by more than fp32 noise
+        shift = rng.choice([0.0, 0.35, -0.35], size=(H, E)).astype(np.float32)
+        logp = (logp + shift).astype(np.float32)
+        buf["logp"] = torch.from_numpy(logp).cuda()
+    idx = None if nmb is None else rng.permutation(n_rows)[:nmb].astype(np.int64)
+    n = n_rows if idx is None else len(idx)
+    grad = torch.empty(pol.n_params, device="cuda")
+    stats = torch.empty(5, device="cuda")
+    ws = torch.empty(simx.ppo_loss_grad_workspace_size(pol, n), dtype=torch.uint8, device="cuda")
+    simx.ppo_loss_grad(pol, buf, torch.from_numpy(ret).cuda(), torch.from_numpy(adv).cuda(),
+                       None if idx is None else torch.from_numpy(idx).cuda(), n, algo, 0.2, 0.5,
+                       0.01, grad, stats, ws)
+    torch.cuda.synchronize()
+    obs = buf["obs"].cpu().numpy()
+    act = buf["action"].cpu().numpy()
+    rows = np.arange(n_rows) if idx is None else idx
+    X, a, lpo = rl.gather_rows(obs, act, logp, rows, E)
+    t, e = rows // E, rows % E
+    Ws, bs, hv = host
+    grads, st = rl.loss_grad(Ws, bs, hv, X, a, lpo, adv[t, e], ret[t, e],
+                             rl.PPO if algo == "ppo" else rl.REINFORCE, 0.2, 0.5, 0.01)
+    _check_grad(grad.cpu().numpy().astype(np.float64), rl.flat(grads), list(zip(Ws, bs)))
+    s = stats.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(s[:4] - st[:4]) <= 1e-5 * (np.abs(st[:4]) + 1.0))
+    assert abs(s[4] - st[4]) <= 1.0 / n  # clip fraction: at most one row on an fp32 edge
