@@ -1,0 +1,381 @@
+#!/usr/bin/env python
+"""Throughput benchmark of the batched rollout engine (one JSON line on rank 0).
+
+Workload: the single-server bursty heterogeneous environment (4096 envs x 512
+decision steps, two-state MMPP 300/3000 req/s, 80/20 short/long requests, per-type
+queues of 256, MLP 16-64-64-12, REINFORCE with a mean-return baseline), inputs
+synthetic and seeded.  One step is one pass of the whole hot path over one batch:
+rollout_collect (simulation + fused policy) -> REINFORCE returns -> mean baseline
+-> loss gradient over all 2,097,152 rows, every stage a kernel of libsimx.so.
+
+metric: simulated decision steps per second (envs x horizon x ranks / step time).
+--impl reference times the oracle (the plain CPU reference) on a bounded sample of
+the same workload on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "simulated decision steps/sec"
+UNIT = "steps/s"
+WORKLOAD = "c2"
+SEED_BASE = 0x5EED0002
+GAMMA = 0.99
+L2_FLUSH_BYTES = 256 << 20
+
+
+def _args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-child", default=None, help=argparse.SUPPRESS)
+    return p.parse_args()
+
+
+# --------------------------------------------------------------------------- #
+# CPU reference (the oracle), run in a child process with single-threaded BLAS
+# --------------------------------------------------------------------------- #
+def _oracle_step(n_envs: int, env0: int, H: int):
+    """One oracle pass of the hot path over envs [env0, env0 + n_envs): rollout,
+    returns, mean baseline, REINFORCE loss gradient (fp64).  Returns seconds."""
+    import numpy as np
+
+    import oracle
+    from oracle import rl
+    from paper_2607_05272_gb300 import workloads as W
+    cfg = W.c2(n_envs)
+    dims, hv = W.mlp_dims(WORKLOAD)
+    Ws, bs = W.mlp_weights(dims, 1)
+    t0 = time.perf_counter()
+    out = oracle.rollout(cfg, (Ws, bs, hv), SEED_BASE, 0, list(range(env0, env0 + n_envs)), H)
+    G = rl.returns(out["reward"], out["done"], GAMMA)
+    adv, _ = rl.baseline(G)
+    X = out["obs"].transpose(0, 2, 1).reshape(-1, dims[0])
+    rl.loss_grad(Ws, bs, hv, X, out["action"].ravel(), out["logp"].ravel(), adv.ravel(),
+                 G.ravel(), rl.REINFORCE, 0.2, 0.0, 0.0)
+    return time.perf_counter() - t0
+
+
+def _cpu_child(spec: str):
+    kind, n_envs, steps, warm = spec.split(",")
+    n_envs, steps, warm = int(n_envs), int(steps), int(warm)
+    H = 512
+    times = []
+    for i in range(warm + steps):
+        dt = _oracle_step(n_envs, (i * n_envs) % 4096, H)
+        if i >= warm:
+            times.append(dt)
+    print(json.dumps({"times": times, "env_steps": n_envs * H}))
+
+
+def _run_cpu(n_envs: int, steps: int, warm: int) -> dict:
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-child",
+                        "x,%d,%d,%d" % (n_envs, steps, warm)], capture_output=True, text=True,
+                       env=env, cwd=ROOT)
+    if r.returncode != 0:
+        raise RuntimeError("oracle child failed:\n" + r.stderr[-2000:])
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def cpu_baseline() -> dict:
+    """The oracle as it stands, single-threaded, on a bounded sample (~10-20 s)."""
+    import oracle
+    oracle.build()
+    probe = _run_cpu(16, 1, 0)
+    per_env = probe["times"][0] / 16.0
+    n = int(max(16, min(4096, 12.0 / max(per_env, 1e-6))))
+    res = _run_cpu(n, 1, 0)
+    v = res["env_steps"] / res["times"][0]
+    return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": "%d envs x 512 steps of the same workload (rollout + returns + baseline + "
+                      "loss gradient), single-threaded" % n}
+
+
+def run_reference(a) -> None:
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    probe = _run_cpu(16, 1, 0)
+    per_env = probe["times"][0] / 16.0
+    budget = min(6.0, 150.0 / max(1, a.steps + a.warmup))  # whole run within a few minutes
+    n = int(max(4, min(4096, budget / max(per_env, 1e-6))))
+    res = _run_cpu(n, a.steps, a.warmup)
+    t = statistics.mean(res["times"])
+    v = res["env_steps"] / t
+    sample = ("%d envs x 512 steps per step (rollout + returns + baseline + loss gradient), "
+              "single-threaded" % n)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": a.gpus,
+        "steps": a.steps, "warmup": a.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "c2: 4096 envs x 512 steps, MMPP 300/3000 req/s, 80/20 short/long, "
+                               "MLP 16-64-64-12, REINFORCE + mean baseline",
+                   "sample_envs": n},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- #
+# GPU arm
+# --------------------------------------------------------------------------- #
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.p = None
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(index), "--query-gpu=" + self.Q,
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return None
+        self.p.terminate()
+        try:
+            out, _ = self.p.communicate(timeout=10)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+            out, _ = self.p.communicate()
+        rows = []
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 7:
+                continue
+            try:
+                rows.append((float(f[0]), float(f[1]), f[3:7]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i in range(4) if r[i].lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "sm_max_mhz": 2070.0}, "fallback"
+
+
+def run_gpu(a) -> None:
+    import numpy as np
+    import torch
+
+    from paper_2607_05272_gb300 import build as B
+    from paper_2607_05272_gb300 import workloads as W
+    B.build()
+    from paper_2607_05272_gb300 import simx
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+
+    # Replicas: every rank simulates its own 4096 envs (seed offset by rank); no
+    # data-path collective, only the timing barrier and max-reduction.
+    E, H = 4096, W.HORIZON[WORKLOAD]
+    cfg = W.c2(E)
+    dims, hv = W.mlp_dims(WORKLOAD)
+    Ws, bs = W.mlp_weights(dims, 1)
+    dWs = [torch.from_numpy(w).cuda() for w in Ws]
+    dbs = [torch.from_numpy(b).cuda() for b in bs]
+    pol = simx.Policy(dWs, dbs, hv)
+    sim = simx.Sim(cfg, device=local)
+    sim.reset(SEED_BASE + rank)
+    D = sim.D
+    n = E * H
+    buf = simx.alloc_rollout(E, D, H)
+    ret = torch.empty((H, E), device="cuda")
+    adv = torch.empty((H, E), device="cuda")
+    mean = torch.empty(1, device="cuda")
+    ws_b = torch.empty(simx.returns_baseline_workspace_size(n), dtype=torch.uint8, device="cuda")
+    grad = torch.empty(pol.n_params, device="cuda")
+    stats = torch.empty(5, device="cuda")
+    ws_l = torch.empty(simx.ppo_loss_grad_workspace_size(pol, n), dtype=torch.uint8, device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        sim.rollout("sample", H, buf, pol)
+        if ev:
+            ev[1].record(stream)
+        simx.compute_returns_gae(buf["reward"], buf["done"], GAMMA, -1.0, ret)
+        if ev:
+            ev[2].record(stream)
+        simx.returns_baseline(ret, adv, mean, ws_b)
+        if ev:
+            ev[3].record(stream)
+        simx.ppo_loss_grad(pol, buf, ret, adv, None, n, "reinforce", 0.2, 0.0, 0.0, grad, stats,
+                           ws_l)
+        if ev:
+            ev[4].record(stream)
+
+    for _ in range(a.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    # candidates generated per rollout launch (for the algorithmic FLOP count)
+    cj0 = sim.save()[:, 2].astype(np.int64)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(a.steps)]
+    clocks = Clocks(local) if rank == 0 else None
+    l0 = simx.launches()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter()
+    for k in range(a.steps):
+        flush.zero_()  # evict L2 between steps (outside the timed events)
+        step(evs[k])
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    t_wall = time.perf_counter() - t_wall
+    launches = simx.launches() - l0
+    clk = clocks.stop() if clocks else None
+    cj1 = sim.save()[:, 2].astype(np.int64)
+    cand_per_launch = float((cj1 - cj0).sum()) / a.steps
+
+    phase_ms = [[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(4)] for k in range(a.steps)]
+    step_ms = [evs[k][0].elapsed_time(evs[k][4]) for k in range(a.steps)]
+    ms = statistics.mean(step_ms)
+    ph = [statistics.mean(p[i] for p in phase_ms) for i in range(4)]
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * n / (ms * 1e-3)
+    st, code = sim.last_status()
+    if st != 0:
+        raise RuntimeError("device status 0x%x after the timed region" % code)
+
+    # end to end through the public API: policy in from pinned host memory, gradient and
+    # statistics back to the host, every step
+    e2e = None
+    if not a.no_e2e:
+        hW = [torch.from_numpy(w).pin_memory() for w in Ws]
+        hb = [torch.from_numpy(b).pin_memory() for b in bs]
+        hg = torch.empty(pol.n_params, dtype=torch.float32).pin_memory()
+        hs = torch.empty(5, dtype=torch.float32).pin_memory()
+        h2d = sum(w.numel() * 4 for w in hW) + sum(b.numel() * 4 for b in hb)
+        d2h = hg.numel() * 4 + hs.numel() * 4
+        k_e2e = max(3, min(a.steps, 50))
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(k_e2e):
+            for d, h in zip(dWs + dbs, hW + hb):
+                d.copy_(h, non_blocking=True)
+            step()
+            hg.copy_(grad, non_blocking=True)
+            hs.copy_(stats, non_blocking=True)
+            torch.cuda.synchronize()
+        t_e2e = (time.perf_counter() - t0) / k_e2e
+        if dist:
+            t = torch.tensor([t_e2e], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            t_e2e = float(t.item())
+        e2e = {"value": world * n / t_e2e, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h}
+
+    # roofline of the dominant kernel
+    peaks, src = _peaks()
+    sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
+    fp32_peak = 152 * 128 * 2 * sm_mhz * 1e6 / 1e12  # TFLOP/s, FP32 FMA lanes x clock
+    P = sum(dims[l] * dims[l + 1] for l in range(len(dims) - 1))
+    hidden = sum(dims[1:-1])
+    A = dims[-1] - (1 if hv else 0)
+    flop_rollout = n * (2.0 * P + 20.0 * hidden + 20.0 * A) + 15.0 * cand_per_launch
+    flop_loss = n * (6.0 * P - 2.0 * dims[0] * dims[1])
+    phases = {"rollout_ms": ph[0], "returns_ms": ph[1], "baseline_ms": ph[2], "loss_grad_ms": ph[3]}
+    dom = max(range(4), key=lambda i: ph[i])
+    if dom == 0:
+        ach = flop_rollout / (ph[0] * 1e-3) / 1e12
+        roof = {"kernel": "k_rollout (simulation + fused policy)", "bound": "alu", "achieved": ach,
+                "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak, "traffic": None,
+                "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz" % sm_mhz}
+    elif dom == 3:
+        ach = flop_loss / (ph[3] * 1e-3) / 1e12
+        roof = {"kernel": "loss gradient (SIMT fp32 GEMMs)", "bound": "alu", "achieved": ach,
+                "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak, "traffic": None,
+                "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz" % sm_mhz}
+    else:
+        hbm = float(peaks.get("hbm_gbs", 6800.0))
+        byts = n * 13.0 if dom == 1 else n * 12.0
+        ach = byts / (ph[dom] * 1e-3) / 1e9
+        roof = {"kernel": "returns" if dom == 1 else "baseline", "bound": "hbm", "achieved": ach,
+                "peak": hbm, "unit": "GB/s", "frac": ach / hbm, "traffic": None,
+                "peak_source": "%s hbm_gbs" % src}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps,
+            "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": "c2: 4096 envs x 512 steps per GPU, MMPP 300/3000 req/s, "
+                                   "80/20 short/long, MLP 16-64-64-12, REINFORCE + mean baseline",
+                       "envs_per_gpu": E, "horizon": H, "l2": "flushed (256 MB write) before every "
+                       "timed step", "parallelism": "replicas" if world > 1 else "single GPU"},
+            "phases_ms": phases,
+            "roofline": roof,
+            "e2e": e2e,
+            "gpu_launches": launches,
+            "clocks": clk,
+            "wall_s": t_wall,
+        }
+        if world == 1 and not a.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline()
+        print(json.dumps(line), flush=True)
+    sim.close()
+    if dist:
+        dist.destroy_process_group()
+
+
+def main():
+    a = _args()
+    if a.cpu_child:
+        _cpu_child(a.cpu_child)
+        return
+    if a.impl == "reference":
+        run_reference(a)
+    else:
+        run_gpu(a)
+
+
+if __name__ == "__main__":
+    main()

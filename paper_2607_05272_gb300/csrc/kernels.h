@@ -33,7 +33,9 @@ struct RolloutArgs {
   float* next_obs;
   int64_t next_ld;
   int act_stride;   // shared floats per env
+  int buf2_off;     // offset of the second activation buffer inside an env's block
   int scratch_off;  // offset of the softmax scratch inside an env's shared block
+  int G;            // lanes per env (8, 16 or 32)
 };
 
 struct PolicyArgs {
@@ -46,7 +48,8 @@ struct PolicyArgs {
   float* value;
   uint8_t* action;
   float* logp;
-  int act_stride, scratch_off;
+  int act_stride, buf2_off, scratch_off;
+  int G;
 };
 
 cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s);
@@ -57,8 +60,7 @@ cudaError_t launch_load(const DevState& st, int32_t cost_type, uint64_t words, c
 cudaError_t launch_stats(const DevState& st, unsigned long long* out, cudaStream_t s);
 cudaError_t launch_repack(const float* W, const float* b, int N, int K, int Npad, float* Wt, float* bias, cudaStream_t s);
 cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s);
-int lanes_per_env();
-int envs_per_block();
+int choose_lanes(int64_t envs);
 
 // returns.cu
 cudaError_t launch_returns_gae(const float* rew, const float* val, const uint8_t* done,

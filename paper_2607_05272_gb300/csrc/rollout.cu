@@ -6,15 +6,31 @@
 // launch runs H decision steps of every environment with its state in registers:
 // rollout_collect uses H = horizon; sim_step_batched uses H = 1.
 #include <cstdint>
+#include <cstdlib>
 
 #include "kernels.h"
 #include "sim.cuh"
 
 namespace simx {
 
-constexpr int kG = 8;
-constexpr int kWarpsPerBlock = 8;
-constexpr int kEnvsPerBlock = kWarpsPerBlock * (32 / kG);
+// Threads per block of the env kernels; an env is a group of G lanes, so a block
+// holds kThreads / G envs.  G (8, 16 or 32) is chosen per launch from the env count.
+constexpr int kThreads = 64;
+// At least 8 resident blocks (16 warps) per SM: caps registers at 128 per thread.
+constexpr int kMinBlocks = 8;
+
+// Two values indexed by a runtime 0/1 through selects, so that the structs below
+// stay in registers (a dynamically indexed array would be placed in local memory).
+struct Pair {
+  uint32_t v0, v1;
+  __device__ __forceinline__ uint32_t operator[](uint32_t i) const { return i ? v1 : v0; }
+  __device__ __forceinline__ void set(uint32_t i, uint32_t x) {
+    if (i) v1 = x; else v0 = x;
+  }
+  __device__ __forceinline__ void add(uint32_t i, uint32_t x) {
+    if (i) v1 += x; else v0 += x;
+  }
+};
 
 struct Scal {
   uint32_t now, tg, cj, cT, swi, swT, mst, ep, epo, pt, pty, pc;
@@ -22,7 +38,7 @@ struct Scal {
   uint64_t swait;
   uint32_t tld, prev, nlast, tlast;
   float lmw, rate;
-  uint32_t na[2], nd[2];
+  Pair na, nd;
   uint32_t status, events;
   uint32_t ep_cached;
   float ep_factor;
@@ -31,7 +47,8 @@ struct Scal {
 // Per-environment queue state: SINGLE mode keeps it replicated in every lane;
 // ROUTE mode keeps server gl's in lane gl.
 struct Srv {
-  uint32_t busy, bsize, qh[2], qc[2];
+  uint32_t busy, bsize;
+  Pair qh, qc;
 };
 
 __device__ __forceinline__ uint32_t add_time(uint32_t a, uint64_t b, uint32_t& status) {
@@ -127,9 +144,9 @@ __device__ void advance_single(const RolloutArgs& A, const Grp<G>& g, uint32_t e
         }
       }
       const uint32_t adm = cnt < room ? cnt : room;
-      q.qc[t] += adm;
-      s.na[t] += cnt;
-      s.nd[t] += cnt - adm;
+      q.qc.add(t, adm);
+      s.na.add(t, cnt);
+      s.nd.add(t, cnt - adm);
       s.narr += cnt;
       s.ndrop += cnt - adm;
     }
@@ -332,8 +349,8 @@ __device__ __forceinline__ void try_start(const simx_config& c, uint32_t* ringS,
     W += (uint64_t)(st - ringS[h * cap + slot]);
     if (costed) csum += costS[slot];
   }
-  L.qh[h] = (L.qh[h] + n) & (cap - 1u);
-  L.qc[h] -= n;
+  L.qh.set(h, (L.qh[h] + n) & (cap - 1u));
+  L.qc.set(h, L.qc[h] - n);
   L.busy = add_time(st, service_us(c, h, n, csum), status);
   stn += n;
   if (h) w1 += W; else w0 += W;
@@ -344,41 +361,71 @@ __device__ __forceinline__ float fdiv_u(uint32_t a, float b) {
   return __fdiv_rn(__uint2float_rn(a), b);
 }
 
-// Observation (Sec. 4.1 state), written to o[0..D).  SINGLE: lane 0 writes all.
+// Observation (Sec. 4.1 state), written to o[0..D).
+// SINGLE: every feature is (num * mul) / den with mul = 1 except for the rate
+// features, so one lane per feature evaluates it without branches; multiplying by
+// 1.0f is exact, so each value has the bits of the plain formula.  Layout for T types:
+// [q_t / cap]_T, (now - t_last) / T_w, head-type one-hot (2), server busy (0),
+// arrivals * rate_scale / dt, n_last / 32, [head-of-line wait_t / T_w]_T, and with
+// obs_extra: type-0 and type-1 arrival rates, last batch type one-hot (2),
+// drops / 32, last batch mean wait / T_w.
 // ROUTE: lane k writes server k's three features, lane 0 the rest.
 template <int G>
 __device__ void observe_single(const simx_config& c, const Grp<G>& g, const Scal& s,
                                const Srv& q, const uint32_t* ringb, float* o) {
-  if (g.gl == 0) {
-    const float fcap = __uint2float_rn(c.queue_cap);
-    const uint32_t T = c.n_types;
-    int i = 0;
-    for (uint32_t t = 0; t < T; ++t) o[i++] = fdiv_u(q.qc[t], fcap);
-    o[i++] = fdiv_u(s.now - s.tld, c.t_window_us);
-    uint32_t head[2] = {0u, 0u};
-    uint32_t h = kNone;
-    for (uint32_t t = 0; t < T; ++t) {
-      if (q.qc[t] == 0) continue;
-      head[t] = ringb[t * c.queue_cap + q.qh[t]];
-      if (h == kNone || head[t] < head[h]) h = t;
+  const int T = (int)c.n_types;
+  const uint32_t cap = c.queue_cap;
+  const bool ne0 = q.qc[0] > 0u, ne1 = T > 1 && q.qc[1] > 0u;
+  const uint32_t h0 = ne0 ? ringb[q.qh[0]] : 0u;
+  const uint32_t h1 = ne1 ? ringb[cap + q.qh[1]] : 0u;
+  const uint32_t head = ne0 ? ((ne1 && h1 < h0) ? 1u : 0u) : (ne1 ? 1u : kNone);
+  uint32_t dt = s.now - s.prev;
+  if (dt < 1u) dt = 1u;
+  const float fdt = __uint2float_rn(dt), fcap = __uint2float_rn(cap), tw = c.t_window_us;
+  const float rs = c.rate_scale;
+  const int D = 2 * T + 6 + (c.obs_extra ? 6 : 0);
+  for (int d = (int)g.gl; d < D; d += G) {
+    float num = 0.0f, mul = 1.0f, den = 1.0f;
+    const int r = d - T;  // position after the queue lengths
+    if (d < T) {
+      num = __uint2float_rn(d ? q.qc[1] : q.qc[0]);
+      den = fcap;
+    } else if (r == 0) {
+      num = __uint2float_rn(s.now - s.tld);
+      den = tw;
+    } else if (r == 1 || r == 2) {
+      num = head == (uint32_t)(r - 1) ? 1.0f : 0.0f;
+    } else if (r == 3) {
+      num = 0.0f;  // server status: always free at a SINGLE-mode decision
+    } else if (r == 4) {
+      num = __uint2float_rn(s.na[0] + s.na[1]);
+      mul = rs;
+      den = fdt;
+    } else if (r == 5) {
+      num = __uint2float_rn(s.nlast);
+      den = 32.0f;
+    } else if (r < 6 + T) {
+      const bool one = (r - 6) != 0;
+      const bool ne = one ? ne1 : ne0;
+      num = ne ? __uint2float_rn(s.now - (one ? h1 : h0)) : 0.0f;
+      den = tw;
+    } else {
+      const int x = r - 6 - T;
+      if (x == 0 || x == 1) {
+        num = __uint2float_rn(x ? s.na[1] : s.na[0]);
+        mul = rs;
+        den = fdt;
+      } else if (x == 2 || x == 3) {
+        num = s.tlast == (uint32_t)(x - 2) ? 1.0f : 0.0f;
+      } else if (x == 4) {
+        num = __uint2float_rn(s.nd[0] + s.nd[1]);
+        den = 32.0f;
+      } else {
+        num = s.lmw;
+        den = tw;
+      }
     }
-    o[i++] = (h == 0) ? 1.0f : 0.0f;
-    o[i++] = (h == 1) ? 1.0f : 0.0f;
-    o[i++] = 0.0f;
-    uint32_t dt = s.now - s.prev;
-    if (dt < 1u) dt = 1u;
-    const float fdt = __uint2float_rn(dt);
-    o[i++] = __fdiv_rn(__fmul_rn(__uint2float_rn(s.na[0] + s.na[1]), c.rate_scale), fdt);
-    o[i++] = fdiv_u(s.nlast, 32.0f);
-    for (uint32_t t = 0; t < T; ++t) o[i++] = q.qc[t] > 0 ? fdiv_u(s.now - head[t], c.t_window_us) : 0.0f;
-    if (c.obs_extra) {
-      o[i++] = __fdiv_rn(__fmul_rn(__uint2float_rn(s.na[0]), c.rate_scale), fdt);
-      o[i++] = __fdiv_rn(__fmul_rn(__uint2float_rn(s.na[1]), c.rate_scale), fdt);
-      o[i++] = (s.tlast == 0) ? 1.0f : 0.0f;
-      o[i++] = (s.tlast == 1) ? 1.0f : 0.0f;
-      o[i++] = fdiv_u(s.nd[0] + s.nd[1], 32.0f);
-      o[i++] = __fdiv_rn(s.lmw, c.t_window_us);
-    }
+    o[d] = __fdiv_rn(__fmul_rn(num, mul), den);
   }
   g.sync();
 }
@@ -432,10 +479,8 @@ __device__ __forceinline__ void load_scal(const DevState& st, uint32_t e, Scal& 
   s.tlast = h[F_TLAST * E + e];
   s.lmw = __uint_as_float(h[F_LMW * E + e]);
   s.rate = __uint_as_float(h[F_RATE * E + e]);
-  s.na[0] = h[F_NA0 * E + e];
-  s.na[1] = h[F_NA1 * E + e];
-  s.nd[0] = h[F_ND0 * E + e];
-  s.nd[1] = h[F_ND1 * E + e];
+  s.na = Pair{h[F_NA0 * E + e], h[F_NA1 * E + e]};
+  s.nd = Pair{h[F_ND0 * E + e], h[F_ND1 * E + e]};
   s.status = h[F_STATUS * E + e];
   s.events = 0;
   s.ep_cached = kNone;
@@ -481,8 +526,8 @@ __device__ __forceinline__ void load_srv(const DevState& st, uint32_t e, uint32_
   L.busy = st.srv[(0 * K + k) * E + e];
   L.bsize = st.srv[(1 * K + k) * E + e];
   for (uint32_t t = 0; t < 2; ++t) {
-    L.qh[t] = t < T ? st.qh[(k * T + t) * E + e] : 0u;
-    L.qc[t] = t < T ? st.qc[(k * T + t) * E + e] : 0u;
+    L.qh.set(t, t < T ? st.qh[(k * T + t) * E + e] : 0u);
+    L.qc.set(t, t < T ? st.qc[(k * T + t) * E + e] : 0u);
   }
 }
 
@@ -500,14 +545,14 @@ __device__ __forceinline__ void store_srv(const DevState& st, uint32_t e, uint32
 // observation in act[0..D).
 template <int G, bool ROUTE>
 __device__ int choose_action(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
-                             const Srv& L, const uint32_t* ringb, float* act, float* scratch,
-                             float& logp, float& value) {
+                             const Srv& L, const uint32_t* ringb, float* act, float* act2,
+                             float* scratch, float& logp, float& value) {
   const simx_config& c = A.cfg;
   logp = 0.0f;
   value = 0.0f;
   const int mode = A.policy_mode;
   if (mode == SIMX_POLICY_SAMPLE || mode == SIMX_POLICY_ARGMAX)
-    return policy_eval<G>(A.mlp, act, scratch, mode, A.key0, A.key1, s.tg, env, logp, value, g);
+    return policy_eval<G>(A.mlp, act, act2, scratch, mode, A.key0, A.key1, s.tg, env, logp, value, g);
   if (mode == SIMX_POLICY_EXTERNAL) {
     const int32_t a = A.ext[env];
     if (a < 0 || (uint32_t)a >= A.n_actions) {
@@ -546,17 +591,21 @@ __device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int D
   for (int d = (int)g.gl; d < D; d += G) dst[(int64_t)d * ld + e] = o[d];
 }
 
-// The rollout / step kernel.  Block: kWarpsPerBlock warps; each G-lane group owns
-// one env.  Shared memory: one activation vector of act_stride floats per env.
-template <bool ROUTE>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32)
+// The rollout / step kernel.  Block: kThreads threads; each G-lane group owns
+// one env.  Shared memory per env: two activation buffers and the softmax scratch.
+// Every lane stays alive to the end (groups past the last env do no work) so that
+// the whole warp reconverges at the __syncwarp() between the phases of a step.
+template <bool ROUTE, int G>
+__global__ void __launch_bounds__(kThreads, kMinBlocks)
 k_rollout(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
-  const Grp<kG> g;
-  const uint32_t slot = threadIdx.x / kG;
-  const uint32_t env = blockIdx.x * kEnvsPerBlock + slot;
-  if (env >= A.st.E) return;  // whole groups exit together (E splits at group bounds)
+  const Grp<G> g;
+  const uint32_t slot = threadIdx.x / G;
+  const uint32_t env_raw = blockIdx.x * (kThreads / G) + slot;
+  const bool live = env_raw < A.st.E;
+  const uint32_t env = live ? env_raw : 0u;
   float* act = smem + (size_t)slot * A.act_stride;
+  float* act2 = act + A.buf2_off;
   float* scratch = act + A.scratch_off;
   const simx_config& c = A.cfg;
   const DevState& st = A.st;
@@ -564,102 +613,120 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
   uint32_t* ringb = st.ring + (size_t)env * K * T * cap;
   uint32_t* costb = st.cost ? st.cost + (size_t)env * K * cap : nullptr;
 
-  Scal s;
-  load_scal(st, env, s);
-  Srv L;
-  if (ROUTE) {
-    if (g.gl < K) load_srv(st, env, g.gl, L);
-    else L = Srv{0u, 0u, {0u, 0u}, {0u, 0u}};
-  } else {
-    load_srv(st, env, 0, L);
+  Scal s{};
+  Srv L{0u, 0u, Pair{0u, 0u}, Pair{0u, 0u}};
+  if (live) {
+    load_scal(st, env, s);
+    if (ROUTE) {
+      if (g.gl < K) load_srv(st, env, g.gl, L);
+    } else {
+      load_srv(st, env, 0, L);
+    }
   }
   uint32_t* ringS = ROUTE ? ringb + (size_t)(g.gl < K ? g.gl : 0) * T * cap : ringb;
   uint32_t* costS = (ROUTE && costb) ? costb + (size_t)(g.gl < K ? g.gl : 0) * cap : costb;
   const int D = A.obs_dim;
 
   for (int t = 0; t < A.H; ++t) {
-    if (ROUTE) observe_route<kG>(c, g, s, L, act);
-    else observe_single<kG>(c, g, s, L, ringb, act);
-    write_obs<kG>(g, act, D, A.obs ? A.obs + (int64_t)t * D * A.ld : nullptr, A.ld, env);
-    g.sync();
-    float logp, value;
-    const int a = choose_action<kG, ROUTE>(A, g, env, s, L, ringb, act, scratch, logp, value);
+    // phase 1: observation (Sec. 4.1)
+    if (live) {
+      if (ROUTE) observe_route<G>(c, g, s, L, act);
+      else observe_single<G>(c, g, s, L, ringb, act);
+      write_obs<G>(g, act, D, A.obs ? A.obs + (int64_t)t * D * A.ld : nullptr, A.ld, env);
+      g.sync();
+    }
+    __syncwarp();
+    // phase 2: action (Sec. 4.2 policy or a Sec. 5.1 baseline)
+    float logp = 0.0f, value = 0.0f;
+    int a = 0;
+    if (live) a = choose_action<G, ROUTE>(A, g, env, s, L, ringb, act, act2, scratch, logp, value);
+    __syncwarp();
     const uint32_t k = (uint32_t)a / c.n_bsizes;
     const uint32_t b = c.bsizes[(uint32_t)a % c.n_bsizes];
     const bool frozen = s.status != 0;
     const uint32_t now = ROUTE ? s.pt : s.now;
     uint32_t n_step = 0, qafter = 0;
     uint64_t w_step = 0;
-    float reward;
+    float reward = 0.0f;
+    // phase 3: apply the action; phase 4: advance to the next decision point
     if (!ROUTE) {
       uint32_t n = 0;
-      uint64_t W = 0, csum = 0;
-      if (!frozen) {
-        n = b < L.qc[k] ? b : L.qc[k];
-        uint64_t wp = 0, cp = 0;
-        for (uint32_t i = g.gl; i < n; i += kG) {
-          const uint32_t sl = (L.qh[k] + i) & (cap - 1u);
-          wp += (uint64_t)(now - ringb[k * cap + sl]);
-          if ((int32_t)k == c.cost_type) cp += costb[sl];
+      if (live) {
+        uint64_t W = 0, csum = 0;
+        if (!frozen) {
+          n = b < L.qc[k] ? b : L.qc[k];
+          uint64_t wp = 0, cp = 0;
+          for (uint32_t i = g.gl; i < n; i += G) {
+            const uint32_t sl = (L.qh[k] + i) & (cap - 1u);
+            wp += (uint64_t)(now - ringb[k * cap + sl]);
+            if ((int32_t)k == c.cost_type) cp += costb[sl];
+          }
+          W = g.sum64(wp);
+          csum = g.sum64(cp);
+          L.qh.set(k, (L.qh[k] + n) & (cap - 1u));
+          L.qc.set(k, L.qc[k] - n);
+          if (n > 0) {
+            L.busy = add_time(now, service_us(c, k, n, csum), s.status);
+            s.nlast = n;
+            s.tlast = k;
+            s.tld = now;
+            s.lmw = __fdiv_rn(__ull2float_rn(W), __uint2float_rn(n));
+            s.nbat += 1u;
+          }
+          s.ndisp += n;
+          s.swait += W;
         }
-        W = g.sum64(wp);
-        csum = g.sum64(cp);
-        L.qh[k] = (L.qh[k] + n) & (cap - 1u);
-        L.qc[k] -= n;
-        if (n > 0) {
-          L.busy = add_time(now, service_us(c, k, n, csum), s.status);
-          s.nlast = n;
-          s.tlast = k;
-          s.tld = now;
-          s.lmw = __fdiv_rn(__ull2float_rn(W), __uint2float_rn(n));
-          s.nbat += 1u;
-        }
-        s.ndisp += n;
-        s.swait += W;
+        reward = __fsub_rn(__uint2float_rn(n), __fmul_rn(c.w_wait[k], __ull2float_rn(W)));
+        n_step = n;
+        w_step = W;
+        qafter = L.qc[0] + (T > 1 ? L.qc[1] : 0u);
+        s.prev = now;
+        s.na = Pair{0u, 0u};
+        s.nd = Pair{0u, 0u};
+        s.tg += 1u;
       }
-      reward = __fsub_rn(__uint2float_rn(n), __fmul_rn(c.w_wait[k], __ull2float_rn(W)));
-      n_step = n;
-      w_step = W;
-      qafter = L.qc[0] + (T > 1 ? L.qc[1] : 0u);
-      s.prev = now;
-      s.na[0] = s.na[1] = 0u;
-      s.nd[0] = s.nd[1] = 0u;
-      s.tg += 1u;
-      if (!frozen) {
+      __syncwarp();
+      if (live && !frozen) {
         s.events = 0;
         if (n > 0) {
           const uint32_t next = L.busy;
-          advance_single<kG>(A, g, env, s, L, ringb, costb, next);
+          advance_single<G>(A, g, env, s, L, ringb, costb, next);
           s.now = next;
-          if (L.qc[0] + (T > 1 ? L.qc[1] : 0u) == 0u) jump_single<kG>(A, g, env, s, L, ringb, costb);
+          if (L.qc[0] + (T > 1 ? L.qc[1] : 0u) == 0u) jump_single<G>(A, g, env, s, L, ringb, costb);
         } else {
-          jump_single<kG>(A, g, env, s, L, ringb, costb);
+          jump_single<G>(A, g, env, s, L, ringb, costb);
         }
       }
+      __syncwarp();
     } else {
       const uint32_t mt = s.pty;
       uint32_t stn = 0, nbat = 0, lstat = 0;
       uint64_t w0 = 0, w1 = 0;
-      if (!frozen) {
-        s.events = 0;
-        uint32_t dropped = 0;
-        if (g.gl == k) {
-          if (L.qc[mt] < cap) {
-            const uint32_t sl = (L.qh[mt] + L.qc[mt]) & (cap - 1u);
-            ringS[mt * cap + sl] = now;
-            if ((int32_t)mt == c.cost_type) costS[sl] = s.pc;
-            L.qc[mt] += 1u;
-          } else {
-            dropped = 1u;
+      if (live) {
+        if (!frozen) {
+          s.events = 0;
+          uint32_t dropped = 0;
+          if (g.gl == k) {
+            if (L.qc[mt] < cap) {
+              const uint32_t sl = (L.qh[mt] + L.qc[mt]) & (cap - 1u);
+              ringS[mt * cap + sl] = now;
+              if ((int32_t)mt == c.cost_type) costS[sl] = s.pc;
+              L.qc.add(mt, 1u);
+            } else {
+              dropped = 1u;
+            }
+            L.bsize = b;
+            if (L.busy <= now) try_start(c, ringS, costS, L, now, stn, w0, w1, nbat, lstat);
           }
-          L.bsize = b;
-          if (L.busy <= now) try_start(c, ringS, costS, L, now, stn, w0, w1, nbat, lstat);
+          dropped = g.shfl(dropped, (int)k);
+          s.ndrop += dropped;
+          s.nd.add(mt, dropped);
         }
-        dropped = g.shfl(dropped, (int)k);
-        s.ndrop += dropped;
-        s.nd[mt] += dropped;
         qafter = g.sum(g.gl < K ? L.qc[0] + L.qc[1] : 0u);
-        next_arrival<kG>(A, g, env, s);
+      }
+      __syncwarp();
+      if (live && !frozen) {
+        next_arrival<G>(A, g, env, s);
         uint32_t gap = s.pt - now;
         if (gap < 1u) gap = 1u;
         const float inst = __fdiv_rn(1.0e6f, __uint2float_rn(gap));
@@ -668,26 +735,28 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
           while (L.busy <= s.pt && (L.qc[0] + L.qc[1]) > 0u)
             try_start(c, ringS, costS, L, L.busy, stn, w0, w1, nbat, lstat);
         s.now = s.pt;
-      } else {
-        qafter = g.sum(g.gl < K ? L.qc[0] + L.qc[1] : 0u);
       }
-      stn = g.sum(stn);
-      w0 = g.sum64(w0);
-      w1 = g.sum64(w1);
-      nbat = g.sum(nbat);
-      s.status |= g.bor(lstat);
-      s.ndisp += stn;
-      s.swait += w0 + w1;
-      s.nbat += nbat;
-      reward = __fsub_rn(__uint2float_rn(stn),
-                         __fadd_rn(__fmul_rn(c.w_wait[0], __ull2float_rn(w0)),
-                                   __fmul_rn(c.w_wait[1], __ull2float_rn(w1))));
-      n_step = stn;
-      w_step = w0 + w1;
-      s.prev = now;
-      s.tg += 1u;
+      __syncwarp();
+      if (live) {
+        stn = g.sum(stn);
+        w0 = g.sum64(w0);
+        w1 = g.sum64(w1);
+        nbat = g.sum(nbat);
+        s.status |= g.bor(lstat);
+        s.ndisp += stn;
+        s.swait += w0 + w1;
+        s.nbat += nbat;
+        reward = __fsub_rn(__uint2float_rn(stn),
+                           __fadd_rn(__fmul_rn(c.w_wait[0], __ull2float_rn(w0)),
+                                     __fmul_rn(c.w_wait[1], __ull2float_rn(w1))));
+        n_step = stn;
+        w_step = w0 + w1;
+        s.prev = now;
+        s.tg += 1u;
+      }
     }
-    if (g.gl == 0) {
+    // phase 5: records of step t
+    if (live && g.gl == 0) {
       const int64_t o = (int64_t)t * A.ld + env;
       if (A.action) A.action[o] = (uint8_t)a;
       if (A.logp) A.logp[o] = logp;
@@ -702,12 +771,13 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
         tr[3 * A.ld] = qafter;
       }
     }
-    g.sync();
+    __syncwarp();
   }
+  if (!live) return;
   if (A.next_obs) {
-    if (ROUTE) observe_route<kG>(c, g, s, L, act);
-    else observe_single<kG>(c, g, s, L, ringb, act);
-    write_obs<kG>(g, act, D, A.next_obs, A.next_ld, env);
+    if (ROUTE) observe_route<G>(c, g, s, L, act);
+    else observe_single<G>(c, g, s, L, ringb, act);
+    write_obs<G>(g, act, D, A.next_obs, A.next_ld, env);
   }
   if (g.gl == 0) store_scal(st, env, s);
   if (ROUTE) {
@@ -719,20 +789,20 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
 
 // Reset: empty queues, idle servers, chain state from the INIT stream, then advance
 // to the first decision point.
-template <bool ROUTE>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32) k_reset(const __grid_constant__ RolloutArgs A) {
-  const Grp<kG> g;
-  const uint32_t slot = threadIdx.x / kG;
-  const uint32_t env = blockIdx.x * kEnvsPerBlock + slot;
+template <bool ROUTE, int G>
+__global__ void __launch_bounds__(kThreads) k_reset(const __grid_constant__ RolloutArgs A) {
+  const Grp<G> g;
+  const uint32_t slot = threadIdx.x / G;
+  const uint32_t env = blockIdx.x * (kThreads / G) + slot;
   if (env >= A.st.E) return;
   const simx_config& c = A.cfg;
   const DevState& st = A.st;
   const uint32_t K = c.n_servers, T = c.n_types, cap = c.queue_cap;
   uint32_t* ringb = st.ring + (size_t)env * K * T * cap;
   uint32_t* costb = st.cost ? st.cost + (size_t)env * K * cap : nullptr;
-  for (uint32_t i = g.gl; i < K * T * cap; i += kG) ringb[i] = 0u;
+  for (uint32_t i = g.gl; i < K * T * cap; i += G) ringb[i] = 0u;
   if (costb)
-    for (uint32_t i = g.gl; i < K * cap; i += kG) costb[i] = 0u;
+    for (uint32_t i = g.gl; i < K * cap; i += G) costb[i] = 0u;
   Scal s;
   s.now = s.tg = s.cj = s.cT = 0u;
   s.ep = s.epo = s.pt = s.pty = s.pc = 0u;
@@ -742,7 +812,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) k_reset(const __grid_cons
   s.tlast = kNone;
   s.lmw = 0.0f;
   s.rate = c.rate_ref;
-  s.na[0] = s.na[1] = s.nd[0] = s.nd[1] = 0u;
+  s.na = Pair{0u, 0u};
+  s.nd = Pair{0u, 0u};
   s.status = 0u;
   s.events = 0u;
   s.ep_cached = kNone;
@@ -759,13 +830,13 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) k_reset(const __grid_cons
   }
   if (c.arrival_kind == SIMX_ARR_DIURNAL)
     s.epo = (uint32_t)(((uint64_t)(w.y >> 8) * c.diurnal_len) >> 24);
-  Srv L{0u, c.bsizes[c.static_bi], {0u, 0u}, {0u, 0u}};
+  Srv L{0u, c.bsizes[c.static_bi], Pair{0u, 0u}, Pair{0u, 0u}};
   __syncwarp(g.mask);
   if (ROUTE) {
-    next_arrival<kG>(A, g, env, s);
+    next_arrival<G>(A, g, env, s);
     s.now = s.pt;
   } else {
-    jump_single<kG>(A, g, env, s, L, ringb, costb);
+    jump_single<G>(A, g, env, s, L, ringb, costb);
   }
   if (g.gl == 0) store_scal(st, env, s);
   if (ROUTE) {
@@ -776,12 +847,12 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) k_reset(const __grid_cons
 }
 
 // Current observation of every env (no state change).
-template <bool ROUTE>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32) k_observe(const __grid_constant__ RolloutArgs A) {
+template <bool ROUTE, int G>
+__global__ void __launch_bounds__(kThreads) k_observe(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
-  const Grp<kG> g;
-  const uint32_t slot = threadIdx.x / kG;
-  const uint32_t env = blockIdx.x * kEnvsPerBlock + slot;
+  const Grp<G> g;
+  const uint32_t slot = threadIdx.x / G;
+  const uint32_t env = blockIdx.x * (kThreads / G) + slot;
   if (env >= A.st.E) return;
   float* act = smem + (size_t)slot * A.act_stride;
   const simx_config& c = A.cfg;
@@ -792,13 +863,13 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) k_observe(const __grid_co
   Srv L;
   if (ROUTE) {
     if (g.gl < K) load_srv(A.st, env, g.gl, L);
-    else L = Srv{0u, 0u, {0u, 0u}, {0u, 0u}};
-    observe_route<kG>(c, g, s, L, act);
+    else L = Srv{0u, 0u, Pair{0u, 0u}, Pair{0u, 0u}};
+    observe_route<G>(c, g, s, L, act);
   } else {
     load_srv(A.st, env, 0, L);
-    observe_single<kG>(c, g, s, L, ringb, act);
+    observe_single<G>(c, g, s, L, ringb, act);
   }
-  write_obs<kG>(g, act, A.obs_dim, A.next_obs, A.next_ld, env);
+  write_obs<G>(g, act, A.obs_dim, A.next_obs, A.next_ld, env);
 }
 
 // Canonical state image of each env (header, servers, queue lengths, FIFO contents
@@ -898,24 +969,26 @@ __global__ void k_repack(const float* __restrict__ W, const float* __restrict__ 
 }
 
 // Batched policy forward (Sec. 4.2) over observation columns [D][ld].
-__global__ void __launch_bounds__(kWarpsPerBlock * 32)
+template <int G>
+__global__ void __launch_bounds__(kThreads)
 k_policy_forward(const __grid_constant__ PolicyArgs P) {
   extern __shared__ float smem[];
-  const Grp<kG> g;
-  const uint32_t slot = threadIdx.x / kG;
-  const int64_t i = (int64_t)blockIdx.x * kEnvsPerBlock + slot;
+  const Grp<G> g;
+  const uint32_t slot = threadIdx.x / G;
+  const int64_t i = (int64_t)blockIdx.x * (kThreads / G) + slot;
   if (i >= P.n) return;
   float* act = smem + (size_t)slot * P.act_stride;
   float* scratch = act + P.scratch_off;
   const int D = P.mlp.dims[0];
-  for (int d = (int)g.gl; d < D; d += kG) act[d] = P.obs[(int64_t)d * P.ld + i];
+  for (int d = (int)g.gl; d < D; d += G) act[d] = P.obs[(int64_t)d * P.ld + i];
   g.sync();
   float logp, value;
   const uint32_t env = P.env_base + (uint32_t)i;
-  const int a = policy_eval<kG>(P.mlp, act, scratch, P.mode, P.key0, P.key1, P.step, env, logp,
-                                value, g);
+  float* z = nullptr;
+  const int a = policy_eval<G>(P.mlp, act, act + P.buf2_off, scratch, P.mode, P.key0, P.key1,
+                                P.step, env, logp, value, g, &z);
   if (P.logits)
-    for (int j = (int)g.gl; j < P.mlp.n_actions; j += kG) P.logits[(int64_t)j * P.ld + i] = act[j];
+    for (int j = (int)g.gl; j < P.mlp.n_actions; j += G) P.logits[(int64_t)j * P.ld + i] = z[j];
   if (g.gl == 0) {
     if (P.value) P.value[i] = value;
     if (P.action) P.action[i] = (uint8_t)a;
@@ -926,35 +999,47 @@ k_policy_forward(const __grid_constant__ PolicyArgs P) {
 // ---------------------------------------------------------------------------
 // Host launchers
 // ---------------------------------------------------------------------------
-static unsigned grid_for(uint32_t E) { return (E + kEnvsPerBlock - 1) / kEnvsPerBlock; }
+template <int G>
+static unsigned grid_for(int64_t E) { return (unsigned)((E + kThreads / G - 1) / (kThreads / G)); }
 
-cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s) {
-  const size_t sh = (size_t)kEnvsPerBlock * a.act_stride * sizeof(float);
-  if (a.cfg.mode == SIMX_MODE_ROUTE) {
-    cudaFuncSetAttribute(k_rollout<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
-    k_rollout<true><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
-  } else {
-    cudaFuncSetAttribute(k_rollout<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
-    k_rollout<false><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
-  }
+template <bool ROUTE, int G>
+static cudaError_t rollout_t(const RolloutArgs& a, cudaStream_t s) {
+  const size_t sh = (size_t)(kThreads / G) * a.act_stride * sizeof(float);
+  cudaFuncSetAttribute(k_rollout<ROUTE, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
+  k_rollout<ROUTE, G><<<grid_for<G>(a.st.E), kThreads, sh, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
 
-cudaError_t launch_reset(const RolloutArgs& a, cudaStream_t s) {
-  if (a.cfg.mode == SIMX_MODE_ROUTE) k_reset<true><<<grid_for(a.st.E), kWarpsPerBlock * 32, 0, s>>>(a);
-  else k_reset<false><<<grid_for(a.st.E), kWarpsPerBlock * 32, 0, s>>>(a);
+template <bool ROUTE, int G>
+static cudaError_t reset_t(const RolloutArgs& a, cudaStream_t s) {
+  k_reset<ROUTE, G><<<grid_for<G>(a.st.E), kThreads, 0, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
 
-cudaError_t launch_observe(const RolloutArgs& a, cudaStream_t s) {
-  const size_t sh = (size_t)kEnvsPerBlock * a.act_stride * sizeof(float);
-  if (a.cfg.mode == SIMX_MODE_ROUTE) k_observe<true><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
-  else k_observe<false><<<grid_for(a.st.E), kWarpsPerBlock * 32, sh, s>>>(a);
+template <bool ROUTE, int G>
+static cudaError_t observe_t(const RolloutArgs& a, cudaStream_t s) {
+  const size_t sh = (size_t)(kThreads / G) * a.act_stride * sizeof(float);
+  k_observe<ROUTE, G><<<grid_for<G>(a.st.E), kThreads, sh, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
+
+#define SIMX_DISPATCH(fn, a, s)                                                        \
+  do {                                                                                 \
+    const bool route = (a).cfg.mode == SIMX_MODE_ROUTE;                                \
+    switch ((a).G) {                                                                   \
+      case 8: return route ? fn<true, 8>(a, s) : fn<false, 8>(a, s);                  \
+      case 16: return route ? fn<true, 16>(a, s) : fn<false, 16>(a, s);               \
+      case 32: return route ? fn<true, 32>(a, s) : fn<false, 32>(a, s);               \
+      default: return cudaErrorInvalidValue;                                           \
+    }                                                                                  \
+  } while (0)
+
+cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s) { SIMX_DISPATCH(rollout_t, a, s); }
+cudaError_t launch_reset(const RolloutArgs& a, cudaStream_t s) { SIMX_DISPATCH(reset_t, a, s); }
+cudaError_t launch_observe(const RolloutArgs& a, cudaStream_t s) { SIMX_DISPATCH(observe_t, a, s); }
 
 cudaError_t launch_save(const DevState& st, int32_t cost_type, uint64_t words, uint32_t* out,
                         cudaStream_t s) {
@@ -984,16 +1069,36 @@ cudaError_t launch_repack(const float* W, const float* b, int N, int K, int Npad
   return cudaGetLastError();
 }
 
-cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s) {
-  const size_t sh = (size_t)kEnvsPerBlock * p.act_stride * sizeof(float);
-  cudaFuncSetAttribute(k_policy_forward, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
-  const unsigned grid = (unsigned)((p.n + kEnvsPerBlock - 1) / kEnvsPerBlock);
-  k_policy_forward<<<grid, kWarpsPerBlock * 32, sh, s>>>(p);
+template <int G>
+static cudaError_t policy_forward_t(const PolicyArgs& p, cudaStream_t s) {
+  const size_t sh = (size_t)(kThreads / G) * p.act_stride * sizeof(float);
+  cudaFuncSetAttribute(k_policy_forward<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
+  k_policy_forward<G><<<grid_for<G>(p.n), kThreads, sh, s>>>(p);
   count_launches(1);
   return cudaGetLastError();
 }
 
-int lanes_per_env() { return kG; }
-int envs_per_block() { return kEnvsPerBlock; }
+cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s) {
+  switch (p.G) {
+    case 8: return policy_forward_t<8>(p, s);
+    case 16: return policy_forward_t<16>(p, s);
+    case 32: return policy_forward_t<32>(p, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+// Lanes per env: enough warps to cover every SM at the occupancy the registers
+// allow (about 16 warps per SM), but never fewer than 8 lanes per env.
+// The environment variable SIMX_LANES (8, 16 or 32) overrides the choice.
+int choose_lanes(int64_t envs) {
+  if (const char* f = getenv("SIMX_LANES")) {
+    const int v = atoi(f);
+    if (v == 8 || v == 16 || v == 32) return v;
+  }
+  const int64_t target_warps = 152 * 16;
+  if (envs * 32 / 32 <= target_warps) return 32;
+  if (envs * 16 / 32 <= target_warps) return 16;
+  return 8;
+}
 
 }  // namespace simx

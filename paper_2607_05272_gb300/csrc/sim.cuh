@@ -93,74 +93,108 @@ struct Grp {
   __device__ __forceinline__ void sync() const { __syncwarp(mask); }
 };
 
-// One tanh MLP layer for one environment, computed by its G lanes in place on the
-// environment's shared-memory activation vector act[0..K) -> act[0..N).
-// Lane gl owns outputs 4 gl + 4 G b + c; every output is the fp32 fused
-// multiply-add chain over k = 0..K-1 in order from 0, then + bias (Sec. 4.2).
-constexpr int kMaxAcc = 36;  // 4 G * 9 >= 288 >= padded 257 outputs
+// One tanh MLP layer for one environment, computed by its G lanes from the
+// shared-memory activation vector x[0..K) into y[0..N) (a second buffer).
+// Lane gl owns outputs 4 gl + 4 G b + c, taken in passes of at most kPass column
+// blocks (16 accumulators); every output is the fp32 fused multiply-add chain over
+// k = 0..K-1 in order from 0, then + bias (Sec. 4.2).  The k loop is unrolled by
+// four (one float4 of activations, four weight rows) with the per-output order
+// unchanged.  tanh is applied afterwards, one output per lane at a time.
+constexpr int kPass = 4;
+
 template <int G>
 __device__ __forceinline__ void mlp_layer(const float* __restrict__ Wt,
                                           const float* __restrict__ bias, int K, int N,
-                                          int Npad, float* act, bool do_tanh,
+                                          int Npad, const float* x, float* y, bool do_tanh,
                                           const Grp<G>& g) {
-  float acc[kMaxAcc];
-#pragma unroll
-  for (int p = 0; p < kMaxAcc; ++p) acc[p] = 0.0f;
   const int nb = Npad / (4 * G);
   const float* wp = Wt + 4 * g.gl;
-  for (int k = 0; k < K; ++k) {
-    const float xk = act[k];
-    const float* wr = wp + (size_t)k * Npad;
+  for (int p0 = 0; p0 < nb; p0 += kPass) {
+    float acc[4 * kPass];
 #pragma unroll
-    for (int b = 0; b < kMaxAcc / 4; ++b) {
-      if (b < nb) {
-        const float4 w4 = __ldg(reinterpret_cast<const float4*>(wr + 4 * G * b));
-        acc[4 * b + 0] = __fmaf_rn(w4.x, xk, acc[4 * b + 0]);
-        acc[4 * b + 1] = __fmaf_rn(w4.y, xk, acc[4 * b + 1]);
-        acc[4 * b + 2] = __fmaf_rn(w4.z, xk, acc[4 * b + 2]);
-        acc[4 * b + 3] = __fmaf_rn(w4.w, xk, acc[4 * b + 3]);
+    for (int q = 0; q < 4 * kPass; ++q) acc[q] = 0.0f;
+    int k = 0;
+    for (; k + 4 <= K; k += 4) {
+      const float4 xv = *reinterpret_cast<const float4*>(x + k);
+      const float* wr = wp + (size_t)k * Npad + 4 * G * p0;
+#pragma unroll
+      for (int b = 0; b < kPass; ++b) {
+        if (p0 + b < nb) {
+          const float4 w0 = __ldg(reinterpret_cast<const float4*>(wr + 4 * G * b));
+          const float4 w1 = __ldg(reinterpret_cast<const float4*>(wr + Npad + 4 * G * b));
+          const float4 w2 = __ldg(reinterpret_cast<const float4*>(wr + 2 * Npad + 4 * G * b));
+          const float4 w3 = __ldg(reinterpret_cast<const float4*>(wr + 3 * Npad + 4 * G * b));
+          float* a4 = acc + 4 * b;
+          a4[0] = __fmaf_rn(w3.x, xv.w, __fmaf_rn(w2.x, xv.z, __fmaf_rn(w1.x, xv.y, __fmaf_rn(w0.x, xv.x, a4[0]))));
+          a4[1] = __fmaf_rn(w3.y, xv.w, __fmaf_rn(w2.y, xv.z, __fmaf_rn(w1.y, xv.y, __fmaf_rn(w0.y, xv.x, a4[1]))));
+          a4[2] = __fmaf_rn(w3.z, xv.w, __fmaf_rn(w2.z, xv.z, __fmaf_rn(w1.z, xv.y, __fmaf_rn(w0.z, xv.x, a4[2]))));
+          a4[3] = __fmaf_rn(w3.w, xv.w, __fmaf_rn(w2.w, xv.z, __fmaf_rn(w1.w, xv.y, __fmaf_rn(w0.w, xv.x, a4[3]))));
+        }
       }
     }
-  }
-  g.sync();
+    for (; k < K; ++k) {
+      const float xk = x[k];
+      const float* wr = wp + (size_t)k * Npad + 4 * G * p0;
 #pragma unroll
-  for (int b = 0; b < kMaxAcc / 4; ++b) {
-    if (b < nb) {
+      for (int b = 0; b < kPass; ++b) {
+        if (p0 + b < nb) {
+          const float4 w4 = __ldg(reinterpret_cast<const float4*>(wr + 4 * G * b));
+          acc[4 * b + 0] = __fmaf_rn(w4.x, xk, acc[4 * b + 0]);
+          acc[4 * b + 1] = __fmaf_rn(w4.y, xk, acc[4 * b + 1]);
+          acc[4 * b + 2] = __fmaf_rn(w4.z, xk, acc[4 * b + 2]);
+          acc[4 * b + 3] = __fmaf_rn(w4.w, xk, acc[4 * b + 3]);
+        }
+      }
+    }
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int j = 4 * (int)g.gl + 4 * G * b + c;
-        if (j < N) {
-          const float z = __fadd_rn(acc[4 * b + c], __ldg(bias + j));
-          act[j] = do_tanh ? det_tanh(z) : z;
+    for (int b = 0; b < kPass; ++b) {
+      if (p0 + b < nb) {
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+          const int j = 4 * (int)g.gl + 4 * G * (p0 + b) + cc;
+          if (j < N) y[j] = __fadd_rn(acc[4 * b + cc], __ldg(bias + j));
         }
       }
     }
   }
   g.sync();
+  if (do_tanh) {
+    for (int j = (int)g.gl; j < N; j += G) y[j] = det_tanh(y[j]);
+    g.sync();
+  }
 }
 
-// Policy head on the environment's activation vector (Sec. 4.2): forward through
-// all layers, then (mode SAMPLE) categorical sampling by inversion of the
-// cumulative softmax with a POLICY-stream uniform, or (ARGMAX) the first largest
-// logit.  p_i = e^{z_i - max} are computed by the lanes in parallel and summed by
-// lane 0 in index order.  Returns the action; logp/value valid in every lane.
-// scratch must hold n_actions floats.
+// Policy head (Sec. 4.2) on the observation in bufA: forward through all layers
+// (alternating bufA / bufB), then (mode SAMPLE) categorical sampling by inversion of
+// the cumulative softmax with a POLICY-stream uniform, or (ARGMAX) the first
+// largest logit.  p_i = e^{z_i - max} are computed by the lanes in parallel and summed
+// by lane 0 in index order.  Returns the action; logp/value valid in every lane;
+// *zout (if given) points at the logits.  scratch holds n_actions floats.
 template <int G>
-__device__ __forceinline__ int policy_eval(const DevMlp& m, float* act, float* scratch,
-                                           int mode, uint32_t key0, uint32_t key1,
-                                           uint32_t step, uint32_t env, float& logp,
-                                           float& value, const Grp<G>& g) {
-  for (int l = 0; l < m.n_layers; ++l)
-    mlp_layer<G>(m.Wt[l], m.bias[l], m.dims[l], m.dims[l + 1], m.npad[l + 1], act,
+__device__ __forceinline__ int policy_eval(const DevMlp& m, float* bufA, float* bufB,
+                                           float* scratch, int mode, uint32_t key0,
+                                           uint32_t key1, uint32_t step, uint32_t env,
+                                           float& logp, float& value, const Grp<G>& g,
+                                           float** zout = nullptr) {
+  float* in = bufA;
+  float* out = bufB;
+  for (int l = 0; l < m.n_layers; ++l) {
+    mlp_layer<G>(m.Wt[l], m.bias[l], m.dims[l], m.dims[l + 1], m.npad[l + 1], in, out,
                  l + 1 < m.n_layers, g);
+    float* t = in;
+    in = out;
+    out = t;
+  }
+  const float* z = in;
+  if (zout) *zout = in;
   const int A = m.n_actions;
   // group argmax (first index of the largest logit)
   float mx = -__uint_as_float(0x7F800000u);
   int ai = 0x7FFFFFFF;
   for (int i = (int)g.gl; i < A; i += G) {
-    const float z = act[i];
-    if (z > mx) {
-      mx = z;
+    const float v = z[i];
+    if (v > mx) {
+      mx = v;
       ai = i;
     }
   }
@@ -173,7 +207,7 @@ __device__ __forceinline__ int policy_eval(const DevMlp& m, float* act, float* s
       ai = oi;
     }
   }
-  for (int i = (int)g.gl; i < A; i += G) scratch[i] = det_exp(__fsub_rn(act[i], mx));
+  for (int i = (int)g.gl; i < A; i += G) scratch[i] = det_exp(__fsub_rn(z[i], mx));
   g.sync();
   int a = 0;
   float lp = 0.0f;
@@ -195,11 +229,11 @@ __device__ __forceinline__ int policy_eval(const DevMlp& m, float* act, float* s
         }
       }
     }
-    lp = __fsub_rn(__fsub_rn(act[a], mx), det_log(S));
+    lp = __fsub_rn(__fsub_rn(z[a], mx), det_log(S));
   }
   a = (int)g.shfl((uint32_t)a, 0);
   logp = g.shflf(lp, 0);
-  value = m.has_value ? act[A] : 0.0f;
+  value = m.has_value ? z[A] : 0.0f;
   g.sync();
   return a;
 }

@@ -80,6 +80,18 @@ def test_rollout_matches_oracle(name, mk, H, mode):
     _assert_same(got, ref, W.MLP_SHAPES[name][1])
 
 
+@pytest.mark.parametrize("lanes", [8, 16, 32])
+@pytest.mark.parametrize("name,mk,H,mode", [c for c in CASES if c[0] != "c1"] +
+                         [("c1", lambda: W.c1(23), 1500, "sample")],
+                         ids=[c[0] for c in CASES if c[0] != "c1"] + ["c1"])
+def test_rollout_every_lane_width(name, mk, H, mode, lanes, monkeypatch):
+    """The same results whichever number of lanes (8, 16, 32) serves an env."""
+    monkeypatch.setenv("SIMX_LANES", str(lanes))
+    got, ref, st, code = _run(name, mk(), min(H, 300), mode)
+    assert st == 0 and code == 0
+    _assert_same(got, ref, W.MLP_SHAPES[name][1])
+
+
 BASELINES = [
     ("c1", lambda: W.c1(33), 2000, "static"),
     ("c2", lambda: W.c2(33), 512, "static"),
