@@ -101,13 +101,11 @@ simx_status validate_config(const simx_config* c) {
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
 
-// Shared floats per env: two activation buffers (widest layer each) + softmax
-// scratch, with a stride that spreads the envs of a warp over distinct banks.
-void act_layout(int maxdim, int n_actions, int& stride, int& buf2_off, int& scratch_off) {
-  buf2_off = round_up(maxdim, 4);
-  scratch_off = 2 * buf2_off;
-  stride = scratch_off + round_up(n_actions > 0 ? n_actions : 1, 4);
-  if (stride % 32 == 0 || stride % 32 == 16) stride += 4;
+// Shared-memory geometry of the env kernels: activation rows (widest layer) and
+// softmax scratch per env, both rounded to float4.
+void act_layout(int maxdim, int n_actions, int& maxd4, int& apad) {
+  maxd4 = round_up(maxdim, 4);
+  apad = round_up(n_actions > 0 ? n_actions : 1, 4);
 }
 
 simx_status validate_mlp(const simx_mlp* m, uint32_t obs_dim, uint32_t n_actions) {
@@ -133,11 +131,11 @@ struct Packed {
   int device = -1;
 };
 
-simx_status pack_mlp(const simx_mlp* m, int G, Packed& P, DevMlp& out, cudaStream_t s) {
+simx_status pack_mlp(const simx_mlp* m, Packed& P, DevMlp& out, cudaStream_t s) {
   size_t need = 0;
   int npad[SIMX_MAX_LAYERS + 1];
   for (int l = 0; l < m->n_layers; ++l) {
-    npad[l + 1] = round_up(m->dims[l + 1], 4 * G);
+    npad[l + 1] = round_up(m->dims[l + 1], 4);
     need += (size_t)m->dims[l] * npad[l + 1] + npad[l + 1];
   }
   if (need > P.cap) {
@@ -302,7 +300,8 @@ static void base_args(simx_ctx* c, RolloutArgs& a) {
   a.ld = c->cfg.n_envs;
   a.next_ld = c->cfg.n_envs;
   a.G = choose_lanes(c->cfg.n_envs);
-  act_layout((int)c->cfg.obs_dim, (int)a.n_actions, a.act_stride, a.buf2_off, a.scratch_off);
+  a.threads = choose_threads(c->cfg.n_envs, a.G);
+  act_layout((int)c->cfg.obs_dim, (int)a.n_actions, a.maxd4, a.apad);
 }
 
 simx_status sim_reset(simx_ctx* c, uint64_t seed, void* stream) {
@@ -342,9 +341,9 @@ static simx_status prepare_policy(simx_ctx* c, const simx_mlp* pol, int mode, Ro
     case SIMX_POLICY_ARGMAX: {
       simx_status v = validate_mlp(pol, c->cfg.obs_dim, a.n_actions);
       if (v != SIMX_OK) return v;
-      v = pack_mlp(pol, a.G, c->pack, a.mlp, s);
+      v = pack_mlp(pol, c->pack, a.mlp, s);
       if (v != SIMX_OK) return v;
-      act_layout(mlp_maxdim(pol), (int)a.n_actions, a.act_stride, a.buf2_off, a.scratch_off);
+      act_layout(mlp_maxdim(pol), (int)a.n_actions, a.maxd4, a.apad);
       break;
     }
     case SIMX_POLICY_STATIC:
@@ -448,9 +447,10 @@ simx_status policy_forward(const simx_mlp* pol, const float* d_obs, int64_t ld, 
   std::memset(&p, 0, sizeof(p));
   const cudaStream_t s = (cudaStream_t)stream;
   p.G = choose_lanes(n);
-  v = pack_mlp(pol, p.G, g_pf_pack[dev], p.mlp, s);
+  p.threads = choose_threads(n, p.G);
+  v = pack_mlp(pol, g_pf_pack[dev], p.mlp, s);
   if (v != SIMX_OK) return v;
-  act_layout(mlp_maxdim(pol), p.mlp.n_actions, p.act_stride, p.buf2_off, p.scratch_off);
+  act_layout(mlp_maxdim(pol), p.mlp.n_actions, p.maxd4, p.apad);
   p.obs = d_obs;
   p.ld = ld;
   p.n = n;

@@ -32,10 +32,10 @@ struct RolloutArgs {
   int64_t* trace;
   float* next_obs;
   int64_t next_ld;
-  int act_stride;   // shared floats per env
-  int buf2_off;     // offset of the second activation buffer inside an env's block
-  int scratch_off;  // offset of the softmax scratch inside an env's shared block
+  int maxd4;        // rows of each activation buffer (widest layer, multiple of 4)
+  int apad;         // softmax scratch floats per env (multiple of 4)
   int G;            // lanes per env (8, 16 or 32)
+  int threads;      // threads per block (64, 128 or 256)
 };
 
 struct PolicyArgs {
@@ -48,8 +48,8 @@ struct PolicyArgs {
   float* value;
   uint8_t* action;
   float* logp;
-  int act_stride, buf2_off, scratch_off;
-  int G;
+  int maxd4, apad;
+  int G, threads;
 };
 
 cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s);
@@ -61,6 +61,7 @@ cudaError_t launch_stats(const DevState& st, unsigned long long* out, cudaStream
 cudaError_t launch_repack(const float* W, const float* b, int N, int K, int Npad, float* Wt, float* bias, cudaStream_t s);
 cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s);
 int choose_lanes(int64_t envs);
+int choose_threads(int64_t envs, int G);
 
 // returns.cu
 cudaError_t launch_returns_gae(const float* rew, const float* val, const uint8_t* done,
@@ -90,6 +91,10 @@ struct LossArgs {
   float* stats;          // [5]
 };
 size_t loss_workspace_bytes(const LossArgs& a);
+// loss_fused.cu
+bool loss_fused_fits(const LossArgs& a);
+size_t loss_fused_workspace(const LossArgs& a);
+cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 
 }  // namespace simx

@@ -279,9 +279,14 @@ static WsLayout layout(const LossArgs& a) {
   return w;
 }
 
-size_t loss_workspace_bytes(const LossArgs& a) { return layout(a).total; }
+size_t loss_workspace_bytes(const LossArgs& a) {
+  return loss_fused_fits(a) ? loss_fused_workspace(a) : layout(a).total;
+}
 
+// Policies whose parameters and per-tile activations fit in shared memory take the
+// fused one-kernel path (loss_fused.cu); wider ones the GEMM pipeline below.
 cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s) {
+  if (loss_fused_fits(a)) return launch_loss_fused(a, ws, ws_bytes, s);
   const WsLayout w = layout(a);
   if (ws_bytes < w.total) return cudaErrorInvalidValue;
   char* base = static_cast<char*>(ws);

@@ -1,0 +1,408 @@
+// loss_fused.cu — REINFORCE / PPO loss gradient (Sec. 4.3) in one persistent kernel
+// for policies whose parameters fit in shared memory.
+//
+// Each block walks row tiles of R = 32 minibatch rows.  Per tile: gather the rows'
+// observations, run the forward pass keeping every activation in shared memory
+// (feature-major, [feature][row]), evaluate the loss head per row (log-softmax,
+// rho, clipped surrogate, entropy, value residual -> dL/dZ), then the backward pass:
+//   dW_l += dZ_l^T H_l   (each thread owns 4 x 4 blocks of dW_l, accumulated in
+//                         shared memory across all of the block's tiles),
+//   db_l += column sums of dZ_l,
+//   dZ_{l-1} = (dZ_l W_l) * (1 - H_l^2).
+// Every GEMM is a register-tiled shared-memory product (4 rows x 4 columns per thread,
+// one float4 of each operand per step).  At the end each block writes its dW/db and
+// fp64 loss statistics; a second kernel sums the blocks in block order, so the result
+// is deterministic for a given launch configuration.  Nothing touches HBM but the
+// gathered observations and the per-block partials.
+#include <cstdint>
+
+#include "devmath.cuh"
+#include "kernels.h"
+
+namespace simx {
+
+constexpr int kLR = 32;                // rows per tile
+constexpr int kLld = kLR + 4;          // row stride of the activation buffers
+constexpr int kLThreads = 256;
+
+// Y[j][r] = sum_k Wt[k][j] X[k][r] (+ epilogue) for rows r < R, outputs j < N.
+// Wt is row-major with row stride ldw (a multiple of 4, 16-byte aligned).
+// epi 0: + bias, tanh when do_tanh; epi 1: * (1 - H[j][r]^2).
+__device__ __forceinline__ void tile_gemm(const float* __restrict__ Wt, int ldw, int K, int N,
+                                          const float* X, float* Y, int epi,
+                                          const float* __restrict__ bias, bool do_tanh,
+                                          const float* H) {
+  const int neb = kLR / 4, nob = (N + 3) / 4;
+  for (int tile = threadIdx.x; tile < neb * nob; tile += blockDim.x) {
+    const int eb = tile % neb, ob = tile / neb;
+    float acc[4][4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+#pragma unroll
+      for (int o = 0; o < 4; ++o) acc[e][o] = 0.0f;
+    const float* wc = Wt + 4 * ob;
+    const float* xc = X + 4 * eb;
+#pragma unroll 4
+    for (int k = 0; k < K; ++k) {
+      const float4 w = *reinterpret_cast<const float4*>(wc + (size_t)k * ldw);
+      const float4 x = *reinterpret_cast<const float4*>(xc + k * kLld);
+      const float xv[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        acc[e][0] = __fmaf_rn(w.x, xv[e], acc[e][0]);
+        acc[e][1] = __fmaf_rn(w.y, xv[e], acc[e][1]);
+        acc[e][2] = __fmaf_rn(w.z, xv[e], acc[e][2]);
+        acc[e][3] = __fmaf_rn(w.w, xv[e], acc[e][3]);
+      }
+    }
+#pragma unroll
+    for (int o = 0; o < 4; ++o) {
+      const int j = 4 * ob + o;
+      if (j >= N) continue;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int r = 4 * eb + e;
+        float v = acc[e][o];
+        if (epi == 0) {
+          v = __fadd_rn(v, bias[j]);
+        } else {
+          const float h = H[j * kLld + r];
+          v = v * (1.0f - h * h);
+        }
+        Y[j * kLld + r] = v;
+      }
+    }
+    if (epi == 0 && do_tanh) {
+#pragma unroll 1
+      for (int q = 0; q < 16; ++q) {
+        const int j = 4 * ob + q / 4;
+        if (j < N) {
+          float* y = Y + j * kLld + 4 * eb + q % 4;
+          *y = det_tanh(*y);
+        }
+      }
+    }
+  }
+}
+
+struct FusedLossArgs {
+  LossArgs a;
+  const float* Wt[SIMX_MAX_LAYERS];  // [K][Npad] transposed (forward)
+  const float* Wn[SIMX_MAX_LAYERS];  // [N][Kpad] row-major copy (backward), Kpad % 4 == 0
+  int npad[SIMX_MAX_LAYERS + 1];     // Npad per layer output (index l + 1)
+  int kpad[SIMX_MAX_LAYERS + 1];     // Kpad per layer input (index l)
+  int act_off[SIMX_MAX_LAYERS + 2];  // row offset of each layer's activation buffer
+  int dz_rows;                       // rows of each dZ buffer
+  int poff[SIMX_MAX_LAYERS];         // offset of layer l's dW in the flat gradient
+  int n_params;
+  float* part;                       // [gridDim.x][n_params]
+  double* spart;                     // [gridDim.x][4]
+  int64_t ntiles;
+};
+
+__global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant__ FusedLossArgs F) {
+  extern __shared__ float sm[];
+  const LossArgs& a = F.a;
+  const int L = a.n_layers;
+  float* acts = sm;                                        // all layers' activations
+  float* dzA = acts + (size_t)F.act_off[L + 1] * kLld;     // two dZ buffers
+  float* dzB = dzA + (size_t)F.dz_rows * kLld;
+  float* gacc = dzB + (size_t)F.dz_rows * kLld;            // dW/db accumulators [n_params]
+  for (int i = threadIdx.x; i < F.n_params; i += blockDim.x) gacc[i] = 0.0f;
+  double st_pg = 0.0, st_v = 0.0, st_h = 0.0, st_cf = 0.0;
+  const int D = a.dims[0];
+  const int A = a.n_actions;
+  const int NL = a.dims[L];
+  const float inv_n = 1.0f / (float)a.n;
+  for (int64_t tile = blockIdx.x; tile < F.ntiles; tile += gridDim.x) {
+    const int64_t r0 = tile * kLR;
+    __syncthreads();
+    // gather X [D][R] (rows past n are zero and have zero dZ)
+    float* X = acts + (size_t)F.act_off[0] * kLld;
+    for (int q = threadIdx.x; q < D * kLR; q += blockDim.x) {
+      const int d = q / kLR, r = q % kLR;
+      const int64_t rr = r0 + r;
+      float v = 0.0f;
+      if (rr < a.n) {
+        const int64_t row = a.idx ? a.idx[rr] : rr;
+        const int64_t t = row / a.E, e = row % a.E;
+        v = a.obs[(t * D + d) * a.E + e];
+      }
+      X[d * kLld + r] = v;
+    }
+    __syncthreads();
+    for (int l = 0; l < L; ++l) {
+      tile_gemm(F.Wt[l], F.npad[l + 1], a.dims[l], a.dims[l + 1],
+                acts + (size_t)F.act_off[l] * kLld, acts + (size_t)F.act_off[l + 1] * kLld, 0,
+                a.b[l], l + 1 < L, nullptr);
+      __syncthreads();
+    }
+    // loss head: 8 lanes per row (32 rows x 8 = 256 threads); lane q takes logits
+    // i = q, q + 8, ... and the row's max / sums are reduced across the 8 lanes
+    const float* Z = acts + (size_t)F.act_off[L] * kLld;
+    float* dz = dzA;
+    {
+      const int r = threadIdx.x / 8, q = threadIdx.x % 8;
+      const unsigned gm = 0xFFu << (threadIdx.x & 24u);  // this row's 8 lanes
+      const int64_t rr = r0 + r;
+      if (rr < a.n) {
+        const int64_t row = a.idx ? a.idx[rr] : rr;
+        const int ac = a.action[row];
+        const float ad = a.adv[row];
+        float m = -__uint_as_float(0x7F800000u);
+        for (int i = q; i < A; i += 8) m = fmaxf(m, Z[i * kLld + r]);
+#pragma unroll
+        for (int d = 4; d > 0; d >>= 1) m = fmaxf(m, __shfl_xor_sync(gm, m, d, 8));
+        float S = 0.0f;
+        for (int i = q; i < A; i += 8) S += det_exp(Z[i * kLld + r] - m);
+#pragma unroll
+        for (int d = 4; d > 0; d >>= 1) S += __shfl_xor_sync(gm, S, d, 8);
+        const float lse = m + det_log(S);
+        float H = 0.0f;
+        for (int i = q; i < A; i += 8) {
+          const float lp = Z[i * kLld + r] - lse;
+          H -= det_exp(lp) * lp;
+        }
+#pragma unroll
+        for (int d = 4; d > 0; d >>= 1) H += __shfl_xor_sync(gm, H, d, 8);
+        const float lpa = Z[ac * kLld + r] - lse;
+        float coef, pg;
+        if (a.algo == SIMX_ALGO_REINFORCE) {
+          coef = ad;
+          pg = -ad * lpa;
+        } else {
+          const float rho = det_exp(lpa - a.logp_old[row]);
+          const float s1 = rho * ad;
+          const float s2 = fminf(fmaxf(rho, 1.0f - a.clip_eps), 1.0f + a.clip_eps) * ad;
+          pg = -fminf(s1, s2);
+          coef = (s1 <= s2 ? ad : 0.0f) * rho;
+          if (q == 0) st_cf += fabsf(rho - 1.0f) > a.clip_eps ? 1.0 : 0.0;
+        }
+        for (int i = q; i < A; i += 8) {
+          const float lp = Z[i * kLld + r] - lse;
+          const float p = det_exp(lp);
+          const float onehot = (i == ac) ? 1.0f : 0.0f;
+          dz[i * kLld + r] = (-coef * (onehot - p) + a.c_entropy * p * (lp + H)) * inv_n;
+        }
+        if (q == 0) {
+          if (a.has_value) {
+            const float dv = Z[A * kLld + r] - a.ret[row];
+            st_v += (double)dv * (double)dv;
+            dz[A * kLld + r] = 2.0f * a.c_value * dv * inv_n;
+          }
+          st_pg += pg;
+          st_h += H;
+        }
+      } else {
+        for (int i = q; i < NL; i += 8) dz[i * kLld + r] = 0.0f;
+      }
+    }
+    __syncthreads();
+    // backward
+    for (int l = L - 1; l >= 0; --l) {
+      const int K = a.dims[l], N = a.dims[l + 1];
+      const float* Hl = acts + (size_t)F.act_off[l] * kLld;
+      float* gW = gacc + F.poff[l];
+      float* gb = gW + (size_t)N * K;
+      // dW += dZ^T H: 4 x 4 blocks of (j, k), rows in float4 steps
+      const int njb = (N + 3) / 4, nkb = (K + 3) / 4;
+      for (int blk = threadIdx.x; blk < njb * nkb; blk += blockDim.x) {
+        const int jb = blk / nkb, kb = blk % nkb;
+        float acc[4][4];
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) acc[p][q] = 0.0f;
+        for (int r = 0; r < kLR; r += 4) {
+          float4 dv[4], hv[4];
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const int j = 4 * jb + p, k = 4 * kb + p;
+            dv[p] = j < N ? *reinterpret_cast<const float4*>(dz + j * kLld + r) : make_float4(0, 0, 0, 0);
+            hv[p] = k < K ? *reinterpret_cast<const float4*>(Hl + k * kLld + r) : make_float4(0, 0, 0, 0);
+          }
+#pragma unroll
+          for (int p = 0; p < 4; ++p)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              acc[p][q] = __fmaf_rn(dv[p].x, hv[q].x, acc[p][q]);
+              acc[p][q] = __fmaf_rn(dv[p].y, hv[q].y, acc[p][q]);
+              acc[p][q] = __fmaf_rn(dv[p].z, hv[q].z, acc[p][q]);
+              acc[p][q] = __fmaf_rn(dv[p].w, hv[q].w, acc[p][q]);
+            }
+        }
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          const int j = 4 * jb + p;
+          if (j >= N) continue;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int k = 4 * kb + q;
+            if (k < K) gW[(size_t)j * K + k] += acc[p][q];
+          }
+        }
+      }
+      for (int j = threadIdx.x; j < N; j += blockDim.x) {
+        float sacc = 0.0f;
+        for (int r = 0; r < kLR; ++r) sacc += dz[j * kLld + r];
+        gb[j] += sacc;
+      }
+      if (l > 0) {
+        float* dzn = (dz == dzA) ? dzB : dzA;
+        // dZ_{l-1}[k][r] = sum_j W_l[j][k] dZ_l[j][r] * (1 - H_l[k][r]^2)
+        tile_gemm(F.Wn[l], F.kpad[l], N, K, dz, dzn, 1, nullptr, false, Hl);
+        __syncthreads();
+        dz = dzn;
+      } else {
+        __syncthreads();
+      }
+    }
+  }
+  __syncthreads();
+  float* out = F.part + (size_t)blockIdx.x * F.n_params;
+  for (int i = threadIdx.x; i < F.n_params; i += blockDim.x) out[i] = gacc[i];
+  // fp64 statistics of the rows this block owned (lane 0 of each row group holds them)
+  __shared__ double sh[4][kLThreads / 8];
+  if (threadIdx.x % 8 == 0) {
+    sh[0][threadIdx.x / 8] = st_pg;
+    sh[1][threadIdx.x / 8] = st_v;
+    sh[2][threadIdx.x / 8] = st_h;
+    sh[3][threadIdx.x / 8] = st_cf;
+  }
+  __syncthreads();
+  if (threadIdx.x < 4) {
+    double sum = 0.0;
+    for (int r = 0; r < kLThreads / 8; ++r) sum += sh[threadIdx.x][r];
+    F.spart[(size_t)blockIdx.x * 4 + threadIdx.x] = sum;
+  }
+}
+
+// Transposed (forward) and row-major padded (backward) copies of each W_l.
+__global__ void k_pack_loss_w(const float* __restrict__ W, int N, int K, int npad, int kpad,
+                              float* __restrict__ Wt, float* __restrict__ Wn) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < K * npad) {
+    const int k = i / npad, j = i % npad;
+    Wt[i] = j < N ? W[(size_t)j * K + k] : 0.0f;
+  }
+  if (i < N * kpad) {
+    const int j = i / kpad, k = i % kpad;
+    Wn[i] = k < K ? W[(size_t)j * K + k] : 0.0f;
+  }
+}
+
+__global__ void k_reduce_blocks(const float* __restrict__ part, int nb, int P, float* __restrict__ out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= P) return;
+  float s = 0.0f;
+  for (int b = 0; b < nb; ++b) s += part[(size_t)b * P + i];
+  out[i] = s;
+}
+
+__global__ void k_fused_stats(const double* __restrict__ sp, int nb, int64_t n, int has_value,
+                              float cv, float ce, float* __restrict__ stats) {
+  if (threadIdx.x != 0) return;
+  double s[4] = {0, 0, 0, 0};
+  for (int b = 0; b < nb; ++b)
+    for (int q = 0; q < 4; ++q) s[q] += sp[(size_t)b * 4 + q];
+  const double pg = s[0] / (double)n, v = s[1] / (double)n, H = s[2] / (double)n;
+  stats[0] = (float)(pg + (has_value ? (double)cv * v : 0.0) - (double)ce * H);
+  stats[1] = (float)pg;
+  stats[2] = (float)v;
+  stats[3] = (float)H;
+  stats[4] = (float)(s[3] / (double)n);
+}
+
+namespace {
+struct FusedPlan {
+  bool ok;
+  int npad[SIMX_MAX_LAYERS + 1], kpad[SIMX_MAX_LAYERS + 1], act_off[SIMX_MAX_LAYERS + 2];
+  int dz_rows, poff[SIMX_MAX_LAYERS], n_params, grid;
+  size_t smem, w_off[SIMX_MAX_LAYERS][2], part_off, spart_off, total;
+};
+
+int r4(int x) { return (x + 3) / 4 * 4; }
+
+FusedPlan plan(const LossArgs& a) {
+  FusedPlan p{};
+  const int L = a.n_layers;
+  int rows = 0, maxd = 0;
+  for (int l = 0; l <= L; ++l) {
+    p.act_off[l] = rows;
+    rows += r4(a.dims[l]);
+    if (l > 0 && a.dims[l] > maxd) maxd = a.dims[l];
+  }
+  p.act_off[L + 1] = rows;
+  p.dz_rows = r4(maxd);
+  int P = 0;
+  for (int l = 0; l < L; ++l) {
+    p.npad[l + 1] = r4(a.dims[l + 1]);
+    p.kpad[l] = r4(a.dims[l]);
+    p.poff[l] = P;
+    P += a.dims[l + 1] * a.dims[l] + a.dims[l + 1];
+  }
+  p.n_params = P;
+  p.smem = ((size_t)rows * kLld + (size_t)2 * p.dz_rows * kLld + (size_t)P) * sizeof(float);
+  p.ok = p.smem <= 200 * 1024;
+  const int64_t ntiles = (a.n + kLR - 1) / kLR;
+  const int per_sm = p.smem <= 70 * 1024 ? 3 : (p.smem <= 110 * 1024 ? 2 : 1);
+  int64_t grid = (int64_t)152 * per_sm;
+  if (grid > ntiles) grid = ntiles;
+  p.grid = (int)(grid < 1 ? 1 : grid);
+  size_t off = 0;
+  auto take = [&](size_t b) {
+    const size_t o = off;
+    off += (b + 255) & ~(size_t)255;
+    return o;
+  };
+  for (int l = 0; l < L; ++l) {
+    p.w_off[l][0] = take((size_t)a.dims[l] * p.npad[l + 1] * sizeof(float));
+    p.w_off[l][1] = take((size_t)a.dims[l + 1] * p.kpad[l] * sizeof(float));
+  }
+  p.part_off = take((size_t)p.grid * P * sizeof(float));
+  p.spart_off = take((size_t)p.grid * 4 * sizeof(double));
+  p.total = off;
+  return p;
+}
+}  // namespace
+
+bool loss_fused_fits(const LossArgs& a) { return plan(a).ok; }
+size_t loss_fused_workspace(const LossArgs& a) { return plan(a).total; }
+
+cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s) {
+  const FusedPlan p = plan(a);
+  if (!p.ok || ws_bytes < p.total) return cudaErrorInvalidValue;
+  char* base = static_cast<char*>(ws);
+  FusedLossArgs F{};
+  F.a = a;
+  for (int l = 0; l < a.n_layers; ++l) {
+    float* Wt = reinterpret_cast<float*>(base + p.w_off[l][0]);
+    float* Wn = reinterpret_cast<float*>(base + p.w_off[l][1]);
+    const int n = a.dims[l] * p.npad[l + 1] > a.dims[l + 1] * p.kpad[l] ? a.dims[l] * p.npad[l + 1]
+                                                                         : a.dims[l + 1] * p.kpad[l];
+    k_pack_loss_w<<<(n + 255) / 256, 256, 0, s>>>(a.W[l], a.dims[l + 1], a.dims[l], p.npad[l + 1],
+                                                  p.kpad[l], Wt, Wn);
+    F.Wt[l] = Wt;
+    F.Wn[l] = Wn;
+  }
+  for (int l = 0; l <= a.n_layers; ++l) {
+    F.npad[l] = p.npad[l];
+    F.kpad[l] = p.kpad[l];
+    F.act_off[l] = p.act_off[l];
+  }
+  F.act_off[a.n_layers + 1] = p.act_off[a.n_layers + 1];
+  F.dz_rows = p.dz_rows;
+  for (int l = 0; l < a.n_layers; ++l) F.poff[l] = p.poff[l];
+  F.n_params = p.n_params;
+  F.part = reinterpret_cast<float*>(base + p.part_off);
+  F.spart = reinterpret_cast<double*>(base + p.spart_off);
+  F.ntiles = (a.n + kLR - 1) / kLR;
+  cudaFuncSetAttribute(k_loss_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+  k_loss_fused<<<p.grid, kLThreads, p.smem, s>>>(F);
+  k_reduce_blocks<<<(p.n_params + 255) / 256, 256, 0, s>>>(F.part, p.grid, p.n_params, a.grad);
+  k_fused_stats<<<1, 32, 0, s>>>(F.spart, p.grid, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
+  count_launches(a.n_layers + 3);
+  return cudaGetLastError();
+}
+
+}  // namespace simx

@@ -13,11 +13,12 @@
 
 namespace simx {
 
-// Threads per block of the env kernels; an env is a group of G lanes, so a block
-// holds kThreads / G envs.  G (8, 16 or 32) is chosen per launch from the env count.
-constexpr int kThreads = 64;
-// At least 8 resident blocks (16 warps) per SM: caps registers at 128 per thread.
-constexpr int kMinBlocks = 8;
+// Env kernels run blocks of 64, 128 or 256 threads (chosen per launch); an env is a
+// group of G lanes (G = 8, 16 or 32, also chosen per launch), so a block holds
+// blockDim.x / G envs.  At least 2 resident 256-thread blocks (16 warps) per SM caps
+// registers at 128 per thread.
+constexpr int kMaxThreads = 256;
+constexpr int kMinBlocks = 2;
 
 // Two values indexed by a runtime 0/1 through selects, so that the structs below
 // stay in registers (a dynamically indexed array would be placed in local memory).
@@ -372,7 +373,7 @@ __device__ __forceinline__ float fdiv_u(uint32_t a, float b) {
 // ROUTE: lane k writes server k's three features, lane 0 the rest.
 template <int G>
 __device__ void observe_single(const simx_config& c, const Grp<G>& g, const Scal& s,
-                               const Srv& q, const uint32_t* ringb, float* o) {
+                               const Srv& q, const uint32_t* ringb, float* o, int B) {
   const int T = (int)c.n_types;
   const uint32_t cap = c.queue_cap;
   const bool ne0 = q.qc[0] > 0u, ne1 = T > 1 && q.qc[1] > 0u;
@@ -425,29 +426,29 @@ __device__ void observe_single(const simx_config& c, const Grp<G>& g, const Scal
         den = tw;
       }
     }
-    o[d] = __fdiv_rn(__fmul_rn(num, mul), den);
+    o[d * B] = __fdiv_rn(__fmul_rn(num, mul), den);
   }
   g.sync();
 }
 
 template <int G>
 __device__ void observe_route(const simx_config& c, const Grp<G>& g, const Scal& s,
-                              const Srv& L, float* o) {
+                              const Srv& L, float* o, int B) {
   const uint32_t K = c.n_servers;
   if (g.gl < K) {
     const float fcap = __uint2float_rn(c.queue_cap);
-    o[3 * g.gl + 0] = fdiv_u(L.qc[0], fcap);
-    o[3 * g.gl + 1] = fdiv_u(c.n_types > 1 ? L.qc[1] : 0u, fcap);
+    o[(3 * g.gl + 0) * B] = fdiv_u(L.qc[0], fcap);
+    o[(3 * g.gl + 1) * B] = fdiv_u(c.n_types > 1 ? L.qc[1] : 0u, fcap);
     const uint32_t rem = L.busy > s.now ? L.busy - s.now : 0u;
-    o[3 * g.gl + 2] = fdiv_u(rem, c.busy_norm_us);
+    o[(3 * g.gl + 2) * B] = fdiv_u(rem, c.busy_norm_us);
   }
   if (g.gl == 0) {
-    o[3 * K] = __fdiv_rn(s.rate, c.rate_ref);
+    o[(3 * K) * B] = __fdiv_rn(s.rate, c.rate_ref);
     if (c.obs_extra) {
-      o[3 * K + 1] = (s.pty == 0) ? 1.0f : 0.0f;
-      o[3 * K + 2] = (s.pty == 1) ? 1.0f : 0.0f;
+      o[(3 * K + 1) * B] = (s.pty == 0) ? 1.0f : 0.0f;
+      o[(3 * K + 2) * B] = (s.pty == 1) ? 1.0f : 0.0f;
       const uint32_t ph = (s.now + s.epo * c.epoch_us) % c.phase_period_us;
-      o[3 * K + 3] = __fdiv_rn(__uint2float_rn(ph), __uint2float_rn(c.phase_period_us));
+      o[(3 * K + 3) * B] = __fdiv_rn(__uint2float_rn(ph), __uint2float_rn(c.phase_period_us));
     }
   }
   g.sync();
@@ -541,18 +542,13 @@ __device__ __forceinline__ void store_srv(const DevState& st, uint32_t e, uint32
   }
 }
 
-// Action from the policy or a baseline (Sec. 4.2, Sec. 5.1).  Needs the
-// observation in act[0..D).
+// Action of a baseline (Sec. 5.1) or an external caller; the policy case is
+// handled by the block-wide MLP in the kernel.
 template <int G, bool ROUTE>
-__device__ int choose_action(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
-                             const Srv& L, const uint32_t* ringb, float* act, float* act2,
-                             float* scratch, float& logp, float& value) {
+__device__ int baseline_action(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
+                               const Srv& L, const uint32_t* ringb) {
   const simx_config& c = A.cfg;
-  logp = 0.0f;
-  value = 0.0f;
   const int mode = A.policy_mode;
-  if (mode == SIMX_POLICY_SAMPLE || mode == SIMX_POLICY_ARGMAX)
-    return policy_eval<G>(A.mlp, act, act2, scratch, mode, A.key0, A.key1, s.tg, env, logp, value, g);
   if (mode == SIMX_POLICY_EXTERNAL) {
     const int32_t a = A.ext[env];
     if (a < 0 || (uint32_t)a >= A.n_actions) {
@@ -585,33 +581,38 @@ __device__ int choose_action(const RolloutArgs& A, const Grp<G>& g, uint32_t env
 }
 
 template <int G>
-__device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int D, float* dst,
+__device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int B, int D, float* dst,
                                           int64_t ld, uint32_t e) {
   if (!dst) return;
-  for (int d = (int)g.gl; d < D; d += G) dst[(int64_t)d * ld + e] = o[d];
+  for (int d = (int)g.gl; d < D; d += G) dst[(int64_t)d * ld + e] = o[d * B];
 }
 
-// The rollout / step kernel.  Block: kThreads threads; each G-lane group owns
-// one env.  Shared memory per env: two activation buffers and the softmax scratch.
+// The rollout / step kernel.  A block of blockDim.x threads owns B = blockDim.x / G
+// envs, one per G-lane group.  Shared memory: two activation buffers X0, X1 of
+// maxd4 x B floats (feature-major) and a softmax scratch of apad floats per env.
 // Every lane stays alive to the end (groups past the last env do no work) so that
-// the whole warp reconverges at the __syncwarp() between the phases of a step.
+// warps reconverge at each phase and the block can run the MLP together.
 template <bool ROUTE, int G>
-__global__ void __launch_bounds__(kThreads, kMinBlocks)
+__global__ void __launch_bounds__(kMaxThreads, kMinBlocks)
 k_rollout(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
   const Grp<G> g;
+  const int B = (int)blockDim.x / G;
+  const int Bs = B + 4;  // row stride of the activation buffers
   const uint32_t slot = threadIdx.x / G;
-  const uint32_t env_raw = blockIdx.x * (kThreads / G) + slot;
+  const uint32_t env_raw = blockIdx.x * (uint32_t)B + slot;
   const bool live = env_raw < A.st.E;
   const uint32_t env = live ? env_raw : 0u;
-  float* act = smem + (size_t)slot * A.act_stride;
-  float* act2 = act + A.buf2_off;
-  float* scratch = act + A.scratch_off;
+  float* X0 = smem;
+  float* X1 = smem + (size_t)A.maxd4 * Bs;
+  float* scratch = smem + (size_t)2 * A.maxd4 * Bs + (size_t)slot * A.apad;
+  float* ocol = X0 + slot;
   const simx_config& c = A.cfg;
   const DevState& st = A.st;
   const uint32_t K = c.n_servers, T = c.n_types, cap = c.queue_cap;
   uint32_t* ringb = st.ring + (size_t)env * K * T * cap;
   uint32_t* costb = st.cost ? st.cost + (size_t)env * K * cap : nullptr;
+  const bool use_mlp = A.policy_mode == SIMX_POLICY_SAMPLE || A.policy_mode == SIMX_POLICY_ARGMAX;
 
   Scal s{};
   Srv L{0u, 0u, Pair{0u, 0u}, Pair{0u, 0u}};
@@ -628,18 +629,24 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
   const int D = A.obs_dim;
 
   for (int t = 0; t < A.H; ++t) {
-    // phase 1: observation (Sec. 4.1)
+    // phase 1: observation (Sec. 4.1) into column `slot` of X0
     if (live) {
-      if (ROUTE) observe_route<G>(c, g, s, L, act);
-      else observe_single<G>(c, g, s, L, ringb, act);
-      write_obs<G>(g, act, D, A.obs ? A.obs + (int64_t)t * D * A.ld : nullptr, A.ld, env);
-      g.sync();
+      if (ROUTE) observe_route<G>(c, g, s, L, ocol, Bs);
+      else observe_single<G>(c, g, s, L, ringb, ocol, Bs);
+      write_obs<G>(g, ocol, Bs, D, A.obs ? A.obs + (int64_t)t * D * A.ld : nullptr, A.ld, env);
     }
     __syncwarp();
-    // phase 2: action (Sec. 4.2 policy or a Sec. 5.1 baseline)
+    // phase 2: action from the policy (Sec. 4.2, block-wide MLP) or a baseline
     float logp = 0.0f, value = 0.0f;
     int a = 0;
-    if (live) a = choose_action<G, ROUTE>(A, g, env, s, L, ringb, act, act2, scratch, logp, value);
+    if (use_mlp) {
+      const float* Z = mlp_forward_block(A.mlp, X0, X1, B, Bs);
+      if (live)
+        a = sample_action<G>(A.mlp, Z + slot, Bs, scratch, A.policy_mode, A.key0, A.key1, s.tg,
+                             env, logp, value, g);
+    } else if (live) {
+      a = baseline_action<G, ROUTE>(A, g, env, s, L, ringb);
+    }
     __syncwarp();
     const uint32_t k = (uint32_t)a / c.n_bsizes;
     const uint32_t b = c.bsizes[(uint32_t)a % c.n_bsizes];
@@ -775,9 +782,9 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
   }
   if (!live) return;
   if (A.next_obs) {
-    if (ROUTE) observe_route<G>(c, g, s, L, act);
-    else observe_single<G>(c, g, s, L, ringb, act);
-    write_obs<G>(g, act, D, A.next_obs, A.next_ld, env);
+    if (ROUTE) observe_route<G>(c, g, s, L, ocol, Bs);
+    else observe_single<G>(c, g, s, L, ringb, ocol, Bs);
+    write_obs<G>(g, ocol, Bs, D, A.next_obs, A.next_ld, env);
   }
   if (g.gl == 0) store_scal(st, env, s);
   if (ROUTE) {
@@ -790,10 +797,10 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
 // Reset: empty queues, idle servers, chain state from the INIT stream, then advance
 // to the first decision point.
 template <bool ROUTE, int G>
-__global__ void __launch_bounds__(kThreads) k_reset(const __grid_constant__ RolloutArgs A) {
+__global__ void __launch_bounds__(kMaxThreads) k_reset(const __grid_constant__ RolloutArgs A) {
   const Grp<G> g;
   const uint32_t slot = threadIdx.x / G;
-  const uint32_t env = blockIdx.x * (kThreads / G) + slot;
+  const uint32_t env = blockIdx.x * (blockDim.x / G) + slot;
   if (env >= A.st.E) return;
   const simx_config& c = A.cfg;
   const DevState& st = A.st;
@@ -848,28 +855,28 @@ __global__ void __launch_bounds__(kThreads) k_reset(const __grid_constant__ Roll
 
 // Current observation of every env (no state change).
 template <bool ROUTE, int G>
-__global__ void __launch_bounds__(kThreads) k_observe(const __grid_constant__ RolloutArgs A) {
+__global__ void __launch_bounds__(kMaxThreads) k_observe(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
   const Grp<G> g;
+  const int B = (int)blockDim.x / G;
   const uint32_t slot = threadIdx.x / G;
-  const uint32_t env = blockIdx.x * (kThreads / G) + slot;
+  const uint32_t env = blockIdx.x * (uint32_t)B + slot;
   if (env >= A.st.E) return;
-  float* act = smem + (size_t)slot * A.act_stride;
+  float* ocol = smem + slot;
   const simx_config& c = A.cfg;
   const uint32_t K = c.n_servers, T = c.n_types, cap = c.queue_cap;
   const uint32_t* ringb = A.st.ring + (size_t)env * K * T * cap;
   Scal s;
   load_scal(A.st, env, s);
-  Srv L;
+  Srv L{0u, 0u, Pair{0u, 0u}, Pair{0u, 0u}};
   if (ROUTE) {
     if (g.gl < K) load_srv(A.st, env, g.gl, L);
-    else L = Srv{0u, 0u, Pair{0u, 0u}, Pair{0u, 0u}};
-    observe_route<G>(c, g, s, L, act);
+    observe_route<G>(c, g, s, L, ocol, B + 4);
   } else {
     load_srv(A.st, env, 0, L);
-    observe_single<G>(c, g, s, L, ringb, act);
+    observe_single<G>(c, g, s, L, ringb, ocol, B + 4);
   }
-  write_obs<G>(g, act, A.obs_dim, A.next_obs, A.next_ld, env);
+  write_obs<G>(g, ocol, B + 4, A.obs_dim, A.next_obs, A.next_ld, env);
 }
 
 // Canonical state image of each env (header, servers, queue lengths, FIFO contents
@@ -968,27 +975,32 @@ __global__ void k_repack(const float* __restrict__ W, const float* __restrict__ 
   if (i < Npad) bias[i] = i < N ? b[i] : 0.0f;
 }
 
-// Batched policy forward (Sec. 4.2) over observation columns [D][ld].
+// Batched policy forward (Sec. 4.2) over observation columns [D][ld]: a block of
+// B = blockDim.x / G columns runs the block-wide MLP, then each column's G lanes
+// sample.  Every lane stays alive for the block barriers.
 template <int G>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kMaxThreads)
 k_policy_forward(const __grid_constant__ PolicyArgs P) {
   extern __shared__ float smem[];
   const Grp<G> g;
+  const int B = (int)blockDim.x / G;
+  const int Bs = B + 4;
   const uint32_t slot = threadIdx.x / G;
-  const int64_t i = (int64_t)blockIdx.x * (kThreads / G) + slot;
-  if (i >= P.n) return;
-  float* act = smem + (size_t)slot * P.act_stride;
-  float* scratch = act + P.scratch_off;
+  const int64_t i = (int64_t)blockIdx.x * B + slot;
+  const bool live = i < P.n;
+  float* X0 = smem;
+  float* X1 = smem + (size_t)P.maxd4 * Bs;
+  float* scratch = smem + (size_t)2 * P.maxd4 * Bs + (size_t)slot * P.apad;
   const int D = P.mlp.dims[0];
-  for (int d = (int)g.gl; d < D; d += G) act[d] = P.obs[(int64_t)d * P.ld + i];
-  g.sync();
+  for (int d = (int)g.gl; d < D; d += G) X0[d * Bs + slot] = live ? P.obs[(int64_t)d * P.ld + i] : 0.0f;
+  const float* Z = mlp_forward_block(P.mlp, X0, X1, B, Bs);
+  if (!live) return;
   float logp, value;
   const uint32_t env = P.env_base + (uint32_t)i;
-  float* z = nullptr;
-  const int a = policy_eval<G>(P.mlp, act, act + P.buf2_off, scratch, P.mode, P.key0, P.key1,
-                                P.step, env, logp, value, g, &z);
+  const int a = sample_action<G>(P.mlp, Z + slot, Bs, scratch, P.mode, P.key0, P.key1, P.step, env,
+                                 logp, value, g);
   if (P.logits)
-    for (int j = (int)g.gl; j < P.mlp.n_actions; j += G) P.logits[(int64_t)j * P.ld + i] = z[j];
+    for (int j = (int)g.gl; j < P.mlp.n_actions; j += G) P.logits[(int64_t)j * P.ld + i] = Z[j * Bs + slot];
   if (g.gl == 0) {
     if (P.value) P.value[i] = value;
     if (P.action) P.action[i] = (uint8_t)a;
@@ -999,29 +1011,37 @@ k_policy_forward(const __grid_constant__ PolicyArgs P) {
 // ---------------------------------------------------------------------------
 // Host launchers
 // ---------------------------------------------------------------------------
-template <int G>
-static unsigned grid_for(int64_t E) { return (unsigned)((E + kThreads / G - 1) / (kThreads / G)); }
+static unsigned grid_for(int64_t n, int envs_per_block) {
+  return (unsigned)((n + envs_per_block - 1) / envs_per_block);
+}
+
+static size_t env_smem(const RolloutArgs& a, int B) {
+  return ((size_t)2 * a.maxd4 * (B + 4) + (size_t)a.apad * B) * sizeof(float);
+}
 
 template <bool ROUTE, int G>
 static cudaError_t rollout_t(const RolloutArgs& a, cudaStream_t s) {
-  const size_t sh = (size_t)(kThreads / G) * a.act_stride * sizeof(float);
+  const int B = a.threads / G;
+  const size_t sh = env_smem(a, B);
   cudaFuncSetAttribute(k_rollout<ROUTE, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
-  k_rollout<ROUTE, G><<<grid_for<G>(a.st.E), kThreads, sh, s>>>(a);
+  k_rollout<ROUTE, G><<<grid_for(a.st.E, B), a.threads, sh, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
 
 template <bool ROUTE, int G>
 static cudaError_t reset_t(const RolloutArgs& a, cudaStream_t s) {
-  k_reset<ROUTE, G><<<grid_for<G>(a.st.E), kThreads, 0, s>>>(a);
+  k_reset<ROUTE, G><<<grid_for(a.st.E, a.threads / G), a.threads, 0, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
 
 template <bool ROUTE, int G>
 static cudaError_t observe_t(const RolloutArgs& a, cudaStream_t s) {
-  const size_t sh = (size_t)(kThreads / G) * a.act_stride * sizeof(float);
-  k_observe<ROUTE, G><<<grid_for<G>(a.st.E), kThreads, sh, s>>>(a);
+  const int B = a.threads / G;
+  const size_t sh = env_smem(a, B);
+  cudaFuncSetAttribute(k_observe<ROUTE, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
+  k_observe<ROUTE, G><<<grid_for(a.st.E, B), a.threads, sh, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
@@ -1071,9 +1091,10 @@ cudaError_t launch_repack(const float* W, const float* b, int N, int K, int Npad
 
 template <int G>
 static cudaError_t policy_forward_t(const PolicyArgs& p, cudaStream_t s) {
-  const size_t sh = (size_t)(kThreads / G) * p.act_stride * sizeof(float);
+  const int B = p.threads / G;
+  const size_t sh = ((size_t)2 * p.maxd4 * (B + 4) + (size_t)p.apad * B) * sizeof(float);
   cudaFuncSetAttribute(k_policy_forward<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
-  k_policy_forward<G><<<grid_for<G>(p.n), kThreads, sh, s>>>(p);
+  k_policy_forward<G><<<grid_for(p.n, B), p.threads, sh, s>>>(p);
   count_launches(1);
   return cudaGetLastError();
 }
@@ -1096,9 +1117,19 @@ int choose_lanes(int64_t envs) {
     if (v == 8 || v == 16 || v == 32) return v;
   }
   const int64_t target_warps = 152 * 16;
-  if (envs * 32 / 32 <= target_warps) return 32;
+  if (envs <= target_warps) return 32;
   if (envs * 16 / 32 <= target_warps) return 16;
   return 8;
+}
+
+// Threads per block: the largest of 256, 128, 64 that still gives at least four
+// blocks per SM (two for 64), so small env counts spread over all 152 SMs.
+int choose_threads(int64_t envs, int G) {
+  for (int t = 256; t >= 64; t /= 2) {
+    const int64_t blocks = (envs + t / G - 1) / (t / G);
+    if (blocks >= (t == 64 ? 2 : 4) * 152 || t == 64) return t;
+  }
+  return 64;
 }
 
 }  // namespace simx

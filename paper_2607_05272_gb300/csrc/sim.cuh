@@ -35,7 +35,7 @@ struct DevState {
 };
 
 // Policy parameters repacked for the device: Wt[l] is [K_l][Npad_l] (transposed,
-// columns padded to a multiple of 4G with zeros), bias[l] is [Npad_l].
+// columns padded to a multiple of 4 with zeros), bias[l] is [Npad_l].
 struct DevMlp {
   const float* Wt[SIMX_MAX_LAYERS];
   const float* bias[SIMX_MAX_LAYERS];
@@ -93,106 +93,111 @@ struct Grp {
   __device__ __forceinline__ void sync() const { __syncwarp(mask); }
 };
 
-// One tanh MLP layer for one environment, computed by its G lanes from the
-// shared-memory activation vector x[0..K) into y[0..N) (a second buffer).
-// Lane gl owns outputs 4 gl + 4 G b + c, taken in passes of at most kPass column
-// blocks (16 accumulators); every output is the fp32 fused multiply-add chain over
-// k = 0..K-1 in order from 0, then + bias (Sec. 4.2).  The k loop is unrolled by
-// four (one float4 of activations, four weight rows) with the per-output order
-// unchanged.  tanh is applied afterwards, one output per lane at a time.
-constexpr int kPass = 4;
-
-template <int G>
-__device__ __forceinline__ void mlp_layer(const float* __restrict__ Wt,
-                                          const float* __restrict__ bias, int K, int N,
-                                          int Npad, const float* x, float* y, bool do_tanh,
-                                          const Grp<G>& g) {
-  const int nb = Npad / (4 * G);
-  const float* wp = Wt + 4 * g.gl;
-  for (int p0 = 0; p0 < nb; p0 += kPass) {
-    float acc[4 * kPass];
+// ---------------------------------------------------------------------------
+// Policy network (Sec. 4.2) evaluated for all envs of a block at once.
+//
+// Activations live in shared memory feature-major, X[k * ld + e] for the block's B
+// envs (row stride ld = B + 4 spreads an env's features over the banks), so one
+// layer is the small GEMM Y = X^T W^T.  Each thread owns tiles of TE
+// envs x 4 outputs; per k it loads one float4 of weights (row k of the transposed,
+// padded Wt) and TE activations and issues 4 TE fused multiply-adds.  Every output
+// is still the fp32 chain acc = fma(W[j][k], x[k], acc) over k = 0..K-1 in order
+// from acc = 0, then + bias: the same bits as evaluating one env at a time.
+// ---------------------------------------------------------------------------
+template <int TE>
+__device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
+                                          const float* __restrict__ bias, int K, int N, int Npad,
+                                          const float* X, float* Y, int B, int ld, bool do_tanh) {
+  const int neb = B / TE, nob = (N + 3) / 4;
+  const int ntiles = neb * nob;
+  for (int tile = threadIdx.x; tile < ntiles; tile += blockDim.x) {
+    const int eb = tile % neb, ob = tile / neb;
+    float acc[TE][4];
 #pragma unroll
-    for (int q = 0; q < 4 * kPass; ++q) acc[q] = 0.0f;
-    int k = 0;
-    for (; k + 4 <= K; k += 4) {
-      const float4 xv = *reinterpret_cast<const float4*>(x + k);
-      const float* wr = wp + (size_t)k * Npad + 4 * G * p0;
+    for (int e = 0; e < TE; ++e)
 #pragma unroll
-      for (int b = 0; b < kPass; ++b) {
-        if (p0 + b < nb) {
-          const float4 w0 = __ldg(reinterpret_cast<const float4*>(wr + 4 * G * b));
-          const float4 w1 = __ldg(reinterpret_cast<const float4*>(wr + Npad + 4 * G * b));
-          const float4 w2 = __ldg(reinterpret_cast<const float4*>(wr + 2 * Npad + 4 * G * b));
-          const float4 w3 = __ldg(reinterpret_cast<const float4*>(wr + 3 * Npad + 4 * G * b));
-          float* a4 = acc + 4 * b;
-          a4[0] = __fmaf_rn(w3.x, xv.w, __fmaf_rn(w2.x, xv.z, __fmaf_rn(w1.x, xv.y, __fmaf_rn(w0.x, xv.x, a4[0]))));
-          a4[1] = __fmaf_rn(w3.y, xv.w, __fmaf_rn(w2.y, xv.z, __fmaf_rn(w1.y, xv.y, __fmaf_rn(w0.y, xv.x, a4[1]))));
-          a4[2] = __fmaf_rn(w3.z, xv.w, __fmaf_rn(w2.z, xv.z, __fmaf_rn(w1.z, xv.y, __fmaf_rn(w0.z, xv.x, a4[2]))));
-          a4[3] = __fmaf_rn(w3.w, xv.w, __fmaf_rn(w2.w, xv.z, __fmaf_rn(w1.w, xv.y, __fmaf_rn(w0.w, xv.x, a4[3]))));
-        }
+      for (int o = 0; o < 4; ++o) acc[e][o] = 0.0f;
+    const float* wc = Wt + 4 * ob;
+    const float* xc = X + TE * eb;
+#pragma unroll 4
+    for (int k = 0; k < K; ++k) {
+      const float4 w = __ldg(reinterpret_cast<const float4*>(wc + (size_t)k * Npad));
+      float xv[TE];
+      if (TE == 4) {
+        const float4 x4 = *reinterpret_cast<const float4*>(xc + k * ld);
+        xv[0] = x4.x;
+        xv[1 % TE] = x4.y;
+        xv[2 % TE] = x4.z;
+        xv[3 % TE] = x4.w;
+      } else {
+        xv[0] = xc[k * ld];
       }
-    }
-    for (; k < K; ++k) {
-      const float xk = x[k];
-      const float* wr = wp + (size_t)k * Npad + 4 * G * p0;
 #pragma unroll
-      for (int b = 0; b < kPass; ++b) {
-        if (p0 + b < nb) {
-          const float4 w4 = __ldg(reinterpret_cast<const float4*>(wr + 4 * G * b));
-          acc[4 * b + 0] = __fmaf_rn(w4.x, xk, acc[4 * b + 0]);
-          acc[4 * b + 1] = __fmaf_rn(w4.y, xk, acc[4 * b + 1]);
-          acc[4 * b + 2] = __fmaf_rn(w4.z, xk, acc[4 * b + 2]);
-          acc[4 * b + 3] = __fmaf_rn(w4.w, xk, acc[4 * b + 3]);
-        }
+      for (int e = 0; e < TE; ++e) {
+        acc[e][0] = __fmaf_rn(w.x, xv[e], acc[e][0]);
+        acc[e][1] = __fmaf_rn(w.y, xv[e], acc[e][1]);
+        acc[e][2] = __fmaf_rn(w.z, xv[e], acc[e][2]);
+        acc[e][3] = __fmaf_rn(w.w, xv[e], acc[e][3]);
       }
     }
 #pragma unroll
-    for (int b = 0; b < kPass; ++b) {
-      if (p0 + b < nb) {
+    for (int o = 0; o < 4; ++o) {
+      const int j = 4 * ob + o;
+      if (j < N) {
+        const float bj = __ldg(bias + j);
 #pragma unroll
-        for (int cc = 0; cc < 4; ++cc) {
-          const int j = 4 * (int)g.gl + 4 * G * (p0 + b) + cc;
-          if (j < N) y[j] = __fadd_rn(acc[4 * b + cc], __ldg(bias + j));
+        for (int e = 0; e < TE; ++e) Y[j * ld + TE * eb + e] = __fadd_rn(acc[e][o], bj);
+      }
+    }
+    if (do_tanh) {  // one det_tanh per output, over this thread's own tile
+#pragma unroll 1
+      for (int q = 0; q < 4 * TE; ++q) {
+        const int j = 4 * ob + q / TE;
+        if (j < N) {
+          float* y = Y + j * ld + TE * eb + q % TE;
+          *y = det_tanh(*y);
         }
       }
     }
-  }
-  g.sync();
-  if (do_tanh) {
-    for (int j = (int)g.gl; j < N; j += G) y[j] = det_tanh(y[j]);
-    g.sync();
   }
 }
 
-// Policy head (Sec. 4.2) on the observation in bufA: forward through all layers
-// (alternating bufA / bufB), then (mode SAMPLE) categorical sampling by inversion of
-// the cumulative softmax with a POLICY-stream uniform, or (ARGMAX) the first
-// largest logit.  p_i = e^{z_i - max} are computed by the lanes in parallel and summed
-// by lane 0 in index order.  Returns the action; logp/value valid in every lane;
-// *zout (if given) points at the logits.  scratch holds n_actions floats.
-template <int G>
-__device__ __forceinline__ int policy_eval(const DevMlp& m, float* bufA, float* bufB,
-                                           float* scratch, int mode, uint32_t key0,
-                                           uint32_t key1, uint32_t step, uint32_t env,
-                                           float& logp, float& value, const Grp<G>& g,
-                                           float** zout = nullptr) {
-  float* in = bufA;
-  float* out = bufB;
+// Forward through every layer for the block's envs: the observation is in X0,
+// layers alternate X0 -> X1 -> X0 ...; returns the buffer holding the last layer
+// (logits rows 0..A-1, value row A).  Contains the block barriers.
+__device__ __forceinline__ float* mlp_forward_block(const DevMlp& m, float* X0, float* X1, int B,
+                                                   int ld) {
+  float* in = X0;
+  float* out = X1;
+  __syncthreads();
   for (int l = 0; l < m.n_layers; ++l) {
-    mlp_layer<G>(m.Wt[l], m.bias[l], m.dims[l], m.dims[l + 1], m.npad[l + 1], in, out,
-                 l + 1 < m.n_layers, g);
+    const int K = m.dims[l], N = m.dims[l + 1], Np = m.npad[l + 1];
+    const bool th = l + 1 < m.n_layers;
+    // 4-env tiles when they keep every thread busy, otherwise 1-env tiles
+    if ((B / 4) * ((N + 3) / 4) >= (int)blockDim.x) mlp_tiles<4>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th);
+    else mlp_tiles<1>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th);
+    __syncthreads();
     float* t = in;
     in = out;
     out = t;
   }
-  const float* z = in;
-  if (zout) *zout = in;
+  return in;
+}
+
+// Action from the logits column z[i * B] of one env (Sec. 4.2): SAMPLE draws by
+// inversion of the cumulative softmax with a POLICY-stream uniform, ARGMAX takes the
+// first largest logit.  p_i = e^{z_i - max} are computed by the env's lanes in
+// parallel and summed by lane 0 in index order.  logp/value valid in every lane.
+template <int G>
+__device__ __forceinline__ int sample_action(const DevMlp& m, const float* z, int B,
+                                             float* scratch, int mode, uint32_t key0,
+                                             uint32_t key1, uint32_t step, uint32_t env,
+                                             float& logp, float& value, const Grp<G>& g) {
   const int A = m.n_actions;
-  // group argmax (first index of the largest logit)
   float mx = -__uint_as_float(0x7F800000u);
   int ai = 0x7FFFFFFF;
   for (int i = (int)g.gl; i < A; i += G) {
-    const float v = z[i];
+    const float v = z[i * B];
     if (v > mx) {
       mx = v;
       ai = i;
@@ -207,7 +212,7 @@ __device__ __forceinline__ int policy_eval(const DevMlp& m, float* bufA, float* 
       ai = oi;
     }
   }
-  for (int i = (int)g.gl; i < A; i += G) scratch[i] = det_exp(__fsub_rn(z[i], mx));
+  for (int i = (int)g.gl; i < A; i += G) scratch[i] = det_exp(__fsub_rn(z[i * B], mx));
   g.sync();
   int a = 0;
   float lp = 0.0f;
@@ -229,11 +234,11 @@ __device__ __forceinline__ int policy_eval(const DevMlp& m, float* bufA, float* 
         }
       }
     }
-    lp = __fsub_rn(__fsub_rn(z[a], mx), det_log(S));
+    lp = __fsub_rn(__fsub_rn(z[a * B], mx), det_log(S));
   }
   a = (int)g.shfl((uint32_t)a, 0);
   logp = g.shflf(lp, 0);
-  value = m.has_value ? z[A] : 0.0f;
+  value = m.has_value ? z[A * B] : 0.0f;
   g.sync();
   return a;
 }

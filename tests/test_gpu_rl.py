@@ -123,6 +123,8 @@ def _check_grad(g, g_ref, layers):
     ("c4", "ppo", 33, 128, 3000),
     ("c2", "reinforce", 40, 512, None),
     ("c1", "reinforce", 16, 700, 5000),
+    ("c3", "ppo", 8, 64, 333),
+    ("c2", "reinforce", 3, 7, None),
 ])
 def test_loss_gradient_matches_oracle(name, algo, E, H, nmb):
     simx = _simx()
