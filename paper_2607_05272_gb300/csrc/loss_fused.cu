@@ -345,7 +345,8 @@ FusedPlan plan(const LossArgs& a) {
   p.smem = ((size_t)rows * kLld + (size_t)2 * p.dz_rows * kLld + (size_t)P) * sizeof(float);
   p.ok = p.smem <= 200 * 1024;
   const int64_t ntiles = (a.n + kLR - 1) / kLR;
-  const int per_sm = p.smem <= 70 * 1024 ? 3 : (p.smem <= 110 * 1024 ? 2 : 1);
+  // resident blocks per SM: 128 registers x 256 threads allow two; shared memory may allow fewer
+  const int per_sm = p.smem <= 110 * 1024 ? 2 : 1;
   int64_t grid = (int64_t)152 * per_sm;
   if (grid > ntiles) grid = ntiles;
   p.grid = (int)(grid < 1 ? 1 : grid);

@@ -1124,7 +1124,12 @@ int choose_lanes(int64_t envs) {
 
 // Threads per block: the largest of 256, 128, 64 that still gives at least four
 // blocks per SM (two for 64), so small env counts spread over all 152 SMs.
+// The environment variable SIMX_THREADS (64, 128 or 256) overrides the choice.
 int choose_threads(int64_t envs, int G) {
+  if (const char* f = getenv("SIMX_THREADS")) {
+    const int v = atoi(f);
+    if ((v == 64 || v == 128 || v == 256) && v >= G) return v;
+  }
   for (int t = 256; t >= 64; t /= 2) {
     const int64_t blocks = (envs + t / G - 1) / (t / G);
     if (blocks >= (t == 64 ? 2 : 4) * 152 || t == 64) return t;
