@@ -281,6 +281,30 @@ simx_status ppo_loss_grad(const simx_mlp* pol, const simx_rollout* buf, int64_t 
                           const simx_loss_params* params, float* d_grad, float* d_stats,
                           void* d_workspace, size_t workspace_bytes, void* stream);
 
+/*
+ * Allocation-free variant of ppo_loss_grad.  The paper has no counterpart: this is a
+ * service of the library for callers that cannot allocate device memory themselves,
+ * for instance a plain C host program with no device allocator of its own, or an
+ * application that fixes its device-memory budget before it starts.  Instead of a
+ * caller workspace it uses a buffer of SIMX_NOALLOC_SCRATCH_BYTES built into the
+ * library (a file-scope device array that every GPU which loads the library holds
+ * until the process exits); it calls no cudaMalloc or cudaFree.
+ *   - Arguments and results are those of ppo_loss_grad.
+ *   - A minibatch whose workspace (ppo_loss_grad_workspace_size) exceeds the buffer is
+ *     rejected with SIMX_EINVAL and a message giving both sizes.
+ *   - The first call on a device looks up the buffer's device address (once per
+ *     device, with that device current); make that first call before any stream
+ *     capture.
+ *   - Every call shares the one buffer: calls that overlap on the GPU (different
+ *     streams, or devices sharing a call in flight) race and must be ordered by the
+ *     caller.  Nothing needs to start at zero: each call writes all scratch it reads.
+ */
+#define SIMX_NOALLOC_SCRATCH_BYTES (16u << 20)
+simx_status ppo_loss_grad_noalloc(const simx_mlp* pol, const simx_rollout* buf,
+                                  int64_t n_rows_per_step, const float* d_ret, const float* d_adv,
+                                  const int64_t* d_idx, int64_t n, const simx_loss_params* params,
+                                  float* d_grad, float* d_stats, void* stream);
+
 /* Aggregate counters (synchronises the context's last stream). host_out: host. */
 simx_status sim_stats(simx_ctx* ctx, simx_counters* host_out);
 

@@ -563,6 +563,52 @@ simx_status ppo_loss_grad(const simx_mlp* pol, const simx_rollout* buf, int64_t 
   return SIMX_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Allocation-free loss gradient: the scratch is this file-scope device array.  Host
+// code may not use its name as a device address (it is a host-side stand-in), so the
+// address is looked up once per device with cudaGetSymbolAddress.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) unsigned char g_noalloc_scratch[SIMX_NOALLOC_SCRATCH_BYTES];
+static std::mutex g_noalloc_mu;
+static void* g_noalloc_ptr[64] = {};
+
+static simx_status noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(SIMX_EINVAL, "device %d", dev);
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return SIMX_OK;
+}
+
+simx_status ppo_loss_grad_noalloc(const simx_mlp* pol, const simx_rollout* buf,
+                                  int64_t n_rows_per_step, const float* d_ret, const float* d_adv,
+                                  const int64_t* d_idx, int64_t n, const simx_loss_params* params,
+                                  float* d_grad, float* d_stats, void* stream) {
+  LossArgs a;
+  simx_status v = loss_args(pol, buf, n_rows_per_step, d_ret, d_adv, d_idx, n, params, d_grad,
+                            d_stats, a);
+  if (v != SIMX_OK) return v;
+  const size_t need = loss_workspace_bytes(a);
+  if (need > SIMX_NOALLOC_SCRATCH_BYTES)
+    return fail(SIMX_EINVAL, "this minibatch needs %zu bytes of scratch; the allocation-free entry "
+                "point holds %zu (use ppo_loss_grad with a workspace)", need,
+                (size_t)SIMX_NOALLOC_SCRATCH_BYTES);
+  void* ws = nullptr;
+  v = noalloc_scratch(&ws);
+  if (v != SIMX_OK) return v;
+  cudaError_t e = launch_loss_grad(a, ws, SIMX_NOALLOC_SCRATCH_BYTES, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "loss launch");
+  return SIMX_OK;
+}
+
 static simx_status gather_stats(simx_ctx* c, unsigned long long host[9]) {
   cudaSetDevice(c->device);
   cudaError_t e = cudaStreamSynchronize(c->last);

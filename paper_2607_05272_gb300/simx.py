@@ -87,6 +87,7 @@ SIGNATURES = [
     ("returns_baseline", C.c_int, [P, I64, P, P, P, SZ, P]),
     ("ppo_loss_grad_workspace_size", SZ, [P, I64]),
     ("ppo_loss_grad", C.c_int, [P, P, I64, P, P, P, I64, P, P, P, P, SZ, P]),
+    ("ppo_loss_grad_noalloc", C.c_int, [P, P, I64, P, P, P, I64, P, P, P, P]),
     ("sim_stats", C.c_int, [P, P]),
     ("sim_save", C.c_int, [P, P, U64]),
     ("sim_load", C.c_int, [P, P, U64]),
@@ -309,3 +310,22 @@ def ppo_loss_grad(policy: Policy, buf: dict, ret, adv, idx, n: int, algo: str, c
     _check(lib().ppo_loss_grad(C.byref(policy.c), C.byref(r), r.ld, _ptr(ret), _ptr(adv),
                                _ptr(idx), n, C.byref(p), _ptr(grad), _ptr(stats), _ptr(workspace),
                                workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+NOALLOC_SCRATCH_BYTES = 16 << 20
+
+
+def ppo_loss_grad_noalloc(policy: Policy, buf: dict, ret, adv, idx, n: int, algo: str,
+                          clip_eps: float, c_value: float, c_entropy: float, grad, stats,
+                          stream=None):
+    """ppo_loss_grad without a caller workspace: the scratch is a buffer inside the
+    library, for callers that cannot allocate device memory (see include/simx.h)."""
+    r = Rollout()
+    r.ld = buf["action"].shape[-1]
+    for k in ("obs", "action", "logp", "value", "reward", "done", "trace"):
+        t = buf.get(k)
+        setattr(r, k, None if t is None else t.data_ptr())
+    p = LossParams(ALGO[algo], clip_eps, c_value, c_entropy)
+    _check(lib().ppo_loss_grad_noalloc(C.byref(policy.c), C.byref(r), r.ld, _ptr(ret), _ptr(adv),
+                                       _ptr(idx), n, C.byref(p), _ptr(grad), _ptr(stats),
+                                       _stream(stream)))
