@@ -41,6 +41,7 @@ def _args():
     p.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-hbm-step", action="store_true")
     p.add_argument("--cpu-child", default=None, help=argparse.SUPPRESS)
     return p.parse_args()
 
@@ -186,6 +187,45 @@ def _peaks():
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "sm_max_mhz": 2070.0}, "fallback"
 
 
+def hbm_step_measure(simx, W, torch, E=65536, steps=200, warm=10) -> dict:
+    """sim_step_batched with the Shortest-Queue baseline on the 4-server environment.
+
+    Counted bytes per env-step: the structure-of-arrays state read and written (29 header
+    words, 2K server words, 2KT queue words), the records written (next observation,
+    reward, done, action) and 8 B per routed request (one ring write, one ring read)."""
+    cfg = W.c5(E)
+    K, T, D = cfg["n_servers"], cfg["n_types"], cfg["obs_dim"]
+    sim = simx.Sim(cfg)
+    sim.reset(SEED_BASE + 5)
+    obs = torch.empty((D, E), device="cuda")
+    rew = torch.empty(E, device="cuda")
+    done = torch.empty(E, dtype=torch.uint8, device="cuda")
+    act = torch.empty(E, dtype=torch.uint8, device="cuda")
+    for _ in range(warm):
+        sim.step("sq", obs=obs, reward=rew, done=done, action=act)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(steps):
+        sim.step("sq", obs=obs, reward=rew, done=done, action=act)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    st, code = sim.last_status()
+    sim.close()
+    if st != 0:
+        raise RuntimeError("device status 0x%x in the HBM step" % code)
+    state = (29 + 2 * K + 2 * K * T) * 4
+    per = 2 * state + (D * 4 + 4 + 1 + 1) + 8
+    gbs = per * E / (ms * 1e-3) / 1e9
+    peaks, src = _peaks()
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    return {"kernel": "k_step_thread (policy-free step, SoA state round trip)", "envs": E,
+            "us_per_step": ms * 1e3, "env_steps_per_s": E / (ms * 1e-3),
+            "bytes_per_env_step": per, "achieved": gbs, "peak": hbm, "unit": "GB/s",
+            "frac": gbs / hbm, "peak_source": "%s hbm_gbs" % src}
+
+
 def run_gpu(a) -> None:
     import numpy as np
     import torch
@@ -313,6 +353,10 @@ def run_gpu(a) -> None:
         e2e = {"value": world * n / t_e2e, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}
 
+    # the policy-free batched step (Sec. 5.1 Shortest-Queue router) of the multi-server
+    # environment at 65,536 envs: state read and written every step, HBM-bound
+    hbm_step = None if a.no_hbm_step else hbm_step_measure(simx, W, torch)
+
     # roofline of the dominant kernel
     peaks, src = _peaks()
     sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
@@ -354,6 +398,7 @@ def run_gpu(a) -> None:
             "phases_ms": phases,
             "roofline": roof,
             "e2e": e2e,
+            "hbm_step": hbm_step,
             "gpu_launches": launches,
             "clocks": clk,
             "wall_s": t_wall,

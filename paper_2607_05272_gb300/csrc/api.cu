@@ -388,7 +388,7 @@ simx_status sim_step_batched(simx_ctx* c, const int32_t* d_actions, const simx_m
   a.logp = d_logp;
   a.next_obs = d_obs;
   a.next_ld = d_obs ? ld : c->cfg.n_envs;
-  cudaError_t e = launch_rollout(a, s);
+  cudaError_t e = step_thread_supported(a) ? launch_step_thread(a, s) : launch_rollout(a, s);
   if (e != cudaSuccess) return cuda_fail(e, "step launch");
   c->last = s;
   return SIMX_OK;
@@ -421,7 +421,7 @@ simx_status rollout_collect(simx_ctx* c, const simx_mlp* pol, int policy_mode, i
   a.reward = out->reward;
   a.done = out->done;
   a.trace = out->trace;
-  cudaError_t e = launch_rollout(a, s);
+  cudaError_t e = step_thread_supported(a) ? launch_step_thread(a, s) : launch_rollout(a, s);
   if (e != cudaSuccess) return cuda_fail(e, "rollout launch");
   c->last = s;
   return SIMX_OK;

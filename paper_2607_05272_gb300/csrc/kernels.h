@@ -53,6 +53,9 @@ struct PolicyArgs {
 };
 
 cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s);
+// step_thread.cu: one thread per env for the policy-free modes
+bool step_thread_supported(const RolloutArgs& a);
+cudaError_t launch_step_thread(const RolloutArgs& a, cudaStream_t s);
 cudaError_t launch_reset(const RolloutArgs& a, cudaStream_t s);
 cudaError_t launch_observe(const RolloutArgs& a, cudaStream_t s);
 cudaError_t launch_save(const DevState& st, int32_t cost_type, uint64_t words, uint32_t* out, cudaStream_t s);

@@ -18,7 +18,16 @@ namespace simx {
 // blockDim.x / G envs.  At least 2 resident 256-thread blocks (16 warps) per SM caps
 // registers at 128 per thread.
 constexpr int kMaxThreads = 256;
-constexpr int kMinBlocks = 2;
+#ifndef SIMX_MIN_BLOCKS
+#define SIMX_MIN_BLOCKS 2
+#endif
+#ifndef SIMX_MIN_BLOCKS_32
+#define SIMX_MIN_BLOCKS_32 SIMX_MIN_BLOCKS
+#endif
+// Resident 256-thread blocks per SM the register allocation must allow (one env per
+// warp needs more warps resident than narrower groups do).
+template <int G>
+constexpr int min_blocks() { return G == 32 ? SIMX_MIN_BLOCKS_32 : SIMX_MIN_BLOCKS; }
 
 // Two values indexed by a runtime 0/1 through selects, so that the structs below
 // stay in registers (a dynamically indexed array would be placed in local memory).
@@ -593,7 +602,7 @@ __device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int B
 // Every lane stays alive to the end (groups past the last env do no work) so that
 // warps reconverge at each phase and the block can run the MLP together.
 template <bool ROUTE, int G>
-__global__ void __launch_bounds__(kMaxThreads, kMinBlocks)
+__global__ void __launch_bounds__(kMaxThreads, min_blocks<G>())
 k_rollout(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
   const Grp<G> g;
