@@ -187,12 +187,14 @@ def _peaks():
         return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "sm_max_mhz": 2070.0}, "fallback"
 
 
-def hbm_step_measure(simx, W, torch, E=65536, steps=200, warm=10) -> dict:
+def hbm_step_measure(simx, W, torch, E=65536, steps=100, warm=10) -> dict:
     """sim_step_batched with the Shortest-Queue baseline on the 4-server environment.
 
-    Counted bytes per env-step: the structure-of-arrays state read and written (29 header
-    words, 2K server words, 2KT queue words), the records written (next observation,
-    reward, done, action) and 8 B per routed request (one ring write, one ring read)."""
+    The timed steps are replayed from a CUDA graph (launch-bound otherwise: one step is a
+    few microseconds).  Counted bytes per env-step: the structure-of-arrays state read and
+    written (29 header words, 2K server words, 2KT queue words), the records written (next
+    observation, reward, done, action) and 8 B per routed request (one ring write and one
+    ring read)."""
     cfg = W.c5(E)
     K, T, D = cfg["n_servers"], cfg["n_types"], cfg["obs_dim"]
     sim = simx.Sim(cfg)
@@ -201,16 +203,27 @@ def hbm_step_measure(simx, W, torch, E=65536, steps=200, warm=10) -> dict:
     rew = torch.empty(E, device="cuda")
     done = torch.empty(E, dtype=torch.uint8, device="cuda")
     act = torch.empty(E, dtype=torch.uint8, device="cuda")
-    for _ in range(warm):
-        sim.step("sq", obs=obs, reward=rew, done=done, action=act)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(warm):
+            sim.step("sq", obs=obs, reward=rew, done=done, action=act)
+    torch.cuda.current_stream().wait_stream(side)
     torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for _ in range(steps):
+            sim.step("sq", obs=obs, reward=rew, done=done, action=act)
+    graph.replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 3
     e0.record()
-    for _ in range(steps):
-        sim.step("sq", obs=obs, reward=rew, done=done, action=act)
+    for _ in range(reps):
+        graph.replay()
     e1.record()
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / steps
+    ms = e0.elapsed_time(e1) / (reps * steps)
     st, code = sim.last_status()
     sim.close()
     if st != 0:
@@ -220,10 +233,12 @@ def hbm_step_measure(simx, W, torch, E=65536, steps=200, warm=10) -> dict:
     gbs = per * E / (ms * 1e-3) / 1e9
     peaks, src = _peaks()
     hbm = float(peaks.get("hbm_gbs", 6800.0))
+    l2 = "state (%.0f MB) %s the 129 MB L2" % (state * E / 1e6, "fits in" if state * E < 100e6 else "exceeds")
     return {"kernel": "k_step_thread (policy-free step, SoA state round trip)", "envs": E,
             "us_per_step": ms * 1e3, "env_steps_per_s": E / (ms * 1e-3),
             "bytes_per_env_step": per, "achieved": gbs, "peak": hbm, "unit": "GB/s",
-            "frac": gbs / hbm, "peak_source": "%s hbm_gbs" % src}
+            "frac": gbs / hbm, "peak_source": "%s hbm_gbs" % src, "l2": l2,
+            "timing": "CUDA graph of %d steps, replayed %d times, CUDA events" % (steps, reps)}
 
 
 def run_gpu(a) -> None:
@@ -355,7 +370,8 @@ def run_gpu(a) -> None:
 
     # the policy-free batched step (Sec. 5.1 Shortest-Queue router) of the multi-server
     # environment at 65,536 envs: state read and written every step, HBM-bound
-    hbm_step = None if a.no_hbm_step else hbm_step_measure(simx, W, torch)
+    hbm_step = None if a.no_hbm_step else [hbm_step_measure(simx, W, torch, E=e)
+                                            for e in (65536, 1048576)]
 
     # roofline of the dominant kernel
     peaks, src = _peaks()

@@ -236,10 +236,17 @@ __device__ __forceinline__ uint32_t t_queued(const TEnv<K>& s) {
 }
 
 // Observation (Sec. 4.1; the layouts of rollout.cu) into obs[d * ld].
+// q / cap for a power-of-two capacity: multiplying by the exact reciprocal 2^-k gives
+// the bits of the IEEE division (no rounding either way for these small integers).
+__device__ __forceinline__ float over_cap(uint32_t q, float inv_cap) {
+  return __fmul_rn(__uint2float_rn(q), inv_cap);
+}
+
 template <bool ROUTE, int K>
 __device__ void t_observe(const Ctx& x, const TEnv<K>& s, float* o, int64_t ld) {
   const simx_config& c = x.A.cfg;
   const float fcap = __uint2float_rn(c.queue_cap);
+  const float inv_cap = __fdiv_rn(1.0f, fcap);
   int i = 0;
   if (!ROUTE) {
     const uint32_t T = c.n_types, cap = c.queue_cap;
@@ -249,8 +256,8 @@ __device__ void t_observe(const Ctx& x, const TEnv<K>& s, float* o, int64_t ld) 
     uint32_t dt = s.now - s.prev;
     if (dt < 1u) dt = 1u;
     const float fdt = __uint2float_rn(dt), tw = c.t_window_us;
-    o[(i++) * ld] = __fdiv_rn(__uint2float_rn(s.qc0[0]), fcap);
-    if (T > 1) o[(i++) * ld] = __fdiv_rn(__uint2float_rn(s.qc1[0]), fcap);
+    o[(i++) * ld] = over_cap(s.qc0[0], inv_cap);
+    if (T > 1) o[(i++) * ld] = over_cap(s.qc1[0], inv_cap);
     o[(i++) * ld] = __fdiv_rn(__uint2float_rn(s.now - s.tld), tw);
     o[(i++) * ld] = head == 0u ? 1.0f : 0.0f;
     o[(i++) * ld] = head == 1u ? 1.0f : 0.0f;
@@ -271,8 +278,8 @@ __device__ void t_observe(const Ctx& x, const TEnv<K>& s, float* o, int64_t ld) 
   } else {
 #pragma unroll
   for (int k = 0; k < K; ++k) {
-    o[(i++) * ld] = __fdiv_rn(__uint2float_rn(s.qc0[k]), fcap);
-    o[(i++) * ld] = __fdiv_rn(__uint2float_rn(c.n_types > 1 ? s.qc1[k] : 0u), fcap);
+    o[(i++) * ld] = over_cap(s.qc0[k], inv_cap);
+    o[(i++) * ld] = over_cap(c.n_types > 1 ? s.qc1[k] : 0u, inv_cap);
     const uint32_t rem = s.busy[k] > s.now ? s.busy[k] - s.now : 0u;
     o[(i++) * ld] = __fdiv_rn(__uint2float_rn(rem), c.busy_norm_us);
   }
@@ -324,8 +331,11 @@ __device__ int t_action(const Ctx& x, TEnv<K>& s) {
   return best * (int)c.n_bsizes + (int)c.static_bi;
 }
 
+#ifndef SIMX_STEP_MIN_BLOCKS
+#define SIMX_STEP_MIN_BLOCKS 1
+#endif
 template <bool ROUTE, int K>
-__global__ void __launch_bounds__(128) k_step_thread(const __grid_constant__ RolloutArgs A) {
+__global__ void __launch_bounds__(128, SIMX_STEP_MIN_BLOCKS) k_step_thread(const __grid_constant__ RolloutArgs A) {
   const uint32_t env = blockIdx.x * blockDim.x + threadIdx.x;
   if (env >= A.st.E) return;
   const DevState& st = A.st;
