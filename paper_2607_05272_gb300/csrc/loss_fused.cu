@@ -1,9 +1,10 @@
 // loss_fused.cu — REINFORCE / PPO loss gradient (Sec. 4.3) in one persistent kernel
 // for policies whose parameters fit in shared memory.
 //
-// Each block walks row tiles of R = 32 minibatch rows.  Per tile: gather the rows'
-// observations, run the forward pass keeping every activation in shared memory
-// (feature-major, [feature][row]), evaluate the loss head per row (log-softmax,
+// Each block walks row tiles of R minibatch rows (64 when two blocks of that size fit
+// in one SM's shared memory, else 32).  Per tile: gather the rows' observations, run
+// the forward pass keeping every activation in shared memory (feature-major,
+// [feature][row]), evaluate the loss head per row (log-softmax,
 // rho, clipped surrogate, entropy, value residual -> dL/dZ), then the backward pass:
 //   dW_l += dZ_l^T H_l   (each thread owns 4 x 4 blocks of dW_l, accumulated in
 //                         shared memory across all of the block's tiles),
@@ -21,18 +22,20 @@
 
 namespace simx {
 
-constexpr int kLR = 32;                // rows per tile
-constexpr int kLld = kLR + 4;          // row stride of the activation buffers
-constexpr int kLThreads = 256;
+constexpr int kLThreads = 256;         // threads per block
+// Rows per tile R (64 when the shared-memory plan allows, else 32); activation
+// buffers have row stride R + 4.
 
 // Y[j][r] = sum_k Wt[k][j] X[k][r] (+ epilogue) for rows r < R, outputs j < N.
 // Wt is row-major with row stride ldw (a multiple of 4, 16-byte aligned).
 // epi 0: + bias, tanh when do_tanh; epi 1: * (1 - H[j][r]^2).
+template <int R>
 __device__ __forceinline__ void tile_gemm(const float* __restrict__ Wt, int ldw, int K, int N,
                                           const float* X, float* Y, int epi,
                                           const float* __restrict__ bias, bool do_tanh,
                                           const float* H) {
-  const int neb = kLR / 4, nob = (N + 3) / 4;
+  constexpr int kLld = R + 4;
+  const int neb = R / 4, nob = (N + 3) / 4;
   for (int tile = threadIdx.x; tile < neb * nob; tile += blockDim.x) {
     const int eb = tile % neb, ob = tile / neb;
     float acc[4][4];
@@ -100,7 +103,9 @@ struct FusedLossArgs {
   int64_t ntiles;
 };
 
+template <int R>
 __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant__ FusedLossArgs F) {
+  constexpr int kLR = R, kLld = R + 4, kLanes = kLThreads / R;  // lanes per row in the head
   extern __shared__ float sm[];
   const LossArgs& a = F.a;
   const int L = a.n_layers;
@@ -132,39 +137,39 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
     }
     __syncthreads();
     for (int l = 0; l < L; ++l) {
-      tile_gemm(F.Wt[l], F.npad[l + 1], a.dims[l], a.dims[l + 1],
+      tile_gemm<R>(F.Wt[l], F.npad[l + 1], a.dims[l], a.dims[l + 1],
                 acts + (size_t)F.act_off[l] * kLld, acts + (size_t)F.act_off[l + 1] * kLld, 0,
                 a.b[l], l + 1 < L, nullptr);
       __syncthreads();
     }
-    // loss head: 8 lanes per row (32 rows x 8 = 256 threads); lane q takes logits
-    // i = q, q + 8, ... and the row's max / sums are reduced across the 8 lanes
+    // loss head: kLanes lanes per row (R rows x kLanes = 256 threads); lane q takes
+    // logits i = q, q + kLanes, ... and the row's max / sums are reduced across them
     const float* Z = acts + (size_t)F.act_off[L] * kLld;
     float* dz = dzA;
     {
-      const int r = threadIdx.x / 8, q = threadIdx.x % 8;
-      const unsigned gm = 0xFFu << (threadIdx.x & 24u);  // this row's 8 lanes
+      const int r = threadIdx.x / kLanes, q = threadIdx.x % kLanes;
+      const unsigned gm = (kLanes == 32 ? 0xFFFFFFFFu : ((1u << kLanes) - 1u)) << (threadIdx.x & (32 - kLanes));
       const int64_t rr = r0 + r;
       if (rr < a.n) {
         const int64_t row = a.idx ? a.idx[rr] : rr;
         const int ac = a.action[row];
         const float ad = a.adv[row];
         float m = -__uint_as_float(0x7F800000u);
-        for (int i = q; i < A; i += 8) m = fmaxf(m, Z[i * kLld + r]);
+        for (int i = q; i < A; i += kLanes) m = fmaxf(m, Z[i * kLld + r]);
 #pragma unroll
-        for (int d = 4; d > 0; d >>= 1) m = fmaxf(m, __shfl_xor_sync(gm, m, d, 8));
+        for (int d = kLanes / 2; d > 0; d >>= 1) m = fmaxf(m, __shfl_xor_sync(gm, m, d, kLanes));
         float S = 0.0f;
-        for (int i = q; i < A; i += 8) S += det_exp(Z[i * kLld + r] - m);
+        for (int i = q; i < A; i += kLanes) S += det_exp(Z[i * kLld + r] - m);
 #pragma unroll
-        for (int d = 4; d > 0; d >>= 1) S += __shfl_xor_sync(gm, S, d, 8);
+        for (int d = kLanes / 2; d > 0; d >>= 1) S += __shfl_xor_sync(gm, S, d, kLanes);
         const float lse = m + det_log(S);
         float H = 0.0f;
-        for (int i = q; i < A; i += 8) {
+        for (int i = q; i < A; i += kLanes) {
           const float lp = Z[i * kLld + r] - lse;
           H -= det_exp(lp) * lp;
         }
 #pragma unroll
-        for (int d = 4; d > 0; d >>= 1) H += __shfl_xor_sync(gm, H, d, 8);
+        for (int d = kLanes / 2; d > 0; d >>= 1) H += __shfl_xor_sync(gm, H, d, kLanes);
         const float lpa = Z[ac * kLld + r] - lse;
         float coef, pg;
         if (a.algo == SIMX_ALGO_REINFORCE) {
@@ -178,7 +183,7 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
           coef = (s1 <= s2 ? ad : 0.0f) * rho;
           if (q == 0) st_cf += fabsf(rho - 1.0f) > a.clip_eps ? 1.0 : 0.0;
         }
-        for (int i = q; i < A; i += 8) {
+        for (int i = q; i < A; i += kLanes) {
           const float lp = Z[i * kLld + r] - lse;
           const float p = det_exp(lp);
           const float onehot = (i == ac) ? 1.0f : 0.0f;
@@ -194,7 +199,7 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
           st_h += H;
         }
       } else {
-        for (int i = q; i < NL; i += 8) dz[i * kLld + r] = 0.0f;
+        for (int i = q; i < NL; i += kLanes) dz[i * kLld + r] = 0.0f;
       }
     }
     __syncthreads();
@@ -250,7 +255,7 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
       if (l > 0) {
         float* dzn = (dz == dzA) ? dzB : dzA;
         // dZ_{l-1}[k][r] = sum_j W_l[j][k] dZ_l[j][r] * (1 - H_l[k][r]^2)
-        tile_gemm(F.Wn[l], F.kpad[l], N, K, dz, dzn, 1, nullptr, false, Hl);
+        tile_gemm<R>(F.Wn[l], F.kpad[l], N, K, dz, dzn, 1, nullptr, false, Hl);
         __syncthreads();
         dz = dzn;
       } else {
@@ -262,17 +267,17 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
   float* out = F.part + (size_t)blockIdx.x * F.n_params;
   for (int i = threadIdx.x; i < F.n_params; i += blockDim.x) out[i] = gacc[i];
   // fp64 statistics of the rows this block owned (lane 0 of each row group holds them)
-  __shared__ double sh[4][kLThreads / 8];
-  if (threadIdx.x % 8 == 0) {
-    sh[0][threadIdx.x / 8] = st_pg;
-    sh[1][threadIdx.x / 8] = st_v;
-    sh[2][threadIdx.x / 8] = st_h;
-    sh[3][threadIdx.x / 8] = st_cf;
+  __shared__ double sh[4][kLR];
+  if (threadIdx.x % kLanes == 0) {
+    sh[0][threadIdx.x / kLanes] = st_pg;
+    sh[1][threadIdx.x / kLanes] = st_v;
+    sh[2][threadIdx.x / kLanes] = st_h;
+    sh[3][threadIdx.x / kLanes] = st_cf;
   }
   __syncthreads();
   if (threadIdx.x < 4) {
     double sum = 0.0;
-    for (int r = 0; r < kLThreads / 8; ++r) sum += sh[threadIdx.x][r];
+    for (int r = 0; r < kLR; ++r) sum += sh[threadIdx.x][r];
     F.spart[(size_t)blockIdx.x * 4 + threadIdx.x] = sum;
   }
 }
@@ -316,6 +321,7 @@ __global__ void k_fused_stats(const double* __restrict__ sp, int nb, int64_t n, 
 namespace {
 struct FusedPlan {
   bool ok;
+  int R;
   int npad[SIMX_MAX_LAYERS + 1], kpad[SIMX_MAX_LAYERS + 1], act_off[SIMX_MAX_LAYERS + 2];
   int dz_rows, poff[SIMX_MAX_LAYERS], n_params, grid;
   size_t smem, w_off[SIMX_MAX_LAYERS][2], part_off, spart_off, total;
@@ -323,8 +329,10 @@ struct FusedPlan {
 
 int r4(int x) { return (x + 3) / 4 * 4; }
 
-FusedPlan plan(const LossArgs& a) {
+FusedPlan plan_r(const LossArgs& a, int R) {
   FusedPlan p{};
+  p.R = R;
+  const int ld = R + 4;
   const int L = a.n_layers;
   int rows = 0, maxd = 0;
   for (int l = 0; l <= L; ++l) {
@@ -342,9 +350,9 @@ FusedPlan plan(const LossArgs& a) {
     P += a.dims[l + 1] * a.dims[l] + a.dims[l + 1];
   }
   p.n_params = P;
-  p.smem = ((size_t)rows * kLld + (size_t)2 * p.dz_rows * kLld + (size_t)P) * sizeof(float);
+  p.smem = ((size_t)rows * ld + (size_t)2 * p.dz_rows * ld + (size_t)P) * sizeof(float);
   p.ok = p.smem <= 200 * 1024;
-  const int64_t ntiles = (a.n + kLR - 1) / kLR;
+  const int64_t ntiles = (a.n + R - 1) / R;
   // resident blocks per SM: 128 registers x 256 threads allow two; shared memory may allow fewer
   const int per_sm = p.smem <= 110 * 1024 ? 2 : 1;
   int64_t grid = (int64_t)152 * per_sm;
@@ -364,6 +372,13 @@ FusedPlan plan(const LossArgs& a) {
   p.spart_off = take((size_t)p.grid * 4 * sizeof(double));
   p.total = off;
   return p;
+}
+
+// 64-row tiles when two blocks of them fit in shared memory, else 32-row tiles.
+FusedPlan plan(const LossArgs& a) {
+  const FusedPlan p64 = plan_r(a, 64);
+  if (p64.ok && p64.smem <= 110 * 1024) return p64;
+  return plan_r(a, 32);
 }
 }  // namespace
 
@@ -397,9 +412,14 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
   F.n_params = p.n_params;
   F.part = reinterpret_cast<float*>(base + p.part_off);
   F.spart = reinterpret_cast<double*>(base + p.spart_off);
-  F.ntiles = (a.n + kLR - 1) / kLR;
-  cudaFuncSetAttribute(k_loss_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
-  k_loss_fused<<<p.grid, kLThreads, p.smem, s>>>(F);
+  F.ntiles = (a.n + p.R - 1) / p.R;
+  if (p.R == 64) {
+    cudaFuncSetAttribute(k_loss_fused<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+    k_loss_fused<64><<<p.grid, kLThreads, p.smem, s>>>(F);
+  } else {
+    cudaFuncSetAttribute(k_loss_fused<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+    k_loss_fused<32><<<p.grid, kLThreads, p.smem, s>>>(F);
+  }
   k_reduce_blocks<<<(p.n_params + 255) / 256, 256, 0, s>>>(F.part, p.grid, p.n_params, a.grad);
   k_fused_stats<<<1, 32, 0, s>>>(F.spart, p.grid, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
   count_launches(a.n_layers + 3);
