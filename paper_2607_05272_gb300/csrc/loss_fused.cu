@@ -27,61 +27,197 @@ constexpr int kLThreads = 256;         // threads per block
 // buffers have row stride R + 4.
 
 // Y[j][r] = sum_k Wt[k][j] X[k][r] (+ epilogue) for rows r < R, outputs j < N.
-// Wt is row-major with row stride ldw (a multiple of 4, 16-byte aligned).
+// Wt is row-major with row stride ldw (a multiple of 4, 16-byte aligned).  Each
+// thread owns TE rows x 4 outputs: 4-row tiles when they give every thread a tile,
+// else 1-row tiles (thin layers such as the logits).
 // epi 0: + bias, tanh when do_tanh; epi 1: * (1 - H[j][r]^2).
-template <int R>
-__device__ __forceinline__ void tile_gemm(const float* __restrict__ Wt, int ldw, int K, int N,
-                                          const float* X, float* Y, int epi,
-                                          const float* __restrict__ bias, bool do_tanh,
-                                          const float* H) {
+template <int R, int TE>
+__device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ldw, int K, int N,
+                                            const float* X, float* Y, int epi,
+                                            const float* __restrict__ bias, bool do_tanh,
+                                            const float* H) {
   constexpr int kLld = R + 4;
-  const int neb = R / 4, nob = (N + 3) / 4;
+  const int neb = R / TE, nob = (N + 3) / 4;
   for (int tile = threadIdx.x; tile < neb * nob; tile += blockDim.x) {
     const int eb = tile % neb, ob = tile / neb;
-    float acc[4][4];
+    float acc[TE][4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e)
+    for (int e = 0; e < TE; ++e)
 #pragma unroll
       for (int o = 0; o < 4; ++o) acc[e][o] = 0.0f;
     const float* wc = Wt + 4 * ob;
-    const float* xc = X + 4 * eb;
+    const float* xc = X + TE * eb;
 #pragma unroll 4
     for (int k = 0; k < K; ++k) {
       const float4 w = *reinterpret_cast<const float4*>(wc + (size_t)k * ldw);
-      const float4 x = *reinterpret_cast<const float4*>(xc + k * kLld);
-      const float xv[4] = {x.x, x.y, x.z, x.w};
+      float xv[TE];
+      if (TE == 4) {
+        const float4 x = *reinterpret_cast<const float4*>(xc + k * kLld);
+        xv[0] = x.x;
+        xv[1 % TE] = x.y;
+        xv[2 % TE] = x.z;
+        xv[3 % TE] = x.w;
+      } else {
+        xv[0] = xc[k * kLld];
+      }
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
+      for (int e = 0; e < TE; ++e) {
         acc[e][0] = __fmaf_rn(w.x, xv[e], acc[e][0]);
         acc[e][1] = __fmaf_rn(w.y, xv[e], acc[e][1]);
         acc[e][2] = __fmaf_rn(w.z, xv[e], acc[e][2]);
         acc[e][3] = __fmaf_rn(w.w, xv[e], acc[e][3]);
       }
     }
+    if (TE == 4) {
+      // the tile's 4 rows of output j are one 16-byte store (conflict-free across
+      // the warp's consecutive row blocks)
 #pragma unroll
-    for (int o = 0; o < 4; ++o) {
-      const int j = 4 * ob + o;
-      if (j >= N) continue;
+      for (int o = 0; o < 4; ++o) {
+        const int j = 4 * ob + o;
+        if (j >= N) continue;
+        float4 v = make_float4(acc[0][o], acc[1 % TE][o], acc[2 % TE][o], acc[3 % TE][o]);
+        if (epi == 0) {
+          const float bj = bias[j];
+          v.x = __fadd_rn(v.x, bj);
+          v.y = __fadd_rn(v.y, bj);
+          v.z = __fadd_rn(v.z, bj);
+          v.w = __fadd_rn(v.w, bj);
+        } else {
+          const float4 h = *reinterpret_cast<const float4*>(H + j * kLld + 4 * eb);
+          v.x = v.x * (1.0f - h.x * h.x);
+          v.y = v.y * (1.0f - h.y * h.y);
+          v.z = v.z * (1.0f - h.z * h.z);
+          v.w = v.w * (1.0f - h.w * h.w);
+        }
+        *reinterpret_cast<float4*>(Y + j * kLld + 4 * eb) = v;
+      }
+      if (epi == 0 && do_tanh) {  // one det_tanh per output, four rows at a time
+#pragma unroll 1
+        for (int o = 0; o < 4; ++o) {
+          const int j = 4 * ob + o;
+          if (j < N) {
+            float4* y = reinterpret_cast<float4*>(Y + j * kLld + 4 * eb);
+            float4 v = *y;
+            v.x = det_tanh(v.x);
+            v.y = det_tanh(v.y);
+            v.z = det_tanh(v.z);
+            v.w = det_tanh(v.w);
+            *y = v;
+          }
+        }
+      }
+    } else {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int r = 4 * eb + e;
-        float v = acc[e][o];
+      for (int o = 0; o < 4; ++o) {
+        const int j = 4 * ob + o;
+        if (j >= N) continue;
+        float v = acc[0][o];
         if (epi == 0) {
           v = __fadd_rn(v, bias[j]);
         } else {
-          const float h = H[j * kLld + r];
+          const float h = H[j * kLld + eb];
           v = v * (1.0f - h * h);
         }
-        Y[j * kLld + r] = v;
+        Y[j * kLld + eb] = v;
+      }
+      if (epi == 0 && do_tanh) {
+#pragma unroll 1
+        for (int o = 0; o < 4; ++o) {
+          const int j = 4 * ob + o;
+          if (j < N) Y[j * kLld + eb] = det_tanh(Y[j * kLld + eb]);
+        }
       }
     }
-    if (epi == 0 && do_tanh) {
-#pragma unroll 1
-      for (int q = 0; q < 16; ++q) {
-        const int j = 4 * ob + q / 4;
-        if (j < N) {
-          float* y = Y + j * kLld + 4 * eb + q % 4;
-          *y = det_tanh(*y);
+  }
+}
+
+template <int R>
+__device__ __forceinline__ void tile_gemm(const float* __restrict__ Wt, int ldw, int K, int N,
+                                          const float* X, float* Y, int epi,
+                                          const float* __restrict__ bias, bool do_tanh,
+                                          const float* H) {
+  if ((R / 4) * ((N + 3) / 4) >= kLThreads)
+    tile_gemm_t<R, 4>(Wt, ldw, K, N, X, Y, epi, bias, do_tanh, H);
+  else
+    tile_gemm_t<R, 1>(Wt, ldw, K, N, X, Y, epi, bias, do_tanh, H);
+}
+
+// Row splits for a reduction over the R rows of a tile shared by `items`
+// independent outputs: the largest power of two S <= min(32, R / 4) with
+// items * S <= the block size (at least 1).
+template <int R>
+__device__ __forceinline__ int row_splits(int items) {
+  int S = 1;
+  while (S * 2 <= 32 && S * 2 <= R / 4 && items * S * 2 <= kLThreads) S *= 2;
+  return S;
+}
+
+// Lane mask of the S adjacent lanes (S a power of two dividing 32) that share an
+// output; their partial sums are combined by a fixed xor butterfly, so the order
+// is the same on every run.
+__device__ __forceinline__ unsigned split_mask(int S) {
+  const unsigned lane = threadIdx.x & 31u;
+  return (S == 32) ? 0xFFFFFFFFu : (((1u << S) - 1u) << (lane & ~(unsigned)(S - 1)));
+}
+
+// dW[j][k] += sum_r dZ[j][r] H[k][r] for one layer and one tile.  Thread block
+// (jb, kb) owns j = jb + p nj4, k = kb + q nk4 (p, q < 4; nj4 = ceil(N/4),
+// nk4 = ceil(K/4)): neighbouring lanes read neighbouring features, whose rows sit
+// R + 4 floats apart, so a warp's 16-byte row loads are free of bank conflicts.
+// Each block is handled by S adjacent lanes, lane sp summing rows
+// [sp R / S, (sp + 1) R / S); the S partial sums are combined by a fixed xor
+// butterfly, so the order is the same on every run.
+template <int R, int S>
+__device__ __forceinline__ void dw_blocks(const float* dz, const float* Hl, int N, int K,
+                                          float* gW) {
+  constexpr int kLld = R + 4, rs = R / S;
+  static_assert(rs % 4 == 0 && 32 % S == 0, "row split");
+  const int nj4 = (N + 3) / 4, nk4 = (K + 3) / 4, nblk = nj4 * nk4;
+  for (int qd = threadIdx.x; qd < nblk * S; qd += blockDim.x) {
+    const int blk = qd / S, sp = qd % S;
+    const int jb = blk / nk4, kb = blk % nk4;
+    float acc[4][4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) acc[p][q] = 0.0f;
+#pragma unroll 2
+    for (int r = sp * rs; r < (sp + 1) * rs; r += 4) {
+      float4 dv[4], hv[4];
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const int j = jb + p * nj4, k = kb + p * nk4;
+        dv[p] = j < N ? *reinterpret_cast<const float4*>(dz + j * kLld + r) : make_float4(0, 0, 0, 0);
+        hv[p] = k < K ? *reinterpret_cast<const float4*>(Hl + k * kLld + r) : make_float4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int p = 0; p < 4; ++p)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          acc[p][q] = __fmaf_rn(dv[p].x, hv[q].x, acc[p][q]);
+          acc[p][q] = __fmaf_rn(dv[p].y, hv[q].y, acc[p][q]);
+          acc[p][q] = __fmaf_rn(dv[p].z, hv[q].z, acc[p][q]);
+          acc[p][q] = __fmaf_rn(dv[p].w, hv[q].w, acc[p][q]);
+        }
+    }
+    if (S > 1) {
+      const unsigned gm = split_mask(S);
+#pragma unroll
+      for (int d = S / 2; d > 0; d >>= 1)
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+#pragma unroll
+          for (int q = 0; q < 4; ++q) acc[p][q] += __shfl_xor_sync(gm, acc[p][q], d, 32);
+    }
+    if (sp == 0) {
+#pragma unroll
+      for (int p = 0; p < 4; ++p) {
+        const int j = jb + p * nj4;
+        if (j >= N) continue;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int k = kb + q * nk4;
+          if (k < K) gW[(size_t)j * K + k] += acc[p][q];
         }
       }
     }
@@ -122,28 +258,32 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
   for (int64_t tile = blockIdx.x; tile < F.ntiles; tile += gridDim.x) {
     const int64_t r0 = tile * kLR;
     __syncthreads();
-    // gather X [D][R] (rows past n are zero and have zero dZ)
+    // gather X [D][R]: thread (r, dq) reads features dq, dq + kLanes, ... of row r
+    // (rows past n are zero and have zero dZ); consecutive threads take consecutive
+    // rows, so for a fixed feature the reads are coalesced along the env axis
     float* X = acts + (size_t)F.act_off[0] * kLld;
-    for (int q = threadIdx.x; q < D * kLR; q += blockDim.x) {
-      const int d = q / kLR, r = q % kLR;
+    {
+      const int r = threadIdx.x % kLR, dq = threadIdx.x / kLR;
       const int64_t rr = r0 + r;
-      float v = 0.0f;
       if (rr < a.n) {
         const int64_t row = a.idx ? a.idx[rr] : rr;
         const int64_t t = row / a.E, e = row % a.E;
-        v = a.obs[(t * D + d) * a.E + e];
+        const float* src = a.obs + t * D * a.E + e;
+        for (int d = dq; d < D; d += kLanes) X[d * kLld + r] = src[(int64_t)d * a.E];
+      } else {
+        for (int d = dq; d < D; d += kLanes) X[d * kLld + r] = 0.0f;
       }
-      X[d * kLld + r] = v;
     }
     __syncthreads();
     for (int l = 0; l < L; ++l) {
       tile_gemm<R>(F.Wt[l], F.npad[l + 1], a.dims[l], a.dims[l + 1],
-                acts + (size_t)F.act_off[l] * kLld, acts + (size_t)F.act_off[l + 1] * kLld, 0,
-                a.b[l], l + 1 < L, nullptr);
+                   acts + (size_t)F.act_off[l] * kLld, acts + (size_t)F.act_off[l + 1] * kLld, 0,
+                   a.b[l], l + 1 < L, nullptr);
       __syncthreads();
     }
     // loss head: kLanes lanes per row (R rows x kLanes = 256 threads); lane q takes
-    // logits i = q, q + kLanes, ... and the row's max / sums are reduced across them
+    // logits i = q, q + kLanes, ... and the row's max / sums are reduced across them.
+    // e_i = exp(z_i - max) is kept in the dZ buffer between the passes; p_i = e_i / S.
     const float* Z = acts + (size_t)F.act_off[L] * kLld;
     float* dz = dzA;
     {
@@ -159,14 +299,19 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
 #pragma unroll
         for (int d = kLanes / 2; d > 0; d >>= 1) m = fmaxf(m, __shfl_xor_sync(gm, m, d, kLanes));
         float S = 0.0f;
-        for (int i = q; i < A; i += kLanes) S += det_exp(Z[i * kLld + r] - m);
+        for (int i = q; i < A; i += kLanes) {
+          const float e = det_exp(Z[i * kLld + r] - m);
+          dz[i * kLld + r] = e;
+          S += e;
+        }
 #pragma unroll
         for (int d = kLanes / 2; d > 0; d >>= 1) S += __shfl_xor_sync(gm, S, d, kLanes);
         const float lse = m + det_log(S);
+        const float invS = 1.0f / S;
         float H = 0.0f;
         for (int i = q; i < A; i += kLanes) {
           const float lp = Z[i * kLld + r] - lse;
-          H -= det_exp(lp) * lp;
+          H -= dz[i * kLld + r] * invS * lp;
         }
 #pragma unroll
         for (int d = kLanes / 2; d > 0; d >>= 1) H += __shfl_xor_sync(gm, H, d, kLanes);
@@ -185,7 +330,7 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
         }
         for (int i = q; i < A; i += kLanes) {
           const float lp = Z[i * kLld + r] - lse;
-          const float p = det_exp(lp);
+          const float p = dz[i * kLld + r] * invS;
           const float onehot = (i == ac) ? 1.0f : 0.0f;
           dz[i * kLld + r] = (-coef * (onehot - p) + a.c_entropy * p * (lp + H)) * inv_n;
         }
@@ -209,48 +354,33 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
       const float* Hl = acts + (size_t)F.act_off[l] * kLld;
       float* gW = gacc + F.poff[l];
       float* gb = gW + (size_t)N * K;
-      // dW += dZ^T H: 4 x 4 blocks of (j, k), rows in float4 steps
-      const int njb = (N + 3) / 4, nkb = (K + 3) / 4;
-      for (int blk = threadIdx.x; blk < njb * nkb; blk += blockDim.x) {
-        const int jb = blk / nkb, kb = blk % nkb;
-        float acc[4][4];
-#pragma unroll
-        for (int p = 0; p < 4; ++p)
-#pragma unroll
-          for (int q = 0; q < 4; ++q) acc[p][q] = 0.0f;
-        for (int r = 0; r < kLR; r += 4) {
-          float4 dv[4], hv[4];
-#pragma unroll
-          for (int p = 0; p < 4; ++p) {
-            const int j = 4 * jb + p, k = 4 * kb + p;
-            dv[p] = j < N ? *reinterpret_cast<const float4*>(dz + j * kLld + r) : make_float4(0, 0, 0, 0);
-            hv[p] = k < K ? *reinterpret_cast<const float4*>(Hl + k * kLld + r) : make_float4(0, 0, 0, 0);
-          }
-#pragma unroll
-          for (int p = 0; p < 4; ++p)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              acc[p][q] = __fmaf_rn(dv[p].x, hv[q].x, acc[p][q]);
-              acc[p][q] = __fmaf_rn(dv[p].y, hv[q].y, acc[p][q]);
-              acc[p][q] = __fmaf_rn(dv[p].z, hv[q].z, acc[p][q]);
-              acc[p][q] = __fmaf_rn(dv[p].w, hv[q].w, acc[p][q]);
-            }
-        }
-#pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          const int j = 4 * jb + p;
-          if (j >= N) continue;
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int k = 4 * kb + q;
-            if (k < K) gW[(size_t)j * K + k] += acc[p][q];
-          }
+      // dW += dZ^T H: 4 x 4 blocks of (j, k); the tile's rows are split over S
+      // adjacent lanes (S > 1 for thin layers) whose partial sums are combined before
+      // the block's accumulator is updated
+      {
+        const int nblk = ((N + 3) / 4) * ((K + 3) / 4);
+        switch (row_splits<R>(nblk)) {
+          case 1: dw_blocks<R, 1>(dz, Hl, N, K, gW); break;
+          case 2: dw_blocks<R, 2>(dz, Hl, N, K, gW); break;
+          case 4: dw_blocks<R, 4>(dz, Hl, N, K, gW); break;
+          case 8: dw_blocks<R, 8>(dz, Hl, N, K, gW); break;
+          default: dw_blocks<R, (R / 4 < 16 ? R / 4 : 16)>(dz, Hl, N, K, gW); break;  // S <= R / 4
         }
       }
-      for (int j = threadIdx.x; j < N; j += blockDim.x) {
-        float sacc = 0.0f;
-        for (int r = 0; r < kLR; ++r) sacc += dz[j * kLld + r];
-        gb[j] += sacc;
+      // db += column sums of dZ, rows split the same way
+      {
+        const int S = row_splits<R>(N), lg = __ffs(S) - 1, rs = kLR >> lg;
+        for (int qd = threadIdx.x; qd < N * S; qd += blockDim.x) {
+          const int j = qd >> lg, sp = qd & (S - 1);
+          float sacc = 0.0f;
+          for (int r = sp * rs; r < (sp + 1) * rs; r += 4) {
+            const float4 v = *reinterpret_cast<const float4*>(dz + j * kLld + r);
+            sacc += (v.x + v.y) + (v.z + v.w);
+          }
+          const unsigned gm = split_mask(S);
+          for (int d = S / 2; d > 0; d >>= 1) sacc += __shfl_xor_sync(gm, sacc, d, 32);
+          if (sp == 0) gb[j] += sacc;
+        }
       }
       if (l > 0) {
         float* dzn = (dz == dzA) ? dzB : dzA;
