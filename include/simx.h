@@ -176,11 +176,20 @@ typedef struct simx_rollout {
 /* Loss selection for ppo_loss_grad (Sec. 4.3). */
 typedef enum { SIMX_ALGO_REINFORCE = 0, SIMX_ALGO_PPO = 1 } simx_algo;
 
+/* Arithmetic of the loss-gradient products (the paper fixes none; Sec. 4.3 trains in
+   PyTorch's default fp32).  SIMX_PREC_FP32: FP32 fused multiply-adds on the CUDA cores
+   (within 1e-5 of the fp64 definition).  SIMX_PREC_TF32: the matrix products on the
+   tensor cores with TF32 inputs (rounded to nearest) and FP32 accumulation, within 1e-2;
+   policies too wide for the tensor-core kernel (a layer wider than 128 outputs, or
+   operands beyond one SM's shared memory) silently take the FP32 path. */
+typedef enum { SIMX_PREC_FP32 = 0, SIMX_PREC_TF32 = 1 } simx_precision;
+
 typedef struct simx_loss_params {
   int32_t algo;        /* simx_algo */
   float   clip_eps;    /* PPO clip range epsilon */
   float   c_value;     /* value-loss coefficient (used when the MLP has a value row) */
   float   c_entropy;   /* entropy bonus coefficient */
+  int32_t precision;   /* simx_precision */
 } simx_loss_params;
 
 /* Aggregate counters over all envs (sim_stats). */

@@ -508,6 +508,8 @@ static simx_status loss_args(const simx_mlp* pol, const simx_rollout* buf, int64
   if (!p) return fail(SIMX_EINVAL, "loss params are NULL");
   if (p->algo != SIMX_ALGO_REINFORCE && p->algo != SIMX_ALGO_PPO) return fail(SIMX_EINVAL, "algo %d", p->algo);
   if (p->algo == SIMX_ALGO_PPO && !buf->logp) return fail(SIMX_EINVAL, "PPO needs logp_old");
+  if (p->precision != SIMX_PREC_FP32 && p->precision != SIMX_PREC_TF32)
+    return fail(SIMX_EINVAL, "precision %d", p->precision);
   if (!d_adv || !d_grad || !d_stats) return fail(SIMX_EINVAL, "adv, grad and stats are required");
   if (pol->has_value && !d_ret) return fail(SIMX_EINVAL, "a value row needs return targets");
   if (E < 1 || buf->ld != E) return fail(SIMX_EINVAL, "n_rows_per_step %lld must equal the rollout ld %lld", (long long)E, (long long)buf->ld);
@@ -532,6 +534,7 @@ static simx_status loss_args(const simx_mlp* pol, const simx_rollout* buf, int64
   a.clip_eps = p->clip_eps;
   a.c_value = p->c_value;
   a.c_entropy = p->c_entropy;
+  a.precision = p->precision;
   a.grad = d_grad;
   a.stats = d_stats;
   return SIMX_OK;

@@ -92,12 +92,19 @@ struct LossArgs {
   float clip_eps, c_value, c_entropy;
   float* grad;           // flat gradient
   float* stats;          // [5]
+  int precision;         // SIMX_PREC_FP32 (SIMT) or SIMX_PREC_TF32 (tensor cores where it fits)
 };
 size_t loss_workspace_bytes(const LossArgs& a);
 // loss_fused.cu
 bool loss_fused_fits(const LossArgs& a);
 size_t loss_fused_workspace(const LossArgs& a);
 cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
+void launch_loss_reduce(const float* part, int nb, int n_params, const double* spart,
+                        const LossArgs& a, cudaStream_t s);
+// loss_tc.cu
+bool loss_tc_fits(const LossArgs& a);
+size_t loss_tc_workspace(const LossArgs& a);
+cudaError_t launch_loss_tc(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 
 }  // namespace simx

@@ -550,10 +550,18 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
     cudaFuncSetAttribute(k_loss_fused<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
     k_loss_fused<32><<<p.grid, kLThreads, p.smem, s>>>(F);
   }
-  k_reduce_blocks<<<(p.n_params + 255) / 256, 256, 0, s>>>(F.part, p.grid, p.n_params, a.grad);
-  k_fused_stats<<<1, 32, 0, s>>>(F.spart, p.grid, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
-  count_launches(a.n_layers + 3);
+  launch_loss_reduce(F.part, p.grid, p.n_params, F.spart, a, s);
+  count_launches(a.n_layers + 1);
   return cudaGetLastError();
+}
+
+// Sums the per-block partial gradients (in block order) into a.grad and the per-block
+// fp64 statistics into a.stats.
+void launch_loss_reduce(const float* part, int nb, int n_params, const double* spart,
+                        const LossArgs& a, cudaStream_t s) {
+  k_reduce_blocks<<<(n_params + 255) / 256, 256, 0, s>>>(part, nb, n_params, a.grad);
+  k_fused_stats<<<1, 32, 0, s>>>(spart, nb, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
+  count_launches(2);
 }
 
 }  // namespace simx

@@ -60,7 +60,10 @@ class Rollout(C.Structure):
 
 class LossParams(C.Structure):
     _fields_ = [("algo", C.c_int32), ("clip_eps", C.c_float), ("c_value", C.c_float),
-                ("c_entropy", C.c_float)]
+                ("c_entropy", C.c_float), ("precision", C.c_int32)]
+
+
+PRECISION = {"fp32": 0, "tf32": 1}
 
 
 class Counters(C.Structure):
@@ -300,13 +303,14 @@ def ppo_loss_grad_workspace_size(policy: Policy, n: int) -> int:
 
 
 def ppo_loss_grad(policy: Policy, buf: dict, ret, adv, idx, n: int, algo: str, clip_eps: float,
-                  c_value: float, c_entropy: float, grad, stats, workspace, stream=None):
+                  c_value: float, c_entropy: float, grad, stats, workspace, stream=None,
+                  precision: str = "fp32"):
     r = Rollout()
     r.ld = buf["action"].shape[-1]
     for k in ("obs", "action", "logp", "value", "reward", "done", "trace"):
         t = buf.get(k)
         setattr(r, k, None if t is None else t.data_ptr())
-    p = LossParams(ALGO[algo], clip_eps, c_value, c_entropy)
+    p = LossParams(ALGO[algo], clip_eps, c_value, c_entropy, PRECISION[precision])
     _check(lib().ppo_loss_grad(C.byref(policy.c), C.byref(r), r.ld, _ptr(ret), _ptr(adv),
                                _ptr(idx), n, C.byref(p), _ptr(grad), _ptr(stats), _ptr(workspace),
                                workspace.numel() * workspace.element_size(), _stream(stream)))
@@ -317,7 +321,7 @@ NOALLOC_SCRATCH_BYTES = 16 << 20
 
 def ppo_loss_grad_noalloc(policy: Policy, buf: dict, ret, adv, idx, n: int, algo: str,
                           clip_eps: float, c_value: float, c_entropy: float, grad, stats,
-                          stream=None):
+                          stream=None, precision: str = "fp32"):
     """ppo_loss_grad without a caller workspace: the scratch is a buffer inside the
     library, for callers that cannot allocate device memory (see include/simx.h)."""
     r = Rollout()
@@ -325,7 +329,7 @@ def ppo_loss_grad_noalloc(policy: Policy, buf: dict, ret, adv, idx, n: int, algo
     for k in ("obs", "action", "logp", "value", "reward", "done", "trace"):
         t = buf.get(k)
         setattr(r, k, None if t is None else t.data_ptr())
-    p = LossParams(ALGO[algo], clip_eps, c_value, c_entropy)
+    p = LossParams(ALGO[algo], clip_eps, c_value, c_entropy, PRECISION[precision])
     _check(lib().ppo_loss_grad_noalloc(C.byref(policy.c), C.byref(r), r.ld, _ptr(ret), _ptr(adv),
                                        _ptr(idx), n, C.byref(p), _ptr(grad), _ptr(stats),
                                        _stream(stream)))

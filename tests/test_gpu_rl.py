@@ -6,7 +6,8 @@ order, so these compare within tolerances derived from the arithmetic:
   same recurrence run on absolute values (the sum of |terms| it adds), and per
   tensor ||x - x_ref|| <= 1e-5 ||x_ref||;
 * loss gradients, per tensor: ||g - g_ref|| <= 1e-5 ||g_ref||, per element:
-  |g - g_ref| <= 1e-5 (|g_ref| + rms(g_ref)).
+  |g - g_ref| <= 1e-5 (|g_ref| + rms(g_ref)); the tensor-core (TF32-input) path is held
+  to 1e-2 under the same definitions.
 Sizes span several blocks with ragged tails, plus the full c1 returns shape.
 """
 import numpy as np
@@ -90,9 +91,11 @@ def test_mean_baseline(n):
     assert np.all(np.abs(adv.cpu().numpy() - a_ref) <= 1e-6 * (np.abs(x) + abs(m_ref)))
 
 
-def _rollout_for_loss(simx, name, E, H):
+def _rollout_for_loss(simx, name, E, H, hidden=None):
     cfg = W.CONFIGS[name](E)
     dims, hv = W.mlp_dims(name)
+    if hidden is not None:
+        dims = [dims[0]] + [hidden] * (len(dims) - 2) + [dims[-1]]
     Ws, bs = W.mlp_weights(dims, 21)
     bs = [(np.random.default_rng(l).standard_normal(b.shape) * 0.05).astype(np.float32)
           for l, b in enumerate(bs)]
@@ -107,15 +110,49 @@ def _rollout_for_loss(simx, name, E, H):
     return cfg, pol, (Ws, bs, hv), buf
 
 
-def _check_grad(g, g_ref, layers):
+def _check_grad(g, g_ref, layers, tol=1e-5):
     off = 0
     for (W_, b_) in layers:
         for size in (W_.size, b_.size):
             gg, rr = g[off:off + size], g_ref[off:off + size]
             off += size
-            assert np.linalg.norm(gg - rr) <= 1e-5 * np.linalg.norm(rr) + 1e-12
+            assert np.linalg.norm(gg - rr) <= tol * np.linalg.norm(rr) + 1e-12
             rms = np.sqrt(np.mean(rr ** 2))
-            assert np.all(np.abs(gg - rr) <= 1e-5 * (np.abs(rr) + rms) + 1e-12)
+            assert np.all(np.abs(gg - rr) <= tol * (np.abs(rr) + rms) + 1e-12)
+
+
+def _loss_case(simx, name, algo, E, H, nmb, precision="fp32", hidden=None):
+    cfg, pol, host, buf = _rollout_for_loss(simx, name, E, H, hidden)
+    n_rows = E * H
+    rng = np.random.default_rng(3)
+    adv = (rng.standard_normal((H, E)) * 2.0).astype(np.float32)
+    ret = rng.standard_normal((H, E)).astype(np.float32)
+    logp = buf["logp"].cpu().numpy()
+    if algo == "ppo":
+        # move half the rows' old log-probabilities so clipping is exercised, keeping
+        # rho away from the clip edges by more than the arithmetic's noise
+        shift = rng.choice([0.0, 0.35, -0.35], size=(H, E)).astype(np.float32)
+        logp = (logp + shift).astype(np.float32)
+        buf["logp"] = torch.from_numpy(logp).cuda()
+    idx = None if nmb is None else rng.permutation(n_rows)[:nmb].astype(np.int64)
+    n = n_rows if idx is None else len(idx)
+    grad = torch.empty(pol.n_params, device="cuda")
+    stats = torch.empty(5, device="cuda")
+    ws = torch.empty(simx.ppo_loss_grad_workspace_size(pol, n), dtype=torch.uint8, device="cuda")
+    simx.ppo_loss_grad(pol, buf, torch.from_numpy(ret).cuda(), torch.from_numpy(adv).cuda(),
+                       None if idx is None else torch.from_numpy(idx).cuda(), n, algo, 0.2, 0.5,
+                       0.01, grad, stats, ws, precision=precision)
+    torch.cuda.synchronize()
+    obs = buf["obs"].cpu().numpy()
+    act = buf["action"].cpu().numpy()
+    rows = np.arange(n_rows) if idx is None else idx
+    X, a, lpo = rl.gather_rows(obs, act, logp, rows, E)
+    t, e = rows // E, rows % E
+    Ws, bs, hv = host
+    grads, st = rl.loss_grad(Ws, bs, hv, X, a, lpo, adv[t, e], ret[t, e],
+                             rl.PPO if algo == "ppo" else rl.REINFORCE, 0.2, 0.5, 0.01)
+    return grad.cpu().numpy().astype(np.float64), stats.cpu().numpy().astype(np.float64), \
+        rl.flat(grads), st, list(zip(Ws, bs)), n
 
 
 @pytest.mark.parametrize("name,algo,E,H,nmb", [
@@ -128,36 +165,32 @@ def _check_grad(g, g_ref, layers):
 ])
 def test_loss_gradient_matches_oracle(name, algo, E, H, nmb):
     simx = _simx()
-    cfg, pol, host, buf = _rollout_for_loss(simx, name, E, H)
-    n_rows = E * H
-    rng = np.random.default_rng(3)
-    adv = (rng.standard_normal((H, E)) * 2.0).astype(np.float32)
-    ret = rng.standard_normal((H, E)).astype(np.float32)
-    logp = buf["logp"].cpu().numpy()
-    if algo == "ppo":
-        # move half the rows' old log-probabilities so clipping is exercised, keeping
-        # rho away from the clip edges by more than fp32 noise
-        shift = rng.choice([0.0, 0.35, -0.35], size=(H, E)).astype(np.float32)
-        logp = (logp + shift).astype(np.float32)
-        buf["logp"] = torch.from_numpy(logp).cuda()
-    idx = None if nmb is None else rng.permutation(n_rows)[:nmb].astype(np.int64)
-    n = n_rows if idx is None else len(idx)
-    grad = torch.empty(pol.n_params, device="cuda")
-    stats = torch.empty(5, device="cuda")
-    ws = torch.empty(simx.ppo_loss_grad_workspace_size(pol, n), dtype=torch.uint8, device="cuda")
-    simx.ppo_loss_grad(pol, buf, torch.from_numpy(ret).cuda(), torch.from_numpy(adv).cuda(),
-                       None if idx is None else torch.from_numpy(idx).cuda(), n, algo, 0.2, 0.5,
-                       0.01, grad, stats, ws)
-    torch.cuda.synchronize()
-    obs = buf["obs"].cpu().numpy()
-    act = buf["action"].cpu().numpy()
-    rows = np.arange(n_rows) if idx is None else idx
-    X, a, lpo = rl.gather_rows(obs, act, logp, rows, E)
-    t, e = rows // E, rows % E
-    Ws, bs, hv = host
-    grads, st = rl.loss_grad(Ws, bs, hv, X, a, lpo, adv[t, e], ret[t, e],
-                             rl.PPO if algo == "ppo" else rl.REINFORCE, 0.2, 0.5, 0.01)
-    _check_grad(grad.cpu().numpy().astype(np.float64), rl.flat(grads), list(zip(Ws, bs)))
-    s = stats.cpu().numpy().astype(np.float64)
+    g, s, g_ref, st, layers, n = _loss_case(simx, name, algo, E, H, nmb)
+    _check_grad(g, g_ref, layers)
     assert np.all(np.abs(s[:4] - st[:4]) <= 1e-5 * (np.abs(st[:4]) + 1.0))
     assert abs(s[4] - st[4]) <= 1.0 / n  # clip fraction: at most one row on an fp32 edge
+
+
+@pytest.mark.parametrize("name,algo,E,H,nmb,hidden", [
+    ("c2", "reinforce", 40, 512, None, None),   # 160 full 128-row tiles
+    ("c2", "reinforce", 3, 7, None, None),      # one partial tile
+    ("c1", "reinforce", 16, 700, 5000, None),   # minibatch, ragged last tile
+    ("c2", "ppo", 37, 300, 9001, None),
+    ("c3", "ppo", 64, 256, 8192, 64),           # value head, 13-64-64-17
+    ("c3", "reinforce", 21, 50, None, 32),
+])
+def test_tensor_core_loss_gradient_matches_oracle(name, algo, E, H, nmb, hidden):
+    """TF32 tensor-core loss gradient against the fp64 oracle, within 1e-2."""
+    simx = _simx()
+    g, s, g_ref, st, layers, n = _loss_case(simx, name, algo, E, H, nmb, "tf32", hidden)
+    _check_grad(g, g_ref, layers, tol=1e-2)
+    assert np.all(np.abs(s[:4] - st[:4]) <= 1e-2 * (np.abs(st[:4]) + 1.0))
+    assert abs(s[4] - st[4]) <= 1.0 / n
+
+
+def test_tensor_core_request_falls_back_for_wide_policies():
+    """A policy too wide for the tensor-core kernel gives the FP32 path's exact bits."""
+    simx = _simx()
+    a = _loss_case(simx, "c3", "ppo", 16, 64, 700, "tf32")
+    b = _loss_case(simx, "c3", "ppo", 16, 64, 700, "fp32")
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
