@@ -141,6 +141,19 @@ __device__ __forceinline__ float4 tm_ld4(uint32_t taddr) {
   return make_float4(__uint_as_float(a), __uint_as_float(b), __uint_as_float(c), __uint_as_float(d));
 }
 
+// Issue a 4-column load without waiting; tm_wait() then completes every load issued,
+// and reg_fence() keeps the compiler from using the registers before that point.
+__device__ __forceinline__ void tm_ld4_nw(uint32_t taddr, uint32_t (&u)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3])
+               : "r"(taddr)
+               : "memory");
+}
+__device__ __forceinline__ void tm_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void reg_fence(uint32_t (&u)[4]) {
+  asm volatile("" : "+r"(u[0]), "+r"(u[1]), "+r"(u[2]), "+r"(u[3]));
+}
+
 // Byte offset of element (r, c) in a row-major operand of width W (core matrices of
 // 8 rows x 4 columns, row-group major).
 __device__ __forceinline__ uint32_t rm_off(int r, int c, int W) {
@@ -244,34 +257,62 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
     fence_after();
   };
 
-  for (int64_t tile = blockIdx.x; tile < A.ntiles; tile += gridDim.x) {
+  // Per-row inputs of the next tile are loaded into registers while the current tile
+  // is computed: observation blocks cb = cq, cq + 4 (the plan keeps C_0 <= 32), and for
+  // the head thread (cq == 0) the action, advantage, old log-probability and target.
+  float px[8];
+  int pact = 0;
+  float padv = 0.0f, plpo = 0.0f, pret = 0.0f;
+  bool plive = false;
+  auto prefetch = [&](int64_t tile) {
     const int64_t rr = tile * kR + r;
-    const bool live = rr < a.n;
+    plive = tile < A.ntiles && rr < a.n;
     int64_t row = 0;
-    if (live) row = a.idx ? a.idx[rr] : rr;
-    // gather X (rows past n are zero; their loss gradient is zero) with the ones column
+    if (plive) row = a.idx ? a.idx[rr] : rr;
+    const int64_t t = row / a.E, e = row % a.E;
+    const float* src = a.obs + t * D * a.E + e;
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int f = 4 * (cq + 4 * j) + i;
+        px[4 * j + i] = (plive && f < D) ? src[(int64_t)f * a.E] : 0.0f;
+      }
+    if (cq == 0 && plive) {
+      pact = a.action[row];
+      padv = a.adv[row];
+      plpo = a.algo == SIMX_ALGO_PPO ? a.logp_old[row] : 0.0f;
+      pret = a.has_value ? a.ret[row] : 0.0f;
+    }
+  };
+  prefetch(blockIdx.x);
+  for (int64_t tile = blockIdx.x; tile < A.ntiles; tile += gridDim.x) {
+    const bool live = plive;
+    const int ac_row = pact;
+    const float adv_row = padv, lpo_row = plpo, ret_row = pret;
+    // X (rows past n are zero; their loss gradient is zero) with the ones column
     {
       const int C = P.C[0];
-      const float* src = nullptr;
-      if (live) {
-        const int64_t t = row / a.E, e = row % a.E;
-        src = a.obs + t * D * a.E + e;
-      }
       unsigned char* hr_lo = hr + kR * C * 4;  // x_lo follows x_hi in the row-major buffer
-      for (int cb = cq; cb < C / 4; cb += 4) {
-        float hi[4], lo[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int f = 4 * cb + i;
-          const float x = f < D ? (live ? src[(int64_t)f * a.E] : 0.0f) : (f == D ? 1.0f : 0.0f);
-          hi[i] = to_tf32(x);
-          lo[i] = to_tf32(x - hi[i]);
-          if (f < D) put1(sm + P.o_ht[0], tr_off(f, r), hi[i]);
+      for (int j = 0; j < 2; ++j) {
+        const int cb = cq + 4 * j;
+        if (cb < C / 4) {
+          float hi[4], lo[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int f = 4 * cb + i;
+            const float x = f < D ? px[4 * j + i] : (f == D ? 1.0f : 0.0f);
+            hi[i] = to_tf32(x);
+            lo[i] = to_tf32(x - hi[i]);
+            if (f < D) put1(sm + P.o_ht[0], tr_off(f, r), hi[i]);
+          }
+          put4(hr, rm_off(r, 4 * cb, C), make_float4(hi[0], hi[1], hi[2], hi[3]));
+          put4(hr_lo, rm_off(r, 4 * cb, C), make_float4(lo[0], lo[1], lo[2], lo[3]));
         }
-        put4(hr, rm_off(r, 4 * cb, C), make_float4(hi[0], hi[1], hi[2], hi[3]));
-        put4(hr_lo, rm_off(r, 4 * cb, C), make_float4(lo[0], lo[1], lo[2], lo[3]));
       }
     }
+    prefetch(tile + gridDim.x);
     if (!stage_sync()) break;
     // forward
     for (int l = 0; l < L; ++l) {
@@ -292,51 +333,63 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
       }
       wait_mma();
       if (l + 1 < L) {
-        // H_{l+1} = tanh(Z_l): row-major with its ones column, and transposed
+        // H_{l+1} = tanh(Z_l): row-major with its ones column, and transposed; the
+        // thread's column blocks cb = cq + 4 j are loaded four at a time, one wait each
         const int Cn = P.C[l + 1];
-        for (int cb = cq; cb < Cn / 4; cb += 4) {
-          float v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-          if (4 * cb < N) {
-            const float4 z = tm_ld4(tlane + P.t_work + 4 * cb);
-            v[0] = z.x;
-            v[1] = z.y;
-            v[2] = z.z;
-            v[3] = z.w;
-          }
+        for (int j0 = 0; cq + 4 * j0 < Cn / 4; j0 += 4) {
+          uint32_t u[4][4];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int f = 4 * cb + i;
-            if (f < N) {
-              const float h = tanhf(v[i]);
-              put1(sm + P.o_ht[l + 1], tr_off(f, r), h);  // FP32 (the MMA reads its TF32 part)
-              v[i] = to_tf32(h);
-            } else {
-              v[i] = f == N ? 1.0f : 0.0f;
-            }
+          for (int j = 0; j < 4; ++j) {
+            const int cb = cq + 4 * (j0 + j);
+            if (cb < Cn / 4 && 4 * cb < N) tm_ld4_nw(tlane + P.t_work + 4 * cb, u[j]);
+            else u[j][0] = u[j][1] = u[j][2] = u[j][3] = 0u;
           }
-          put4(hr, rm_off(r, 4 * cb, Cn), make_float4(v[0], v[1], v[2], v[3]));
+          tm_wait();
+#pragma unroll
+          for (int j = 0; j < 4; ++j) reg_fence(u[j]);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int cb = cq + 4 * (j0 + j);
+            if (cb >= Cn / 4) break;
+            float v[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int f = 4 * cb + i;
+              if (f < N) {
+                const float h = tanhf(__uint_as_float(u[j][i]));
+                put1(sm + P.o_ht[l + 1], tr_off(f, r), h);  // FP32 (the MMA reads its TF32 part)
+                v[i] = to_tf32(h);
+              } else {
+                v[i] = f == N ? 1.0f : 0.0f;
+              }
+            }
+            put4(hr, rm_off(r, 4 * cb, Cn), make_float4(v[0], v[1], v[2], v[3]));
+          }
         }
       } else if (cq == 0) {
         // loss head for row r: G_L = dL/dZ (logits, then the value row)
         float z[kMaxNL];
+        {
+          uint32_t u[kMaxNL / 4][4];
 #pragma unroll
-        for (int cb = 0; cb < kMaxNL / 4; ++cb) {
-          if (4 * cb < N) {
-            const float4 q = tm_ld4(tlane + P.t_work + 4 * cb);
-            z[4 * cb] = q.x;
-            z[4 * cb + 1] = q.y;
-            z[4 * cb + 2] = q.z;
-            z[4 * cb + 3] = q.w;
-          } else {
-            z[4 * cb] = z[4 * cb + 1] = z[4 * cb + 2] = z[4 * cb + 3] = 0.0f;
+          for (int cb = 0; cb < kMaxNL / 4; ++cb) {
+            if (4 * cb < N) tm_ld4_nw(tlane + P.t_work + 4 * cb, u[cb]);
+            else u[cb][0] = u[cb][1] = u[cb][2] = u[cb][3] = 0u;
+          }
+          tm_wait();
+#pragma unroll
+          for (int cb = 0; cb < kMaxNL / 4; ++cb) {
+            reg_fence(u[cb]);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) z[4 * cb + i] = __uint_as_float(u[cb][i]);
           }
         }
         float g[kMaxNL];
 #pragma unroll
         for (int i = 0; i < kMaxNL; ++i) g[i] = 0.0f;
         if (live) {
-          const int ac = a.action[row];
-          const float ad = a.adv[row];
+          const int ac = ac_row;
+          const float ad = adv_row;
           float m = -__uint_as_float(0x7F800000u);
 #pragma unroll
           for (int i = 0; i < kMaxNL; ++i)
@@ -363,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
             coef = ad;
             pg = -ad * lpa;
           } else {
-            const float rho = expf(lpa - a.logp_old[row]);
+            const float rho = expf(lpa - lpo_row);
             const float s1 = rho * ad;
             const float s2 = fminf(fmaxf(rho, 1.0f - a.clip_eps), 1.0f + a.clip_eps) * ad;
             pg = -fminf(s1, s2);
@@ -383,7 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
 #pragma unroll
             for (int i = 0; i < kMaxNL; ++i)
               if (i == NA) zv = z[i];
-            const float dv = zv - a.ret[row];
+            const float dv = zv - ret_row;
             st_v += (double)dv * (double)dv;
 #pragma unroll
             for (int i = 0; i < kMaxNL; ++i)
@@ -434,27 +487,35 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
         // G_{l-1} = dH_l * (1 - H_l^2), row-major (width Gw_{l-1}) and transposed
         const int Gn = P.Gw[l - 1];
         (void)Kp;
-        for (int cb = cq; cb < Gn / 4; cb += 4) {
-          float v[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-          if (4 * cb < K) {
-            const float4 d = tm_ld4(tlane + P.t_work + 4 * cb);
-            v[0] = d.x;
-            v[1] = d.y;
-            v[2] = d.z;
-            v[3] = d.w;
-          }
+        for (int j0 = 0; cq + 4 * j0 < Gn / 4; j0 += 4) {
+          uint32_t u[4][4];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int f = 4 * cb + i;
-            if (f < K) {
-              const float h = get1(sm + P.o_ht[l], tr_off(f, r));
-              v[i] = to_tf32(v[i] * (1.0f - h * h));
-              put1(dat, tr_off(f, r), v[i]);
-            } else {
-              v[i] = 0.0f;
-            }
+          for (int j = 0; j < 4; ++j) {
+            const int cb = cq + 4 * (j0 + j);
+            if (cb < Gn / 4 && 4 * cb < K) tm_ld4_nw(tlane + P.t_work + 4 * cb, u[j]);
+            else u[j][0] = u[j][1] = u[j][2] = u[j][3] = 0u;
           }
-          put4(hr, rm_off(r, 4 * cb, Gn), make_float4(v[0], v[1], v[2], v[3]));
+          tm_wait();
+#pragma unroll
+          for (int j = 0; j < 4; ++j) reg_fence(u[j]);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int cb = cq + 4 * (j0 + j);
+            if (cb >= Gn / 4) break;
+            float v[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int f = 4 * cb + i;
+              if (f < K) {
+                const float h = get1(sm + P.o_ht[l], tr_off(f, r));
+                v[i] = to_tf32(__uint_as_float(u[j][i]) * (1.0f - h * h));
+                put1(dat, tr_off(f, r), v[i]);
+              } else {
+                v[i] = 0.0f;
+              }
+            }
+            put4(hr, rm_off(r, 4 * cb, Gn), make_float4(v[0], v[1], v[2], v[3]));
+          }
         }
       }
       if (!stage_sync()) break;
@@ -532,7 +593,7 @@ Plan plan(const LossArgs& a) {
     hr_w = hr_w > p.Gw[l] ? hr_w : p.Gw[l];
     maxN = maxN > N ? maxN : N;
   }
-  if (a.dims[L] > kMaxNL) return p;
+  if (a.dims[L] > kMaxNL || p.C[0] > 32) return p;  // head registers; prefetch of 2 blocks
   p.n_params = P;
   // shared memory: the transposed G block first, because its M = 128 reads run past its
   // own rows into the following buffers (those result rows are never read)
