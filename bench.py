@@ -42,6 +42,8 @@ def _args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-hbm-step", action="store_true")
+    p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
+                   help="loss-gradient products: tf32 tensor cores (parity 1e-2) or fp32 (1e-5)")
     p.add_argument("--cpu-child", default=None, help=argparse.SUPPRESS)
     return p.parse_args()
 
@@ -179,6 +181,12 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
+# DRAM bytes (read + write) of one k_rollout launch of the benchmark workload, from an
+# ncu capture of the current kernel; to be re-measured (or set to None) whenever the
+# rollout kernel changes.
+ROLLOUT_DRAM_BYTES = 116.2e6
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -296,7 +304,7 @@ def run_gpu(a) -> None:
         if ev:
             ev[3].record(stream)
         simx.ppo_loss_grad(pol, buf, ret, adv, None, n, "reinforce", 0.2, 0.0, 0.0, grad, stats,
-                           ws_l)
+                           ws_l, precision=a.loss_precision)
         if ev:
             ev[4].record(stream)
 
@@ -368,6 +376,20 @@ def run_gpu(a) -> None:
         e2e = {"value": world * n / t_e2e, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}
 
+    # the loss gradient in the other precision, on the same buffer, for comparison
+    other = "fp32" if a.loss_precision == "tf32" else "tf32"
+    lo_ms = []
+    for _ in range(5):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        simx.ppo_loss_grad(pol, buf, ret, adv, None, n, "reinforce", 0.2, 0.0, 0.0, grad, stats,
+                           ws_l, precision=other)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        lo_ms.append(e0.elapsed_time(e1))
+    loss_other_ms = statistics.median(lo_ms[1:])
+
     # the policy-free batched step (Sec. 5.1 Shortest-Queue router) of the multi-server
     # environment at 65,536 envs: state read and written every step, HBM-bound
     hbm_step = None if a.no_hbm_step else [hbm_step_measure(simx, W, torch, E=e)
@@ -382,18 +404,32 @@ def run_gpu(a) -> None:
     A = dims[-1] - (1 if hv else 0)
     flop_rollout = n * (2.0 * P + 20.0 * hidden + 20.0 * A) + 15.0 * cand_per_launch
     flop_loss = n * (6.0 * P - 2.0 * dims[0] * dims[1])
-    phases = {"rollout_ms": ph[0], "returns_ms": ph[1], "baseline_ms": ph[2], "loss_grad_ms": ph[3]}
+    phases = {"rollout_ms": ph[0], "returns_ms": ph[1], "baseline_ms": ph[2], "loss_grad_ms": ph[3],
+              "loss_grad_%s_ms" % other: loss_other_ms}
+    # the loss kernel against its own bound: FP32 lanes, or the TF32 tensor pipe (nominally
+    # half the bf16 rate; the measured bf16 GEMM peak x 0.5)
+    if a.loss_precision == "tf32":
+        tf32_peak = float(peaks.get("bf16_tflops", 1900.0)) * 0.5
+        ach_l = flop_loss / (ph[3] * 1e-3) / 1e12
+        roof_loss = {"kernel": "k_loss_tc (tcgen05 kind::tf32)", "bound": "tensor", "achieved": ach_l,
+                     "peak": tf32_peak, "unit": "TFLOP/s", "frac": ach_l / tf32_peak, "traffic": None,
+                     "peak_source": "%s bf16_tflops x 0.5 (nominal tf32 / bf16 rate)" % src}
+    else:
+        ach_l = flop_loss / (ph[3] * 1e-3) / 1e12
+        roof_loss = {"kernel": "k_loss_fused (FP32 SIMT)", "bound": "alu", "achieved": ach_l,
+                     "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach_l / fp32_peak, "traffic": None,
+                     "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz" % sm_mhz}
     dom = max(range(4), key=lambda i: ph[i])
     if dom == 0:
         ach = flop_rollout / (ph[0] * 1e-3) / 1e12
         roof = {"kernel": "k_rollout (simulation + fused policy)", "bound": "alu", "achieved": ach,
-                "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak, "traffic": None,
+                "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak,
+                "traffic": ROLLOUT_DRAM_BYTES,
+                "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one "
+                                  "k_rollout launch of this workload (5.8 MB + 110.4 MB)",
                 "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz" % sm_mhz}
     elif dom == 3:
-        ach = flop_loss / (ph[3] * 1e-3) / 1e12
-        roof = {"kernel": "loss gradient (SIMT fp32 GEMMs)", "bound": "alu", "achieved": ach,
-                "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak, "traffic": None,
-                "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz" % sm_mhz}
+        roof = roof_loss
     else:
         hbm = float(peaks.get("hbm_gbs", 6800.0))
         byts = n * 13.0 if dom == 1 else n * 12.0
@@ -406,13 +442,18 @@ def run_gpu(a) -> None:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": a.steps,
             "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "vs_baseline": None, "dtype": "f32+tf32" if a.loss_precision == "tf32" else "f32",
+            "data": "synthetic",
             "config": {"workload": "c2: 4096 envs x 512 steps per GPU, MMPP 300/3000 req/s, "
                                    "80/20 short/long, MLP 16-64-64-12, REINFORCE + mean baseline",
                        "envs_per_gpu": E, "horizon": H, "l2": "flushed (256 MB write) before every "
-                       "timed step", "parallelism": "replicas" if world > 1 else "single GPU"},
+                       "timed step", "parallelism": "replicas" if world > 1 else "single GPU",
+                       "loss_precision": "tf32 tensor cores, split tf32 first layer, fp32 "
+                       "accumulation (parity 1e-2)" if a.loss_precision == "tf32" else
+                       "fp32 (parity 1e-5)"},
             "phases_ms": phases,
             "roofline": roof,
+            "roofline_loss": roof_loss,
             "e2e": e2e,
             "hbm_step": hbm_step,
             "gpu_launches": launches,

@@ -141,6 +141,13 @@ __device__ __forceinline__ float4 tm_ld4(uint32_t taddr) {
   return make_float4(__uint_as_float(a), __uint_as_float(b), __uint_as_float(c), __uint_as_float(d));
 }
 
+// tanh(x) = 1 - 2 / (e^{2x} + 1) with the hardware exponential and reciprocal: absolute
+// error near 1e-7 (far below the TF32 rounding that follows), exactly +-1 once e^{2x}
+// overflows or underflows.
+__device__ __forceinline__ float tanh_fast(float x) {
+  return 1.0f - __fdividef(2.0f, __expf(2.0f * x) + 1.0f);
+}
+
 // Issue a 4-column load without waiting; tm_wait() then completes every load issued,
 // and reg_fence() keeps the compiler from using the registers before that point.
 __device__ __forceinline__ void tm_ld4_nw(uint32_t taddr, uint32_t (&u)[4]) {
@@ -317,17 +324,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
     // forward
     for (int l = 0; l < L; ++l) {
       const int C = P.C[l], Np = P.Np[l], N = P.N[l];
-      if (tid == 0) {
+      if (tid == kThreads - 32) {
+        // descriptors advance by 256 bytes (16 in the address field) per K step of 8
         const uint32_t id = idesc(kR, Np);
         const uint32_t sbo = (C / 4) * 128;
+        uint64_t xh = sdesc(su32(hr), 128, sbo), wh = sdesc(su32(sm + P.o_wa[l]), 128, sbo);
+        uint64_t wl = sdesc(su32(sm + P.o_wl0), 128, sbo), xl = sdesc(su32(hr) + kR * C * 4, 128, sbo);
+        const uint32_t d = tmem + P.t_work;
         for (int ks = 0; ks < C / 8; ++ks) {
-          const uint64_t xh = sdesc(su32(hr) + 256 * ks, 128, sbo);
-          const uint64_t wh = sdesc(su32(sm + P.o_wa[l]) + 256 * ks, 128, sbo);
-          mma(tmem + P.t_work, xh, wh, id, ks > 0);
+          mma(d, xh, wh, id, ks > 0);
           if (l == 0) {  // split TF32: + x_hi w_lo + x_lo w_hi
-            mma(tmem + P.t_work, xh, sdesc(su32(sm + P.o_wl0) + 256 * ks, 128, sbo), id, 1u);
-            mma(tmem + P.t_work, sdesc(su32(hr) + kR * C * 4 + 256 * ks, 128, sbo), wh, id, 1u);
+            mma(d, xh, wl, id, 1u);
+            mma(d, xl, wh, id, 1u);
           }
+          xh += 16;
+          wh += 16;
+          wl += 16;
+          xl += 16;
         }
         commit(mbar);
       }
@@ -356,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
             for (int i = 0; i < 4; ++i) {
               const int f = 4 * cb + i;
               if (f < N) {
-                const float h = tanhf(__uint_as_float(u[j][i]));
+                const float h = tanh_fast(__uint_as_float(u[j][i]));
                 put1(sm + P.o_ht[l + 1], tr_off(f, r), h);  // FP32 (the MMA reads its TF32 part)
                 v[i] = to_tf32(h);
               } else {
@@ -398,11 +411,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
 #pragma unroll
           for (int i = 0; i < kMaxNL; ++i)
             if (i < NA) {
-              g[i] = expf(z[i] - m);
+              g[i] = __expf(z[i] - m);
               S += g[i];
             }
-          const float lse = m + logf(S);
-          const float invS = 1.0f / S;
+          const float lse = m + __logf(S);
+          const float invS = __fdividef(1.0f, S);
           float H = 0.0f, lpa = 0.0f;
 #pragma unroll
           for (int i = 0; i < kMaxNL; ++i)
@@ -416,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
             coef = ad;
             pg = -ad * lpa;
           } else {
-            const float rho = expf(lpa - lpo_row);
+            const float rho = __expf(lpa - lpo_row);
             const float s1 = rho * ad;
             const float s2 = fminf(fmaxf(rho, 1.0f - a.clip_eps), 1.0f + a.clip_eps) * ad;
             pg = -fminf(s1, s2);
@@ -464,21 +477,31 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
     // backward
     for (int l = L - 1; l >= 0; --l) {
       const int K = P.K[l], Gw = P.Gw[l], Kp = P.Kp[l];
-      if (tid == 0) {
+      if (tid == kThreads - 32) {
+        // transposed operands advance 2 x 144 bytes (18 in the address field) per K step
         const uint32_t acc0 = first ? 0u : 1u;
         const uint32_t idw = idesc(kR, Kp), idb = idesc(kR, 16);
+        uint64_t ad = sdesc(su32(dat), kRowLd, kTGroup);
+        uint64_t hd = sdesc(su32(sm + P.o_ht[l]), kRowLd, kTGroup);
+        uint64_t od = sdesc(su32(sm + P.o_ones), kRowLd, kTGroup);
+        const uint32_t dw = tmem + P.t_dw[l], db = tmem + P.t_db[l];
         for (int ks = 0; ks < kR / 8; ++ks) {
-          const uint64_t ad = sdesc(su32(dat) + 2 * kRowLd * ks, kRowLd, kTGroup);
-          mma(tmem + P.t_dw[l], ad, sdesc(su32(sm + P.o_ht[l]) + 2 * kRowLd * ks, kRowLd, kTGroup),
-              idw, ks > 0 ? 1u : acc0);
-          mma(tmem + P.t_db[l], ad, sdesc(su32(sm + P.o_ones) + 2 * kRowLd * ks, kRowLd, kTGroup),
-              idb, ks > 0 ? 1u : acc0);
+          const uint32_t acc = ks > 0 ? 1u : acc0;
+          mma(dw, ad, hd, idw, acc);
+          mma(db, ad, od, idb, acc);
+          ad += (2 * kRowLd) >> 4;
+          hd += (2 * kRowLd) >> 4;
+          od += (2 * kRowLd) >> 4;
         }
         if (l > 0) {
           const uint32_t idh = idesc(kR, Kp);
-          for (int ks = 0; ks < Gw / 8; ++ks)
-            mma(tmem + P.t_work, sdesc(su32(hr) + 256 * ks, 128, (Gw / 4) * 128),
-                sdesc(su32(sm + P.o_wt[l]) + 256 * ks, 128, (Gw / 4) * 128), idh, ks > 0);
+          uint64_t gd = sdesc(su32(hr), 128, (Gw / 4) * 128);
+          uint64_t wd = sdesc(su32(sm + P.o_wt[l]), 128, (Gw / 4) * 128);
+          for (int ks = 0; ks < Gw / 8; ++ks) {
+            mma(tmem + P.t_work, gd, wd, idh, ks > 0);
+            gd += 16;
+            wd += 16;
+          }
         }
         commit(mbar);
       }
