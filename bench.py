@@ -42,6 +42,9 @@ def _args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-hbm-step", action="store_true")
+    p.add_argument("--sweep", action="store_true",
+                   help="every configuration (c1-c5, c5 at every env count): one JSON line each")
+    p.add_argument("--sweep-child", default=None, help=argparse.SUPPRESS)
     p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
                    help="loss-gradient products: tf32 tensor cores (parity 1e-2) or fp32 (1e-5)")
     p.add_argument("--cpu-child", default=None, help=argparse.SUPPRESS)
@@ -134,6 +137,181 @@ def run_reference(a) -> None:
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
+
+
+def _sweep_child(spec: str):
+    """Oracle rollout of one configuration over envs [env0, env0 + n) for H steps."""
+    import oracle
+    from paper_2607_05272_gb300 import workloads as W
+    name, E, env0, n, H = spec.split(",")
+    E, env0, n, H = int(E), int(env0), int(n), int(H)
+    cfg = W.CONFIGS[name](E)
+    dims, hv = W.mlp_dims(name)
+    Ws, bs = W.mlp_weights(dims, 1)
+    mode = 1 if name == "c5" else 0
+    t0 = time.perf_counter()
+    oracle.rollout(cfg, (Ws, bs, hv), W.SEED[name], mode, list(range(env0, env0 + n)), H)
+    print(json.dumps({"seconds": time.perf_counter() - t0, "env_steps": n * H}))
+
+
+def _oracle_rate(name: str, E: int, H: int, budget_s: float = 3.0) -> dict:
+    """Oracle rollout env-steps/s on one core and on every host core (one fresh process per
+    core over disjoint env ranges); each sample sized to about budget_s seconds."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+
+    def child(env0, n, h):
+        return subprocess.Popen([sys.executable, os.path.abspath(__file__), "--sweep-child",
+                                 "%s,%d,%d,%d,%d" % (name, E, env0, n, h)], stdout=subprocess.PIPE,
+                                stderr=subprocess.PIPE, text=True, env=env, cwd=ROOT)
+
+    def result(p):
+        out, err = p.communicate()
+        if p.returncode != 0:
+            raise RuntimeError("oracle child failed:\n" + err[-2000:])
+        return json.loads(out.strip().splitlines()[-1])
+
+    h = min(H, 64)
+    probe = result(child(0, 1, h))
+    per_step = probe["seconds"] / probe["env_steps"]
+    target = max(h, int(budget_s / max(per_step, 1e-9)))  # env-steps for about budget_s
+    h = min(H, max(h, target // E))                        # whole-E samples grow the horizon
+    n = max(1, min(E, target // h))
+    one = result(child(0, n, h))
+    cores = os.cpu_count() or 1
+    n_each = max(1, min(n, -(-E // cores)))
+    h_each = min(H, max(h, target // n_each))
+    procs = [child((i * n_each) % E, n_each, h_each) for i in range(cores)]
+    res = [result(p) for p in procs]
+    # every process runs concurrently; the rate uses each one's own compute time (process
+    # start-up excluded), bounded by the slowest
+    wall = max(r["seconds"] for r in res)
+    return {"oracle_1core_steps_per_s": one["env_steps"] / one["seconds"],
+            "oracle_ncore_steps_per_s": sum(r["env_steps"] for r in res) / wall,
+            "oracle_cores": cores,
+            "oracle_sample": "%d envs x %d steps (1 core); %d processes x %d envs x %d steps"
+                             % (n, h, cores, n_each, h_each)}
+
+
+def measure_fp32_peak(simx, torch) -> dict:
+    """FP32 FMA rate of this GPU from the library's probe kernel (best of 5 launches)."""
+    sink = torch.empty(simx.fma_probe_sink_floats(), device="cuda")
+    simx.fma_probe(1000, sink)
+    best = 0.0
+    for _ in range(5):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fl = simx.fma_probe(20000, sink)
+        e1.record()
+        torch.cuda.synchronize()
+        best = max(best, fl / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    return {"tflops": best, "sms": props.multi_processor_count}
+
+
+def run_sweep(a) -> None:
+    """Every configuration on one GPU (rollout steps/s and FP32 fraction; GAE samples/s and
+    HBM fraction; PPO loss minibatches/s) beside the oracle's 1-core and all-core rates."""
+    import numpy as np
+    import torch
+
+    from paper_2607_05272_gb300 import build as B
+    from paper_2607_05272_gb300 import workloads as W
+    B.build()
+    import oracle
+    oracle.build()
+    from paper_2607_05272_gb300 import simx
+    peaks, src = _peaks()
+    fp = measure_fp32_peak(simx, torch)
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    tf32_peak = float(peaks.get("bf16_tflops", 1900.0)) * 0.5
+    print(json.dumps({"fp32_fma_probe_tflops": fp["tflops"], "sms": fp["sms"], "hbm_gbs": hbm,
+                      "hbm_source": src}), flush=True)
+    cases = [("c1", 64, 10000, "sample"), ("c2", 4096, 512, "sample"), ("c3", 16384, 256, "sample"),
+             ("c4", 65536, 512, "sample")]
+    cases += [("c5", e, 1024, "argmax") for e in (1024, 4096, 16384, 65536, 262144, 1048576)]
+    oracle_cache = {}
+    for name, E, H, mode in cases:
+        cfg = W.CONFIGS[name](E)
+        dims, hv = W.mlp_dims(name)
+        Ws, bs = W.mlp_weights(dims, 1)
+        pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws],
+                          [torch.from_numpy(b).cuda() for b in bs], hv)
+        sim = simx.Sim(cfg)
+        sim.reset(W.SEED[name])
+        warm = simx.alloc_rollout(E, sim.D, 4, has_value=hv)
+        sim.rollout(mode, 4, warm, pol)
+        del warm
+        buf = simx.alloc_rollout(E, sim.D, H, has_value=hv)
+        arr0 = sim.stats()["arrived"]
+        reps = 3 if E * H <= 50_000_000 else 1
+        ts = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            sim.rollout(mode, H, buf, pol)
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        st, code = sim.last_status()
+        arrivals = (sim.stats()["arrived"] - arr0) / reps
+        ms = statistics.median(ts)
+        P = sum(dims[l] * dims[l + 1] for l in range(len(dims) - 1))
+        A = dims[-1] - (1 if hv else 0)
+        flop = E * H * (2.0 * P + 20.0 * sum(dims[1:-1]) + 20.0 * A) + 15.0 * arrivals
+        line = {"config": name, "envs": E, "horizon": H, "policy": mode,
+                "rollout_ms": ms, "decision_steps_per_s": E * H / (ms * 1e-3),
+                "fp32_tflops": flop / (ms * 1e-3) / 1e12,
+                "fp32_frac": flop / (ms * 1e-3) / 1e12 / fp["tflops"], "status": st}
+        n = E * H
+        if hv:  # GAE over the rollout buffer: reward, value, done in; advantage, return out
+            adv = torch.empty((H, E), device="cuda")
+            ret = torch.empty((H, E), device="cuda")
+            last = torch.zeros(E, device="cuda")
+            gts = []
+            for _ in range(3):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                simx.compute_returns_gae(buf["reward"], buf["done"], 0.99, 0.95, ret, adv=adv,
+                                         val=buf["value"], last_val=last)
+                e1.record()
+                torch.cuda.synchronize()
+                gts.append(e0.elapsed_time(e1))
+            g = min(gts)
+            line.update({"gae_ms": g, "gae_samples_per_s": n / (g * 1e-3),
+                         "gae_gbs": 17.0 * n / (g * 1e-3) / 1e9,
+                         "gae_hbm_frac": 17.0 * n / (g * 1e-3) / 1e9 / hbm})
+            # PPO loss gradient on one minibatch of 8192 rows, both precisions
+            rng = np.random.default_rng(1)
+            idx = torch.from_numpy(rng.permutation(n)[:8192].astype(np.int64)).cuda()
+            grad = torch.empty(pol.n_params, device="cuda")
+            stats = torch.empty(5, device="cuda")
+            ws = torch.empty(simx.ppo_loss_grad_workspace_size(pol, 8192), dtype=torch.uint8,
+                             device="cuda")
+            lflop = 8192 * (6.0 * P - 2.0 * dims[0] * dims[1])
+            for prec in ("fp32", "tf32"):
+                lts = []
+                for _ in range(6):
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record()
+                    simx.ppo_loss_grad(pol, buf, ret, adv, idx, 8192, "ppo", 0.2, 0.5, 0.01, grad,
+                                       stats, ws, precision=prec)
+                    e1.record()
+                    torch.cuda.synchronize()
+                    lts.append(e0.elapsed_time(e1))
+                lm = statistics.median(lts[1:])
+                line["loss8192_%s_ms" % prec] = lm
+                line["loss8192_%s_minibatches_per_s" % prec] = 1e3 / lm
+                line["loss8192_%s_tflops" % prec] = lflop / (lm * 1e-3) / 1e12
+            del adv, ret, grad, ws
+        key = name if name != "c5" else "c5"
+        if key not in oracle_cache:
+            oracle_cache[key] = _oracle_rate(name, E, H)
+        line.update(oracle_cache[key])
+        line["gpu_vs_oracle_ncore"] = line["decision_steps_per_s"] / line["oracle_ncore_steps_per_s"]
+        print(json.dumps(line), flush=True)
+        sim.close()
+        del buf, sim, pol
+        torch.cuda.empty_cache()
 
 
 # --------------------------------------------------------------------------- #
@@ -289,6 +467,7 @@ def run_gpu(a) -> None:
     stats = torch.empty(5, device="cuda")
     ws_l = torch.empty(simx.ppo_loss_grad_workspace_size(pol, n), dtype=torch.uint8, device="cuda")
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    fp = measure_fp32_peak(simx, torch)  # FP32 roofline denominator, measured on this GPU
     stream = torch.cuda.current_stream()
 
     def step(ev=None):
@@ -398,7 +577,11 @@ def run_gpu(a) -> None:
     # roofline of the dominant kernel
     peaks, src = _peaks()
     sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
-    fp32_peak = 152 * 128 * 2 * sm_mhz * 1e6 / 1e12  # TFLOP/s, FP32 FMA lanes x clock
+    fp32_nominal = fp["sms"] * 128 * 2 * sm_mhz * 1e6 / 1e12  # FMA lanes x clock
+    fp32_peak = fp["tflops"]
+    fp32_src = ("measured FMA probe (libsimx k_fma_probe, best of 5): %.1f TFLOP/s; nominal "
+                "%d SMs x 128 lanes x 2 x %.0f MHz = %.1f" % (fp32_peak, fp["sms"], sm_mhz,
+                                                            fp32_nominal))
     P = sum(dims[l] * dims[l + 1] for l in range(len(dims) - 1))
     hidden = sum(dims[1:-1])
     A = dims[-1] - (1 if hv else 0)
@@ -418,7 +601,7 @@ def run_gpu(a) -> None:
         ach_l = flop_loss / (ph[3] * 1e-3) / 1e12
         roof_loss = {"kernel": "k_loss_fused (FP32 SIMT)", "bound": "alu", "achieved": ach_l,
                      "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach_l / fp32_peak, "traffic": None,
-                     "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz" % sm_mhz}
+                     "peak_source": fp32_src}
     dom = max(range(4), key=lambda i: ph[i])
     if dom == 0:
         ach = flop_rollout / (ph[0] * 1e-3) / 1e12
@@ -427,7 +610,7 @@ def run_gpu(a) -> None:
                 "traffic": ROLLOUT_DRAM_BYTES,
                 "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one "
                                   "k_rollout launch of this workload (5.8 MB + 110.4 MB)",
-                "peak_source": "FP32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz" % sm_mhz}
+                "peak_source": fp32_src}
     elif dom == 3:
         roof = roof_loss
     else:
@@ -472,6 +655,12 @@ def main():
     a = _args()
     if a.cpu_child:
         _cpu_child(a.cpu_child)
+        return
+    if a.sweep_child:
+        _sweep_child(a.sweep_child)
+        return
+    if a.sweep:
+        run_sweep(a)
         return
     if a.impl == "reference":
         run_reference(a)

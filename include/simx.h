@@ -329,6 +329,15 @@ simx_status simx_last_status(simx_ctx* ctx, uint32_t* device_code);
    a tracing aid: the difference across a region counts the region's launches. */
 uint64_t simx_launches(void);
 
+/* FP32 fused multiply-add probe (no counterpart in the paper: the denominator of the FP32
+   roofline fractions).  Launches, on `stream`, one block of 256 threads per quarter warp
+   slot (4 blocks per SM), each thread running 16 independent FMA chains `iters` long, and
+   stores one float per thread into d_sink (device, at least simx_fma_probe_sink_floats()
+   floats).  host_flops receives the FLOPs the launch performs (2 per FMA); the caller
+   times the launch on the stream.  SIMX_EINVAL for iters < 1 or a NULL pointer. */
+simx_status simx_fma_probe(int64_t iters, float* d_sink, double* host_flops, void* stream);
+size_t simx_fma_probe_sink_floats(void);
+
 const char* simx_strerror(simx_status s);
 const char* simx_last_error(void);
 

@@ -210,6 +210,15 @@ const char* simx_last_error(void) { return g_err.c_str(); }
 
 uint64_t simx_launches(void) { return g_launches.load(std::memory_order_relaxed); }
 
+simx_status simx_fma_probe(int64_t iters, float* d_sink, double* host_flops, void* stream) {
+  if (iters < 1 || !d_sink || !host_flops) return fail(SIMX_EINVAL, "fma probe: iters %lld", (long long)iters);
+  const cudaError_t e = launch_fma_probe(iters, d_sink, host_flops, (cudaStream_t)stream);
+  if (e != cudaSuccess) return fail(SIMX_ECUDA, "fma probe: %s", cudaGetErrorString(e));
+  return SIMX_OK;
+}
+
+size_t simx_fma_probe_sink_floats(void) { return fma_probe_sink_floats(); }
+
 uint32_t simx_obs_dim(const simx_config* cfg) {
   if (!cfg || cfg->mode > SIMX_MODE_ROUTE || cfg->n_types < 1 || cfg->n_types > SIMX_MAX_TYPES ||
       cfg->n_servers < 1 || cfg->n_servers > SIMX_MAX_SERVERS)

@@ -101,6 +101,9 @@ size_t loss_fused_workspace(const LossArgs& a);
 cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 void launch_loss_reduce(const float* part, int nb, int n_params, const double* spart,
                         const LossArgs& a, cudaStream_t s);
+// fma_probe.cu
+cudaError_t launch_fma_probe(int64_t iters, float* sink, double* flops, cudaStream_t s);
+size_t fma_probe_sink_floats();
 // loss_tc.cu
 bool loss_tc_fits(const LossArgs& a);
 size_t loss_tc_workspace(const LossArgs& a);

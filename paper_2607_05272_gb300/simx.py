@@ -96,6 +96,8 @@ SIGNATURES = [
     ("sim_load", C.c_int, [P, P, U64]),
     ("simx_last_status", C.c_int, [P, P]),
     ("simx_launches", U64, []),
+    ("simx_fma_probe", C.c_int, [I64, P, P, P]),
+    ("simx_fma_probe_sink_floats", SZ, []),
     ("simx_strerror", C.c_char_p, [C.c_int]),
     ("simx_last_error", C.c_char_p, []),
 ]
@@ -333,3 +335,14 @@ def ppo_loss_grad_noalloc(policy: Policy, buf: dict, ret, adv, idx, n: int, algo
     _check(lib().ppo_loss_grad_noalloc(C.byref(policy.c), C.byref(r), r.ld, _ptr(ret), _ptr(adv),
                                        _ptr(idx), n, C.byref(p), _ptr(grad), _ptr(stats),
                                        _stream(stream)))
+
+
+def fma_probe_sink_floats() -> int:
+    return lib().simx_fma_probe_sink_floats()
+
+
+def fma_probe(iters: int, sink, stream=None) -> float:
+    """Launch the FP32 FMA-rate probe on the stream; returns the FLOPs it performs."""
+    fl = C.c_double(0.0)
+    _check(lib().simx_fma_probe(iters, _ptr(sink), C.byref(fl), _stream(stream)))
+    return fl.value
