@@ -6,7 +6,11 @@
 // REINFORCE: x = G, delta_t = r_t, c_t = gamma (1 - d_t), x_T = last_value;
 // GAE:       x = A, delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t,
 //            c_t = gamma lambda (1 - d_t), x_T = 0.
-// A block owns 32 envs (threadIdx.x) and splits time into S chunks (threadIdx.y).
+// Large env counts with 16-byte aligned rows take k_returns_wide: one thread owns four
+// adjacent envs for the whole horizon (one pass: every input read once, every output
+// written once, 17 bytes per sample for GAE), loading 8 time steps ahead with 16-byte
+// loads, so a block reads 4 KB of each row per step.  Otherwise:
+// a block owns 32 envs (threadIdx.x) and splits time into S chunks (threadIdx.y).
 // Each thread composes its chunk's map x_{t0} = a x_{t1} + b, one thread per env
 // chains the S maps in shared memory, then every thread replays its chunk from the
 // right carry.  Loads are coalesced across envs; no global scratch is needed.
@@ -90,10 +94,94 @@ k_returns_gae(const float* __restrict__ rew, const float* __restrict__ val,
   }
 }
 
+constexpr int kWideU = 8;                 // time steps loaded ahead
+constexpr int kWideThreads = 256;         // 1024 envs per block
+constexpr int64_t kWideMinEnvs = 65536;
+
+__device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ void st4(float* p, float4 v) { *reinterpret_cast<float4*>(p) = v; }
+
+template <bool GAE>
+__global__ void __launch_bounds__(kWideThreads, 2)
+k_returns_wide(const float* __restrict__ rew, const float* __restrict__ val,
+               const uint8_t* __restrict__ done, const float* __restrict__ last_val, int64_t T,
+               int64_t E, int64_t ld, float gamma, float lam, float* __restrict__ ret,
+               float* __restrict__ adv) {
+  const int64_t e = ((int64_t)blockIdx.x * kWideThreads + threadIdx.x) * 4;
+  if (e >= E) return;
+  const float cmul = GAE ? gamma * lam : gamma;
+  float4 last = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+  if (last_val) last = ld4(last_val + e);
+  float x[4] = {GAE ? 0.0f : last.x, GAE ? 0.0f : last.y, GAE ? 0.0f : last.z, GAE ? 0.0f : last.w};
+  float vn[4] = {last.x, last.y, last.z, last.w};
+  for (int64_t tb = T; tb > 0; tb -= kWideU) {
+    const int n = tb < kWideU ? (int)tb : kWideU;
+    float4 r[kWideU], v[kWideU];
+    uint32_t d[kWideU];
+#pragma unroll
+    for (int i = 0; i < kWideU; ++i) {
+      if (i < n) {
+        const int64_t o = (tb - 1 - i) * ld + e;
+        r[i] = ld4(rew + o);
+        d[i] = *reinterpret_cast<const uint32_t*>(done + o);
+        if (GAE) v[i] = ld4(val + o);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kWideU; ++i) {
+      if (i < n) {
+        const int64_t o = (tb - 1 - i) * ld + e;
+        const float rv[4] = {r[i].x, r[i].y, r[i].z, r[i].w};
+        float vv[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        if (GAE) {
+          vv[0] = v[i].x;
+          vv[1] = v[i].y;
+          vv[2] = v[i].z;
+          vv[3] = v[i].w;
+        }
+        float o4[4], g4[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float mask = ((d[i] >> (8 * k)) & 0xFFu) ? 0.0f : 1.0f;
+          float delta = rv[k];
+          if (GAE) {
+            delta = delta + gamma * mask * vn[k] - vv[k];
+            vn[k] = vv[k];
+          }
+          x[k] = delta + cmul * mask * x[k];
+          o4[k] = x[k];
+          g4[k] = x[k] + vv[k];
+        }
+        if (GAE) {
+          st4(adv + o, make_float4(o4[0], o4[1], o4[2], o4[3]));
+          st4(ret + o, make_float4(g4[0], g4[1], g4[2], g4[3]));
+        } else {
+          st4(ret + o, make_float4(o4[0], o4[1], o4[2], o4[3]));
+          if (adv) st4(adv + o, make_float4(o4[0], o4[1], o4[2], o4[3]));
+        }
+      }
+    }
+  }
+}
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
 cudaError_t launch_returns_gae(const float* rew, const float* val, const uint8_t* done,
                                const float* last_val, int64_t T, int64_t E, int64_t ld,
                                float gamma, float lam, float* ret, float* adv, cudaStream_t s) {
   if (T <= 0 || E <= 0) return cudaSuccess;
+  const bool gae = lam >= 0.0f;
+  if (E >= kWideMinEnvs && E % 4 == 0 && ld % 4 == 0 && aligned16(rew) && aligned16(ret) &&
+      ((uintptr_t)done & 3u) == 0 && (!gae || aligned16(val)) && (!adv || aligned16(adv)) &&
+      (!last_val || aligned16(last_val))) {
+    const unsigned grid = (unsigned)((E / 4 + kWideThreads - 1) / kWideThreads);
+    if (gae)
+      k_returns_wide<true><<<grid, kWideThreads, 0, s>>>(rew, val, done, last_val, T, E, ld, gamma, lam, ret, adv);
+    else
+      k_returns_wide<false><<<grid, kWideThreads, 0, s>>>(rew, val, done, last_val, T, E, ld, gamma, lam, ret, adv);
+    count_launches(1);
+    return cudaGetLastError();
+  }
   // Enough (env, chunk) threads to fill the GPU: ~300k threads, chunks of >= 16 steps.
   int S = 1;
   while (S < kRetMaxChunks && E * S * 2 <= 311296 && T / (S * 2) >= 16) S *= 2;
