@@ -8,9 +8,10 @@ order, so these compare within tolerances derived from the arithmetic:
 * loss gradients, per tensor: ||g - g_ref|| <= 1e-5 ||g_ref||, per element:
   |g - g_ref| <= 1e-5 (|g_ref| + rms(g_ref)); the tensor-core (TF32-input) path is held
   to 1e-2 under the same definitions.
-Sizes span several blocks with ragged tails (horizons that are not a multiple of the
-16-step chunk), plus the full c1 returns shape, whose 10,000-step horizon takes the
-two-pass chunked kernel; shorter horizons take the register-cached one.
+Sizes span several blocks with ragged tails, plus the full c1 returns shape; env counts
+from 65,536 that are a multiple of 4 take the one-pass four-envs-per-thread kernel (with
+horizons that are not a multiple of its 8-step lookahead), the rest the chunked two-pass
+one (262,145 envs among them).
 """
 import numpy as np
 import pytest
