@@ -331,11 +331,11 @@ __device__ int t_action(const Ctx& x, TEnv<K>& s) {
   return best * (int)c.n_bsizes + (int)c.static_bi;
 }
 
-#ifndef SIMX_STEP_MIN_BLOCKS
-#define SIMX_STEP_MIN_BLOCKS 1
-#endif
-template <bool ROUTE, int K>
-__global__ void __launch_bounds__(128, SIMX_STEP_MIN_BLOCKS) k_step_thread(const __grid_constant__ RolloutArgs A) {
+// MINB resident 128-thread blocks per SM bound the registers (4: 128, 5: 96; a few bytes
+// spill).  The latency of one env-step is a long dependent chain, so the step rate is the
+// number of resident threads over that latency: more residency beats more registers.
+template <bool ROUTE, int K, int MINB>
+__global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant__ RolloutArgs A) {
   const uint32_t env = blockIdx.x * blockDim.x + threadIdx.x;
   if (env >= A.st.E) return;
   const DevState& st = A.st;
@@ -548,9 +548,14 @@ __global__ void __launch_bounds__(128, SIMX_STEP_MIN_BLOCKS) k_step_thread(const
   }
 }
 
+// Up to one wave (152 SMs x 4 x 128 threads = 77,824 envs) and a little beyond, 4 blocks per
+// SM finish a step soonest; many waves (from 262,144 envs) run faster at 5, except with 8
+// servers, whose state does not fit 96 registers.
 template <bool ROUTE, int K>
 cudaError_t step_thread_t(const RolloutArgs& a, cudaStream_t s) {
-  k_step_thread<ROUTE, K><<<(a.st.E + 127) / 128, 128, 0, s>>>(a);
+  const unsigned grid = (a.st.E + 127) / 128;
+  if (a.st.E >= 262144 && K <= 4) k_step_thread<ROUTE, K, (K <= 4 ? 5 : 4)><<<grid, 128, 0, s>>>(a);
+  else k_step_thread<ROUTE, K, 4><<<grid, 128, 0, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
