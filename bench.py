@@ -44,6 +44,8 @@ def _args():
     p.add_argument("--no-hbm-step", action="store_true")
     p.add_argument("--sweep", action="store_true",
                    help="every configuration (c1-c5, c5 at every env count): one JSON line each")
+    p.add_argument("--sweep-configs", default="c1,c2,c3,c4,c5",
+                   help="comma-separated subset of the sweep's configurations")
     p.add_argument("--sweep-child", default=None, help=argparse.SUPPRESS)
     p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
                    help="loss-gradient products: tf32 tensor cores (parity 1e-2) or fp32 (1e-5)")
@@ -229,6 +231,8 @@ def run_sweep(a) -> None:
     cases = [("c1", 64, 10000, "sample"), ("c2", 4096, 512, "sample"), ("c3", 16384, 256, "sample"),
              ("c4", 65536, 512, "sample")]
     cases += [("c5", e, 1024, "argmax") for e in (1024, 4096, 16384, 65536, 262144, 1048576)]
+    keep = set(a.sweep_configs.split(","))
+    cases = [c for c in cases if c[0] in keep]
     oracle_cache = {}
     for name, E, H, mode in cases:
         cfg = W.CONFIGS[name](E)

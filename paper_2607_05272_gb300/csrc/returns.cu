@@ -9,7 +9,7 @@
 // Large env counts with 16-byte aligned rows take k_returns_wide: one thread owns four
 // adjacent envs for the whole horizon (one pass: every input read once, every output
 // written once, 17 bytes per sample for GAE), loading 8 time steps ahead with 16-byte
-// loads, so a block reads 4 KB of each row per step.  Otherwise:
+// loads, so a block reads 1 KB of each row per step.  Otherwise:
 // a block owns 32 envs (threadIdx.x) and splits time into S chunks (threadIdx.y).
 // Each thread composes its chunk's map x_{t0} = a x_{t1} + b, one thread per env
 // chains the S maps in shared memory, then every thread replays its chunk from the
@@ -95,14 +95,14 @@ k_returns_gae(const float* __restrict__ rew, const float* __restrict__ val,
 }
 
 constexpr int kWideU = 8;                 // time steps loaded ahead
-constexpr int kWideThreads = 256;         // 1024 envs per block
+constexpr int kWideThreads = 64;          // 256 envs per block: every SM gets blocks from 65,536 envs
 constexpr int64_t kWideMinEnvs = 65536;
 
 __device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
 __device__ __forceinline__ void st4(float* p, float4 v) { *reinterpret_cast<float4*>(p) = v; }
 
 template <bool GAE>
-__global__ void __launch_bounds__(kWideThreads, 2)
+__global__ void __launch_bounds__(kWideThreads, 8)
 k_returns_wide(const float* __restrict__ rew, const float* __restrict__ val,
                const uint8_t* __restrict__ done, const float* __restrict__ last_val, int64_t T,
                int64_t E, int64_t ld, float gamma, float lam, float* __restrict__ ret,
