@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define SIMX_ABI_VERSION 1u
+#define SIMX_ABI_VERSION 2u
 #define SIMX_MAX_TYPES 2
 #define SIMX_MAX_SERVERS 8
 #define SIMX_MAX_BSIZES 8
@@ -142,6 +142,11 @@ typedef struct simx_config {
   float    rate_ref;           /* ROUTE: EWMA rate normaliser and its initial value */
   float    busy_norm_us;       /* ROUTE: busy-remaining normaliser */
   uint32_t phase_period_us;    /* ROUTE extra: diurnal phase period */
+  /* workload variants (Sec. 3.1 K heterogeneous GPUs; Sec. 3.2 Extreme Burst) */
+  uint32_t dwell_kind;         /* 0: exponential dwell of mean dwell_mean_us; 1: fixed dwell of
+                                  round(dwell_mean_us) (a square wave between the two rates) */
+  uint32_t srv_speed16[SIMX_MAX_SERVERS]; /* batch time factor of server k in 1/16 (0 means 16):
+                                  L_k = (L * s_k + 8) / 16 in integer microseconds, 1 .. 255 */
 } simx_config;
 
 /*

@@ -336,7 +336,17 @@ static void request_attrs(const orc_env* e, const uint32_t w[4], uint32_t* type,
   *cost = cst;
 }
 
-/* Modulating chain: switch i >= 1 at S_i = S_{i-1} + round(dwell * E_i), S_0 = 0.
+/* Dwell of the modulating chain before switch i: round(dwell * E_i) with E_i the
+   exponential of the switch's draw, or exactly round(dwell) for a fixed dwell (the
+   square wave of the paper's Extreme Burst workload, Sec. 3.2). */
+static uint32_t dwell_us(orc_env* e, uint32_t i) {
+  if (e->c.dwell_kind == 1) return orc_duration(e->c.dwell_mean_us);
+  uint32_t w[4];
+  draw(e, i, ORC_STREAM_SWITCH, w);
+  return orc_duration(e->c.dwell_mean_us * expo1(w[0]));
+}
+
+/* Modulating chain: switch i >= 1 at S_i = S_{i-1} + dwell_i, S_0 = 0.
    All switches at times <= limit take effect. */
 static void process_switches(orc_env* e, uint32_t limit) {
   if (e->c.n_mod_states < 2) return;
@@ -344,9 +354,7 @@ static void process_switches(orc_env* e, uint32_t limit) {
     if (count_event(e)) return;
     e->mstate ^= 1u;
     e->sw_i += 1u;
-    uint32_t w[4];
-    draw(e, e->sw_i, ORC_STREAM_SWITCH, w);
-    e->sw_T = add_time(e, e->sw_T, orc_duration(e->c.dwell_mean_us * expo1(w[0])));
+    e->sw_T = add_time(e, e->sw_T, dwell_us(e, e->sw_i));
   }
 }
 
@@ -458,11 +466,16 @@ static void next_arrival(orc_env* e) {
   }
 }
 
-/* Batch latency (Sec. 3.1 execution model): alpha + beta n, or alpha + the sum of
-   the batch's per-request costs for the cost type. */
-static uint64_t service_time(const orc_env* e, uint32_t type, uint32_t n, uint64_t csum) {
-  if ((int32_t)type == e->c.cost_type) return (uint64_t)e->c.alpha_us[type] + csum;
-  return (uint64_t)e->c.alpha_us[type] + (uint64_t)e->c.beta_us[type] * n;
+/* Batch latency on server k (Sec. 3.1 execution model; K heterogeneous GPUs): L =
+   alpha + beta n, or alpha + the sum of the batch's per-request costs for the cost type,
+   scaled by the server's speed factor s/16 and rounded to the nearest microsecond
+   (halves up): (L s + 8) / 16 in integers, which is L itself for s = 16. */
+static uint64_t service_time(const orc_env* e, uint32_t k, uint32_t type, uint32_t n, uint64_t csum) {
+  uint64_t L;
+  if ((int32_t)type == e->c.cost_type) L = (uint64_t)e->c.alpha_us[type] + csum;
+  else L = (uint64_t)e->c.alpha_us[type] + (uint64_t)e->c.beta_us[type] * n;
+  const uint64_t s = e->c.srv_speed16[k] ? e->c.srv_speed16[k] : 16u;
+  return (L * s + 8u) / 16u;
 }
 
 /* ROUTE mode: server k starts a batch at time s from the queue whose head is
@@ -479,7 +492,7 @@ static void try_start(orc_env* e, uint32_t k, uint32_t s) {
     W += (uint64_t)(s - arr);
     csum += cost;
   }
-  uint64_t L = service_time(e, h, n, csum);
+  uint64_t L = service_time(e, k, h, n, csum);
   e->busy_until[k] = add_time(e, s, L);
   e->step_n += n;
   e->step_w[h] += W;
@@ -564,9 +577,7 @@ void orc_env_reset(orc_env* e) {
   if (c.n_mod_states == 2) {
     e->mstate = w[0] >> 31;
     e->sw_i = 1;
-    uint32_t ws[4];
-    draw(e, 1, ORC_STREAM_SWITCH, ws);
-    e->sw_T = add_time(e, 0, orc_duration(c.dwell_mean_us * expo1(ws[0])));
+    e->sw_T = add_time(e, 0, dwell_us(e, 1));
   } else {
     e->mstate = 0;
     e->sw_i = 0;
@@ -750,7 +761,7 @@ static void step_single(orc_env* e, const orc_mlp* m, int mode, int32_t ext, orc
       csum += cost;
     }
     if (n > 0) {
-      e->busy_until[0] = add_time(e, now, service_time(e, k, n, csum));
+      e->busy_until[0] = add_time(e, now, service_time(e, 0, k, n, csum));
       e->n_last = n;
       e->type_last = k;
       e->t_last_dispatch = now;

@@ -51,6 +51,8 @@ typedef struct {
   uint32_t obs_extra, obs_dim;
   float t_window_us, rate_scale, rate_ref, busy_norm_us;
   uint32_t phase_period_us;
+  uint32_t dwell_kind;                      /* 0 exponential dwell, 1 fixed dwell (square wave) */
+  uint32_t srv_speed16[ORC_MAX_SERVERS];    /* batch time factor of each server, in 1/16 (0: 16) */
 } orc_config;
 
 /* Host-memory MLP (row-major W[l] of dims[l+1] x dims[l]). */

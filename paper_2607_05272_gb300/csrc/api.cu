@@ -57,6 +57,8 @@ simx_status validate_config(const simx_config* c) {
   if (c->n_types < 1 || c->n_types > SIMX_MAX_TYPES) return fail(SIMX_EINVAL, "n_types %u", c->n_types);
   if (c->mode == SIMX_MODE_SINGLE && c->n_servers != 1) return fail(SIMX_EINVAL, "SINGLE mode needs n_servers = 1");
   if (c->n_servers < 1 || c->n_servers > SIMX_MAX_SERVERS) return fail(SIMX_EINVAL, "n_servers %u", c->n_servers);
+  for (uint32_t k = 0; k < SIMX_MAX_SERVERS; ++k)
+    if (c->srv_speed16[k] > 255) return fail(SIMX_EINVAL, "srv_speed16[%u] = %u (at most 255)", k, c->srv_speed16[k]);
   if (!pow2(c->queue_cap) || c->queue_cap > 4096) return fail(SIMX_EINVAL, "queue_cap %u must be a power of two <= 4096", c->queue_cap);
   if (c->episode_len < 1) return fail(SIMX_EINVAL, "episode_len must be >= 1");
   if (c->arrival_kind == SIMX_ARR_THINNED) {
@@ -65,6 +67,9 @@ simx_status validate_config(const simx_config* c) {
     for (uint32_t i = 0; i < c->n_mod_states; ++i)
       if (c->accept_thr[i] > (1u << 24)) return fail(SIMX_EINVAL, "accept_thr[%u] > 2^24", i);
     if (c->n_mod_states == 2 && !finite_pos(c->dwell_mean_us)) return fail(SIMX_EINVAL, "dwell_mean_us must be > 0");
+    if (c->dwell_kind > 1) return fail(SIMX_EINVAL, "dwell_kind %u", c->dwell_kind);
+    if (c->n_mod_states == 2 && c->dwell_kind == 1 && !(c->dwell_mean_us >= 0.5f))
+      return fail(SIMX_EINVAL, "a fixed dwell must be at least 1 us");
   } else if (c->arrival_kind == SIMX_ARR_DIURNAL) {
     if (c->mode != SIMX_MODE_ROUTE) return fail(SIMX_EINVAL, "DIURNAL arrivals need ROUTE mode");
     if (c->epoch_us < 1) return fail(SIMX_EINVAL, "epoch_us must be >= 1");

@@ -80,15 +80,23 @@ __device__ __forceinline__ uint32_t req_type(const simx_config& c, uint32_t w1) 
   return (c.n_types > 1 && (w1 >> 8) >= c.type0_thr) ? 1u : 0u;
 }
 
-__device__ __forceinline__ uint64_t service_us(const simx_config& c, uint32_t type, uint32_t n,
-                                               uint64_t csum) {
-  if ((int32_t)type == c.cost_type) return (uint64_t)c.alpha_us[type] + csum;
-  return (uint64_t)c.alpha_us[type] + (uint64_t)c.beta_us[type] * n;
+// Batch time of `n` requests of `type` on server k: alpha + beta n (or alpha + the sum
+// of the requests' costs for the cost type), times the server's speed s/16, rounded to
+// the nearest microsecond in integers.
+__device__ __forceinline__ uint64_t service_us(const simx_config& c, uint32_t k, uint32_t type,
+                                               uint32_t n, uint64_t csum) {
+  const uint64_t L = ((int32_t)type == c.cost_type)
+                         ? (uint64_t)c.alpha_us[type] + csum
+                         : (uint64_t)c.alpha_us[type] + (uint64_t)c.beta_us[type] * n;
+  const uint64_t s = c.srv_speed16[k] ? c.srv_speed16[k] : 16u;
+  return (L * s + 8u) >> 4;
 }
 
-// Time of the modulating chain's switch number i, given switch i-1 at t.
+// Time of the modulating chain's switch number i, given switch i-1 at t: an exponential
+// dwell drawn from the SWITCH stream, or the fixed dwell of a square wave.
 __device__ __forceinline__ uint32_t switch_time(const RolloutArgs& A, uint32_t env, uint32_t i,
                                                 uint32_t t, uint32_t& status) {
+  if (A.cfg.dwell_kind == 1) return add_time(t, duration_us(A.cfg.dwell_mean_us), status);
   const U4 w = philox(i, env, kStreamSwitch, 0u, A.key0, A.key1);
   return add_time(t, duration_us(__fmul_rn(A.cfg.dwell_mean_us, expo1(w.x))), status);
 }
@@ -336,9 +344,10 @@ __device__ void next_arrival(const RolloutArgs& A, const Grp<G>& g, uint32_t env
 
 // ROUTE mode, executed by the lane that owns the server: start a batch at time
 // st from the queue whose head arrived first (tie: type 0).
-__device__ __forceinline__ void try_start(const simx_config& c, uint32_t* ringS, uint32_t* costS,
-                                          Srv& L, uint32_t st, uint32_t& stn, uint64_t& w0,
-                                          uint64_t& w1, uint32_t& nbat, uint32_t& status) {
+__device__ __forceinline__ void try_start(const simx_config& c, uint32_t srv, uint32_t* ringS,
+                                          uint32_t* costS, Srv& L, uint32_t st, uint32_t& stn,
+                                          uint64_t& w0, uint64_t& w1, uint32_t& nbat,
+                                          uint32_t& status) {
   const uint32_t cap = c.queue_cap;
   uint32_t h;
   if (L.qc[0] > 0 && L.qc[1] > 0) {
@@ -361,7 +370,7 @@ __device__ __forceinline__ void try_start(const simx_config& c, uint32_t* ringS,
   }
   L.qh.set(h, (L.qh[h] + n) & (cap - 1u));
   L.qc.set(h, L.qc[h] - n);
-  L.busy = add_time(st, service_us(c, h, n, csum), status);
+  L.busy = add_time(st, service_us(c, srv, h, n, csum), status);
   stn += n;
   if (h) w1 += W; else w0 += W;
   nbat += 1u;
@@ -682,7 +691,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
           L.qh.set(k, (L.qh[k] + n) & (cap - 1u));
           L.qc.set(k, L.qc[k] - n);
           if (n > 0) {
-            L.busy = add_time(now, service_us(c, k, n, csum), s.status);
+            L.busy = add_time(now, service_us(c, 0u, k, n, csum), s.status);
             s.nlast = n;
             s.tlast = k;
             s.tld = now;
@@ -732,7 +741,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
               dropped = 1u;
             }
             L.bsize = b;
-            if (L.busy <= now) try_start(c, ringS, costS, L, now, stn, w0, w1, nbat, lstat);
+            if (L.busy <= now) try_start(c, g.gl, ringS, costS, L, now, stn, w0, w1, nbat, lstat);
           }
           dropped = g.shfl(dropped, (int)k);
           s.ndrop += dropped;
@@ -749,7 +758,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
         s.rate = __fadd_rn(s.rate, __fmul_rn(0.0625f, __fsub_rn(inst, s.rate)));
         if (g.gl < K)
           while (L.busy <= s.pt && (L.qc[0] + L.qc[1]) > 0u)
-            try_start(c, ringS, costS, L, L.busy, stn, w0, w1, nbat, lstat);
+            try_start(c, g.gl, ringS, costS, L, L.busy, stn, w0, w1, nbat, lstat);
         s.now = s.pt;
       }
       __syncwarp();

@@ -68,8 +68,12 @@ __device__ void t_switches(const Ctx& x, TEnv<K>& s, uint32_t limit) {
     if (t_count(s)) return;
     s.mst ^= 1u;
     s.swi += 1u;
-    const U4 w = philox(s.swi, x.env, kStreamSwitch, 0u, x.A.key0, x.A.key1);
-    s.swT = t_add(s.swT, duration_us(__fmul_rn(x.A.cfg.dwell_mean_us, expo1(w.x))), s.status);
+    if (x.A.cfg.dwell_kind == 1) {  // fixed dwell: a square wave
+      s.swT = t_add(s.swT, duration_us(x.A.cfg.dwell_mean_us), s.status);
+    } else {
+      const U4 w = philox(s.swi, x.env, kStreamSwitch, 0u, x.A.key0, x.A.key1);
+      s.swT = t_add(s.swT, duration_us(__fmul_rn(x.A.cfg.dwell_mean_us, expo1(w.x))), s.status);
+    }
   }
 }
 
@@ -183,6 +187,12 @@ __device__ void t_next_arrival(const Ctx& x, TEnv<K>& s) {
   }
 }
 
+// Batch time L on server k scaled by its speed s/16, rounded to the nearest microsecond.
+__device__ __forceinline__ uint64_t t_speed(const simx_config& c, int k, uint64_t L) {
+  const uint64_t s = c.srv_speed16[k] ? c.srv_speed16[k] : 16u;
+  return (L * s + 8u) >> 4;
+}
+
 // ROUTE mode: server i starts a batch at time st (the oldest-head type, tie: type 0).
 template <int K>
 __device__ __forceinline__ void t_start(const Ctx& x, TEnv<K>& s, int i, uint32_t st,
@@ -219,7 +229,7 @@ __device__ __forceinline__ void t_start(const Ctx& x, TEnv<K>& s, int i, uint32_
   }
   const uint64_t L = costed ? (uint64_t)c.alpha_us[h] + csum
                             : (uint64_t)c.alpha_us[h] + (uint64_t)c.beta_us[h] * n;
-  s.busy[i] = t_add(st, L, s.status);
+  s.busy[i] = t_add(st, t_speed(c, i, L), s.status);
   stn += n;
   if (h) w1 += W; else w0 += W;
   s.ndisp += n;
@@ -331,9 +341,9 @@ __device__ int t_action(const Ctx& x, TEnv<K>& s) {
   return best * (int)c.n_bsizes + (int)c.static_bi;
 }
 
-// MINB resident 128-thread blocks per SM bound the registers (4: 128, 5: 96; a few bytes
-// spill).  The latency of one env-step is a long dependent chain, so the step rate is the
-// number of resident threads over that latency: more residency beats more registers.
+// MINB resident 128-thread blocks per SM bound the registers (4: 128).  The latency of
+// one env-step is a long dependent chain, so the step rate is the number of resident
+// threads over that latency: more residency beats more registers.
 template <bool ROUTE, int K, int MINB>
 __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant__ RolloutArgs A) {
   const uint32_t env = blockIdx.x * blockDim.x + threadIdx.x;
@@ -418,7 +428,7 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
           const uint64_t L = ((int32_t)kk == c.cost_type)
                                  ? (uint64_t)c.alpha_us[kk] + csum
                                  : (uint64_t)c.alpha_us[kk] + (uint64_t)c.beta_us[kk] * n;
-          s.busy[0] = t_add(now, L, s.status);
+          s.busy[0] = t_add(now, t_speed(c, 0, L), s.status);
           s.nlast = n;
           s.tlast = kk;
           s.tld = now;
@@ -548,14 +558,11 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
   }
 }
 
-// Up to one wave (152 SMs x 4 x 128 threads = 77,824 envs) and a little beyond, 4 blocks per
-// SM finish a step soonest; many waves (from 262,144 envs) run faster at 5, except with 8
-// servers, whose state does not fit 96 registers.
+// 4 resident blocks per SM (128 registers): one wave of 77,824 envs; fewer registers
+// spill the server state of the router.
 template <bool ROUTE, int K>
 cudaError_t step_thread_t(const RolloutArgs& a, cudaStream_t s) {
-  const unsigned grid = (a.st.E + 127) / 128;
-  if (a.st.E >= 262144 && K <= 4) k_step_thread<ROUTE, K, (K <= 4 ? 5 : 4)><<<grid, 128, 0, s>>>(a);
-  else k_step_thread<ROUTE, K, 4><<<grid, 128, 0, s>>>(a);
+  k_step_thread<ROUTE, K, 4><<<(a.st.E + 127) / 128, 128, 0, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }

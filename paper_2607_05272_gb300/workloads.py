@@ -30,7 +30,7 @@ import math
 
 import numpy as np
 
-ABI_VERSION = 1
+ABI_VERSION = 2
 MODE_SINGLE, MODE_ROUTE = 0, 1
 ARR_THINNED, ARR_DIURNAL = 0, 1
 POLICY = {"sample": 0, "argmax": 1, "static": 2, "rr": 3, "sq": 4, "random": 5, "external": 6}
@@ -47,7 +47,8 @@ CONFIG_FIELDS = [
     ("cost_scale_us", "f32"), ("pareto_inv_alpha", "f32"), ("w_wait", "f32[2]"),
     ("n_bsizes", "u32"), ("bsizes", "u32[8]"), ("static_bi", "u32"), ("obs_extra", "u32"),
     ("obs_dim", "u32"), ("t_window_us", "f32"), ("rate_scale", "f32"), ("rate_ref", "f32"),
-    ("busy_norm_us", "f32"), ("phase_period_us", "u32"),
+    ("busy_norm_us", "f32"), ("phase_period_us", "u32"), ("dwell_kind", "u32"),
+    ("srv_speed16", "u32[8]"),
 ]
 
 
@@ -75,7 +76,7 @@ def _base(**kw) -> dict:
         cost_type=-1, cost_kind=0, cost_scale_us=0.0, pareto_inv_alpha=0.0,
         w_wait=[0.001, 0.0], n_bsizes=6, bsizes=[1, 2, 4, 8, 16, 32, 0, 0], static_bi=3,
         obs_extra=0, obs_dim=8, t_window_us=10000.0, rate_scale=1250.0, rate_ref=800.0,
-        busy_norm_us=100000.0, phase_period_us=0,
+        busy_norm_us=100000.0, phase_period_us=0, dwell_kind=0, srv_speed16=[0] * 8,
     )
     c.update(kw)
     return c
@@ -141,7 +142,28 @@ def mm1(lam: float, mean_service_us: float = 2100.0, n_envs: int = 64) -> dict:
                  cost_type=0, cost_kind=1, cost_scale_us=float(mean_service_us))
 
 
-CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5}
+def burst(n_envs: int = 64) -> dict:
+    """Extreme Burst (Sec. 3.2): c1's server under a square wave between 0 and 100 req/s.
+
+    The paper switches "every 200 steps"; here the rate switches every 2 s of simulated
+    time (200 steps at the high rate's 10 ms mean gap) through the modulating chain with a
+    fixed dwell: candidates at 100/s, all kept in the high state and none in the low one.
+    """
+    return _base(n_envs=n_envs, cand_mean_gap_us=10000.0, n_mod_states=2,
+                 accept_thr=[0, TWO24], dwell_mean_us=2_000_000.0, dwell_kind=1,
+                 rate_scale=10000.0, rate_ref=100.0)
+
+
+def c3h(n_envs: int = 16384) -> dict:
+    """Heterogeneous multi-GPU routing (Sec. 3.1 K heterogeneous GPUs, Sec. 3.2 Multi-GPU
+    Routing): c3's router with a 50/50 fast/slow request mix over two full-speed servers
+    and two at half speed (batch times x 2)."""
+    c = c3(n_envs)
+    c.update(type0_thr=_thr(0.5), srv_speed16=[16, 16, 32, 32, 0, 0, 0, 0])
+    return c
+
+
+CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5, "burst": burst, "c3h": c3h}
 
 # Policy network shapes (input, hidden..., actions) and whether a value row follows.
 MLP_SHAPES = {
@@ -150,10 +172,13 @@ MLP_SHAPES = {
     "c3": ([13, 128, 128, 16], True),
     "c4": ([28, 256, 256, 48], True),
     "c5": ([13, 128, 128, 16], True),
+    "burst": ([8, 32, 6], False),
+    "c3h": ([13, 128, 128, 16], True),
 }
 
-HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024}
-SEED = {name: 0x5EED0000 + i + 1 for i, name in enumerate(["c1", "c2", "c3", "c4", "c5"])}
+HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024, "burst": 2000, "c3h": 256}
+SEED = {name: 0x5EED0000 + i + 1
+        for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h"])}
 
 
 def mlp_dims(name: str) -> tuple:

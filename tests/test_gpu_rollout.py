@@ -70,6 +70,8 @@ CASES = [
     ("c3", lambda: W.c3(45), 256, "sample"),
     ("c4", lambda: W.c4(21), 512, "sample"),
     ("c5", lambda: W.c5(40), 1024, "argmax"),
+    ("burst", lambda: W.burst(37), 2000, "sample"),  # square-wave arrivals (fixed dwell)
+    ("c3h", lambda: W.c3h(45), 256, "sample"),        # heterogeneous server speeds
 ]
 
 
@@ -100,6 +102,9 @@ BASELINES = [
     ("c3", lambda: W.c3(33), 256, "rr"),
     ("c3", lambda: W.c3(33), 256, "random"),
     ("c4", lambda: W.c4(33), 512, "sq"),
+    ("burst", lambda: W.burst(35), 2000, "static"),
+    ("c3h", lambda: W.c3h(41), 256, "sq"),
+    ("c3h", lambda: W.c3h(39), 256, "rr"),
 ]
 
 
@@ -122,7 +127,8 @@ def test_single_env_and_zero_horizon():
     assert np.array_equal(sim.save(), before)
 
 
-@pytest.mark.parametrize("name,mk", [("c2", lambda: W.c2(36)), ("c4", lambda: W.c4(13))])
+@pytest.mark.parametrize("name,mk", [("c2", lambda: W.c2(36)), ("c4", lambda: W.c4(13)),
+                                     ("c3h", lambda: W.c3h(17))])
 def test_step_batched_equals_rollout(name, mk):
     """H single-step launches with the internal policy give the rollout's records."""
     simx = _simx()

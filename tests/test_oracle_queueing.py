@@ -7,6 +7,10 @@
 * Request conservation after every step: arrived = dropped + dispatched + queued.
 * The latency model L(b) = alpha + beta b and the reward on hand-built states.
 * The two-state MMPP's long-run arrival rate.
+* The Extreme Burst square wave: switch times exactly periodic, arrivals only in the
+  high-rate phases, and their count against 100 req/s over those phases.
+* Heterogeneous server speeds: batch times scaled by s/16 on hand-built states and in
+  traces.
 """
 import math
 
@@ -178,3 +182,110 @@ def test_mmpp_long_run_rate():
     per_env_mean = rate.mean()
     se = rate.std(ddof=1) / math.sqrt(rate.size)
     assert abs(per_env_mean - 1650.0) < 4.0 * se + 0.02 * 1650.0
+
+
+def _burst_state_at(t, init, D):
+    """Modulating state at time t of a square wave that starts in `init` and switches at
+    every multiple of D (a candidate at a switch time sees the new state)."""
+    return init ^ ((t // D) & 1)
+
+
+def test_square_wave_switches_and_arrival_phases():
+    """Extreme Burst: switch i is at exactly i D; every queued request arrived in a
+    high-rate phase; the arrival count matches 100 req/s over the high phases only."""
+    cfg = W.burst(6)
+    D = int(cfg["dwell_mean_us"])
+    expected = observed = 0.0
+    for env_id in range(6):
+        e = oracle.OracleEnv(cfg, env_id, 31)
+        e.reset()
+        s = e.export()
+        init = int(s[6]) ^ ((int(s[4]) - 1) & 1)   # each processed switch toggled the state
+        for _ in range(1500):
+            assert s[5] == s[4] * D                            # S_i = i D exactly
+            assert int(s[6]) == _burst_state_at(int(s[5]) - 1, init, D)
+            q = int(s[34])
+            for t in s[35:35 + q]:
+                assert _burst_state_at(int(t), init, D) == 1   # only the 100 req/s state
+            e.step(STATIC, None)
+            s = e.export()
+        now = int(s[0])
+        high = sum(min(now, (p + 1) * D) - p * D
+                   for p in range(now // D + 1) if p * D < now and _burst_state_at(p * D, init, D))
+        expected += 100.0 * high * 1e-6
+        observed += float(s[12])
+    assert expected > 1000.0
+    assert abs(observed - expected) < 4.0 * math.sqrt(expected) + 2.0
+
+
+def test_server_speed_single_hand_scenario():
+    """c1 with the server at speed 24/16: a batch of 2 takes (2200 x 24 + 8) / 16 = 3300 us."""
+    cfg = W.c1(1)
+    cfg["srv_speed16"] = [24, 0, 0, 0, 0, 0, 0, 0]
+    e = oracle.OracleEnv(cfg, 0, 5)
+    e.reset()
+    s = np.zeros(e.SW, np.uint32)
+    s[0] = 10000
+    s[2], s[3] = 5, 10000
+    s[5] = 0xFFFFFFFF
+    s[21] = 0xFFFFFFFF
+    s[23] = np.float32(800.0).view(np.uint32)
+    s[19] = 8000
+    base = 32 + 2 * 1
+    s[33] = 8
+    s[base] = 4
+    s[base + 1: base + 5] = [1000, 3000, 9000, 9500]
+    s[12], s[14] = 4, 0
+    e.load(s)
+    e.step(EXTERNAL, None, action=1)
+    s2 = e.export()
+    assert s2[32] == 10000 + 3300
+    assert s2[0] == 13300
+
+
+def test_server_speed_route_hand_scenario():
+    """c3h-style speeds: a long request routed to idle server 0 at speed 40/16 runs
+    (22000 x 40 + 8) / 16 = 55000 us; server 1 (busy) keeps its completion time."""
+    cfg = W.c3(1)
+    cfg["srv_speed16"] = [40, 32, 16, 16, 0, 0, 0, 0]
+    e = oracle.OracleEnv(cfg, 0, 5)
+    e.reset()
+    K = 4
+    s = np.zeros(e.SW, np.uint32)
+    s[0] = 50000
+    s[2], s[3] = 10, 50000
+    s[5] = 0xFFFFFFFF
+    s[9], s[10] = 50000, 1
+    s[21] = 0xFFFFFFFF
+    s[23] = np.float32(4000.0).view(np.uint32)
+    srv = 32
+    for k in range(K):
+        s[srv + 2 * k + 1] = 4
+    s[srv + 2 * 1] = 60000
+    s[12] = 1
+    e.load(s)
+    e.step(EXTERNAL, None, action=0 * 4 + 2)
+    s2 = e.export()
+    assert s2[srv + 0] == 50000 + 55000
+    assert s2[srv + 2] == 60000
+
+
+def test_server_speed_latency_from_traces():
+    """With speed s/16 the next decision after a dispatch with work still queued comes
+    exactly (L s + 8) / 16 later, L = alpha_k + beta_k n."""
+    cfg = W.c2(8)
+    cfg["srv_speed16"] = [21, 0, 0, 0, 0, 0, 0, 0]
+    out = oracle.rollout(cfg, _policy_for("c2"), W.SEED["c2"], SAMPLE, list(range(8)), 300)
+    tr, act = out["trace"], out["action"]
+    nb = cfg["n_bsizes"]
+    checked = 0
+    for t in range(299):
+        for e in range(8):
+            n, qafter = int(tr[t, 1, e]), int(tr[t, 3, e])
+            if n == 0 or qafter == 0:
+                continue
+            k = act[t, e] // nb
+            L = cfg["alpha_us"][k] + cfg["beta_us"][k] * n
+            assert tr[t + 1, 0, e] == tr[t, 0, e] + (L * 21 + 8) // 16
+            checked += 1
+    assert checked > 100
