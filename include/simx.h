@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define SIMX_ABI_VERSION 2u
+#define SIMX_ABI_VERSION 3u
 #define SIMX_MAX_TYPES 2
 #define SIMX_MAX_SERVERS 8
 #define SIMX_MAX_BSIZES 8
@@ -147,6 +147,12 @@ typedef struct simx_config {
                                   round(dwell_mean_us) (a square wave between the two rates) */
   uint32_t srv_speed16[SIMX_MAX_SERVERS]; /* batch time factor of server k in 1/16 (0 means 16):
                                   L_k = (L * s_k + 8) / 16 in integer microseconds, 1 .. 255 */
+  uint32_t action_layout;      /* 0: a = major * n_bsizes + i, batch bsizes[i];
+                                  1 (SINGLE only; Sec. 4.1 action 0 = Wait): a = 0 waits (no
+                                  dispatch; the next decision is at the next arrival), a >= 1 is
+                                  type (a-1) / n_bsizes with batch ((a-1) % n_bsizes) + 1;
+                                  n_bsizes <= 64, static batch static_bi + 1.  Actions:
+                                  1 + T * n_bsizes (33 for T = 1, 65 for T = 2 at n_bsizes 32) */
 } simx_config;
 
 /*

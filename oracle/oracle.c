@@ -518,7 +518,8 @@ orc_env* orc_env_new(const orc_config* c, uint32_t env_id, uint64_t seed) {
   e->K = c->n_servers;
   e->T = c->n_types;
   e->cap = c->queue_cap;
-  e->A = (c->mode == ORC_SINGLE ? c->n_types : c->n_servers) * c->n_bsizes;
+  e->A = (c->mode == ORC_SINGLE ? c->n_types : c->n_servers) * c->n_bsizes +
+         (c->action_layout == 1 ? 1u : 0u);
   e->qarr = (uint32_t*)calloc((size_t)e->K * 2 * e->cap, sizeof(uint32_t));
   e->qcost = (uint32_t*)calloc((size_t)e->K * e->cap, sizeof(uint32_t));
   if (!e->qarr || !e->qcost) {
@@ -571,7 +572,8 @@ void orc_env_reset(orc_env* e) {
   memset(qc, 0, (size_t)K * cap * sizeof(uint32_t));
   e->type_last = NONE;
   e->rate_est = c.rate_ref;
-  for (uint32_t k = 0; k < K; ++k) e->bsize[k] = c.bsizes[c.static_bi];
+  for (uint32_t k = 0; k < K; ++k)
+    e->bsize[k] = c.action_layout == 1 ? c.static_bi + 1u : c.bsizes[c.static_bi];
   uint32_t w[4];
   draw(e, 0, ORC_STREAM_INIT, w);
   if (c.n_mod_states == 2) {
@@ -727,7 +729,7 @@ static int32_t choose_action(orc_env* e, const orc_mlp* m, int mode, int32_t ext
   if (mode == ORC_STATIC) {
     uint32_t h = head_type(e, 0);
     if (h == NONE) h = 0;
-    return (int32_t)(h * c->n_bsizes + c->static_bi);
+    return (int32_t)((c->action_layout == 1 ? 1u : 0u) + h * c->n_bsizes + c->static_bi);
   }
   if (mode == ORC_RR) return (int32_t)((e->t_global % e->K) * c->n_bsizes + c->static_bi);
   /* ORC_SQ: fewest queued requests, first such server */
@@ -742,13 +744,32 @@ static int32_t choose_action(orc_env* e, const orc_mlp* m, int mode, int32_t ext
   return (int32_t)(best * c->n_bsizes + c->static_bi);
 }
 
+/* Action a -> (major, batch size) (Sec. 4.1).  Layout 0: major a / n_bsizes, batch
+   bsizes[a % n_bsizes].  Layout 1: a = 0 is "Wait" (batch 0: nothing is dispatched and the
+   next decision is at the next arrival), a >= 1 is major (a - 1) / n_bsizes with batch
+   ((a - 1) % n_bsizes) + 1. */
+static void decode_action(const orc_config* c, int32_t a, uint32_t* major, uint32_t* b) {
+  if (c->action_layout == 1) {
+    if (a == 0) {
+      *major = 0;
+      *b = 0;
+    } else {
+      *major = (uint32_t)(a - 1) / c->n_bsizes;
+      *b = (uint32_t)(a - 1) % c->n_bsizes + 1u;
+    }
+    return;
+  }
+  *major = (uint32_t)a / c->n_bsizes;
+  *b = c->bsizes[(uint32_t)a % c->n_bsizes];
+}
+
 static void step_single(orc_env* e, const orc_mlp* m, int mode, int32_t ext, orc_step_out* o) {
   const orc_config* c = &e->c;
   int frozen = e->status != 0;
   orc_env_observe(e, o->obs);
   int32_t a = choose_action(e, m, mode, ext, o->obs, o);
-  uint32_t k = (uint32_t)a / c->n_bsizes;
-  uint32_t b = c->bsizes[(uint32_t)a % c->n_bsizes];
+  uint32_t k, b;
+  decode_action(c, a, &k, &b);
   uint32_t now = e->now;
   uint32_t n = 0;
   uint64_t W = 0, csum = 0;
@@ -799,8 +820,8 @@ static void step_route(orc_env* e, const orc_mlp* m, int mode, int32_t ext, orc_
   int frozen = e->status != 0;
   orc_env_observe(e, o->obs);
   int32_t a = choose_action(e, m, mode, ext, o->obs, o);
-  uint32_t k = (uint32_t)a / c->n_bsizes;
-  uint32_t b = c->bsizes[(uint32_t)a % c->n_bsizes];
+  uint32_t k, b;
+  decode_action(c, a, &k, &b);
   uint32_t A = e->pend_time;
   e->step_n = 0;
   e->step_w[0] = e->step_w[1] = 0;

@@ -53,6 +53,7 @@ typedef struct {
   uint32_t phase_period_us;
   uint32_t dwell_kind;                      /* 0 exponential dwell, 1 fixed dwell (square wave) */
   uint32_t srv_speed16[ORC_MAX_SERVERS];    /* batch time factor of each server, in 1/16 (0: 16) */
+  uint32_t action_layout;                   /* 0: major x table index; 1: Wait + sizes 1..n */
 } orc_config;
 
 /* Host-memory MLP (row-major W[l] of dims[l+1] x dims[l]). */

@@ -39,7 +39,8 @@ simx_status cuda_fail(cudaError_t e, const char* what) {
 bool pow2(uint32_t x) { return x && !(x & (x - 1)); }
 
 uint32_t n_actions_of(const simx_config& c) {
-  return (c.mode == SIMX_MODE_SINGLE ? c.n_types : c.n_servers) * c.n_bsizes;
+  return (c.mode == SIMX_MODE_SINGLE ? c.n_types : c.n_servers) * c.n_bsizes +
+         (c.action_layout == 1 ? 1u : 0u);
 }
 
 uint32_t obs_dim_of(const simx_config& c) {
@@ -87,9 +88,15 @@ simx_status validate_config(const simx_config* c) {
     if (!finite_pos(c->cost_scale_us)) return fail(SIMX_EINVAL, "cost_scale_us must be > 0");
     if (c->cost_kind == 0 && !finite_pos(c->pareto_inv_alpha)) return fail(SIMX_EINVAL, "pareto_inv_alpha must be > 0");
   }
-  if (c->n_bsizes < 1 || c->n_bsizes > SIMX_MAX_BSIZES) return fail(SIMX_EINVAL, "n_bsizes %u", c->n_bsizes);
-  for (uint32_t i = 0; i < c->n_bsizes; ++i)
-    if (c->bsizes[i] < 1) return fail(SIMX_EINVAL, "bsizes[%u] must be >= 1", i);
+  if (c->action_layout > 1) return fail(SIMX_EINVAL, "action_layout %u", c->action_layout);
+  if (c->action_layout == 1) {  // Wait + batch sizes 1 .. n_bsizes (no table)
+    if (c->mode != SIMX_MODE_SINGLE) return fail(SIMX_EINVAL, "the Wait action layout is single-server only");
+    if (c->n_bsizes < 1 || c->n_bsizes > 64) return fail(SIMX_EINVAL, "n_bsizes %u (1 .. 64 with the Wait layout)", c->n_bsizes);
+  } else {
+    if (c->n_bsizes < 1 || c->n_bsizes > SIMX_MAX_BSIZES) return fail(SIMX_EINVAL, "n_bsizes %u", c->n_bsizes);
+    for (uint32_t i = 0; i < c->n_bsizes; ++i)
+      if (c->bsizes[i] < 1) return fail(SIMX_EINVAL, "bsizes[%u] must be >= 1", i);
+  }
   if (c->static_bi >= c->n_bsizes) return fail(SIMX_EINVAL, "static_bi %u >= n_bsizes", c->static_bi);
   if (n_actions_of(*c) > 255) return fail(SIMX_EINVAL, "more than 255 actions");
   if (c->obs_dim != obs_dim_of(*c)) return fail(SIMX_EINVAL, "obs_dim %u != %u implied by the configuration", c->obs_dim, obs_dim_of(*c));

@@ -92,6 +92,25 @@ __device__ __forceinline__ uint64_t service_us(const simx_config& c, uint32_t k,
   return (L * s + 8u) >> 4;
 }
 
+// Action a -> (major, batch size) (Sec. 4.1): layout 0, major a / n_bsizes and batch
+// bsizes[a % n_bsizes]; layout 1, a = 0 is Wait (batch 0) and a >= 1 is major
+// (a - 1) / n_bsizes with batch ((a - 1) % n_bsizes) + 1.
+__device__ __forceinline__ void decode_action(const simx_config& c, uint32_t a, uint32_t& major,
+                                              uint32_t& b) {
+  if (c.action_layout == 1) {
+    major = a == 0u ? 0u : (a - 1u) / c.n_bsizes;
+    b = a == 0u ? 0u : (a - 1u) % c.n_bsizes + 1u;
+  } else {
+    major = a / c.n_bsizes;
+    b = c.bsizes[a % c.n_bsizes];
+  }
+}
+
+// Initial per-server batch size: the static one.
+__device__ __forceinline__ uint32_t static_bsize(const simx_config& c) {
+  return c.action_layout == 1 ? c.static_bi + 1u : c.bsizes[c.static_bi];
+}
+
 // Time of the modulating chain's switch number i, given switch i-1 at t: an exponential
 // dwell drawn from the SWITCH stream, or the fixed dwell of a square wave.
 __device__ __forceinline__ uint32_t switch_time(const RolloutArgs& A, uint32_t env, uint32_t i,
@@ -586,7 +605,7 @@ __device__ int baseline_action(const RolloutArgs& A, const Grp<G>& g, uint32_t e
     } else if (L.qc[0] == 0 && c.n_types > 1 && L.qc[1] > 0) {
       h = 1u;
     }
-    return (int)(h * c.n_bsizes + c.static_bi);
+    return (int)((c.action_layout == 1 ? 1u : 0u) + h * c.n_bsizes + c.static_bi);
   }
   if (mode == SIMX_POLICY_RR) return (int)((s.tg % c.n_servers) * c.n_bsizes + c.static_bi);
   // SQ: server with the fewest queued requests (first such)
@@ -666,8 +685,8 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
       a = baseline_action<G, ROUTE>(A, g, env, s, L, ringb);
     }
     __syncwarp();
-    const uint32_t k = (uint32_t)a / c.n_bsizes;
-    const uint32_t b = c.bsizes[(uint32_t)a % c.n_bsizes];
+    uint32_t k, b;
+    decode_action(c, (uint32_t)a, k, b);
     const bool frozen = s.status != 0;
     const uint32_t now = ROUTE ? s.pt : s.now;
     uint32_t n_step = 0, qafter = 0;
@@ -855,7 +874,7 @@ __global__ void __launch_bounds__(kMaxThreads) k_reset(const __grid_constant__ R
   }
   if (c.arrival_kind == SIMX_ARR_DIURNAL)
     s.epo = (uint32_t)(((uint64_t)(w.y >> 8) * c.diurnal_len) >> 24);
-  Srv L{0u, c.bsizes[c.static_bi], Pair{0u, 0u}, Pair{0u, 0u}};
+  Srv L{0u, static_bsize(c), Pair{0u, 0u}, Pair{0u, 0u}};
   __syncwarp(g.mask);
   if (ROUTE) {
     next_arrival<G>(A, g, env, s);

@@ -325,7 +325,7 @@ __device__ int t_action(const Ctx& x, TEnv<K>& s) {
     const uint32_t cap = c.queue_cap;
     if (s.qc0[0] > 0u && c.n_types > 1 && s.qc1[0] > 0u) h = x.ring[cap + s.qh1[0]] < x.ring[s.qh0[0]] ? 1u : 0u;
     else if (s.qc0[0] == 0u && c.n_types > 1 && s.qc1[0] > 0u) h = 1u;
-    return (int)(h * c.n_bsizes + c.static_bi);
+    return (int)((c.action_layout == 1 ? 1u : 0u) + h * c.n_bsizes + c.static_bi);
   }
   if (mode == SIMX_POLICY_RR) return (int)((s.tg % c.n_servers) * c.n_bsizes + c.static_bi);
   int best = 0;
@@ -398,8 +398,14 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
   for (int t = 0; t < A.H; ++t) {
     if (A.obs) t_observe<ROUTE, K>(x, s, A.obs + (int64_t)t * A.obs_dim * A.ld + env, A.ld);
     const int a = t_action<ROUTE, K>(x, s);
-    const uint32_t kk = (uint32_t)a / c.n_bsizes;
-    const uint32_t b = c.bsizes[(uint32_t)a % c.n_bsizes];
+    uint32_t kk, b;
+    if (c.action_layout == 1) {  // a = 0: Wait (batch 0); a >= 1: type, batch 1 .. n_bsizes
+      kk = a == 0 ? 0u : (uint32_t)(a - 1) / c.n_bsizes;
+      b = a == 0 ? 0u : (uint32_t)(a - 1) % c.n_bsizes + 1u;
+    } else {
+      kk = (uint32_t)a / c.n_bsizes;
+      b = c.bsizes[(uint32_t)a % c.n_bsizes];
+    }
     const bool frozen = s.status != 0;
     const uint32_t now = ROUTE ? s.pt : s.now;
     uint32_t n_step = 0, qafter;

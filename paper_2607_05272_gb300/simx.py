@@ -45,6 +45,7 @@ class Config(C.Structure):
         ("obs_dim", C.c_uint32), ("t_window_us", C.c_float), ("rate_scale", C.c_float),
         ("rate_ref", C.c_float), ("busy_norm_us", C.c_float), ("phase_period_us", C.c_uint32),
         ("dwell_kind", C.c_uint32), ("srv_speed16", C.c_uint32 * 8),
+        ("action_layout", C.c_uint32),
     ]
 
 

@@ -30,7 +30,7 @@ import math
 
 import numpy as np
 
-ABI_VERSION = 2
+ABI_VERSION = 3
 MODE_SINGLE, MODE_ROUTE = 0, 1
 ARR_THINNED, ARR_DIURNAL = 0, 1
 POLICY = {"sample": 0, "argmax": 1, "static": 2, "rr": 3, "sq": 4, "random": 5, "external": 6}
@@ -48,7 +48,7 @@ CONFIG_FIELDS = [
     ("n_bsizes", "u32"), ("bsizes", "u32[8]"), ("static_bi", "u32"), ("obs_extra", "u32"),
     ("obs_dim", "u32"), ("t_window_us", "f32"), ("rate_scale", "f32"), ("rate_ref", "f32"),
     ("busy_norm_us", "f32"), ("phase_period_us", "u32"), ("dwell_kind", "u32"),
-    ("srv_speed16", "u32[8]"),
+    ("srv_speed16", "u32[8]"), ("action_layout", "u32"),
 ]
 
 
@@ -77,6 +77,7 @@ def _base(**kw) -> dict:
         w_wait=[0.001, 0.0], n_bsizes=6, bsizes=[1, 2, 4, 8, 16, 32, 0, 0], static_bi=3,
         obs_extra=0, obs_dim=8, t_window_us=10000.0, rate_scale=1250.0, rate_ref=800.0,
         busy_norm_us=100000.0, phase_period_us=0, dwell_kind=0, srv_speed16=[0] * 8,
+        action_layout=0,
     )
     c.update(kw)
     return c
@@ -163,7 +164,21 @@ def c3h(n_envs: int = 16384) -> dict:
     return c
 
 
-CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5, "burst": burst, "c3h": c3h}
+def c1w(n_envs: int = 64) -> dict:
+    """c1 with the paper's action space (Sec. 4.1): action 0 waits, actions 1..32 dispatch
+    a batch of that size (33 actions)."""
+    return _base(n_envs=n_envs, action_layout=1, n_bsizes=32, static_bi=7)
+
+
+def c2w(n_envs: int = 4096) -> dict:
+    """c2 with Wait plus (type, batch size 1..32): 65 actions (Sec. 4.1)."""
+    c = c2(n_envs)
+    c.update(action_layout=1, n_bsizes=32, static_bi=7)
+    return c
+
+
+CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5, "burst": burst, "c3h": c3h,
+           "c1w": c1w, "c2w": c2w}
 
 # Policy network shapes (input, hidden..., actions) and whether a value row follows.
 MLP_SHAPES = {
@@ -174,11 +189,14 @@ MLP_SHAPES = {
     "c5": ([13, 128, 128, 16], True),
     "burst": ([8, 32, 6], False),
     "c3h": ([13, 128, 128, 16], True),
+    "c1w": ([8, 32, 33], False),
+    "c2w": ([16, 64, 64, 65], False),
 }
 
-HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024, "burst": 2000, "c3h": 256}
+HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024, "burst": 2000, "c3h": 256,
+           "c1w": 2000, "c2w": 512}
 SEED = {name: 0x5EED0000 + i + 1
-        for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h"])}
+        for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h", "c1w", "c2w"])}
 
 
 def mlp_dims(name: str) -> tuple:

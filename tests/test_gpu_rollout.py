@@ -72,6 +72,8 @@ CASES = [
     ("c5", lambda: W.c5(40), 1024, "argmax"),
     ("burst", lambda: W.burst(37), 2000, "sample"),  # square-wave arrivals (fixed dwell)
     ("c3h", lambda: W.c3h(45), 256, "sample"),        # heterogeneous server speeds
+    ("c1w", lambda: W.c1w(33), 2000, "sample"),       # Wait + batch 1..32: 33 actions
+    ("c2w", lambda: W.c2w(37), 512, "sample"),        # Wait + (type, batch 1..32): 65
 ]
 
 
@@ -105,6 +107,8 @@ BASELINES = [
     ("burst", lambda: W.burst(35), 2000, "static"),
     ("c3h", lambda: W.c3h(41), 256, "sq"),
     ("c3h", lambda: W.c3h(39), 256, "rr"),
+    ("c2w", lambda: W.c2w(34), 512, "static"),
+    ("c1w", lambda: W.c1w(30), 2000, "random"),
 ]
 
 
@@ -159,12 +163,13 @@ def test_step_batched_equals_rollout(name, mk):
 
 
 @pytest.mark.parametrize("name,mk", [("c1", lambda: W.c1(9)), ("c2", lambda: W.c2(17)),
-                                     ("c3", lambda: W.c3(19)), ("c4", lambda: W.c4(11))])
+                                     ("c3", lambda: W.c3(19)), ("c4", lambda: W.c4(11)),
+                                     ("c2w", lambda: W.c2w(15))])
 def test_external_actions_match_oracle(name, mk):
     simx = _simx()
     cfg = mk()
     E, H = cfg["n_envs"], 60
-    A = (cfg["n_types"] if cfg["mode"] == 0 else cfg["n_servers"]) * cfg["n_bsizes"]
+    A = (cfg["n_types"] if cfg["mode"] == 0 else cfg["n_servers"]) * cfg["n_bsizes"] + cfg["action_layout"]
     rng = np.random.default_rng(5)
     acts = rng.integers(0, A, size=(H, E)).astype(np.int32)
     sim = simx.Sim(cfg)

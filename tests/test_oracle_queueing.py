@@ -289,3 +289,40 @@ def test_server_speed_latency_from_traces():
             assert tr[t + 1, 0, e] == tr[t, 0, e] + (L * 21 + 8) // 16
             checked += 1
     assert checked > 100
+
+
+def test_wait_action_layout_hand_scenario():
+    """c1w (Sec. 4.1 action space): from queue [1000, 3000, 9000, 9500] at t = 10,000 us,
+    action 0 waits (nothing dispatched, reward 0, queue kept, next decision later), and
+    action 3 dispatches a batch of 3 (waits 9000 + 7000 + 1000 us)."""
+    cfg = W.c1w(1)
+    def state():
+        s = np.zeros(oracle.OracleEnv(cfg, 0, 5).SW, np.uint32)
+        s[0] = 10000
+        s[2], s[3] = 5, 10000
+        s[5] = 0xFFFFFFFF
+        s[21] = 0xFFFFFFFF
+        s[23] = np.float32(800.0).view(np.uint32)
+        s[19] = 8000
+        s[33] = 8
+        s[34] = 4
+        s[35:39] = [1000, 3000, 9000, 9500]
+        s[12], s[14] = 4, 0
+        return s
+    e = oracle.OracleEnv(cfg, 0, 5)
+    e.reset()
+    e.load(state())
+    o = e.step(EXTERNAL, None, action=0)
+    assert o["trace"][1] == 0 and o["reward"] == 0.0
+    s2 = e.export()
+    assert s2[14] == 0                                   # nothing dispatched
+    assert s2[0] > 10000                                 # the next decision is at an arrival
+    assert list(s2[35:39]) == [1000, 3000, 9000, 9500]   # the queue is kept, in order
+    e2 = oracle.OracleEnv(cfg, 0, 5)
+    e2.reset()
+    e2.load(state())
+    o2 = e2.step(EXTERNAL, None, action=3)
+    assert o2["trace"][:3] == [10000, 3, 9000 + 7000 + 1000]
+    s3 = e2.export()
+    assert s3[32] == 10000 + 2000 + 100 * 3
+    assert list(s3[35:36]) == [9500]
