@@ -44,7 +44,7 @@ def _args():
     p.add_argument("--no-hbm-step", action="store_true")
     p.add_argument("--sweep", action="store_true",
                    help="every configuration (c1-c5, c5 at every env count): one JSON line each")
-    p.add_argument("--sweep-configs", default="c1,c2,c3,c4,c5",
+    p.add_argument("--sweep-configs", default="c1,c2,c3,c4,c5,c1p",
                    help="comma-separated subset of the sweep's configurations")
     p.add_argument("--sweep-child", default=None, help=argparse.SUPPRESS)
     p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
@@ -149,10 +149,11 @@ def _sweep_child(spec: str):
     E, env0, n, H = int(E), int(env0), int(n), int(H)
     cfg = W.CONFIGS[name](E)
     dims, hv = W.mlp_dims(name)
-    Ws, bs = W.mlp_weights(dims, 1)
+    Ws, bs = W.policy_weights(name, dims, 1)
     mode = 1 if name == "c5" else 0
     t0 = time.perf_counter()
-    oracle.rollout(cfg, (Ws, bs, hv), W.SEED[name], mode, list(range(env0, env0 + n)), H)
+    oracle.rollout(cfg, (Ws, bs, hv, W.mlp_acts(name)), W.SEED[name], mode,
+                   list(range(env0, env0 + n)), H)
     print(json.dumps({"seconds": time.perf_counter() - t0, "env_steps": n * H}))
 
 
@@ -229,7 +230,7 @@ def run_sweep(a) -> None:
     print(json.dumps({"fp32_fma_probe_tflops": fp["tflops"], "sms": fp["sms"], "hbm_gbs": hbm,
                       "hbm_source": src}), flush=True)
     cases = [("c1", 64, 10000, "sample"), ("c2", 4096, 512, "sample"), ("c3", 16384, 256, "sample"),
-             ("c4", 65536, 512, "sample")]
+             ("c4", 65536, 512, "sample"), ("c1p", 4096, 2000, "sample")]
     cases += [("c5", e, 1024, "argmax") for e in (1024, 4096, 16384, 65536, 262144, 1048576)]
     keep = set(a.sweep_configs.split(","))
     cases = [c for c in cases if c[0] in keep]
@@ -237,9 +238,9 @@ def run_sweep(a) -> None:
     for name, E, H, mode in cases:
         cfg = W.CONFIGS[name](E)
         dims, hv = W.mlp_dims(name)
-        Ws, bs = W.mlp_weights(dims, 1)
+        Ws, bs = W.policy_weights(name, dims, 1)
         pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws],
-                          [torch.from_numpy(b).cuda() for b in bs], hv)
+                          [torch.from_numpy(b).cuda() for b in bs], hv, W.mlp_acts(name))
         sim = simx.Sim(cfg)
         sim.reset(W.SEED[name])
         warm = simx.alloc_rollout(E, sim.D, 4, has_value=hv)

@@ -38,11 +38,11 @@
 extern "C" {
 #endif
 
-#define SIMX_ABI_VERSION 3u
+#define SIMX_ABI_VERSION 4u
 #define SIMX_MAX_TYPES 2
 #define SIMX_MAX_SERVERS 8
 #define SIMX_MAX_BSIZES 8
-#define SIMX_MAX_LAYERS 4
+#define SIMX_MAX_LAYERS 6
 #define SIMX_MAX_WIDTH 256      /* widest hidden layer */
 #define SIMX_MAX_OUT 257        /* widest output layer: actions + value row */
 #define SIMX_MAX_OBS 64
@@ -155,12 +155,21 @@ typedef struct simx_config {
                                   1 + T * n_bsizes (33 for T = 1, 65 for T = 2 at n_bsizes 32) */
 } simx_config;
 
+/* Activation after a hidden layer (simx_mlp.act). */
+typedef enum { SIMX_ACT_TANH = 0, SIMX_ACT_IDENTITY = 1, SIMX_ACT_GELU = 2 } simx_act;
+
 /*
- * Policy network (Sec. 4.2): a tanh MLP.  Layer l maps dims[l] -> dims[l+1] with
+ * Policy network (Sec. 4.2): an MLP.  Layer l maps dims[l] -> dims[l+1] with
  * z_j = (sum_k W_l[j][k] x_k, accumulated in fp32 by fused multiply-adds in k order
- * from k = 0) + b_l[j]; hidden layers apply tanh.  The last layer has n_actions rows
- * followed by one value row when has_value (the value head of Sec. 4.2 sharing the
- * trunk).  W_l is row-major [dims[l+1]][dims[l]] fp32, device memory.
+ * from k = 0) + b_l[j]; every layer but the last applies act[l]: tanh (the default, 0),
+ * identity, or GELU in its tanh form, 0.5 z (1 + tanh(c (z + 0.044715 z^3))),
+ * c = sqrt(2/pi), evaluated as u = fma(0.044715, (z*z)*z, z), t = tanh(c*u),
+ * (0.5*z)*(1 + t) with the library's deterministic tanh.  The last layer has n_actions
+ * rows followed by one value row when has_value.  The paper's network (projection,
+ * 2-head attention over its single token, GELU policy and value heads) is such an MLP:
+ * attention over one token is a linear map, and separate heads are one hidden layer with
+ * zero blocks in the output layer.  W_l is row-major [dims[l+1]][dims[l]] fp32, device
+ * memory.
  */
 typedef struct simx_mlp {
   int32_t n_layers;                     /* 1 .. SIMX_MAX_LAYERS */
@@ -168,6 +177,7 @@ typedef struct simx_mlp {
   const float* W[SIMX_MAX_LAYERS];
   const float* b[SIMX_MAX_LAYERS];
   int32_t has_value;
+  int32_t act[SIMX_MAX_LAYERS];         /* simx_act after layer l < n_layers - 1 */
 } simx_mlp;
 
 /* Rollout buffer (device memory, caller-owned).  ld >= n_envs is the env stride. */
@@ -293,7 +303,8 @@ simx_status returns_baseline(const float* d_x, int64_t n, float* d_adv_out, floa
  *   both     : + c_value mean((V - ret)^2) (value row only) - c_entropy mean(H[pi]).
  * d_grad [n_params] fp32 is overwritten with dL/dtheta in the order W0,b0,W1,b1,...;
  * d_stats [5] = {L, policy term, mean (V-ret)^2, mean entropy, clip fraction}.
- * d_workspace must hold ppo_loss_grad_workspace_size(pol, n) bytes.
+ * d_workspace must hold ppo_loss_grad_workspace_size(pol, n) bytes (the size depends on
+ * pol's layer widths and activations, not on its weights).
  */
 size_t ppo_loss_grad_workspace_size(const simx_mlp* pol, int64_t n);
 simx_status ppo_loss_grad(const simx_mlp* pol, const simx_rollout* buf, int64_t n_rows_per_step,

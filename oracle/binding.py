@@ -12,6 +12,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "oracle.c")
 _HDR = os.path.join(_HERE, "oracle.h")
 _SO = os.path.join(_HERE, "_build", "liboracle.so")
+MAX_LAYERS = 6  # ORC_MAX_LAYERS
 _lock = threading.Lock()
 _lib = None
 
@@ -53,8 +54,9 @@ class OrcConfig(C.Structure):
 
 
 class OrcMlp(C.Structure):
-    _fields_ = [("n_layers", C.c_int32), ("dims", C.c_int32 * 5),
-                ("W", C.c_void_p * 4), ("b", C.c_void_p * 4), ("has_value", C.c_int32)]
+    _fields_ = [("n_layers", C.c_int32), ("dims", C.c_int32 * (MAX_LAYERS + 1)),
+                ("W", C.c_void_p * MAX_LAYERS), ("b", C.c_void_p * MAX_LAYERS),
+                ("has_value", C.c_int32), ("act", C.c_int32 * MAX_LAYERS)]
 
 
 class OrcStepOut(C.Structure):
@@ -118,7 +120,7 @@ def make_config(cfg: dict) -> OrcConfig:
 class _Mlp:
     """Keeps the numpy weight arrays alive while the C struct points at them."""
 
-    def __init__(self, Ws, bs, has_value):
+    def __init__(self, Ws, bs, has_value, acts=None):
         self.Ws = [np.ascontiguousarray(w, dtype=np.float32) for w in Ws]
         self.bs = [np.ascontiguousarray(b, dtype=np.float32) for b in bs]
         m = OrcMlp()
@@ -129,14 +131,16 @@ class _Mlp:
             m.W[l] = w.ctypes.data
             m.b[l] = self.bs[l].ctypes.data
         m.has_value = int(bool(has_value))
+        for l, a in enumerate(acts or []):
+            m.act[l] = {"tanh": 0, "identity": 1, "gelu": 2}.get(a, a)
         self.c = m
 
 
 def _mlp(mlp):
     if mlp is None:
         return None, None
-    Ws, bs, hv = mlp
-    m = _Mlp(Ws, bs, hv)
+    Ws, bs, hv = mlp[:3]
+    m = _Mlp(Ws, bs, hv, mlp[3] if len(mlp) > 3 else None)
     return m, C.byref(m.c)
 
 
@@ -153,10 +157,10 @@ def philox(ctr, key) -> np.ndarray:
 
 
 def map_fn(fn: str, x) -> np.ndarray:
-    """Apply detlog / detexp / dettanh / detcos2pi to an fp32 array."""
+    """Apply detlog / detexp / dettanh / detcos2pi / detgelu to an fp32 array."""
     x = np.ascontiguousarray(x, dtype=np.float32)
     y = np.empty_like(x)
-    code = {"log": 0, "exp": 1, "tanh": 2, "cos2pi": 3}[fn]
+    code = {"log": 0, "exp": 1, "tanh": 2, "cos2pi": 3, "gelu": 4}[fn]
     lib().orc_map(code, x.ctypes.data, y.ctypes.data, x.size)
     return y
 

@@ -157,6 +157,16 @@ float orc_dettanh(float z) {
   return copysignf(t, z);
 }
 
+/* GELU in its tanh form (Sec. 4.2 policy head): 0.5 x (1 + tanh(c (x + a x^3))),
+   c = sqrt(2/pi), a = 0.044715, in this order: u = fma(a, (x*x)*x, x), t = tanh(c*u),
+   (0.5*x) * (1 + t). */
+float orc_detgelu(float x) {
+  float x3 = (x * x) * x;
+  float u = fmaf(0.044715f, x3, x);
+  float t = orc_dettanh(0.7978845608028654f * u);
+  return (0.5f * x) * (1.0f + t);
+}
+
 /* cos(2 pi u) for u in [0, 1): quadrant from 4u, reflection to [0, pi/4],
    Taylor series of sin to theta^11 and of cos to theta^12. */
 float orc_detcos2pi(float u) {
@@ -657,7 +667,13 @@ void orc_policy(const orc_mlp* m, const float* obs, int mode, uint64_t seed, uin
       float acc = 0.0f;
       for (int k = 0; k < K; ++k) acc = fmaf(W[(size_t)j * K + k], x[k], acc);
       float z = acc + m->b[l][j];
-      y[j] = (l + 1 < m->n_layers) ? orc_dettanh(z) : z;
+      if (l + 1 < m->n_layers) {
+        if (m->act[l] == 1) y[j] = z;
+        else if (m->act[l] == 2) y[j] = orc_detgelu(z);
+        else y[j] = orc_dettanh(z);
+      } else {
+        y[j] = z;
+      }
     }
     x = y;
     y = (y == bufa) ? bufb : bufa;
@@ -1015,6 +1031,7 @@ void orc_map(int fn, const float* x, float* y, int64_t n) {
       case 0: y[i] = orc_detlog(x[i]); break;
       case 1: y[i] = orc_detexp(x[i]); break;
       case 2: y[i] = orc_dettanh(x[i]); break;
+      case 4: y[i] = orc_detgelu(x[i]); break;
       default: y[i] = orc_detcos2pi(x[i]); break;
     }
   }

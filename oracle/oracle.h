@@ -15,7 +15,7 @@
 #define ORC_MAX_TYPES 2
 #define ORC_MAX_SERVERS 8
 #define ORC_MAX_BSIZES 8
-#define ORC_MAX_LAYERS 4
+#define ORC_MAX_LAYERS 6
 #define ORC_DIURNAL_MAX 128
 #define ORC_HEADER_WORDS 32
 
@@ -63,6 +63,7 @@ typedef struct {
   const float* W[ORC_MAX_LAYERS];
   const float* b[ORC_MAX_LAYERS];
   int32_t has_value;
+  int32_t act[ORC_MAX_LAYERS];   /* after layer l < n_layers - 1: 0 tanh, 1 identity, 2 GELU */
 } orc_mlp;
 
 typedef struct orc_env orc_env;
@@ -85,6 +86,7 @@ void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t ou
 float orc_detlog(float x);
 float orc_detexp(float x);
 float orc_dettanh(float x);
+float orc_detgelu(float x);
 float orc_detcos2pi(float u);
 float orc_normal(uint32_t w0, uint32_t w1);
 uint32_t orc_duration(float x);

@@ -8,6 +8,8 @@ of the tanh MLP for the gradients.
 """
 from __future__ import annotations
 
+import math
+
 import numpy as np
 
 REINFORCE, PPO = 0, 1
@@ -52,20 +54,54 @@ def baseline(x):
     return x - m, m
 
 
-def forward(Ws, bs, X):
-    """tanh MLP forward in fp64; returns the list of layer inputs and the last layer's output."""
+TANH, IDENTITY, GELU = 0, 1, 2
+ACT_NAMES = {"tanh": TANH, "identity": IDENTITY, "gelu": GELU}
+GELU_C, GELU_A = math.sqrt(2.0 / math.pi), 0.044715
+
+
+def act_fn(kind, z):
+    """Hidden-layer activation (Sec. 4.2): tanh, identity, or GELU in its tanh form
+    0.5 z (1 + tanh(sqrt(2/pi) (z + 0.044715 z^3))); kind is a code or a name."""
+    kind = ACT_NAMES.get(kind, kind)
+    if kind == IDENTITY:
+        return z
+    if kind == GELU:
+        return 0.5 * z * (1.0 + np.tanh(GELU_C * (z + GELU_A * z ** 3)))
+    return np.tanh(z)
+
+
+def act_grad(kind, z):
+    """d act / d z."""
+    kind = ACT_NAMES.get(kind, kind)
+    if kind == IDENTITY:
+        return np.ones_like(z)
+    if kind == GELU:
+        t = np.tanh(GELU_C * (z + GELU_A * z ** 3))
+        return 0.5 * (1.0 + t) + 0.5 * z * (1.0 - t * t) * GELU_C * (1.0 + 3.0 * GELU_A * z * z)
+    return 1.0 - np.tanh(z) ** 2
+
+
+def _forward(Ws, bs, X, acts=None):
     h = np.asarray(X, np.float64)
-    inputs = []
+    inputs, zs = [], []
     L = len(Ws)
     for l in range(L):
         inputs.append(h)
         z = h @ np.asarray(Ws[l], np.float64).T + np.asarray(bs[l], np.float64)
-        h = np.tanh(z) if l + 1 < L else z
+        zs.append(z)
+        h = act_fn(acts[l] if acts else TANH, z) if l + 1 < L else z
+    return inputs, zs, h
+
+
+def forward(Ws, bs, X, acts=None):
+    """MLP forward in fp64 (tanh hidden layers unless acts says otherwise); returns the
+    list of layer inputs and the last layer's output."""
+    inputs, _, h = _forward(Ws, bs, X, acts)
     return inputs, h
 
 
 def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=0.2,
-              c_value=0.5, c_entropy=0.01):
+              c_value=0.5, c_entropy=0.01, acts=None):
     """Loss, statistics and the gradient with respect to every W_l, b_l (fp64).
 
     pi = softmax(logits); policy term REINFORCE -mean(adv log pi(a)) or PPO
@@ -73,7 +109,7 @@ def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=
     plus c_value mean((V - ret)^2) when a value row exists, minus c_entropy mean(H[pi]).
     Returns (grads [(gW, gb) per layer], stats [L, pg, v, H, clipfrac]).
     """
-    inputs, Z = forward(Ws, bs, X)
+    inputs, zs, Z = _forward(Ws, bs, X, acts)
     n = Z.shape[0]
     A = Z.shape[1] - (1 if has_value else 0)
     logits = Z[:, :A]
@@ -118,7 +154,7 @@ def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=
         grads[l] = (dz.T @ h_in, dz.sum(axis=0))
         if l > 0:
             dh = dz @ np.asarray(Ws[l], np.float64)
-            dz = dh * (1.0 - h_in ** 2)
+            dz = dh * act_grad(acts[l - 1] if acts else TANH, zs[l - 1])
     stats = np.array([loss, pg, vloss, H.mean(), clipfrac])
     return grads, stats
 

@@ -133,6 +133,8 @@ simx_status validate_mlp(const simx_mlp* m, uint32_t obs_dim, uint32_t n_actions
   if (n_actions && (uint32_t)A != n_actions) return fail(SIMX_EINVAL, "policy has %d actions, environment %u", A, n_actions);
   for (int l = 0; l < m->n_layers; ++l)
     if (!m->W[l] || !m->b[l]) return fail(SIMX_EINVAL, "layer %d weights are NULL", l);
+  for (int l = 0; l + 1 < m->n_layers; ++l)
+    if (m->act[l] < SIMX_ACT_TANH || m->act[l] > SIMX_ACT_GELU) return fail(SIMX_EINVAL, "act[%d] = %d", l, m->act[l]);
   return SIMX_OK;
 }
 
@@ -168,6 +170,7 @@ simx_status pack_mlp(const simx_mlp* m, Packed& P, DevMlp& out, cudaStream_t s) 
     if (e != cudaSuccess) return cuda_fail(e, "repack");
     out.Wt[l] = Wt;
     out.bias[l] = bias;
+    out.act[l] = (l + 1 < m->n_layers) ? m->act[l] : -1;  // -1: no activation (output layer)
     p = bias + npad[l + 1];
   }
   for (int l = 0; l <= m->n_layers; ++l) {
@@ -541,6 +544,7 @@ static simx_status loss_args(const simx_mlp* pol, const simx_rollout* buf, int64
   for (int l = 0; l < pol->n_layers; ++l) {
     a.W[l] = pol->W[l];
     a.b[l] = pol->b[l];
+    a.act[l] = (l + 1 < pol->n_layers) ? pol->act[l] : -1;
   }
   a.n_actions = pol->dims[pol->n_layers] - a.has_value;
   a.obs = buf->obs;
@@ -567,6 +571,7 @@ size_t ppo_loss_grad_workspace_size(const simx_mlp* pol, int64_t n) {
   std::memset(&a, 0, sizeof(a));
   a.n_layers = pol->n_layers;
   for (int l = 0; l <= pol->n_layers; ++l) a.dims[l] = pol->dims[l];
+  for (int l = 0; l < pol->n_layers; ++l) a.act[l] = (l + 1 < pol->n_layers) ? pol->act[l] : -1;
   a.n = n;
   return loss_workspace_bytes(a);
 }

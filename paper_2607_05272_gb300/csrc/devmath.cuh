@@ -122,6 +122,25 @@ __device__ __forceinline__ float det_tanh(float z) {
   return copysignf(t, z);
 }
 
+// GELU in its tanh form: 0.5 x (1 + tanh(c (x + 0.044715 x^3))), c = sqrt(2/pi), as
+// u = fma(0.044715, (x*x)*x, x), t = tanh(c*u), (0.5*x)*(1 + t).
+__device__ __forceinline__ float det_gelu(float x) {
+  const float x3 = __fmul_rn(__fmul_rn(x, x), x);
+  const float u = __fmaf_rn(0.044715f, x3, x);
+  const float t = det_tanh(__fmul_rn(0.7978845608028654f, u));
+  return __fmul_rn(__fmul_rn(0.5f, x), __fadd_rn(1.0f, t));
+}
+
+// GELU of x into g (the same operations as det_gelu) and its derivative
+// 0.5 (1 + t) + 0.5 x (1 - t^2) c (1 + 3 a x^2), t = tanh(c (x + a x^3)), into d.
+__device__ __forceinline__ void det_gelu_grad(float x, float& g, float& d) {
+  const float c = 0.7978845608028654f, a = 0.044715f;
+  const float u = __fmaf_rn(a, __fmul_rn(__fmul_rn(x, x), x), x);
+  const float t = det_tanh(__fmul_rn(c, u));
+  d = 0.5f * (1.0f + t) + 0.5f * x * (1.0f - t * t) * c * (1.0f + 3.0f * a * x * x);
+  g = __fmul_rn(__fmul_rn(0.5f, x), __fadd_rn(1.0f, t));
+}
+
 // cos(2 pi u), u in [0, 1): quadrant of 4u, reflection to [0, pi/4], Taylor series.
 __device__ __forceinline__ float det_cos2pi(float u) {
   const float v = __fmul_rn(u, 4.0f);

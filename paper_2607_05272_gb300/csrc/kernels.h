@@ -93,6 +93,7 @@ struct LossArgs {
   float* grad;           // flat gradient
   float* stats;          // [5]
   int precision;         // SIMX_PREC_FP32 (SIMT) or SIMX_PREC_TF32 (tensor cores where it fits)
+  int act[SIMX_MAX_LAYERS];  // simx_act after layer l, -1 for the output layer
 };
 size_t loss_workspace_bytes(const LossArgs& a);
 // loss_fused.cu

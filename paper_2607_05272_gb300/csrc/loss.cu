@@ -3,7 +3,7 @@
 //
 // Pipeline (fp32, deterministic for a given launch configuration):
 //   1. gather the minibatch observations X [n][D] from the [T][D][E] buffer;
-//   2. forward GEMMs H_l = tanh(H_{l-1} W_l^T + b_l), keeping every activation;
+//   2. forward GEMMs H_l = act_l(H_{l-1} W_l^T + b_l), keeping every activation;
 //   3. loss head per row: log-softmax, rho, clipped surrogate, entropy, value
 //      residual -> dL/dZ of the last layer and per-block fp64 statistics;
 //   4. backward per layer: dW_l = dZ_l^T H_{l-1} (split over rows, partial tiles
@@ -19,7 +19,10 @@
 namespace simx {
 
 constexpr int kBM = 64, kBN = 64, kBK = 16, kGemmThreads = 256;
-enum Epi : int { EPI_NONE = 0, EPI_BIAS = 1, EPI_BIAS_TANH = 2, EPI_DTANH = 3 };
+// EPI_BIAS_ACT: + bias, then the activation `act` (0 tanh, 1 identity, 2 GELU, which also
+// writes its derivative to D); EPI_DACT: times the derivative of `act` (1 - H^2 for tanh,
+// D for GELU, 1 for identity).
+enum Epi : int { EPI_NONE = 0, EPI_BIAS = 1, EPI_BIAS_ACT = 2, EPI_DACT = 3 };
 
 struct Gemm {
   const float* A;  // A(i, k) = A[i * sai + k * sak]
@@ -32,8 +35,10 @@ struct Gemm {
   int64_t k_per_split;
   int64_t split_stride;
   const float* bias;  // [N]
-  const float* H;     // EPI_DTANH: multiply by (1 - H(i, j)^2), H(i, j) = H[i * ldc + j]
+  const float* H;     // EPI_DACT, tanh: multiply by (1 - H(i, j)^2), H(i, j) = H[i * ldc + j]
+  float* D;           // GELU derivative, D(i, j) = D[i * ldc + j]: written by EPI_BIAS_ACT, read by EPI_DACT
   int epi;
+  int act;
 };
 
 __global__ void __launch_bounds__(kGemmThreads) k_gemm(const __grid_constant__ Gemm g) {
@@ -98,11 +103,18 @@ __global__ void __launch_bounds__(kGemmThreads) k_gemm(const __grid_constant__ G
       const int64_t j = j0 + tx + 16 * b;
       if (j >= g.N) continue;
       float v = acc[a][b];
-      if (g.epi == EPI_BIAS || g.epi == EPI_BIAS_TANH) v = __fadd_rn(v, g.bias[j]);
-      if (g.epi == EPI_BIAS_TANH) v = det_tanh(v);
-      if (g.epi == EPI_DTANH) {
-        const float h = g.H[i * g.ldc + j];
-        v = v * (1.0f - h * h);
+      if (g.epi == EPI_BIAS || g.epi == EPI_BIAS_ACT) v = __fadd_rn(v, g.bias[j]);
+      if (g.epi == EPI_BIAS_ACT) {
+        if (g.act == 0) v = det_tanh(v);
+        else if (g.act == 2) det_gelu_grad(v, v, g.D[i * g.ldc + j]);
+      }
+      if (g.epi == EPI_DACT) {
+        if (g.act == 0) {
+          const float h = g.H[i * g.ldc + j];
+          v = v * (1.0f - h * h);
+        } else if (g.act == 2) {
+          v = v * g.D[i * g.ldc + j];
+        }
       }
       C[i * g.ldc + j] = v;
     }
@@ -243,7 +255,7 @@ __global__ void k_colsum(const float* __restrict__ dZ, int64_t n, int N, int64_t
 }
 
 struct WsLayout {
-  size_t X, H[SIMX_MAX_LAYERS], Z, part, statp, total;
+  size_t X, H[SIMX_MAX_LAYERS], Dg[SIMX_MAX_LAYERS], Z, part, statp, total;
   int splits, head_blocks;
 };
 
@@ -265,6 +277,8 @@ static WsLayout layout(const LossArgs& a) {
   const int64_t n = a.n;
   w.X = take((size_t)n * a.dims[0] * sizeof(float));
   for (int l = 1; l < a.n_layers; ++l) w.H[l] = take((size_t)n * a.dims[l] * sizeof(float));
+  for (int l = 1; l < a.n_layers; ++l)  // GELU derivative of layer l's input
+    w.Dg[l] = a.act[l - 1] == 2 ? take((size_t)n * a.dims[l] * sizeof(float)) : 0;
   w.Z = take((size_t)n * a.dims[a.n_layers] * sizeof(float));
   w.splits = dw_splits(n);
   size_t maxw = 0;
@@ -300,7 +314,11 @@ cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
   float* X = reinterpret_cast<float*>(base + w.X);
   float* Hs[SIMX_MAX_LAYERS + 1];
   Hs[0] = X;
-  for (int l = 1; l < L; ++l) Hs[l] = reinterpret_cast<float*>(base + w.H[l]);
+  float* Dg[SIMX_MAX_LAYERS + 1] = {};
+  for (int l = 1; l < L; ++l) {
+    Hs[l] = reinterpret_cast<float*>(base + w.H[l]);
+    if (a.act[l - 1] == 2) Dg[l] = reinterpret_cast<float*>(base + w.Dg[l]);
+  }
   float* Z = reinterpret_cast<float*>(base + w.Z);
   float* part = reinterpret_cast<float*>(base + w.part);
   double* statp = reinterpret_cast<double*>(base + w.statp);
@@ -328,7 +346,9 @@ cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
     g.k_per_split = K;
     g.split_stride = 0;
     g.bias = a.b[l];
-    g.epi = (l + 1 < L) ? EPI_BIAS_TANH : EPI_BIAS;
+    g.epi = (l + 1 < L) ? EPI_BIAS_ACT : EPI_BIAS;
+    g.act = a.act[l];
+    g.D = (l + 1 < L) ? Dg[l + 1] : nullptr;
     cudaError_t e = gemm(g, 1, s);
     if (e != cudaSuccess) return e;
   }
@@ -379,7 +399,7 @@ cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
     k_reduce_splits<<<(unsigned)((N + 255) / 256), 256, 0, s>>>(bpart, splits, N, gb);
     count_launches(3);
     if (l > 0) {
-      // dZ of layer l-1 = (dZ W) * (1 - H^2) with H = Hs[l] (layer l's input), in place
+      // dZ of layer l-1 = (dZ W) * act'(Z_{l-1}) (1 - H^2 for tanh, H = Hs[l]), in place
       Gemm d{};
       d.A = dZ;  // A(i, k) = dZ[i][k], k over N
       d.sai = N;
@@ -395,7 +415,9 @@ cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
       d.k_per_split = N;
       d.split_stride = 0;
       d.H = Hs[l];
-      d.epi = EPI_DTANH;
+      d.D = Dg[l];
+      d.act = a.act[l - 1];
+      d.epi = EPI_DACT;
       e = gemm(d, 1, s);
       if (e != cudaSuccess) return e;
       dZ = Hs[l];

@@ -30,12 +30,15 @@ constexpr int kLThreads = 256;         // threads per block
 // Wt is row-major with row stride ldw (a multiple of 4, 16-byte aligned).  Each
 // thread owns TE rows x 4 outputs: 4-row tiles when they give every thread a tile,
 // else 1-row tiles (thin layers such as the logits).
-// epi 0: + bias, tanh when do_tanh; epi 1: * (1 - H[j][r]^2).
+// epi 0: + bias, then the activation `act` (-1 none, 0 tanh, 1 identity, 2 GELU; for
+// GELU its derivative is written to D as well); epi 1: times the derivative of the
+// activation `act` of H's layer: 1 - H^2 (tanh, H = the activations), 1 (identity), or
+// H itself (GELU: H = the stored derivative).
 template <int R, int TE>
 __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ldw, int K, int N,
                                             const float* X, float* Y, int epi,
-                                            const float* __restrict__ bias, bool do_tanh,
-                                            const float* H) {
+                                            const float* __restrict__ bias, int act,
+                                            const float* H, float* D) {
   constexpr int kLld = R + 4;
   const int neb = R / TE, nob = (N + 3) / 4;
   for (int tile = threadIdx.x; tile < neb * nob; tile += blockDim.x) {
@@ -82,16 +85,22 @@ __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ld
           v.y = __fadd_rn(v.y, bj);
           v.z = __fadd_rn(v.z, bj);
           v.w = __fadd_rn(v.w, bj);
-        } else {
+        } else if (act == 0) {
           const float4 h = *reinterpret_cast<const float4*>(H + j * kLld + 4 * eb);
           v.x = v.x * (1.0f - h.x * h.x);
           v.y = v.y * (1.0f - h.y * h.y);
           v.z = v.z * (1.0f - h.z * h.z);
           v.w = v.w * (1.0f - h.w * h.w);
+        } else if (act == 2) {
+          const float4 dd = *reinterpret_cast<const float4*>(H + j * kLld + 4 * eb);
+          v.x = v.x * dd.x;
+          v.y = v.y * dd.y;
+          v.z = v.z * dd.z;
+          v.w = v.w * dd.w;
         }
         *reinterpret_cast<float4*>(Y + j * kLld + 4 * eb) = v;
       }
-      if (epi == 0 && do_tanh) {  // one det_tanh per output, four rows at a time
+      if (epi == 0 && act == 0) {  // one det_tanh per output, four rows at a time
 #pragma unroll 1
         for (int o = 0; o < 4; ++o) {
           const int j = 4 * ob + o;
@@ -105,6 +114,15 @@ __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ld
             *y = v;
           }
         }
+      } else if (epi == 0 && act == 2) {  // GELU and its derivative, four rows at a time
+#pragma unroll 1
+        for (int q = 0; q < 16; ++q) {
+          const int j = 4 * ob + q / 4;
+          if (j < N) {
+            float* y = Y + j * kLld + 4 * eb + q % 4;
+            det_gelu_grad(*y, *y, D[j * kLld + 4 * eb + q % 4]);
+          }
+        }
       }
     } else {
 #pragma unroll
@@ -114,17 +132,22 @@ __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ld
         float v = acc[0][o];
         if (epi == 0) {
           v = __fadd_rn(v, bias[j]);
-        } else {
+        } else if (act == 0) {
           const float h = H[j * kLld + eb];
           v = v * (1.0f - h * h);
+        } else if (act == 2) {
+          v = v * H[j * kLld + eb];
         }
         Y[j * kLld + eb] = v;
       }
-      if (epi == 0 && do_tanh) {
+      if (epi == 0 && (act == 0 || act == 2)) {
 #pragma unroll 1
         for (int o = 0; o < 4; ++o) {
           const int j = 4 * ob + o;
-          if (j < N) Y[j * kLld + eb] = det_tanh(Y[j * kLld + eb]);
+          if (j < N) {
+            if (act == 0) Y[j * kLld + eb] = det_tanh(Y[j * kLld + eb]);
+            else det_gelu_grad(Y[j * kLld + eb], Y[j * kLld + eb], D[j * kLld + eb]);
+          }
         }
       }
     }
@@ -134,12 +157,12 @@ __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ld
 template <int R>
 __device__ __forceinline__ void tile_gemm(const float* __restrict__ Wt, int ldw, int K, int N,
                                           const float* X, float* Y, int epi,
-                                          const float* __restrict__ bias, bool do_tanh,
-                                          const float* H) {
+                                          const float* __restrict__ bias, int act,
+                                          const float* H, float* D) {
   if ((R / 4) * ((N + 3) / 4) >= kLThreads)
-    tile_gemm_t<R, 4>(Wt, ldw, K, N, X, Y, epi, bias, do_tanh, H);
+    tile_gemm_t<R, 4>(Wt, ldw, K, N, X, Y, epi, bias, act, H, D);
   else
-    tile_gemm_t<R, 1>(Wt, ldw, K, N, X, Y, epi, bias, do_tanh, H);
+    tile_gemm_t<R, 1>(Wt, ldw, K, N, X, Y, epi, bias, act, H, D);
 }
 
 // Row splits for a reduction over the R rows of a tile shared by `items`
@@ -231,6 +254,7 @@ struct FusedLossArgs {
   int npad[SIMX_MAX_LAYERS + 1];     // Npad per layer output (index l + 1)
   int kpad[SIMX_MAX_LAYERS + 1];     // Kpad per layer input (index l)
   int act_off[SIMX_MAX_LAYERS + 2];  // row offset of each layer's activation buffer
+  int dact_off[SIMX_MAX_LAYERS + 1]; // row offset of the GELU derivative of layer l's input (-1: none)
   int dz_rows;                       // rows of each dZ buffer
   int poff[SIMX_MAX_LAYERS];         // offset of layer l's dW in the flat gradient
   int n_params;
@@ -278,7 +302,8 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
     for (int l = 0; l < L; ++l) {
       tile_gemm<R>(F.Wt[l], F.npad[l + 1], a.dims[l], a.dims[l + 1],
                    acts + (size_t)F.act_off[l] * kLld, acts + (size_t)F.act_off[l + 1] * kLld, 0,
-                   a.b[l], l + 1 < L, nullptr);
+                   a.b[l], a.act[l], nullptr,
+                   F.dact_off[l + 1] >= 0 ? acts + (size_t)F.dact_off[l + 1] * kLld : nullptr);
       __syncthreads();
     }
     // loss head: kLanes lanes per row (R rows x kLanes = 256 threads); lane q takes
@@ -385,7 +410,9 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
       if (l > 0) {
         float* dzn = (dz == dzA) ? dzB : dzA;
         // dZ_{l-1}[k][r] = sum_j W_l[j][k] dZ_l[j][r] * (1 - H_l[k][r]^2)
-        tile_gemm<R>(F.Wn[l], F.kpad[l], N, K, dz, dzn, 1, nullptr, false, Hl);
+        const int pa = a.act[l - 1];  // activation whose derivative applies
+        tile_gemm<R>(F.Wn[l], F.kpad[l], N, K, dz, dzn, 1, nullptr, pa,
+                     pa == 2 ? acts + (size_t)F.dact_off[l] * kLld : Hl, nullptr);
         __syncthreads();
         dz = dzn;
       } else {
@@ -453,6 +480,7 @@ struct FusedPlan {
   bool ok;
   int R;
   int npad[SIMX_MAX_LAYERS + 1], kpad[SIMX_MAX_LAYERS + 1], act_off[SIMX_MAX_LAYERS + 2];
+  int dact_off[SIMX_MAX_LAYERS + 1];
   int dz_rows, poff[SIMX_MAX_LAYERS], n_params, grid;
   size_t smem, w_off[SIMX_MAX_LAYERS][2], part_off, spart_off, total;
 };
@@ -469,6 +497,13 @@ FusedPlan plan_r(const LossArgs& a, int R) {
     p.act_off[l] = rows;
     rows += r4(a.dims[l]);
     if (l > 0 && a.dims[l] > maxd) maxd = a.dims[l];
+  }
+  for (int l = 0; l <= L; ++l) {  // GELU derivative of layer l's input (output of l - 1)
+    p.dact_off[l] = -1;
+    if (l >= 1 && l < L && a.act[l - 1] == 2) {
+      p.dact_off[l] = rows;
+      rows += r4(a.dims[l]);
+    }
   }
   p.act_off[L + 1] = rows;
   p.dz_rows = r4(maxd);
@@ -537,6 +572,7 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
     F.act_off[l] = p.act_off[l];
   }
   F.act_off[a.n_layers + 1] = p.act_off[a.n_layers + 1];
+  for (int l = 0; l <= a.n_layers; ++l) F.dact_off[l] = p.dact_off[l];
   F.dz_rows = p.dz_rows;
   for (int l = 0; l < a.n_layers; ++l) F.poff[l] = p.poff[l];
   F.n_params = p.n_params;

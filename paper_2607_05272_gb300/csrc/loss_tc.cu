@@ -599,6 +599,8 @@ Plan plan(const LossArgs& a) {
   p.ok = false;
   const int L = a.n_layers;
   if (L < 1 || L > SIMX_MAX_LAYERS) return p;
+  for (int l = 0; l + 1 < L; ++l)
+    if (a.act[l] != 0) return p;  // the hidden layers' epilogues here are tanh only
   p.L = L;
   int P = 0, hr_w = 0, maxN = 0;
   for (int l = 0; l < L; ++l) {

@@ -42,6 +42,7 @@ struct DevMlp {
   int dims[SIMX_MAX_LAYERS + 1];
   int npad[SIMX_MAX_LAYERS + 1];
   int n_layers, has_value, n_actions;
+  int act[SIMX_MAX_LAYERS];  // simx_act after layer l, -1 for the output layer
 };
 
 template <int G>
@@ -104,10 +105,19 @@ struct Grp {
 // is still the fp32 chain acc = fma(W[j][k], x[k], acc) over k = 0..K-1 in order
 // from acc = 0, then + bias: the same bits as evaluating one env at a time.
 // ---------------------------------------------------------------------------
+// GELU over rows j0 .. min(j0 + 4, N) - 1, columns 0 .. te - 1 of Y.  Out of line: inlined,
+// its code inside the rollout kernel's loop slowed the tanh policies that never run it.
+static __device__ __noinline__ void gelu_tile(float* Y, int ld, int j0, int N, int te) {
+  for (int j = j0; j < j0 + 4 && j < N; ++j)
+    for (int e = 0; e < te; ++e) Y[j * ld + e] = det_gelu(Y[j * ld + e]);
+}
+
+// act: the activation after this layer: -1 none (output layer), 0 tanh, 1 identity,
+// 2 GELU (det_gelu).
 template <int TE>
 __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
                                           const float* __restrict__ bias, int K, int N, int Npad,
-                                          const float* X, float* Y, int B, int ld, bool do_tanh) {
+                                          const float* X, float* Y, int B, int ld, int act) {
   const int neb = B / TE, nob = (N + 3) / 4;
   const int ntiles = neb * nob;
   for (int tile = threadIdx.x; tile < ntiles; tile += blockDim.x) {
@@ -149,7 +159,8 @@ __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
         for (int e = 0; e < TE; ++e) Y[j * ld + TE * eb + e] = __fadd_rn(acc[e][o], bj);
       }
     }
-    if (do_tanh) {  // one det_tanh per output, over this thread's own tile
+    // one activation per output, over this thread's own tile
+    if (act == 0) {
 #pragma unroll 1
       for (int q = 0; q < 4 * TE; ++q) {
         const int j = 4 * ob + q / TE;
@@ -158,6 +169,8 @@ __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
           *y = det_tanh(*y);
         }
       }
+    } else if (act == 2) {
+      gelu_tile(Y + TE * eb, ld, 4 * ob, N, TE);
     }
   }
 }
@@ -172,7 +185,7 @@ __device__ __forceinline__ float* mlp_forward_block(const DevMlp& m, float* X0, 
   __syncthreads();
   for (int l = 0; l < m.n_layers; ++l) {
     const int K = m.dims[l], N = m.dims[l + 1], Np = m.npad[l + 1];
-    const bool th = l + 1 < m.n_layers;
+    const int th = m.act[l];
     // 4-env tiles when they keep every thread busy, otherwise 1-env tiles
     if ((B / 4) * ((N + 3) / 4) >= (int)blockDim.x) mlp_tiles<4>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th);
     else mlp_tiles<1>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th);

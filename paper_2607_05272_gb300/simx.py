@@ -20,6 +20,7 @@ OK, EINVAL, ENOMEM, ECUDA, EOVERFLOW, ESTATE = range(6)
 POLICY = {"sample": 0, "argmax": 1, "static": 2, "rr": 3, "sq": 4, "random": 5, "external": 6}
 ALGO = {"reinforce": 0, "ppo": 1}
 TRACE_WIDTH = 4
+MAX_LAYERS = 6  # SIMX_MAX_LAYERS
 STATE_HEADER_WORDS = 32
 
 
@@ -50,8 +51,12 @@ class Config(C.Structure):
 
 
 class Mlp(C.Structure):
-    _fields_ = [("n_layers", C.c_int32), ("dims", C.c_int32 * 5), ("W", C.c_void_p * 4),
-                ("b", C.c_void_p * 4), ("has_value", C.c_int32)]
+    _fields_ = [("n_layers", C.c_int32), ("dims", C.c_int32 * (MAX_LAYERS + 1)),
+                ("W", C.c_void_p * MAX_LAYERS), ("b", C.c_void_p * MAX_LAYERS),
+                ("has_value", C.c_int32), ("act", C.c_int32 * MAX_LAYERS)]
+
+
+ACT = {"tanh": 0, "identity": 1, "gelu": 2}
 
 
 class Rollout(C.Structure):
@@ -152,9 +157,11 @@ def _stream(stream=None):
 
 
 class Policy:
-    """A simx_mlp over device tensors W_l [out, in] and b_l [out] (fp32, contiguous)."""
+    """A simx_mlp over device tensors W_l [out, in] and b_l [out] (fp32, contiguous);
+    acts: the activation after each hidden layer ("tanh", "identity" or "gelu"; default
+    tanh)."""
 
-    def __init__(self, Ws, bs, has_value: bool):
+    def __init__(self, Ws, bs, has_value: bool, acts=None):
         self.Ws = [w.contiguous() for w in Ws]
         self.bs = [b.contiguous() for b in bs]
         self.has_value = bool(has_value)
@@ -167,6 +174,8 @@ class Policy:
             m.W[l] = w.data_ptr()
             m.b[l] = self.bs[l].data_ptr()
         m.has_value = int(self.has_value)
+        for l, a in enumerate(acts or []):
+            m.act[l] = ACT[a] if isinstance(a, str) else int(a)
         self.c = m
 
     @property

@@ -30,7 +30,7 @@ import math
 
 import numpy as np
 
-ABI_VERSION = 3
+ABI_VERSION = 4
 MODE_SINGLE, MODE_ROUTE = 0, 1
 ARR_THINNED, ARR_DIURNAL = 0, 1
 POLICY = {"sample": 0, "argmax": 1, "static": 2, "rr": 3, "sq": 4, "random": 5, "external": 6}
@@ -177,8 +177,14 @@ def c2w(n_envs: int = 4096) -> dict:
     return c
 
 
+def c1p(n_envs: int = 64) -> dict:
+    """c1w's env and action space, served by the paper's policy network (Sec. 4.2; the
+    network is described at ``PAPER_NET``)."""
+    return c1w(n_envs)
+
+
 CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5, "burst": burst, "c3h": c3h,
-           "c1w": c1w, "c2w": c2w}
+           "c1w": c1w, "c2w": c2w, "c1p": c1p}
 
 # Policy network shapes (input, hidden..., actions) and whether a value row follows.
 MLP_SHAPES = {
@@ -191,12 +197,26 @@ MLP_SHAPES = {
     "c3h": ([13, 128, 128, 16], True),
     "c1w": ([8, 32, 33], False),
     "c2w": ([16, 64, 64, 65], False),
+    "c1p": ([8, 4, 4, 4, 128, 33], True),
 }
 
+# The paper's network (Sec. 4.2) as a plain MLP.  The 8-dim state is projected to a
+# 4-dim embedding; self-attention (2 heads, embedding 4) then sees that single token, so
+# its softmax weight is 1 and it returns the output projection of the value projection:
+# two linear 4 -> 4 maps (query and key projections do not reach the output).  The
+# policy head (4 -> 64 GELU -> 33 logits) and the value head (4 -> 64 GELU -> 1) become
+# one 4 -> 128 GELU layer and a 128 -> 34 output layer whose logit rows read hidden
+# units 0..63 and whose value row reads 64..127; the other entries start at zero
+# (a trainer that keeps the heads separate leaves them there by masking their gradient).
+PAPER_NET = ("c1p",)
+
+# Activation after each hidden layer where it is not tanh (simx_act names).
+MLP_ACTS = {"c1p": ["identity", "identity", "identity", "gelu"]}
+
 HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024, "burst": 2000, "c3h": 256,
-           "c1w": 2000, "c2w": 512}
+           "c1w": 2000, "c2w": 512, "c1p": 2000}
 SEED = {name: 0x5EED0000 + i + 1
-        for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h", "c1w", "c2w"])}
+        for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h", "c1w", "c2w", "c1p"])}
 
 
 def mlp_dims(name: str) -> tuple:
@@ -214,6 +234,32 @@ def mlp_weights(dims, seed: int, sigma: float = 0.1):
     for k, n in zip(dims[:-1], dims[1:]):
         Ws.append((rng.standard_normal((n, k)) * sigma).astype(np.float32))
         bs.append(np.zeros(n, dtype=np.float32))
+    return Ws, bs
+
+
+def mlp_acts(name: str) -> list:
+    """The activation after each hidden layer of `name`'s policy."""
+    n_hidden = len(MLP_SHAPES[name][0]) - 2
+    return list(MLP_ACTS.get(name, ["tanh"] * n_hidden))
+
+
+def policy_weights(name: str, dims, seed: int):
+    """Initial fp32 weights and biases of `name`'s policy with layer widths `dims`.
+
+    Tanh policies: ``mlp_weights``.  The paper's network: N(0, 1 / (3 fan_in)) weights
+    (the spread of a uniform +-1/sqrt(fan_in) draw), small random biases, and the last
+    layer block-diagonal between the policy and value heads (the last hidden layer split
+    in halves)."""
+    if name not in PAPER_NET:
+        return mlp_weights(dims, seed)
+    rng = np.random.default_rng(seed)
+    Ws, bs = [], []
+    for k, n in zip(dims[:-1], dims[1:]):
+        Ws.append((rng.standard_normal((n, k)) / np.sqrt(3.0 * k)).astype(np.float32))
+        bs.append((rng.standard_normal(n) * 0.05).astype(np.float32))
+    half = dims[-2] // 2
+    Ws[-1][:-1, half:] = 0.0
+    Ws[-1][-1, :half] = 0.0
     return Ws, bs
 
 

@@ -101,18 +101,19 @@ def _rollout_for_loss(simx, name, E, H, hidden=None):
     dims, hv = W.mlp_dims(name)
     if hidden is not None:
         dims = [dims[0]] + [hidden] * (len(dims) - 2) + [dims[-1]]
-    Ws, bs = W.mlp_weights(dims, 21)
+    Ws, bs = W.policy_weights(name, dims, 21)
     bs = [(np.random.default_rng(l).standard_normal(b.shape) * 0.05).astype(np.float32)
           for l, b in enumerate(bs)]
+    acts = W.mlp_acts(name)
     pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws],
-                      [torch.from_numpy(b).cuda() for b in bs], hv)
+                      [torch.from_numpy(b).cuda() for b in bs], hv, acts)
     sim = simx.Sim(cfg)
     sim.reset(W.SEED[name])
     buf = simx.alloc_rollout(E, sim.D, H, has_value=hv)
     sim.rollout("sample", H, buf, pol)
     torch.cuda.synchronize()
     sim.close()
-    return cfg, pol, (Ws, bs, hv), buf
+    return cfg, pol, (Ws, bs, hv, acts), buf
 
 
 def _check_grad(g, g_ref, layers, tol=1e-5):
@@ -153,9 +154,9 @@ def _loss_case(simx, name, algo, E, H, nmb, precision="fp32", hidden=None):
     rows = np.arange(n_rows) if idx is None else idx
     X, a, lpo = rl.gather_rows(obs, act, logp, rows, E)
     t, e = rows // E, rows % E
-    Ws, bs, hv = host
+    Ws, bs, hv, acts = host
     grads, st = rl.loss_grad(Ws, bs, hv, X, a, lpo, adv[t, e], ret[t, e],
-                             rl.PPO if algo == "ppo" else rl.REINFORCE, 0.2, 0.5, 0.01)
+                             rl.PPO if algo == "ppo" else rl.REINFORCE, 0.2, 0.5, 0.01, acts)
     return grad.cpu().numpy().astype(np.float64), stats.cpu().numpy().astype(np.float64), \
         rl.flat(grads), st, list(zip(Ws, bs)), n
 
@@ -167,6 +168,8 @@ def _loss_case(simx, name, algo, E, H, nmb, precision="fp32", hidden=None):
     ("c1", "reinforce", 16, 700, 5000),
     ("c3", "ppo", 8, 64, 333),
     ("c2", "reinforce", 3, 7, None),
+    ("c1p", "reinforce", 40, 300, None),   # the paper's network: identity and GELU layers
+    ("c1p", "ppo", 17, 500, 4001),
 ])
 def test_loss_gradient_matches_oracle(name, algo, E, H, nmb):
     simx = _simx()
@@ -193,9 +196,24 @@ def test_tensor_core_loss_gradient_matches_oracle(name, algo, E, H, nmb, hidden)
     assert abs(s[4] - st[4]) <= 1.0 / n
 
 
-def test_tensor_core_request_falls_back_for_wide_policies():
-    """A policy too wide for the tensor-core kernel gives the FP32 path's exact bits."""
+@pytest.mark.parametrize("name,hidden", [("c3", None), ("c1p", None)])
+def test_tensor_core_request_falls_back(name, hidden):
+    """A policy the tensor-core kernel does not take (too wide, or with identity / GELU
+    layers) gives the FP32 path's exact bits."""
     simx = _simx()
-    a = _loss_case(simx, "c3", "ppo", 16, 64, 700, "tf32")
-    b = _loss_case(simx, "c3", "ppo", 16, 64, 700, "fp32")
+    a = _loss_case(simx, name, "ppo", 16, 64, 700, "tf32", hidden)
+    b = _loss_case(simx, name, "ppo", 16, 64, 700, "fp32", hidden)
     assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+@pytest.mark.parametrize("name,algo,E,H,nmb,hidden", [
+    ("c1p", "ppo", 24, 200, 3001, 256),     # 8-256-256-256-256-34: identity and GELU layers
+    ("c4", "reinforce", 9, 100, None, None),  # 28-256-256-49 tanh
+])
+def test_gemm_pipeline_loss_gradient_matches_oracle(name, algo, E, H, nmb, hidden):
+    """Policies too wide for the fused one-kernel path take the GEMM pipeline."""
+    simx = _simx()
+    g, s, g_ref, st, layers, n = _loss_case(simx, name, algo, E, H, nmb, "fp32", hidden)
+    _check_grad(g, g_ref, layers)
+    assert np.all(np.abs(s[:4] - st[:4]) <= 1e-5 * (np.abs(st[:4]) + 1.0))
+    assert abs(s[4] - st[4]) <= 1.0 / n

@@ -28,10 +28,11 @@ def _simx():
 
 def _policy(simx, name, seed=7):
     dims, hv = W.mlp_dims(name)
-    Ws, bs = W.mlp_weights(dims, seed)
+    Ws, bs = W.policy_weights(name, dims, seed)
+    acts = W.mlp_acts(name)
     pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws],
-                      [torch.from_numpy(b).cuda() for b in bs], hv)
-    return pol, (Ws, bs, hv)
+                      [torch.from_numpy(b).cuda() for b in bs], hv, acts)
+    return pol, (Ws, bs, hv, acts)
 
 
 def _run(name, cfg, H, mode, seed=None, trace=True):
@@ -74,6 +75,7 @@ CASES = [
     ("c3h", lambda: W.c3h(45), 256, "sample"),        # heterogeneous server speeds
     ("c1w", lambda: W.c1w(33), 2000, "sample"),       # Wait + batch 1..32: 33 actions
     ("c2w", lambda: W.c2w(37), 512, "sample"),        # Wait + (type, batch 1..32): 65
+    ("c1p", lambda: W.c1p(41), 2000, "sample"),       # the paper's network (GELU heads)
 ]
 
 
@@ -132,7 +134,7 @@ def test_single_env_and_zero_horizon():
 
 
 @pytest.mark.parametrize("name,mk", [("c2", lambda: W.c2(36)), ("c4", lambda: W.c4(13)),
-                                     ("c3h", lambda: W.c3h(17))])
+                                     ("c3h", lambda: W.c3h(17)), ("c1p", lambda: W.c1p(19))])
 def test_step_batched_equals_rollout(name, mk):
     """H single-step launches with the internal policy give the rollout's records."""
     simx = _simx()
@@ -241,7 +243,7 @@ def test_save_load_resume_is_bit_exact(name, mk, H):
 
 def test_policy_forward_matches_oracle():
     simx = _simx()
-    for name, mode in (("c3", "sample"), ("c4", "argmax"), ("c2", "sample")):
+    for name, mode in (("c3", "sample"), ("c4", "argmax"), ("c2", "sample"), ("c1p", "sample")):
         pol, host = _policy(simx, name, seed=3)
         D = host[0][0].shape[1]
         n = 77

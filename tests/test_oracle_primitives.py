@@ -86,6 +86,21 @@ def test_dettanh():
     assert oracle.dettanh(float(tiny)) == pytest.approx(float(tiny), rel=1e-6)
 
 
+def test_detgelu():
+    """GELU's tanh form against the same formula in fp64.  Bound: 8 eps relative, plus
+    eps |x| absolute: tanh's error (<= 4 ulp of |t| <= 1) and the rounding of 1 + t,
+    scaled by 0.5 |x|, which dominate where 1 + t cancels (x well below 0)."""
+    x = np.linspace(-12.0, 12.0, 1 << 21).astype(np.float32)
+    y = oracle.map_fn("gelu", x).astype(np.float64)
+    xd = x.astype(np.float64)
+    ref = 0.5 * xd * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (xd + 0.044715 * xd ** 3)))
+    eps = 2.0 ** -23
+    assert np.all(np.abs(y - ref) <= 8.0 * eps * np.abs(ref) + eps * np.abs(xd))
+    assert oracle.map_fn("gelu", np.zeros(1, np.float32))[0] == 0.0
+    big = x > 6.0
+    assert np.array_equal(y[big], xd[big])     # tanh saturates at 1: gelu(x) = x exactly
+
+
 def test_detcos2pi_all_inputs():
     j = np.arange(1 << 24, dtype=np.float64)
     u = (j * 2.0 ** -24).astype(np.float32)
@@ -199,3 +214,27 @@ def test_policy_mlp_against_fp64():
         tol = 1e-5 * (np.abs(h) + mag)
         assert np.all(np.abs(lg - h[:A]) <= tol[:A])
         assert abs(v - h[A]) <= tol[A]
+
+
+@pytest.mark.parametrize("acts", [(1, 2, 1), (2, 0, 2)])
+def test_policy_mlp_activations_against_fp64(acts):
+    """The oracle's fp32 policy with identity (1) / GELU (2) / tanh (0) hidden layers
+    against an fp64 evaluation of the same network (the paper's projection, attention
+    over one token and GELU head are such layers)."""
+    from oracle import rl
+    dims = [8, 4, 4, 64, 7]
+    rng = np.random.default_rng(8)
+    Ws = [(rng.standard_normal((n, k)) * 0.4).astype(np.float32) for k, n in zip(dims[:-1], dims[1:])]
+    bs = [(rng.standard_normal(n) * 0.1).astype(np.float32) for n in dims[1:]]
+    for i in range(50):
+        obs = (rng.standard_normal(dims[0]) * 2.0).astype(np.float32)
+        lg, v, a, lp = oracle.policy((Ws, bs, True, list(acts)), obs, 0, 1, i, 0)
+        h = obs.astype(np.float64)
+        for l in range(len(Ws)):
+            Wd = Ws[l].astype(np.float64)
+            z = Wd @ h + bs[l]
+            mag = np.abs(Wd) @ np.abs(h) + np.abs(bs[l])
+            h = rl.act_fn(acts[l], z) if l + 1 < len(Ws) else z
+        tol = 1e-4 * (np.abs(h) + mag)
+        assert np.all(np.abs(lg - h[:6]) <= tol[:6])
+        assert abs(v - h[6]) <= tol[6]

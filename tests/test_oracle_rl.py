@@ -104,14 +104,16 @@ def _tiny(has_value, seed=0, dims=(5, 7, 6, 4)):
     return Ws, bs, X, a, adv, ret, logp_old
 
 
-def _torch_loss(Ws, bs, has_value, X, a, logp_old, adv, ret, algo, eps, cv, ce):
+def _torch_loss(Ws, bs, has_value, X, a, logp_old, adv, ret, algo, eps, cv, ce, acts=None):
     torch = pytest.importorskip("torch")
     tW = [torch.tensor(w, dtype=torch.float64, requires_grad=True) for w in Ws]
     tb = [torch.tensor(b, dtype=torch.float64, requires_grad=True) for b in bs]
     h = torch.tensor(X, dtype=torch.float64)
+    fns = {rl.TANH: torch.tanh, rl.IDENTITY: lambda z: z,
+           rl.GELU: lambda z: torch.nn.functional.gelu(z, approximate="tanh")}
     for l in range(len(Ws)):
         z = h @ tW[l].T + tb[l]
-        h = torch.tanh(z) if l + 1 < len(Ws) else z
+        h = fns[acts[l] if acts else rl.TANH](z) if l + 1 < len(Ws) else z
     A = h.shape[1] - (1 if has_value else 0)
     logpi = torch.log_softmax(h[:, :A], dim=1)
     lpa = logpi[torch.arange(len(a)), torch.tensor(a)]
@@ -135,6 +137,20 @@ def test_loss_grad_matches_autograd(algo, has_value):
     Ws, bs, X, a, adv, ret, lpo = _tiny(has_value, seed=algo * 2 + has_value)
     grads, stats = rl.loss_grad(Ws, bs, has_value, X, a, lpo, adv, ret, algo, 0.2, 0.5, 0.01)
     L, tg = _torch_loss(Ws, bs, has_value, X, a, lpo, adv, ret, algo, 0.2, 0.5, 0.01)
+    assert stats[0] == pytest.approx(L, rel=1e-12, abs=1e-12)
+    for (gW, gb), (tW, tb) in zip(grads, tg):
+        assert np.allclose(gW, tW, rtol=1e-10, atol=1e-12)
+        assert np.allclose(gb, tb, rtol=1e-10, atol=1e-12)
+
+
+@pytest.mark.parametrize("acts", [(rl.IDENTITY, rl.GELU), (rl.GELU, rl.TANH), (rl.GELU, rl.GELU)])
+def test_loss_grad_with_activations_matches_autograd(acts):
+    """Identity and GELU hidden layers (the paper's network shape) against PyTorch autograd
+    with its own tanh-form GELU."""
+    Ws, bs, X, a, adv, ret, lpo = _tiny(True, seed=11)
+    grads, stats = rl.loss_grad(Ws, bs, True, X, a, lpo, adv, ret, rl.PPO, 0.2, 0.5, 0.01,
+                                acts=list(acts))
+    L, tg = _torch_loss(Ws, bs, True, X, a, lpo, adv, ret, rl.PPO, 0.2, 0.5, 0.01, acts=list(acts))
     assert stats[0] == pytest.approx(L, rel=1e-12, abs=1e-12)
     for (gW, gb), (tW, tb) in zip(grads, tg):
         assert np.allclose(gW, tW, rtol=1e-10, atol=1e-12)
