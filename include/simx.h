@@ -76,8 +76,11 @@ typedef enum {
 typedef enum {
   SIMX_ARR_THINNED = 0,  /* Poisson candidate stream thinned by a 1- or 2-state modulating
                             chain: Poisson when n_mod_states = 1, MMPP when 2            */
-  SIMX_ARR_DIURNAL = 1   /* piecewise-constant rate per epoch: diurnal table x lognormal
-                            burst factor; stands in for the trace replay of Sec. 3.2      */
+  SIMX_ARR_DIURNAL = 1,  /* piecewise-constant rate per epoch: diurnal table x lognormal
+                            burst factor; a synthetic stand-in for a trace               */
+  SIMX_ARR_TRACE = 2     /* trace replay (Sec. 3.2 real-world traces): as THINNED, but the
+                            gap before candidate j, and optionally its type and cost,
+                            come from entry j mod n of the trace given by sim_set_trace  */
 } simx_arrival_kind;
 
 /* Action selection (Sec. 4.2 stochastic policy; Sec. 5.1 baselines). */
@@ -233,8 +236,31 @@ uint64_t simx_state_words(const simx_config* cfg);
 simx_status sim_create(const simx_config* cfg, int device, simx_ctx** out);
 void sim_destroy(simx_ctx* ctx);
 
+/*
+ * Trace replay input (Sec. 3.2: the paper replays Azure Functions and BurstGPT traces;
+ * no trace ships with this library, the caller supplies one in this format).
+ *   d_gap_us [n]  : gap in integer us between request i - 1 and request i of the trace
+ *                   (absolute timestamps t_i give gap_i = t_i - t_{i-1}; gap_0 is the
+ *                   gap taken when the replay wraps from entry n - 1 back to entry 0);
+ *   d_type [n]    : request type (values >= n_types count as n_types - 1), or NULL to
+ *                   draw types as THINNED does (type0_thr);
+ *   d_cost_us [n] : per-request cost in us for requests of cfg.cost_type, or NULL to
+ *                   draw costs as THINNED does (cost_kind, cost_scale_us).
+ * Env e replays the trace from entry o_e = floor(u * n / 2^32), u the third word of its
+ * INIT draw, so envs see different windows of one trace; candidate j of an env uses
+ * entry j mod n with its candidate counter starting at o_e (32-bit, wrapping).  The
+ * thinning and the modulating chain of THINNED still apply on top (accept_thr[s] =
+ * 2^24 keeps every entry).  Arrays are device memory owned by the caller and must stay
+ * valid while the context uses them; the call records the pointers and copies nothing.
+ * Required before sim_reset when cfg.arrival_kind == SIMX_ARR_TRACE, refused (EINVAL)
+ * for other arrival kinds; 1 <= n < 2^31.  A new trace takes effect at the next reset.
+ */
+simx_status sim_set_trace(simx_ctx* ctx, const uint32_t* d_gap_us, const uint8_t* d_type,
+                          const uint32_t* d_cost_us, uint32_t n);
+
 /* Reset every env to time 0 with empty queues and idle servers, keyed by `seed`
-   (Philox key), and advance each to its first decision point. */
+   (Philox key), and advance each to its first decision point.  SIMX_ESTATE for a
+   TRACE context without a trace. */
 simx_status sim_reset(simx_ctx* ctx, uint64_t seed, void* stream);
 
 /* Write the current observation of every env to d_obs [obs_dim][ld]. */

@@ -50,7 +50,11 @@ class OrcConfig(C.Structure):
         ("rate_ref", C.c_float), ("busy_norm_us", C.c_float), ("phase_period_us", C.c_uint32),
         ("dwell_kind", C.c_uint32), ("srv_speed16", C.c_uint32 * 8),
         ("action_layout", C.c_uint32),
+        ("trace_gap", C.c_void_p), ("trace_type", C.c_void_p), ("trace_cost", C.c_void_p),
+        ("trace_len", C.c_uint32),
     ]
+
+_TRACE_FIELDS = ("trace_gap", "trace_type", "trace_cost", "trace_len")
 
 
 class OrcMlp(C.Structure):
@@ -105,8 +109,22 @@ def lib():
 
 
 def make_config(cfg: dict) -> OrcConfig:
+    """cfg: the library's configuration fields, plus for trace replay ``trace`` =
+    (gap_us, type or None, cost_us or None) arrays, kept alive by the returned struct."""
     c = OrcConfig()
+    tr = cfg.get("trace")
+    if tr is not None:
+        gap = np.ascontiguousarray(tr[0], dtype=np.uint32)
+        typ = None if tr[1] is None else np.ascontiguousarray(tr[1], dtype=np.uint8)
+        cst = None if tr[2] is None else np.ascontiguousarray(tr[2], dtype=np.uint32)
+        c._keep = (gap, typ, cst)
+        c.trace_gap = gap.ctypes.data
+        c.trace_type = None if typ is None else typ.ctypes.data
+        c.trace_cost = None if cst is None else cst.ctypes.data
+        c.trace_len = len(gap)
     for name, _ in OrcConfig._fields_:
+        if name in _TRACE_FIELDS:
+            continue
         v = cfg[name]
         if isinstance(v, (list, tuple)):
             arr = getattr(c, name)

@@ -329,11 +329,20 @@ static uint32_t head_type(orc_env* e, uint32_t k) {
 
 /* Request type from word w1 and, for the cost type, its per-request cost from
    word w3 with E ~ Exp(1): Pareto by inversion, cost = round(x_m exp(E / alpha));
-   exponential, cost = round(mean E). */
-static void request_attrs(const orc_env* e, const uint32_t w[4], uint32_t* type, uint32_t* cost) {
+   exponential, cost = round(mean E).  Under trace replay, candidate j takes the type
+   (clamped to the last type) and the cost of trace entry j mod n where the trace has
+   them. */
+static void request_attrs(const orc_env* e, uint32_t j, const uint32_t w[4], uint32_t* type,
+                          uint32_t* cost) {
   uint32_t t = (e->T > 1 && (w[1] >> 8) >= e->c.type0_thr) ? 1u : 0u;
+  if (e->c.trace_type) {
+    t = e->c.trace_type[j % e->c.trace_len];
+    if (t >= e->T) t = e->T - 1u;
+  }
   uint32_t cst = 0;
-  if ((int32_t)t == e->c.cost_type) {
+  if ((int32_t)t == e->c.cost_type && e->c.trace_cost) {
+    cst = e->c.trace_cost[j % e->c.trace_len];
+  } else if ((int32_t)t == e->c.cost_type) {
     float E = expo1(w[3]);
     if (e->c.cost_kind == 0) {
       float y = e->c.pareto_inv_alpha * E;
@@ -368,9 +377,11 @@ static void process_switches(orc_env* e, uint32_t limit) {
   }
 }
 
-/* Time of candidate j given the previous candidate's time. */
+/* Time of candidate j given the previous candidate's time: a drawn exponential gap,
+   or under trace replay the gap of trace entry j mod n. */
 static uint32_t cand_time(orc_env* e, uint32_t j, uint32_t base, uint32_t w[4]) {
   draw(e, j, ORC_STREAM_ARRIVAL, w);
+  if (e->c.arrival_kind == ORC_ARR_TRACE) return add_time(e, base, e->c.trace_gap[j % e->c.trace_len]);
   return add_time(e, base, orc_duration(e->c.cand_mean_gap_us * expo1(w[0])));
 }
 
@@ -384,7 +395,7 @@ static int accepted(const orc_env* e, const uint32_t w[4]) {
 static int consume_single(orc_env* e, const uint32_t w[4], uint32_t T) {
   if (!accepted(e, w)) return 0;
   uint32_t type, cost;
-  request_attrs(e, w, &type, &cost);
+  request_attrs(e, e->cand_j, w, &type, &cost);
   e->n_arrived += 1;
   e->narr_since[type] += 1;
   if (e->qcnt[0][type] < e->cap) {
@@ -435,14 +446,15 @@ static void next_arrival(orc_env* e) {
   for (;;) {
     if (count_event(e)) return;
     uint32_t w[4];
-    if (e->c.arrival_kind == ORC_ARR_THINNED) {
-      uint32_t T = cand_time(e, e->cand_j, e->cand_T, w);
+    if (e->c.arrival_kind != ORC_ARR_DIURNAL) { /* THINNED or TRACE */
+      uint32_t j = e->cand_j;
+      uint32_t T = cand_time(e, j, e->cand_T, w);
       process_switches(e, T);
       int acc = accepted(e, w);
       e->cand_j += 1;
       e->cand_T = T;
       if (!acc) continue;
-      request_attrs(e, w, &e->pend_type, &e->pend_cost);
+      request_attrs(e, j, w, &e->pend_type, &e->pend_cost);
       e->pend_time = T;
       e->n_arrived += 1;
       return;
@@ -461,7 +473,7 @@ static void next_arrival(orc_env* e) {
     uint64_t end = (uint64_t)(e->epoch + 1u) * (uint64_t)e->c.epoch_us;
     if ((uint64_t)e->cand_T + g < end) {
       e->cand_T = add_time(e, e->cand_T, g);
-      request_attrs(e, w, &e->pend_type, &e->pend_cost);
+      request_attrs(e, 0, w, &e->pend_type, &e->pend_cost);
       e->pend_time = e->cand_T;
       e->n_arrived += 1;
       return;
@@ -597,6 +609,8 @@ void orc_env_reset(orc_env* e) {
   }
   if (c.arrival_kind == ORC_ARR_DIURNAL)
     e->epoch_off = (uint32_t)(((uint64_t)(w[1] >> 8) * c.diurnal_len) >> 24);
+  if (c.arrival_kind == ORC_ARR_TRACE) /* this env's first trace entry: floor(u n / 2^32) */
+    e->cand_j = (uint32_t)(((uint64_t)w[2] * c.trace_len) >> 32);
   if (c.mode == ORC_SINGLE) {
     jump_single(e);
   } else {
@@ -1056,6 +1070,8 @@ void orc_samplers(const orc_config* c, int kind, float scale, const uint32_t* w,
   orc_env e;
   memset(&e, 0, sizeof(e));
   e.c = *c;
+  e.c.trace_type = NULL;
+  e.c.trace_cost = NULL;
   e.T = c->n_types;
   for (int64_t i = 0; i < n; ++i) {
     const uint32_t* q = w + 4 * i;
@@ -1064,10 +1080,10 @@ void orc_samplers(const orc_config* c, int kind, float scale, const uint32_t* w,
       case 0: out[i] = expo1(q[0]); break;
       case 1: out[i] = (float)orc_duration(scale * expo1(q[0])); break;
       case 2: out[i] = orc_normal(q[0], q[1]); break;
-      case 3: request_attrs(&e, q, &t, &cost); out[i] = (float)t; break;
+      case 3: request_attrs(&e, 0, q, &t, &cost); out[i] = (float)t; break;
       default: {
         uint32_t qq[4] = {q[0], (uint32_t)c->cost_type == 1u ? 0xFFFFFFFFu : 0u, q[2], q[3]};
-        request_attrs(&e, qq, &t, &cost);
+        request_attrs(&e, 0, qq, &t, &cost);
         out[i] = (float)cost;
       }
     }

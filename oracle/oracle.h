@@ -20,7 +20,7 @@
 #define ORC_HEADER_WORDS 32
 
 enum { ORC_SINGLE = 0, ORC_ROUTE = 1 };
-enum { ORC_ARR_THINNED = 0, ORC_ARR_DIURNAL = 1 };
+enum { ORC_ARR_THINNED = 0, ORC_ARR_DIURNAL = 1, ORC_ARR_TRACE = 2 };
 enum { ORC_SAMPLE = 0, ORC_ARGMAX = 1, ORC_STATIC = 2, ORC_RR = 3, ORC_SQ = 4,
        ORC_RANDOM = 5, ORC_EXTERNAL = 6 };
 
@@ -54,6 +54,12 @@ typedef struct {
   uint32_t dwell_kind;                      /* 0 exponential dwell, 1 fixed dwell (square wave) */
   uint32_t srv_speed16[ORC_MAX_SERVERS];    /* batch time factor of each server, in 1/16 (0: 16) */
   uint32_t action_layout;                   /* 0: major x table index; 1: Wait + sizes 1..n */
+  /* Trace replay (arrival_kind TRACE, Sec. 3.2): host arrays of trace_len entries; the
+     gap before each request, its type (or NULL: drawn), its cost (or NULL: drawn). */
+  const uint32_t* trace_gap;
+  const uint8_t* trace_type;
+  const uint32_t* trace_cost;
+  uint32_t trace_len;
 } orc_config;
 
 /* Host-memory MLP (row-major W[l] of dims[l+1] x dims[l]). */

@@ -62,8 +62,9 @@ simx_status validate_config(const simx_config* c) {
     if (c->srv_speed16[k] > 255) return fail(SIMX_EINVAL, "srv_speed16[%u] = %u (at most 255)", k, c->srv_speed16[k]);
   if (!pow2(c->queue_cap) || c->queue_cap > 4096) return fail(SIMX_EINVAL, "queue_cap %u must be a power of two <= 4096", c->queue_cap);
   if (c->episode_len < 1) return fail(SIMX_EINVAL, "episode_len must be >= 1");
-  if (c->arrival_kind == SIMX_ARR_THINNED) {
-    if (!finite_pos(c->cand_mean_gap_us)) return fail(SIMX_EINVAL, "cand_mean_gap_us must be > 0");
+  if (c->arrival_kind == SIMX_ARR_THINNED || c->arrival_kind == SIMX_ARR_TRACE) {
+    if (c->arrival_kind == SIMX_ARR_THINNED && !finite_pos(c->cand_mean_gap_us))
+      return fail(SIMX_EINVAL, "cand_mean_gap_us must be > 0");
     if (c->n_mod_states < 1 || c->n_mod_states > 2) return fail(SIMX_EINVAL, "n_mod_states %u", c->n_mod_states);
     for (uint32_t i = 0; i < c->n_mod_states; ++i)
       if (c->accept_thr[i] > (1u << 24)) return fail(SIMX_EINVAL, "accept_thr[%u] > 2^24", i);
@@ -194,9 +195,17 @@ Packed g_pf_pack[64];  // per-device policy repack buffers for policy_forward
 
 }  // namespace
 
+struct Trace {
+  const uint32_t* gap = nullptr;
+  const uint8_t* type = nullptr;
+  const uint32_t* cost = nullptr;
+  uint32_t n = 0;
+};
+
 struct simx_ctx {
   simx_config cfg;
   int device = 0;
+  Trace trace_next, trace;  // set by sim_set_trace; taken over by sim_reset
   DevState st{};
   uint32_t key0 = 0, key1 = 0;
   bool seeded = false;
@@ -326,11 +335,30 @@ static void base_args(simx_ctx* c, RolloutArgs& a) {
   a.G = choose_lanes(c->cfg.n_envs);
   a.threads = choose_threads(c->cfg.n_envs, a.G);
   act_layout((int)c->cfg.obs_dim, (int)a.n_actions, a.maxd4, a.apad);
+  a.tr_gap = c->trace.gap;
+  a.tr_type = c->trace.type;
+  a.tr_cost = c->trace.cost;
+  a.tr_n = c->trace.n;
+}
+
+simx_status sim_set_trace(simx_ctx* c, const uint32_t* d_gap_us, const uint8_t* d_type,
+                          const uint32_t* d_cost_us, uint32_t n) {
+  if (!c || !d_gap_us) return fail(SIMX_EINVAL, "ctx or d_gap_us is NULL");
+  if (c->cfg.arrival_kind != SIMX_ARR_TRACE) return fail(SIMX_EINVAL, "arrival_kind is not TRACE");
+  if (n < 1 || n >= (1u << 31)) return fail(SIMX_EINVAL, "trace length %u outside [1, 2^31)", n);
+  c->trace_next.gap = d_gap_us;
+  c->trace_next.type = d_type;
+  c->trace_next.cost = d_cost_us;
+  c->trace_next.n = n;
+  return SIMX_OK;
 }
 
 simx_status sim_reset(simx_ctx* c, uint64_t seed, void* stream) {
   if (!c) return fail(SIMX_EINVAL, "ctx is NULL");
   cudaSetDevice(c->device);
+  if (c->cfg.arrival_kind == SIMX_ARR_TRACE && !c->trace_next.gap)
+    return fail(SIMX_ESTATE, "TRACE arrivals need sim_set_trace before sim_reset");
+  c->trace = c->trace_next;
   c->key0 = (uint32_t)seed;
   c->key1 = (uint32_t)(seed >> 32);
   RolloutArgs a;

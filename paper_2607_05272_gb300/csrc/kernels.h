@@ -36,6 +36,11 @@ struct RolloutArgs {
   int apad;         // softmax scratch floats per env (multiple of 4)
   int G;            // lanes per env (8, 16 or 32)
   int threads;      // threads per block (64, 128 or 256)
+  // trace replay (arrival_kind TRACE): gaps, types (or null), costs (or null), length
+  const uint32_t* tr_gap;
+  const uint8_t* tr_type;
+  const uint32_t* tr_cost;
+  uint32_t tr_n;
 };
 
 struct PolicyArgs {

@@ -80,6 +80,25 @@ __device__ __forceinline__ uint32_t req_type(const simx_config& c, uint32_t w1) 
   return (c.n_types > 1 && (w1 >> 8) >= c.type0_thr) ? 1u : 0u;
 }
 
+// Type and cost of candidate j with Philox words w1, w3: under trace replay (TR) the
+// trace's when it has them, else drawn.  TR is a template parameter of the kernels
+// because the trace lookups, even untaken, slowed the candidate loop of generated-
+// arrival workloads by up to a sixth.
+template <bool TR>
+__device__ __forceinline__ uint32_t cand_type(const RolloutArgs& A, uint32_t j, uint32_t w1) {
+  if (TR && A.tr_type) {
+    const uint32_t t = A.tr_type[j % A.tr_n];
+    return t < A.cfg.n_types ? t : A.cfg.n_types - 1u;
+  }
+  return req_type(A.cfg, w1);
+}
+
+template <bool TR>
+__device__ __forceinline__ uint32_t cand_cost(const RolloutArgs& A, uint32_t j, uint32_t w3) {
+  if (TR && A.tr_cost) return A.tr_cost[j % A.tr_n];
+  return req_cost(A.cfg, w3);
+}
+
 // Batch time of `n` requests of `type` on server k: alpha + beta n (or alpha + the sum
 // of the requests' costs for the cost type), times the server's speed s/16, rounded to
 // the nearest microsecond in integers.
@@ -121,12 +140,15 @@ __device__ __forceinline__ uint32_t switch_time(const RolloutArgs& A, uint32_t e
 }
 
 // G consecutive candidates from (cand_j, cand_T): lane gl holds candidate cj + gl with
-// its Philox block; times are the prefix sums of integer gaps (exact in any order).
-template <int G>
+// its Philox block; times are the prefix sums of integer gaps (exact in any order).  The
+// gap is drawn, or read from entry j mod n of a replayed trace.
+template <int G, bool TR>
 __device__ __forceinline__ void gen_chunk(const RolloutArgs& A, const Grp<G>& g, uint32_t env,
                                           const Scal& s, uint32_t& T, bool& over, U4& w) {
-  w = philox(s.cj + g.gl, env, kStreamArrival, 0u, A.key0, A.key1);
-  const uint32_t gap = duration_us(__fmul_rn(A.cfg.cand_mean_gap_us, expo1(w.x)));
+  const uint32_t j = s.cj + g.gl;
+  w = philox(j, env, kStreamArrival, 0u, A.key0, A.key1);
+  const uint32_t gap = TR ? A.tr_gap[j % A.tr_n]
+                          : duration_us(__fmul_rn(A.cfg.cand_mean_gap_us, expo1(w.x)));
   const uint64_t t64 = (uint64_t)s.cT + g.scan_incl(gap);
   over = t64 >= kTimeLimit;
   T = over ? kTimeLimit : (uint32_t)t64;
@@ -134,7 +156,7 @@ __device__ __forceinline__ void gen_chunk(const RolloutArgs& A, const Grp<G>& g,
 
 // SINGLE mode: consume every candidate with time <= target; accepted ones join
 // their type's FIFO (or are dropped when it is full); switches <= target apply.
-template <int G>
+template <int G, bool TR>
 __device__ void advance_single(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
                                Srv& q, uint32_t* ringb, uint32_t* costb, uint32_t target) {
   const simx_config& c = A.cfg;
@@ -143,7 +165,7 @@ __device__ void advance_single(const RolloutArgs& A, const Grp<G>& g, uint32_t e
     uint32_t T;
     bool over;
     U4 w;
-    gen_chunk<G>(A, g, env, s, T, over, w);
+    gen_chunk<G, TR>(A, g, env, s, T, over, w);
     const bool cons = T <= target;
     const int m = __popc(g.ballot(cons));
     const int peek = m < G ? m : G - 1;
@@ -164,8 +186,8 @@ __device__ void advance_single(const RolloutArgs& A, const Grp<G>& g, uint32_t e
       }
     }
     const bool acc = cons && ((w.z >> 8) < c.accept_thr[st]);
-    const uint32_t type = req_type(c, w.y);
-    const uint32_t cst = (acc && (int32_t)type == c.cost_type) ? req_cost(c, w.w) : 0u;
+    const uint32_t type = cand_type<TR>(A, s.cj + g.gl, w.y);
+    const uint32_t cst = (acc && (int32_t)type == c.cost_type) ? cand_cost<TR>(A, s.cj + g.gl, w.w) : 0u;
     for (uint32_t t = 0; t < c.n_types; ++t) {
       const bool mine = acc && type == t;
       const uint32_t bt = g.ballot(mine);
@@ -234,7 +256,7 @@ __device__ __forceinline__ void tentative_states(const RolloutArgs& A, uint32_t 
 
 // SINGLE mode: advance to the next accepted arrival and take in all candidates up
 // to its time (the next decision point when nothing is queued).
-template <int G>
+template <int G, bool TR>
 __device__ void jump_single(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s,
                             Srv& q, uint32_t* ringb, uint32_t* costb) {
   const simx_config& c = A.cfg;
@@ -242,7 +264,7 @@ __device__ void jump_single(const RolloutArgs& A, const Grp<G>& g, uint32_t env,
     uint32_t T;
     bool over;
     U4 w;
-    gen_chunk<G>(A, g, env, s, T, over, w);
+    gen_chunk<G, TR>(A, g, env, s, T, over, w);
     const uint32_t Tmax = g.shfl(T, G - 1);
     uint32_t st, ms, si, sT, tflag, nsw;
     tentative_states<G>(A, env, s, T, Tmax, st, ms, si, sT, tflag, nsw);
@@ -250,7 +272,7 @@ __device__ void jump_single(const RolloutArgs& A, const Grp<G>& g, uint32_t env,
     const uint32_t bm = g.ballot(acc);
     if (bm) {
       const uint32_t Tf = g.shfl(T, __ffs(bm) - 1);
-      advance_single<G>(A, g, env, s, q, ringb, costb, Tf);
+      advance_single<G, TR>(A, g, env, s, q, ringb, costb, Tf);
       s.now = Tf;
       return;
     }
@@ -270,15 +292,15 @@ __device__ void jump_single(const RolloutArgs& A, const Grp<G>& g, uint32_t env,
 }
 
 // ROUTE mode: draw the next request arrival into the pending slot.
-template <int G>
+template <int G, bool TR>
 __device__ void next_arrival(const RolloutArgs& A, const Grp<G>& g, uint32_t env, Scal& s) {
   const simx_config& c = A.cfg;
-  if (c.arrival_kind == SIMX_ARR_THINNED) {
+  if (TR || c.arrival_kind != SIMX_ARR_DIURNAL) {  // THINNED or TRACE
     for (;;) {
       uint32_t T;
       bool over;
       U4 w;
-      gen_chunk<G>(A, g, env, s, T, over, w);
+      gen_chunk<G, TR>(A, g, env, s, T, over, w);
       const uint32_t Tmax = g.shfl(T, G - 1);
       uint32_t st, ms, si, sT, tflag, nsw;
       tentative_states<G>(A, env, s, T, Tmax, st, ms, si, sT, tflag, nsw);
@@ -300,12 +322,13 @@ __device__ void next_arrival(const RolloutArgs& A, const Grp<G>& g, uint32_t env
             }
           }
         }
+        const uint32_t jf = s.cj + (uint32_t)f;
         s.cj += (uint32_t)f + 1u;
         s.cT = Tf;
         s.events += (uint32_t)f + 1u;
         s.pt = Tf;
-        s.pty = req_type(c, wy);
-        s.pc = ((int32_t)s.pty == c.cost_type) ? req_cost(c, ww) : 0u;
+        s.pty = cand_type<TR>(A, jf, wy);
+        s.pc = ((int32_t)s.pty == c.cost_type) ? cand_cost<TR>(A, jf, ww) : 0u;
         s.narr += 1u;
         if (s.events > kEventCap) s.status |= kStEvent;
         return;
@@ -629,7 +652,7 @@ __device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int B
 // maxd4 x B floats (feature-major) and a softmax scratch of apad floats per env.
 // Every lane stays alive to the end (groups past the last env do no work) so that
 // warps reconverge at each phase and the block can run the MLP together.
-template <bool ROUTE, int G>
+template <bool ROUTE, int G, bool TR>
 __global__ void __launch_bounds__(kMaxThreads, min_blocks<G>())
 k_rollout(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
@@ -734,11 +757,11 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
         s.events = 0;
         if (n > 0) {
           const uint32_t next = L.busy;
-          advance_single<G>(A, g, env, s, L, ringb, costb, next);
+          advance_single<G, TR>(A, g, env, s, L, ringb, costb, next);
           s.now = next;
-          if (L.qc[0] + (T > 1 ? L.qc[1] : 0u) == 0u) jump_single<G>(A, g, env, s, L, ringb, costb);
+          if (L.qc[0] + (T > 1 ? L.qc[1] : 0u) == 0u) jump_single<G, TR>(A, g, env, s, L, ringb, costb);
         } else {
-          jump_single<G>(A, g, env, s, L, ringb, costb);
+          jump_single<G, TR>(A, g, env, s, L, ringb, costb);
         }
       }
       __syncwarp();
@@ -770,7 +793,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
       }
       __syncwarp();
       if (live && !frozen) {
-        next_arrival<G>(A, g, env, s);
+        next_arrival<G, TR>(A, g, env, s);
         uint32_t gap = s.pt - now;
         if (gap < 1u) gap = 1u;
         const float inst = __fdiv_rn(1.0e6f, __uint2float_rn(gap));
@@ -833,7 +856,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
 
 // Reset: empty queues, idle servers, chain state from the INIT stream, then advance
 // to the first decision point.
-template <bool ROUTE, int G>
+template <bool ROUTE, int G, bool TR>
 __global__ void __launch_bounds__(kMaxThreads) k_reset(const __grid_constant__ RolloutArgs A) {
   const Grp<G> g;
   const uint32_t slot = threadIdx.x / G;
@@ -874,13 +897,15 @@ __global__ void __launch_bounds__(kMaxThreads) k_reset(const __grid_constant__ R
   }
   if (c.arrival_kind == SIMX_ARR_DIURNAL)
     s.epo = (uint32_t)(((uint64_t)(w.y >> 8) * c.diurnal_len) >> 24);
+  if (TR)  // this env's starting entry of the trace
+    s.cj = (uint32_t)(((uint64_t)w.z * A.tr_n) >> 32);
   Srv L{0u, static_bsize(c), Pair{0u, 0u}, Pair{0u, 0u}};
   __syncwarp(g.mask);
   if (ROUTE) {
-    next_arrival<G>(A, g, env, s);
+    next_arrival<G, TR>(A, g, env, s);
     s.now = s.pt;
   } else {
-    jump_single<G>(A, g, env, s, L, ringb, costb);
+    jump_single<G, TR>(A, g, env, s, L, ringb, costb);
   }
   if (g.gl == 0) store_scal(st, env, s);
   if (ROUTE) {
@@ -1060,15 +1085,17 @@ template <bool ROUTE, int G>
 static cudaError_t rollout_t(const RolloutArgs& a, cudaStream_t s) {
   const int B = a.threads / G;
   const size_t sh = env_smem(a, B);
-  cudaFuncSetAttribute(k_rollout<ROUTE, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
-  k_rollout<ROUTE, G><<<grid_for(a.st.E, B), a.threads, sh, s>>>(a);
+  auto k = a.cfg.arrival_kind == SIMX_ARR_TRACE ? k_rollout<ROUTE, G, true> : k_rollout<ROUTE, G, false>;
+  cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
+  k<<<grid_for(a.st.E, B), a.threads, sh, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }
 
 template <bool ROUTE, int G>
 static cudaError_t reset_t(const RolloutArgs& a, cudaStream_t s) {
-  k_reset<ROUTE, G><<<grid_for(a.st.E, a.threads / G), a.threads, 0, s>>>(a);
+  auto k = a.cfg.arrival_kind == SIMX_ARR_TRACE ? k_reset<ROUTE, G, true> : k_reset<ROUTE, G, false>;
+  k<<<grid_for(a.st.E, a.threads / G), a.threads, 0, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -77,18 +77,38 @@ __device__ void t_switches(const Ctx& x, TEnv<K>& s, uint32_t limit) {
   }
 }
 
-template <int K>
+// Candidate s.cj: its Philox words and its time (a drawn gap, or under trace replay,
+// TR, entry cj mod n of the trace).  TR is a template parameter so that the generated-
+// arrival kernels carry none of the trace code.
+template <int K, bool TR>
 __device__ __forceinline__ uint32_t t_cand(const Ctx& x, TEnv<K>& s, U4& w) {
   w = philox(s.cj, x.env, kStreamArrival, 0u, x.A.key0, x.A.key1);
-  return t_add(s.cT, duration_us(__fmul_rn(x.A.cfg.cand_mean_gap_us, expo1(w.x))), s.status);
+  const uint32_t gap = TR ? x.A.tr_gap[s.cj % x.A.tr_n]
+                          : duration_us(__fmul_rn(x.A.cfg.cand_mean_gap_us, expo1(w.x)));
+  return t_add(s.cT, gap, s.status);
+}
+
+// Type and cost of candidate j: the trace's when it has them, else drawn.
+template <bool TR>
+__device__ __forceinline__ uint32_t t_cand_type(const RolloutArgs& A, uint32_t j, uint32_t w1) {
+  if (TR && A.tr_type) {
+    const uint32_t t = A.tr_type[j % A.tr_n];
+    return t < A.cfg.n_types ? t : A.cfg.n_types - 1u;
+  }
+  return t_type(A.cfg, w1);
+}
+
+template <bool TR>
+__device__ __forceinline__ uint32_t t_cand_cost(const RolloutArgs& A, uint32_t j, uint32_t w3) {
+  return (TR && A.tr_cost) ? A.tr_cost[j % A.tr_n] : t_cost(A.cfg, w3);
 }
 
 // SINGLE mode: an accepted candidate joins its type's FIFO or is dropped.
-template <int K>
+template <int K, bool TR>
 __device__ bool t_consume(const Ctx& x, TEnv<K>& s, const U4& w, uint32_t T) {
   const simx_config& c = x.A.cfg;
   if (!((w.z >> 8) < c.accept_thr[s.mst])) return false;
-  const uint32_t ty = t_type(c, w.y);
+  const uint32_t ty = t_cand_type<TR>(x.A, s.cj, w.y);
   const uint32_t cap = c.queue_cap;
   s.narr += 1u;
   if (ty) s.na1 += 1u; else s.na0 += 1u;
@@ -96,7 +116,7 @@ __device__ bool t_consume(const Ctx& x, TEnv<K>& s, const U4& w, uint32_t T) {
   if (q < cap) {
     const uint32_t slot = ((ty ? s.qh1[0] : s.qh0[0]) + q) & (cap - 1u);
     x.ring[ty * cap + slot] = T;
-    if ((int32_t)ty == c.cost_type) x.cost[slot] = t_cost(c, w.w);
+    if ((int32_t)ty == c.cost_type) x.cost[slot] = t_cand_cost<TR>(x.A, s.cj, w.w);
     if (ty) s.qc1[0] += 1u; else s.qc0[0] += 1u;
   } else {
     s.ndrop += 1u;
@@ -105,55 +125,56 @@ __device__ bool t_consume(const Ctx& x, TEnv<K>& s, const U4& w, uint32_t T) {
   return true;
 }
 
-template <int K>
+template <int K, bool TR>
 __device__ void t_advance(const Ctx& x, TEnv<K>& s, uint32_t target) {
   for (;;) {
     U4 w;
-    const uint32_t T = t_cand(x, s, w);
+    const uint32_t T = t_cand<K, TR>(x, s, w);
     if (T > target) break;
     if (t_count(s)) return;
     t_switches(x, s, T);
-    t_consume(x, s, w, T);
+    t_consume<K, TR>(x, s, w, T);
     s.cj += 1u;
     s.cT = T;
   }
   t_switches(x, s, target);
 }
 
-template <int K>
+template <int K, bool TR>
 __device__ void t_jump(const Ctx& x, TEnv<K>& s) {
   for (;;) {
     U4 w;
-    const uint32_t T = t_cand(x, s, w);
+    const uint32_t T = t_cand<K, TR>(x, s, w);
     if (t_count(s)) return;
     t_switches(x, s, T);
-    const bool acc = t_consume(x, s, w, T);
+    const bool acc = t_consume<K, TR>(x, s, w, T);
     s.cj += 1u;
     s.cT = T;
     if (acc) {
       s.now = T;
-      t_advance(x, s, T);
+      t_advance<K, TR>(x, s, T);
       return;
     }
   }
 }
 
 // ROUTE mode: the next arrival into the pending slot.
-template <int K>
+template <int K, bool TR>
 __device__ void t_next_arrival(const Ctx& x, TEnv<K>& s) {
   const simx_config& c = x.A.cfg;
   for (;;) {
     if (t_count(s)) return;
     U4 w;
-    if (c.arrival_kind == SIMX_ARR_THINNED) {
-      const uint32_t T = t_cand(x, s, w);
+    if (TR || c.arrival_kind != SIMX_ARR_DIURNAL) {  // THINNED or TRACE
+      const uint32_t T = t_cand<K, TR>(x, s, w);
       t_switches(x, s, T);
       const bool acc = (w.z >> 8) < c.accept_thr[s.mst];
+      const uint32_t j = s.cj;
       s.cj += 1u;
       s.cT = T;
       if (!acc) continue;
-      s.pty = t_type(c, w.y);
-      s.pc = ((int32_t)s.pty == c.cost_type) ? t_cost(c, w.w) : 0u;
+      s.pty = t_cand_type<TR>(x.A, j, w.y);
+      s.pc = ((int32_t)s.pty == c.cost_type) ? t_cand_cost<TR>(x.A, j, w.w) : 0u;
       s.pt = T;
       s.narr += 1u;
       return;
@@ -344,7 +365,7 @@ __device__ int t_action(const Ctx& x, TEnv<K>& s) {
 // MINB resident 128-thread blocks per SM bound the registers (4: 128).  The latency of
 // one env-step is a long dependent chain, so the step rate is the number of resident
 // threads over that latency: more residency beats more registers.
-template <bool ROUTE, int K, int MINB>
+template <bool ROUTE, int K, int MINB, bool TR>
 __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant__ RolloutArgs A) {
   const uint32_t env = blockIdx.x * blockDim.x + threadIdx.x;
   if (env >= A.st.E) return;
@@ -455,11 +476,11 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
         s.events = 0;
         if (n > 0) {
           const uint32_t next = s.busy[0];
-          t_advance(x, s, next);
+          t_advance<K, TR>(x, s, next);
           s.now = next;
-          if (t_queued(s) == 0u) t_jump(x, s);
+          if (t_queued(s) == 0u) t_jump<K, TR>(x, s);
         } else {
-          t_jump(x, s);
+          t_jump<K, TR>(x, s);
         }
       }
     } else {
@@ -485,7 +506,7 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
           if (s.busy[k] <= now) t_start<K>(x, s, k, now, stn, w0, w1);
         }
         qafter = t_queued(s);
-        t_next_arrival(x, s);
+        t_next_arrival<K, TR>(x, s);
         uint32_t gap = s.pt - now;
         if (gap < 1u) gap = 1u;
         const float inst = __fdiv_rn(1.0e6f, __uint2float_rn(gap));
@@ -568,7 +589,10 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
 // spill the server state of the router.
 template <bool ROUTE, int K>
 cudaError_t step_thread_t(const RolloutArgs& a, cudaStream_t s) {
-  k_step_thread<ROUTE, K, 4><<<(a.st.E + 127) / 128, 128, 0, s>>>(a);
+  if (a.cfg.arrival_kind == SIMX_ARR_TRACE)
+    k_step_thread<ROUTE, K, 4, true><<<(a.st.E + 127) / 128, 128, 0, s>>>(a);
+  else
+    k_step_thread<ROUTE, K, 4, false><<<(a.st.E + 127) / 128, 128, 0, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }

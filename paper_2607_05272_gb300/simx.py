@@ -11,6 +11,8 @@ import ctypes as C
 import os
 import threading
 
+import numpy as np
+
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libsimx.so")
 _lock = threading.Lock()
@@ -88,6 +90,7 @@ SIGNATURES = [
     ("sim_create", C.c_int, [P, C.c_int, P]),
     ("sim_destroy", None, [P]),
     ("sim_reset", C.c_int, [P, U64, P]),
+    ("sim_set_trace", C.c_int, [P, P, P, P, U32]),
     ("sim_observe", C.c_int, [P, P, I64, P]),
     ("sim_step_batched", C.c_int, [P, P, P, C.c_int, P, I64, P, P, P, P, P]),
     ("rollout_collect", C.c_int, [P, P, C.c_int, I32, P, P]),
@@ -214,6 +217,26 @@ class Sim:
         self.E = cfg["n_envs"]
         self.D = obs_dim(cfg)
         self.words = state_words(cfg)
+        self._trace = None
+        if cfg.get("trace") is not None:
+            self.set_trace(*cfg["trace"])
+
+    def set_trace(self, gap_us, type=None, cost_us=None):
+        """Trace replay input (sim_set_trace): per-request gaps in us, types and costs;
+        numpy arrays are copied to the device, device tensors are used as they are
+        (int32 / uint8 / int32, values below 2^31).  Takes effect at the next reset."""
+        import torch
+
+        def dev(x, dt):
+            if x is None:
+                return None
+            t = x if isinstance(x, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(x).astype(dt))
+            return t.contiguous().cuda()
+        g = dev(gap_us, np.int32)
+        ty = dev(type, np.uint8)
+        co = dev(cost_us, np.int32)
+        _check(lib().sim_set_trace(self._h, g.data_ptr(), _ptr(ty), _ptr(co), len(g)))
+        self._trace = (g, ty, co)
 
     def close(self):
         if getattr(self, "_h", None):

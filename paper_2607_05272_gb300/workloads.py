@@ -32,7 +32,7 @@ import numpy as np
 
 ABI_VERSION = 4
 MODE_SINGLE, MODE_ROUTE = 0, 1
-ARR_THINNED, ARR_DIURNAL = 0, 1
+ARR_THINNED, ARR_DIURNAL, ARR_TRACE = 0, 1, 2
 POLICY = {"sample": 0, "argmax": 1, "static": 2, "rr": 3, "sq": 4, "random": 5, "external": 6}
 TWO24 = 1 << 24
 
@@ -177,6 +177,55 @@ def c2w(n_envs: int = 4096) -> dict:
     return c
 
 
+def synthetic_trace(n: int, seed: int, mean_gap_us: float = 300.0, cv: float = 2.0,
+                    p_long: float = 0.2, stay: float = 0.9, cost_median_us: float = 8000.0,
+                    cost_sigma: float = 1.0):
+    """A seeded request trace of n entries in the trace replay format (gap_us u32,
+    type u8, cost_us u32), shaped like an LLM serving log of the BurstGPT kind: Gamma
+    inter-arrival gaps with coefficient of variation `cv` (bursty when cv > 1), request
+    types from a two-state chain that stays on its type with probability `stay` (runs of
+    one model; a fraction `p_long` of long requests overall), and lognormal per-request
+    costs (response-length shaped).  Synthetic: no real trace is reproduced."""
+    rng = np.random.default_rng(seed)
+    k = 1.0 / (cv * cv)
+    gap = np.rint(rng.gamma(k, mean_gap_us / k, n)).astype(np.uint32)
+    # chain with stationary P(long) = p_long: P(short -> long) = (1 - stay) p_long / (1 - p_long)
+    # scaled so that both switch rates stay in [0, 1]
+    a = (1.0 - stay) * min(1.0, p_long / (1.0 - p_long))
+    b = a * (1.0 - p_long) / p_long
+    u = rng.random(n)
+    typ = np.zeros(n, np.uint8)
+    t = 1 if rng.random() < p_long else 0
+    for i in range(n):
+        typ[i] = t
+        if u[i] < (b if t else a):
+            t ^= 1
+    cost = np.rint(cost_median_us * np.exp(cost_sigma * rng.standard_normal(n)))
+    cost = np.minimum(cost, 2.0 ** 26).astype(np.uint32)
+    return gap, typ, cost
+
+
+def c2t(n_envs: int = 4096) -> dict:
+    """Trace replay (Sec. 3.2 real-world traces) on c2's server: every arrival, its gap
+    and its type come from a 100,000-entry synthetic BurstGPT-shaped trace (mean gap
+    600 us, CV 2, 20 % long requests in runs); each env starts at its own entry."""
+    c = c2(n_envs)
+    c.update(arrival_kind=ARR_TRACE, n_mod_states=1, accept_thr=[TWO24, TWO24],
+             trace=synthetic_trace(100_000, 0x7ACE0002, mean_gap_us=600.0))
+    return c
+
+
+def c3t(n_envs: int = 16384) -> dict:
+    """Trace replay on c3's 4-server router: gaps, types and the long requests' costs
+    (batch time alpha + the sum of its requests' costs) from a synthetic trace (mean gap
+    250 us, CV 2, 30 % long, lognormal costs with median 8 ms)."""
+    c = c3(n_envs)
+    c.update(arrival_kind=ARR_TRACE, n_mod_states=1, accept_thr=[TWO24, TWO24],
+             cost_type=1, cost_kind=1, cost_scale_us=8000.0, beta_us=[50, 0],
+             trace=synthetic_trace(100_000, 0x7ACE0003, mean_gap_us=250.0, p_long=0.3))
+    return c
+
+
 def c1p(n_envs: int = 64) -> dict:
     """c1w's env and action space, served by the paper's policy network (Sec. 4.2; the
     network is described at ``PAPER_NET``)."""
@@ -184,7 +233,7 @@ def c1p(n_envs: int = 64) -> dict:
 
 
 CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5, "burst": burst, "c3h": c3h,
-           "c1w": c1w, "c2w": c2w, "c1p": c1p}
+           "c1w": c1w, "c2w": c2w, "c1p": c1p, "c2t": c2t, "c3t": c3t}
 
 # Policy network shapes (input, hidden..., actions) and whether a value row follows.
 MLP_SHAPES = {
@@ -198,6 +247,8 @@ MLP_SHAPES = {
     "c1w": ([8, 32, 33], False),
     "c2w": ([16, 64, 64, 65], False),
     "c1p": ([8, 4, 4, 4, 128, 33], True),
+    "c2t": ([16, 64, 64, 12], False),
+    "c3t": ([13, 128, 128, 16], True),
 }
 
 # The paper's network (Sec. 4.2) as a plain MLP.  The 8-dim state is projected to a
@@ -214,9 +265,10 @@ PAPER_NET = ("c1p",)
 MLP_ACTS = {"c1p": ["identity", "identity", "identity", "gelu"]}
 
 HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024, "burst": 2000, "c3h": 256,
-           "c1w": 2000, "c2w": 512, "c1p": 2000}
+           "c1w": 2000, "c2w": 512, "c1p": 2000, "c2t": 512, "c3t": 256}
 SEED = {name: 0x5EED0000 + i + 1
-        for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h", "c1w", "c2w", "c1p"])}
+        for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h", "c1w", "c2w", "c1p",
+                                  "c2t", "c3t"])}
 
 
 def mlp_dims(name: str) -> tuple:

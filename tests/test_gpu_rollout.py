@@ -76,6 +76,8 @@ CASES = [
     ("c1w", lambda: W.c1w(33), 2000, "sample"),       # Wait + batch 1..32: 33 actions
     ("c2w", lambda: W.c2w(37), 512, "sample"),        # Wait + (type, batch 1..32): 65
     ("c1p", lambda: W.c1p(41), 2000, "sample"),       # the paper's network (GELU heads)
+    ("c2t", lambda: W.c2t(37), 512, "sample"),        # trace replay: gaps and types
+    ("c3t", lambda: W.c3t(45), 256, "sample"),        # trace replay: gaps, types, costs
 ]
 
 
@@ -111,6 +113,9 @@ BASELINES = [
     ("c3h", lambda: W.c3h(39), 256, "rr"),
     ("c2w", lambda: W.c2w(34), 512, "static"),
     ("c1w", lambda: W.c1w(30), 2000, "random"),
+    ("c2t", lambda: W.c2t(33), 512, "static"),
+    ("c3t", lambda: W.c3t(41), 256, "sq"),
+    ("c3t", lambda: W.c3t(35), 256, "random"),
 ]
 
 
@@ -166,7 +171,7 @@ def test_step_batched_equals_rollout(name, mk):
 
 @pytest.mark.parametrize("name,mk", [("c1", lambda: W.c1(9)), ("c2", lambda: W.c2(17)),
                                      ("c3", lambda: W.c3(19)), ("c4", lambda: W.c4(11)),
-                                     ("c2w", lambda: W.c2w(15))])
+                                     ("c2w", lambda: W.c2w(15)), ("c3t", lambda: W.c3t(13))])
 def test_external_actions_match_oracle(name, mk):
     simx = _simx()
     cfg = mk()
@@ -211,7 +216,8 @@ def test_bad_external_action_sets_status():
     sim.close()
 
 
-@pytest.mark.parametrize("name,mk,H", [("c2", lambda: W.c2(21), 300), ("c4", lambda: W.c4(19), 300)])
+@pytest.mark.parametrize("name,mk,H", [("c2", lambda: W.c2(21), 300), ("c4", lambda: W.c4(19), 300),
+                                      ("c3t", lambda: W.c3t(23), 200)])
 def test_save_load_resume_is_bit_exact(name, mk, H):
     simx = _simx()
     cfg = mk()
@@ -239,6 +245,47 @@ def test_save_load_resume_is_bit_exact(name, mk, H):
         joined = torch.cat([h1[k], h2[k]], 0)
         assert torch.equal(full[k], joined), k
     assert np.array_equal(a.save(), c.save())
+
+
+def _tiny_trace_cfg(E, with_costs):
+    gap = np.array([5, 0, 12, 3, 100, 7, 1, 0, 0, 40, 2], np.uint32)
+    typ = np.array([0, 1, 1, 0, 5, 0, 1, 1, 0, 0, 1], np.uint8)   # 5: the last type
+    cost = np.array([11, 22, 33, 44, 55, 66, 77, 88, 99, 1, 0], np.uint32)
+    cfg = W.c3t(E)
+    cfg["trace"] = (gap, typ, cost if with_costs else None)
+    return cfg
+
+
+@pytest.mark.parametrize("mode", ["sample", "sq"])
+@pytest.mark.parametrize("with_costs", [True, False])
+def test_short_trace_wraps_like_the_oracle(mode, with_costs):
+    """An 11-entry trace with zero gaps and an out-of-range type, replayed hundreds of
+    times over by every env from its own starting entry."""
+    got, ref, st, code = _run("c3t", _tiny_trace_cfg(43, with_costs), 300, mode)
+    assert st == 0 and code == 0
+    _assert_same(got, ref, mode == "sample")
+
+
+def test_trace_call_order_and_arguments():
+    simx = _simx()
+    g = torch.ones(4, dtype=torch.int32, device="cuda")
+    plain = simx.Sim(W.c3(8))
+    with pytest.raises(simx.SimxError) as e:   # not a trace workload
+        plain.set_trace(g)
+    assert e.value.status == simx.EINVAL
+    plain.close()
+    cfg = W.c3t(8)
+    cfg["trace"] = None
+    sim = simx.Sim(cfg)
+    with pytest.raises(simx.SimxError) as e:   # reset before any trace
+        sim.reset(1)
+    assert e.value.status == simx.ESTATE
+    with pytest.raises(simx.SimxError) as e:   # empty trace
+        sim.set_trace(g[:0])
+    assert e.value.status == simx.EINVAL
+    sim.set_trace(g)
+    sim.reset(1)
+    sim.close()
 
 
 def test_policy_forward_matches_oracle():

@@ -60,7 +60,8 @@ def _policy_for(name):
 
 CASES = [("c1", W.c1(4), SAMPLE), ("c2", W.c2(4), SAMPLE), ("c3", W.c3(4), SAMPLE),
          ("c4", W.c4(4), SAMPLE), ("c3", W.c3(4), SQ), ("c2", W.c2(4), STATIC),
-         ("c4", W.c4(4), RANDOM)]
+         ("c4", W.c4(4), RANDOM), ("c2t", W.c2t(4), SAMPLE), ("c2t", W.c2t(4), STATIC),
+         ("c3t", W.c3t(4), SAMPLE), ("c3t", W.c3t(4), SQ)]
 
 
 def _conserved(cfg, s):
