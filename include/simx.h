@@ -362,6 +362,32 @@ simx_status ppo_loss_grad_noalloc(const simx_mlp* pol, const simx_rollout* buf,
                                   const int64_t* d_idx, int64_t n, const simx_loss_params* params,
                                   float* d_grad, float* d_stats, void* stream);
 
+/*
+ * Optimiser step of the training loop (Sec. 4.3 trains REINFORCE and PPO; the paper
+ * names no optimiser, so this is Adam, Kingma & Ba 2015).  On a flat fp32 parameter
+ * vector in the gradient's order (W0, b0, W1, b1, ...; a policy whose W_l, b_l are views
+ * into it updates in place):
+ *   s   = min(1, max_grad_norm / ||g||_2)  when max_grad_norm > 0, else 1;
+ *   m   = beta1 m + (1 - beta1) s g;   v = beta2 v + (1 - beta2) (s g)^2;
+ *   p  -= (lr / (1 - beta1^t)) m / (sqrt(v) / sqrt(1 - beta2^t) + eps),
+ * for every i with d_mask == NULL or d_mask[i] != 0 (masked entries keep p, m and v:
+ * the zero blocks of a block-diagonal head stay zero).  t >= 1 is the step number;
+ * m and v start at zero.  ||g||_2 is taken over the unmasked entries.
+ * All arrays are device memory of n entries (mask: bytes), owned by the caller;
+ * d_workspace holds simx_adam_workspace_size(n) bytes (used only when clipping).
+ * SIMX_EINVAL for n < 1, t < 1, NULL arrays, a short workspace or a parameter outside
+ * lr >= 0, 0 <= beta < 1, eps > 0.
+ */
+typedef struct simx_adam_params {
+  float lr, beta1, beta2, eps;
+  float max_grad_norm;  /* <= 0: no clipping */
+} simx_adam_params;
+size_t simx_adam_workspace_size(int64_t n);
+simx_status simx_adam_step(float* d_params, const float* d_grad, float* d_m, float* d_v,
+                           const uint8_t* d_mask, int64_t n, int64_t t,
+                           const simx_adam_params* params, void* d_workspace,
+                           size_t workspace_bytes, void* stream);
+
 /* Aggregate counters (synchronises the context's last stream). host_out: host. */
 simx_status sim_stats(simx_ctx* ctx, simx_counters* host_out);
 

@@ -170,3 +170,25 @@ def gather_rows(obs, actions, logp, idx, E):
     t, e = idx // E, idx % E
     X = obs[t, :, e]
     return X, np.asarray(actions)[t, e], np.asarray(logp)[t, e]
+
+
+def adam_step(p, g, m, v, t, lr, beta1=0.9, beta2=0.999, eps=1e-8, max_grad_norm=0.0,
+              mask=None):
+    """One Adam step (Kingma & Ba 2015, Algorithm 1) in fp64, the optimiser of the
+    training loop (Sec. 4.3 names none).  When max_grad_norm > 0 the gradient is first
+    scaled by min(1, max_grad_norm / ||g||_2); entries with mask == 0 are left as they
+    are and do not count in the norm.  Returns the new (p, m, v)."""
+    p, g, m, v = (np.array(x, np.float64) for x in (p, g, m, v))
+    sel = np.ones(p.shape, bool) if mask is None else np.asarray(mask) != 0
+    s = 1.0
+    if max_grad_norm > 0.0:
+        norm = math.sqrt(float(np.sum(g[sel] ** 2)))
+        if norm > max_grad_norm:
+            s = max_grad_norm / norm
+    gs = g[sel] * s
+    m[sel] = beta1 * m[sel] + (1.0 - beta1) * gs
+    v[sel] = beta2 * v[sel] + (1.0 - beta2) * gs * gs
+    m_hat = m[sel] / (1.0 - beta1 ** t)
+    v_hat = v[sel] / (1.0 - beta2 ** t)
+    p[sel] = p[sel] - lr * m_hat / (np.sqrt(v_hat) + eps)
+    return p, m, v

@@ -109,6 +109,12 @@ void launch_loss_reduce(const float* part, int nb, int n_params, const double* s
                         const LossArgs& a, cudaStream_t s);
 // fma_probe.cu
 cudaError_t launch_fma_probe(int64_t iters, float* sink, double* flops, cudaStream_t s);
+
+// optim.cu
+size_t adam_workspace_bytes(int64_t n);
+cudaError_t launch_adam(float* p, const float* g, float* m, float* v, const uint8_t* mask,
+                        int64_t n, int64_t t, float lr, float b1, float b2, float eps,
+                        float max_norm, void* ws, cudaStream_t s);
 size_t fma_probe_sink_floats();
 // loss_tc.cu
 bool loss_tc_fits(const LossArgs& a);

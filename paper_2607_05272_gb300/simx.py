@@ -91,6 +91,8 @@ SIGNATURES = [
     ("sim_destroy", None, [P]),
     ("sim_reset", C.c_int, [P, U64, P]),
     ("sim_set_trace", C.c_int, [P, P, P, P, U32]),
+    ("simx_adam_workspace_size", SZ, [I64]),
+    ("simx_adam_step", C.c_int, [P, P, P, P, P, I64, I64, P, P, SZ, P]),
     ("sim_observe", C.c_int, [P, P, I64, P]),
     ("sim_step_batched", C.c_int, [P, P, P, C.c_int, P, I64, P, P, P, P, P]),
     ("rollout_collect", C.c_int, [P, P, C.c_int, I32, P, P]),
@@ -180,6 +182,23 @@ class Policy:
         for l, a in enumerate(acts or []):
             m.act[l] = ACT[a] if isinstance(a, str) else int(a)
         self.c = m
+
+    flat = None  # the flat parameter vector when built by from_flat
+
+    @classmethod
+    def from_flat(cls, flat, dims, has_value: bool, acts=None):
+        """A policy whose W_l, b_l are views into one flat fp32 device vector in the
+        gradient's order (W0, b0, W1, b1, ...): the optimiser updates it in place."""
+        Ws, bs, off = [], [], 0
+        for k, n in zip(dims[:-1], dims[1:]):
+            Ws.append(flat[off:off + n * k].view(n, k))
+            off += n * k
+            bs.append(flat[off:off + n])
+            off += n
+        assert off == flat.numel()
+        pol = cls(Ws, bs, has_value, acts)
+        pol.flat = flat
+        return pol
 
     @property
     def n_actions(self) -> int:
@@ -350,6 +369,26 @@ def ppo_loss_grad(policy: Policy, buf: dict, ret, adv, idx, n: int, algo: str, c
     _check(lib().ppo_loss_grad(C.byref(policy.c), C.byref(r), r.ld, _ptr(ret), _ptr(adv),
                                _ptr(idx), n, C.byref(p), _ptr(grad), _ptr(stats), _ptr(workspace),
                                workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+class AdamParams(C.Structure):
+    _fields_ = [("lr", C.c_float), ("beta1", C.c_float), ("beta2", C.c_float),
+                ("eps", C.c_float), ("max_grad_norm", C.c_float)]
+
+
+def adam_workspace_size(n: int) -> int:
+    return lib().simx_adam_workspace_size(n)
+
+
+def adam_step(params, grad, m, v, t: int, lr: float, beta1: float = 0.9, beta2: float = 0.999,
+              eps: float = 1e-8, max_grad_norm: float = 0.0, mask=None, workspace=None,
+              stream=None):
+    """simx_adam_step on flat fp32 device vectors (mask: uint8 or None)."""
+    p = AdamParams(lr, beta1, beta2, eps, max_grad_norm)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib().simx_adam_step(_ptr(params), _ptr(grad), _ptr(m), _ptr(v), _ptr(mask),
+                                params.numel(), t, C.byref(p), _ptr(workspace), ws_bytes,
+                                _stream(stream)))
 
 
 NOALLOC_SCRATCH_BYTES = 16 << 20

@@ -226,6 +226,20 @@ def c3t(n_envs: int = 16384) -> dict:
     return c
 
 
+def c3s(n_envs: int = 4096) -> dict:
+    """Multi-GPU Routing (Heterogeneous) of Sec. 3.2, the setting of the segregation
+    result of Sec. 5: two servers, Poisson 60 req/s, a 50/50 mix of fast and slow
+    requests with the paper's V100 batch times (alpha 2 ms; beta 5 ms fast, 20 ms slow),
+    batch sizes {1, 2, 4, 8} per server, and an observation that includes the arriving
+    request's type (obs_extra), which segregation needs."""
+    return _base(mode=MODE_ROUTE, n_envs=n_envs, n_servers=2, n_types=2, queue_cap=256,
+                 episode_len=256, cand_mean_gap_us=float(np.float32(1e6 / 60.0)),
+                 type0_thr=_thr(0.5), alpha_us=[2000, 2000], beta_us=[5000, 20000],
+                 w_wait=[0.001, 0.0001], n_bsizes=4, bsizes=[1, 2, 4, 8, 0, 0, 0, 0],
+                 static_bi=0, obs_extra=1, obs_dim=10, rate_scale=0.0, rate_ref=60.0,
+                 phase_period_us=60_000_000)
+
+
 def c1p(n_envs: int = 64) -> dict:
     """c1w's env and action space, served by the paper's policy network (Sec. 4.2; the
     network is described at ``PAPER_NET``)."""
@@ -233,7 +247,7 @@ def c1p(n_envs: int = 64) -> dict:
 
 
 CONFIGS = {"c1": c1, "c2": c2, "c3": c3, "c4": c4, "c5": c5, "burst": burst, "c3h": c3h,
-           "c1w": c1w, "c2w": c2w, "c1p": c1p, "c2t": c2t, "c3t": c3t}
+           "c1w": c1w, "c2w": c2w, "c1p": c1p, "c2t": c2t, "c3t": c3t, "c3s": c3s}
 
 # Policy network shapes (input, hidden..., actions) and whether a value row follows.
 MLP_SHAPES = {
@@ -249,6 +263,7 @@ MLP_SHAPES = {
     "c1p": ([8, 4, 4, 4, 128, 33], True),
     "c2t": ([16, 64, 64, 12], False),
     "c3t": ([13, 128, 128, 16], True),
+    "c3s": ([10, 128, 128, 8], True),
 }
 
 # The paper's network (Sec. 4.2) as a plain MLP.  The 8-dim state is projected to a
@@ -261,14 +276,21 @@ MLP_SHAPES = {
 # (a trainer that keeps the heads separate leaves them there by masking their gradient).
 PAPER_NET = ("c1p",)
 
+# Policies whose value head is a separate network (Sec. 4.2), as one MLP: every layer
+# after the first is block-diagonal between a policy tower (the first half of the hidden
+# units) and a value tower (the second half), and the value row reads only the value
+# tower.  A value row on a shared trunk let the value loss (returns of order -200 on c3s)
+# drown the policy gradient; separate towers learn.
+TWO_TOWER = ("c3s",)
+
 # Activation after each hidden layer where it is not tanh (simx_act names).
 MLP_ACTS = {"c1p": ["identity", "identity", "identity", "gelu"]}
 
 HORIZON = {"c1": 10000, "c2": 512, "c3": 256, "c4": 512, "c5": 1024, "burst": 2000, "c3h": 256,
-           "c1w": 2000, "c2w": 512, "c1p": 2000, "c2t": 512, "c3t": 256}
+           "c1w": 2000, "c2w": 512, "c1p": 2000, "c2t": 512, "c3t": 256, "c3s": 256}
 SEED = {name: 0x5EED0000 + i + 1
         for i, name in enumerate(["c1", "c2", "c3", "c4", "c5", "burst", "c3h", "c1w", "c2w", "c1p",
-                                  "c2t", "c3t"])}
+                                  "c2t", "c3t", "c3s"])}
 
 
 def mlp_dims(name: str) -> tuple:
@@ -295,24 +317,56 @@ def mlp_acts(name: str) -> list:
     return list(MLP_ACTS.get(name, ["tanh"] * n_hidden))
 
 
+def _block_masks(name: str, dims):
+    """Per-layer 0/1 masks of the weight entries that exist, or None for a dense MLP."""
+    if name not in PAPER_NET and name not in TWO_TOWER:
+        return None
+    L = len(dims) - 1
+    masks = []
+    for l, (k, n) in enumerate(zip(dims[:-1], dims[1:])):
+        m = np.ones((n, k), np.uint8)
+        hk = k // 2
+        if l == L - 1:                       # heads: logits <- first half, value <- second
+            m[:-1, hk:] = 0
+            m[-1, :hk] = 0
+        elif name in TWO_TOWER and l > 0:    # towers: hidden layers block-diagonal
+            hn = n // 2
+            m[:hn, hk:] = 0
+            m[hn:, :hk] = 0
+        masks.append(m)
+    return masks
+
+
 def policy_weights(name: str, dims, seed: int):
     """Initial fp32 weights and biases of `name`'s policy with layer widths `dims`.
 
-    Tanh policies: ``mlp_weights``.  The paper's network: N(0, 1 / (3 fan_in)) weights
-    (the spread of a uniform +-1/sqrt(fan_in) draw), small random biases, and the last
-    layer block-diagonal between the policy and value heads (the last hidden layer split
-    in halves)."""
+    Tanh policies: ``mlp_weights`` (two-tower ones with their off-diagonal blocks zeroed).
+    The paper's network: N(0, 1 / (3 fan_in)) weights (the spread of a uniform
+    +-1/sqrt(fan_in) draw), small random biases, and the last layer block-diagonal between
+    the policy and value heads (the last hidden layer split in halves)."""
+    masks = _block_masks(name, dims)
     if name not in PAPER_NET:
-        return mlp_weights(dims, seed)
-    rng = np.random.default_rng(seed)
-    Ws, bs = [], []
-    for k, n in zip(dims[:-1], dims[1:]):
-        Ws.append((rng.standard_normal((n, k)) / np.sqrt(3.0 * k)).astype(np.float32))
-        bs.append((rng.standard_normal(n) * 0.05).astype(np.float32))
-    half = dims[-2] // 2
-    Ws[-1][:-1, half:] = 0.0
-    Ws[-1][-1, :half] = 0.0
+        Ws, bs = mlp_weights(dims, seed)
+    else:
+        rng = np.random.default_rng(seed)
+        Ws, bs = [], []
+        for k, n in zip(dims[:-1], dims[1:]):
+            Ws.append((rng.standard_normal((n, k)) / np.sqrt(3.0 * k)).astype(np.float32))
+            bs.append((rng.standard_normal(n) * 0.05).astype(np.float32))
+    if masks is not None:
+        Ws = [np.where(m != 0, w, np.float32(0.0)).astype(np.float32) for w, m in zip(Ws, masks)]
     return Ws, bs
+
+
+def param_mask(name: str, dims):
+    """Trainable-entry mask (uint8, the flat W0, b0, W1, b1, ... order) or None: the
+    zero blocks of the paper's network and of two-tower policies stay frozen at zero,
+    which keeps their policy and value heads separate."""
+    masks = _block_masks(name, dims)
+    if masks is None:
+        return None
+    return np.concatenate([np.concatenate([m.ravel(), np.ones(m.shape[0], np.uint8)])
+                           for m in masks])
 
 
 def minibatch_perm(n_rows: int, seed: int, epoch: int) -> np.ndarray:

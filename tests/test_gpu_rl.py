@@ -217,3 +217,44 @@ def test_gemm_pipeline_loss_gradient_matches_oracle(name, algo, E, H, nmb, hidde
     _check_grad(g, g_ref, layers)
     assert np.all(np.abs(s[:4] - st[:4]) <= 1e-5 * (np.abs(st[:4]) + 1.0))
     assert abs(s[4] - st[4]) <= 1.0 / n
+
+
+@pytest.mark.parametrize("n,clip,masked", [(1, 0.0, False), (1000, 0.0, False), (100003, 0.5, False),
+                                           (77777, 0.0, True), (5102, 1.0, True)])
+def test_adam_matches_oracle(n, clip, masked):
+    """Six Adam steps on fp32 device vectors against the fp64 oracle: parameters within
+    1e-6 of their size plus 1e-4 of the total step length, moments within 1e-5."""
+    f32 = lambda x: float(np.float32(x))
+    simx = _simx()
+    rng = np.random.default_rng(n)
+    p0 = rng.standard_normal(n).astype(np.float32)
+    mask = (rng.random(n) < 0.6).astype(np.uint8) if masked else None
+    p, m, v = (torch.from_numpy(x).cuda() for x in (p0.copy(), np.zeros(n, np.float32),
+                                                    np.zeros(n, np.float32)))
+    tm = None if mask is None else torch.from_numpy(mask).cuda()
+    ws = torch.empty(simx.adam_workspace_size(n), dtype=torch.uint8, device="cuda")
+    rp, rm, rv = p0.astype(np.float64), np.zeros(n), np.zeros(n)
+    lr = 1e-3
+    for t in range(1, 7):
+        g = (rng.standard_normal(n) * 10.0 ** rng.uniform(-3, 1, n)).astype(np.float32)
+        simx.adam_step(p, torch.from_numpy(g).cuda(), m, v, t, lr, 0.9, 0.999, 1e-8, clip, tm, ws)
+        # the oracle takes the hyper-parameters the ABI carries: fp32 values
+        rp, rm, rv = rl.adam_step(rp, g, rm, rv, t, *map(f32, (lr, 0.9, 0.999, 1e-8, clip)), mask)
+    torch.cuda.synchronize()
+    gp, gm, gv = (x.cpu().numpy().astype(np.float64) for x in (p, m, v))
+    assert np.all(np.abs(gp - rp) <= 1e-6 * np.abs(rp) + 1e-4 * 6 * lr)
+    assert np.all(np.abs(gm - rm) <= 1e-5 * np.abs(rm) + 1e-7 * np.abs(rm).max())
+    assert np.all(np.abs(gv - rv) <= 1e-5 * np.abs(rv) + 1e-7 * np.abs(rv).max())
+    if masked:
+        sel = mask == 0
+        assert np.array_equal(gp[sel], p0[sel]) and not gm[sel].any() and not gv[sel].any()
+
+
+def test_adam_rejects_bad_arguments():
+    simx = _simx()
+    x = torch.zeros(8, device="cuda")
+    for kw in (dict(t=0, lr=1e-3), dict(t=1, lr=-1.0), dict(t=1, lr=1e-3, beta1=1.0),
+               dict(t=1, lr=1e-3, eps=0.0), dict(t=1, lr=1e-3, max_grad_norm=1.0)):
+        with pytest.raises(simx.SimxError) as e:   # the last: clipping without a workspace
+            simx.adam_step(x, x, x, x, **kw)
+        assert e.value.status == simx.EINVAL

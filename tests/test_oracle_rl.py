@@ -207,3 +207,68 @@ def test_gather_rows_layout():
     X, a, _ = rl.gather_rows(obs, act, act, [0, 5, 11], E)
     assert X.tolist() == [[0, 4], [9, 13], [19, 23]]
     assert a.tolist() == [0, 5, 11]
+
+
+def _adam_case(masked):
+    rng = np.random.default_rng(8)
+    n = 300
+    p0 = rng.standard_normal(n)
+    grads = [rng.standard_normal(n) * (0.1 + i) for i in range(5)]
+    mask = (rng.random(n) < 0.7).astype(np.uint8) if masked else None
+    sel = np.ones(n, bool) if mask is None else mask != 0
+    return p0, grads, mask, sel
+
+
+@pytest.mark.parametrize("masked", [False, True])
+def test_adam_matches_torch_optimiser(masked):
+    """Five Adam steps against torch.optim.Adam in fp64; masked entries stay put and the
+    rest follow torch on the unmasked sub-vector."""
+    torch = pytest.importorskip("torch")
+    p0, grads, mask, sel = _adam_case(masked)
+    n = len(p0)
+    tp = torch.tensor(p0[sel], requires_grad=True)
+    opt = torch.optim.Adam([tp], lr=3e-3, betas=(0.9, 0.99), eps=1e-6)
+    p, m, v = p0.copy(), np.zeros(n), np.zeros(n)
+    for t, g in enumerate(grads, start=1):
+        tp.grad = torch.tensor(g[sel])
+        opt.step()
+        p, m, v = rl.adam_step(p, g, m, v, t, 3e-3, 0.9, 0.99, 1e-6, 0.0, mask)
+    assert np.allclose(p[sel], tp.detach().numpy(), rtol=1e-12, atol=1e-14)
+    assert np.array_equal(p[~sel], p0[~sel]) and np.all(m[~sel] == 0) and np.all(v[~sel] == 0)
+    st = opt.state[tp]
+    assert np.allclose(m[sel], st["exp_avg"].numpy(), rtol=1e-12, atol=1e-15)
+    assert np.allclose(v[sel], st["exp_avg_sq"].numpy(), rtol=1e-12, atol=1e-15)
+
+
+@pytest.mark.parametrize("masked", [False, True])
+def test_adam_clipping_matches_torch_clip_grad_norm(masked):
+    """Global-norm clipping over the unmasked entries against torch's clip_grad_norm_,
+    whose scale max_norm / (norm + 1e-6) differs from min(1, max_norm / norm) by 1e-6 in
+    the denominator: moments and movement equal within 1e-5 of their magnitude (entries
+    where m nearly cancels amplify the difference).  A bound above the norm changes
+    nothing."""
+    torch = pytest.importorskip("torch")
+    p0, grads, mask, sel = _adam_case(masked)
+    n = len(p0)
+    p, m, v = p0.copy(), np.zeros(n), np.zeros(n)
+    q, mq, vq = p0.copy(), np.zeros(n), np.zeros(n)
+    for t, g in enumerate(grads, start=1):
+        tg = torch.tensor(g[sel])
+        tg.grad = tg.clone()
+        torch.nn.utils.clip_grad_norm_([tg], 0.5)
+        gc = g.copy()
+        gc[sel] = tg.grad.numpy()
+        p, m, v = rl.adam_step(p, g, m, v, t, 3e-3, 0.9, 0.99, 1e-6, 0.5, mask)
+        q, mq, vq = rl.adam_step(q, gc, mq, vq, t, 3e-3, 0.9, 0.99, 1e-6, 0.0, mask)
+        assert np.max(np.abs(m - mq)) <= 1e-5 * np.max(np.abs(m))
+    assert np.max(np.abs(p - q)) <= 1e-5 * np.max(np.abs(p - p0))   # of the total movement
+    a = rl.adam_step(p0, grads[0], np.zeros(n), np.zeros(n), 1, 3e-3, max_grad_norm=1e9, mask=mask)
+    b = rl.adam_step(p0, grads[0], np.zeros(n), np.zeros(n), 1, 3e-3, mask=mask)
+    assert all(np.array_equal(x, y) for x, y in zip(a, b))
+
+
+def test_adam_first_step_moves_each_entry_by_lr():
+    """A textbook property: at t = 1 with eps -> 0 the step is lr sign(g) per entry."""
+    g = np.array([3.0, -0.01, 1e-4, -250.0])
+    p, _, _ = rl.adam_step(np.zeros(4), g, np.zeros(4), np.zeros(4), 1, 0.01, eps=1e-300)
+    assert np.allclose(p, -0.01 * np.sign(g), rtol=1e-12)
