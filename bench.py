@@ -432,6 +432,29 @@ def hbm_step_measure(simx, W, torch, E=65536, steps=100, warm=10) -> dict:
             "timing": "CUDA graph of %d steps, replayed %d times, CUDA events" % (steps, reps)}
 
 
+# --- replicas (N > 1): every rank simulates its own envs, no data-path collective -------
+
+def replica_seed(rank: int) -> int:
+    """Seed of rank `rank`'s replica: envs are keyed by (seed, env id), so replicas with
+    different seeds are independent problems (weak scaling)."""
+    return SEED_BASE + rank
+
+
+def max_over_ranks(x: float, dist=None, device="cpu") -> float:
+    """The largest of the ranks' values (the step time the job is charged)."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(world: int, units_per_rank: int, ms: float) -> float:
+    """Whole-job throughput: the units all ranks processed over the slowest rank's time."""
+    return world * units_per_rank / (ms * 1e-3)
+
+
 def run_gpu(a) -> None:
     import numpy as np
     import torch
@@ -460,7 +483,7 @@ def run_gpu(a) -> None:
     dbs = [torch.from_numpy(b).cuda() for b in bs]
     pol = simx.Policy(dWs, dbs, hv)
     sim = simx.Sim(cfg, device=local)
-    sim.reset(SEED_BASE + rank)
+    sim.reset(replica_seed(rank))
     D = sim.D
     n = E * H
     buf = simx.alloc_rollout(E, D, H)
@@ -521,11 +544,8 @@ def run_gpu(a) -> None:
     step_ms = [evs[k][0].elapsed_time(evs[k][4]) for k in range(a.steps)]
     ms = statistics.mean(step_ms)
     ph = [statistics.mean(p[i] for p in phase_ms) for i in range(4)]
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * n / (ms * 1e-3)
+    ms = max_over_ranks(ms, dist, "cuda")
+    value = job_value(world, n, ms)
     st, code = sim.last_status()
     if st != 0:
         raise RuntimeError("device status 0x%x after the timed region" % code)
@@ -553,11 +573,8 @@ def run_gpu(a) -> None:
             hs.copy_(stats, non_blocking=True)
             torch.cuda.synchronize()
         t_e2e = (time.perf_counter() - t0) / k_e2e
-        if dist:
-            t = torch.tensor([t_e2e], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            t_e2e = float(t.item())
-        e2e = {"value": world * n / t_e2e, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        t_e2e = max_over_ranks(t_e2e, dist, "cuda")
+        e2e = {"value": job_value(world, n, t_e2e * 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h}
 
     # the loss gradient in the other precision, on the same buffer, for comparison
