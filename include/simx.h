@@ -371,12 +371,15 @@ simx_status ppo_loss_grad_noalloc(const simx_mlp* pol, const simx_rollout* buf,
  *   m   = beta1 m + (1 - beta1) s g;   v = beta2 v + (1 - beta2) (s g)^2;
  *   p  -= (lr / (1 - beta1^t)) m / (sqrt(v) / sqrt(1 - beta2^t) + eps),
  * for every i with d_mask == NULL or d_mask[i] != 0 (masked entries keep p, m and v:
- * the zero blocks of a block-diagonal head stay zero).  t >= 1 is the step number;
- * m and v start at zero.  ||g||_2 is taken over the unmasked entries.
+ * the zero blocks of a block-diagonal head stay zero).  m and v start at zero.
+ * ||g||_2 is taken over the unmasked entries.
+ * The step number: t >= 1 from the host when d_t is NULL; otherwise d_t is a device
+ * int64 counter that the step increments before use (t = ++*d_t, on the stream), so a
+ * captured CUDA graph of training steps advances it on every replay.
  * All arrays are device memory of n entries (mask: bytes), owned by the caller;
- * d_workspace holds simx_adam_workspace_size(n) bytes (used only when clipping).
- * SIMX_EINVAL for n < 1, t < 1, NULL arrays, a short workspace or a parameter outside
- * lr >= 0, 0 <= beta < 1, eps > 0.
+ * d_workspace holds simx_adam_workspace_size(n) bytes (used when clipping or with d_t).
+ * SIMX_EINVAL for n < 1, t < 1 without d_t, NULL arrays, a short workspace or a
+ * parameter outside lr >= 0, 0 <= beta < 1, eps > 0.
  */
 typedef struct simx_adam_params {
   float lr, beta1, beta2, eps;
@@ -384,7 +387,7 @@ typedef struct simx_adam_params {
 } simx_adam_params;
 size_t simx_adam_workspace_size(int64_t n);
 simx_status simx_adam_step(float* d_params, const float* d_grad, float* d_m, float* d_v,
-                           const uint8_t* d_mask, int64_t n, int64_t t,
+                           const uint8_t* d_mask, int64_t n, int64_t t, int64_t* d_t,
                            const simx_adam_params* params, void* d_workspace,
                            size_t workspace_bytes, void* stream);
 

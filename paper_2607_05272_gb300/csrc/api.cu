@@ -246,18 +246,18 @@ size_t simx_fma_probe_sink_floats(void) { return fma_probe_sink_floats(); }
 size_t simx_adam_workspace_size(int64_t n) { return n < 1 ? 0 : adam_workspace_bytes(n); }
 
 simx_status simx_adam_step(float* d_params, const float* d_grad, float* d_m, float* d_v,
-                           const uint8_t* d_mask, int64_t n, int64_t t,
+                           const uint8_t* d_mask, int64_t n, int64_t t, int64_t* d_t,
                            const simx_adam_params* p, void* d_workspace, size_t workspace_bytes,
                            void* stream) {
   if (!d_params || !d_grad || !d_m || !d_v || !p) return fail(SIMX_EINVAL, "adam: NULL array or params");
-  if (n < 1 || t < 1) return fail(SIMX_EINVAL, "adam: n %lld, t %lld", (long long)n, (long long)t);
+  if (n < 1 || (!d_t && t < 1)) return fail(SIMX_EINVAL, "adam: n %lld, t %lld", (long long)n, (long long)t);
   if (!(p->lr >= 0.0f) || !(p->beta1 >= 0.0f && p->beta1 < 1.0f) ||
       !(p->beta2 >= 0.0f && p->beta2 < 1.0f) || !(p->eps > 0.0f) || !std::isfinite(p->lr) ||
       std::isnan(p->max_grad_norm))
     return fail(SIMX_EINVAL, "adam: lr %g beta1 %g beta2 %g eps %g", p->lr, p->beta1, p->beta2, p->eps);
-  if (p->max_grad_norm > 0.0f && (!d_workspace || workspace_bytes < adam_workspace_bytes(n)))
+  if ((p->max_grad_norm > 0.0f || d_t) && (!d_workspace || workspace_bytes < adam_workspace_bytes(n)))
     return fail(SIMX_EINVAL, "adam: workspace of %zu bytes needed", adam_workspace_bytes(n));
-  const cudaError_t e = launch_adam(d_params, d_grad, d_m, d_v, d_mask, n, t, p->lr, p->beta1,
+  const cudaError_t e = launch_adam(d_params, d_grad, d_m, d_v, d_mask, n, t, d_t, p->lr, p->beta1,
                                     p->beta2, p->eps, p->max_grad_norm, d_workspace,
                                     (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "adam launch");

@@ -113,8 +113,8 @@ cudaError_t launch_fma_probe(int64_t iters, float* sink, double* flops, cudaStre
 // optim.cu
 size_t adam_workspace_bytes(int64_t n);
 cudaError_t launch_adam(float* p, const float* g, float* m, float* v, const uint8_t* mask,
-                        int64_t n, int64_t t, float lr, float b1, float b2, float eps,
-                        float max_norm, void* ws, cudaStream_t s);
+                        int64_t n, int64_t t, int64_t* d_t, float lr, float b1, float b2,
+                        float eps, float max_norm, void* ws, cudaStream_t s);
 size_t fma_probe_sink_floats();
 // loss_tc.cu
 bool loss_tc_fits(const LossArgs& a);

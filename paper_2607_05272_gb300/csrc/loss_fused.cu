@@ -461,12 +461,19 @@ __global__ void k_reduce_blocks(const float* __restrict__ part, int nb, int P, f
   out[i] = s;
 }
 
+// One warp per statistic: lane l sums blocks l, l + 32, ... in order, then a fixed
+// butterfly combines the lanes (the same order on every run).
 __global__ void k_fused_stats(const double* __restrict__ sp, int nb, int64_t n, int has_value,
                               float cv, float ce, float* __restrict__ stats) {
+  __shared__ double sh[4];
+  const int q = threadIdx.x / 32, lane = threadIdx.x % 32;
+  double acc = 0.0;
+  for (int b = lane; b < nb; b += 32) acc += sp[(size_t)b * 4 + q];
+  for (int d = 16; d > 0; d /= 2) acc += __shfl_xor_sync(0xffffffffu, acc, d);
+  if (lane == 0) sh[q] = acc;
+  __syncthreads();
   if (threadIdx.x != 0) return;
-  double s[4] = {0, 0, 0, 0};
-  for (int b = 0; b < nb; ++b)
-    for (int q = 0; q < 4; ++q) s[q] += sp[(size_t)b * 4 + q];
+  const double s[4] = {sh[0], sh[1], sh[2], sh[3]};
   const double pg = s[0] / (double)n, v = s[1] / (double)n, H = s[2] / (double)n;
   stats[0] = (float)(pg + (has_value ? (double)cv * v : 0.0) - (double)ce * H);
   stats[1] = (float)pg;
@@ -596,7 +603,7 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
 void launch_loss_reduce(const float* part, int nb, int n_params, const double* spart,
                         const LossArgs& a, cudaStream_t s) {
   k_reduce_blocks<<<(n_params + 255) / 256, 256, 0, s>>>(part, nb, n_params, a.grad);
-  k_fused_stats<<<1, 32, 0, s>>>(spart, nb, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
+  k_fused_stats<<<1, 128, 0, s>>>(spart, nb, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
   count_launches(2);
 }
 

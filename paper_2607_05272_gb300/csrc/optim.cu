@@ -1,7 +1,9 @@
 // Adam (Kingma & Ba 2015), the optimiser step of the policy-gradient training loop
 // (Sec. 4.3), on a flat parameter vector.  One elementwise kernel; with gradient
 // clipping a fixed-grid sum of squares (fp64 partials, reduced in a fixed order, so the
-// scale is the same bits on every run) and a one-block finish run first.
+// scale is the same bits on every run) and a one-thread finish run first.  With a device
+// step counter the finish also advances the counter and computes the bias corrections,
+// so that a captured CUDA graph of training steps needs no host argument per step.
 #include "kernels.h"
 
 namespace simx {
@@ -31,23 +33,42 @@ __global__ void __launch_bounds__(kAdamThreads) k_sumsq(const float* __restrict_
   if (threadIdx.x == 0) part[blockIdx.x] = red[0];
 }
 
-// scale = min(1, max_norm / ||g||), 1 for a zero gradient.
-__global__ void k_clip_scale(const double* part, int nb, float max_norm, float* scale) {
+// scal[0] = min(1, max_norm / ||g||) (1 for a zero gradient, or without clipping);
+// with a device step counter also t = ++*d_t, scal[1] = lr / (1 - b1^t) and
+// scal[2] = 1 / sqrt(1 - b2^t), the bias corrections the host computes otherwise.
+__global__ void k_adam_scalars(const double* part, int nb, float max_norm, int64_t* d_t,
+                               float lr, float b1, float b2, float* scal) {
+  double s = 0.0;  // lane l sums partials l, l + 32, ...; a fixed butterfly combines lanes
+  if (part)
+    for (int b = (int)threadIdx.x; b < nb; b += 32) s += part[b];
+  for (int d = 16; d > 0; d /= 2) s += __shfl_xor_sync(0xffffffffu, s, d);
   if (threadIdx.x != 0) return;
-  double s = 0.0;
-  for (int b = 0; b < nb; ++b) s += part[b];
-  const double norm = sqrt(s);
-  *scale = (norm > (double)max_norm) ? (float)((double)max_norm / norm) : 1.0f;
+  float sc = 1.0f;
+  if (part) {
+    const double norm = sqrt(s);
+    if (norm > (double)max_norm) sc = (float)((double)max_norm / norm);
+  }
+  scal[0] = sc;
+  if (d_t) {
+    const int64_t t = *d_t + 1;
+    *d_t = t;
+    scal[1] = (float)((double)lr / (1.0 - pow((double)b1, (double)t)));
+    scal[2] = (float)(1.0 / sqrt(1.0 - pow((double)b2, (double)t)));
+  }
 }
 
 __global__ void __launch_bounds__(kAdamThreads) k_adam(float* __restrict__ p,
                                                        const float* __restrict__ g,
                                                        float* __restrict__ m, float* __restrict__ v,
                                                        const uint8_t* __restrict__ mask, int64_t n,
-                                                       const float* scale, float step_size,
-                                                       float inv_sqrt_c2, float b1, float b2,
-                                                       float eps) {
-  const float s = scale ? *scale : 1.0f;
+                                                       const float* scal, bool dev_t,
+                                                       float step_size, float inv_sqrt_c2,
+                                                       float b1, float b2, float eps) {
+  const float s = scal ? scal[0] : 1.0f;
+  if (dev_t) {
+    step_size = scal[1];
+    inv_sqrt_c2 = scal[2];
+  }
   for (int64_t i = (int64_t)blockIdx.x * kAdamThreads + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * kAdamThreads) {
     if (mask && !mask[i]) continue;
@@ -65,25 +86,34 @@ __global__ void __launch_bounds__(kAdamThreads) k_adam(float* __restrict__ p,
 
 size_t adam_workspace_bytes(int64_t) { return (size_t)kNormBlocks * sizeof(double) + 16; }
 
+// t >= 1: the step number from the host; d_t: a device counter incremented by the step
+// (then t is ignored and the workspace is always used).
 cudaError_t launch_adam(float* p, const float* g, float* m, float* v, const uint8_t* mask,
-                        int64_t n, int64_t t, float lr, float b1, float b2, float eps,
-                        float max_norm, void* ws, cudaStream_t s) {
-  const double c1 = 1.0 - pow((double)b1, (double)t);
-  const double c2 = 1.0 - pow((double)b2, (double)t);
-  const float step_size = (float)((double)lr / c1);
-  const float inv_sqrt_c2 = (float)(1.0 / sqrt(c2));
-  float* scale = nullptr;
-  if (max_norm > 0.0f) {
+                        int64_t n, int64_t t, int64_t* d_t, float lr, float b1, float b2,
+                        float eps, float max_norm, void* ws, cudaStream_t s) {
+  float step_size = 0.0f, inv_sqrt_c2 = 0.0f;
+  if (!d_t) {
+    const double c1 = 1.0 - pow((double)b1, (double)t);
+    const double c2 = 1.0 - pow((double)b2, (double)t);
+    step_size = (float)((double)lr / c1);
+    inv_sqrt_c2 = (float)(1.0 / sqrt(c2));
+  }
+  float* scal = nullptr;
+  if (max_norm > 0.0f || d_t) {
     double* part = static_cast<double*>(ws);
-    scale = reinterpret_cast<float*>(static_cast<char*>(ws) + (size_t)kNormBlocks * sizeof(double));
-    k_sumsq<<<kNormBlocks, kAdamThreads, 0, s>>>(g, mask, n, part);
-    k_clip_scale<<<1, 32, 0, s>>>(part, kNormBlocks, max_norm, scale);
-    count_launches(2);
+    scal = reinterpret_cast<float*>(static_cast<char*>(ws) + (size_t)kNormBlocks * sizeof(double));
+    if (max_norm > 0.0f) {
+      k_sumsq<<<kNormBlocks, kAdamThreads, 0, s>>>(g, mask, n, part);
+      count_launches(1);
+    }
+    k_adam_scalars<<<1, 32, 0, s>>>(max_norm > 0.0f ? part : nullptr, kNormBlocks, max_norm, d_t,
+                                    lr, b1, b2, scal);
+    count_launches(1);
   }
   int64_t blocks = (n + kAdamThreads - 1) / kAdamThreads;
   if (blocks > 152 * 8) blocks = 152 * 8;
-  k_adam<<<(unsigned)blocks, kAdamThreads, 0, s>>>(p, g, m, v, mask, n, scale, step_size,
-                                                   inv_sqrt_c2, b1, b2, eps);
+  k_adam<<<(unsigned)blocks, kAdamThreads, 0, s>>>(p, g, m, v, mask, n, scal, d_t != nullptr,
+                                                   step_size, inv_sqrt_c2, b1, b2, eps);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -92,7 +92,7 @@ SIGNATURES = [
     ("sim_reset", C.c_int, [P, U64, P]),
     ("sim_set_trace", C.c_int, [P, P, P, P, U32]),
     ("simx_adam_workspace_size", SZ, [I64]),
-    ("simx_adam_step", C.c_int, [P, P, P, P, P, I64, I64, P, P, SZ, P]),
+    ("simx_adam_step", C.c_int, [P, P, P, P, P, I64, I64, P, P, P, SZ, P]),
     ("sim_observe", C.c_int, [P, P, I64, P]),
     ("sim_step_batched", C.c_int, [P, P, P, C.c_int, P, I64, P, P, P, P, P]),
     ("rollout_collect", C.c_int, [P, P, C.c_int, I32, P, P]),
@@ -380,15 +380,17 @@ def adam_workspace_size(n: int) -> int:
     return lib().simx_adam_workspace_size(n)
 
 
-def adam_step(params, grad, m, v, t: int, lr: float, beta1: float = 0.9, beta2: float = 0.999,
+def adam_step(params, grad, m, v, t, lr: float, beta1: float = 0.9, beta2: float = 0.999,
               eps: float = 1e-8, max_grad_norm: float = 0.0, mask=None, workspace=None,
               stream=None):
-    """simx_adam_step on flat fp32 device vectors (mask: uint8 or None)."""
+    """simx_adam_step on flat fp32 device vectors (mask: uint8 or None).  t: the step
+    number (int), or an int64 device tensor of one element that the step increments."""
     p = AdamParams(lr, beta1, beta2, eps, max_grad_norm)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    dev = not isinstance(t, int)
     _check(lib().simx_adam_step(_ptr(params), _ptr(grad), _ptr(m), _ptr(v), _ptr(mask),
-                                params.numel(), t, C.byref(p), _ptr(workspace), ws_bytes,
-                                _stream(stream)))
+                                params.numel(), 0 if dev else t, _ptr(t) if dev else None,
+                                C.byref(p), _ptr(workspace), ws_bytes, _stream(stream)))
 
 
 NOALLOC_SCRATCH_BYTES = 16 << 20

@@ -33,7 +33,8 @@ class Trainer:
                  algo: str = "reinforce", horizon: int = 256, lr: float = 3e-4,
                  gamma: float = 0.99, lam: float = 0.95, epochs: int = 4, minibatch: int = 8192,
                  clip_eps: float = 0.2, c_value: float = 0.5, c_entropy: float = 0.01,
-                 max_grad_norm: float = 0.5, seed: int = 1, precision: str = "fp32"):
+                 max_grad_norm: float = 0.5, seed: int = 1, precision: str = "fp32",
+                 graph: bool = False):
         import torch
         self.torch = torch
         self.cfg, self.algo, self.H = cfg, algo, horizon
@@ -52,7 +53,8 @@ class Trainer:
         self.grad = torch.empty(n, device="cuda")
         self.stats = torch.empty(5, device="cuda")
         self.adam_ws = torch.empty(simx.adam_workspace_size(n), dtype=torch.uint8, device="cuda")
-        self.t = 0
+        self.t = 0                                                      # updates so far (host)
+        self.t_dev = torch.zeros(1, dtype=torch.int64, device="cuda")   # Adam's step counter
         E = cfg["n_envs"]
         self.E = E
         self.sim = simx.Sim(cfg)
@@ -71,18 +73,44 @@ class Trainer:
         self.mean = torch.empty(1, device="cuda")
         self.gen = torch.Generator(device="cuda")
         self.gen.manual_seed(seed)
+        # PPO minibatch rows of every epoch, drawn before each iteration (outside a graph)
+        self.perm = torch.empty((epochs, self.n_rows), dtype=torch.int64, device="cuda")
+        self.n_mb = self.n_rows // minibatch if algo == "ppo" else 1
+        self.use_graph = graph
+        self.graph = None
 
     def _update(self, idx, n):
         simx.ppo_loss_grad(self.policy, self.buf, self.ret, self.adv, idx, n, self.algo,
                            self.clip_eps, self.c_value if self.has_value else 0.0,
                            self.c_entropy, self.grad, self.stats, self.loss_ws,
                            precision=self.precision)
-        self.t += 1
-        simx.adam_step(self.params, self.grad, self.m, self.v, self.t, self.lr,
+        simx.adam_step(self.params, self.grad, self.m, self.v, self.t_dev, self.lr,
                        max_grad_norm=self.max_grad_norm, mask=self.mask, workspace=self.adam_ws)
 
     def iteration(self) -> dict:
-        """One rollout of H decisions per env and the policy update(s) on it."""
+        """One rollout of H decisions per env and the policy update(s) on it.  With
+        graph=True the first iteration runs eagerly (it sizes the library's internal
+        buffers), the second captures the whole iteration in a CUDA graph, and every
+        iteration from then on replays it: the same kernels on the same buffers, with
+        Adam's step counter advanced on the device."""
+        if self.algo == "ppo":
+            for e in range(self.epochs):
+                self.perm[e] = self.torch.randperm(self.n_rows, device="cuda", generator=self.gen)
+        if not self.use_graph or self.t == 0:
+            self._body()
+        else:
+            if self.graph is None:
+                self.graph = self.torch.cuda.CUDAGraph()
+                # relaxed: the library's host side sets kernel attributes, no stream work
+                with self.torch.cuda.graph(self.graph, capture_error_mode="relaxed"):
+                    self._body()
+            self.graph.replay()
+        self.t += self.n_mb * (self.epochs if self.algo == "ppo" else 1)
+        st = self.stats.cpu().numpy()
+        return {"mean_reward": float(self.buf["reward"].mean().item()), "loss": float(st[0]),
+                "entropy": float(st[3]), "updates": self.t}
+
+    def _body(self):
         b = self.buf
         self.sim.rollout("sample", self.H, b, self.policy)
         if self.has_value:  # bootstrap value of each env's current state
@@ -101,13 +129,9 @@ class Trainer:
         else:
             simx.compute_returns_gae(b["reward"], b["done"], self.gamma, self.lam, self.ret,
                                      adv=self.adv, val=b["value"], last_val=self.last)
-            for _ in range(self.epochs):
-                perm = self.torch.randperm(self.n_rows, device="cuda", generator=self.gen)
-                for s in range(0, self.n_rows - self.mb + 1, self.mb):
-                    self._update(perm[s:s + self.mb], self.mb)
-        st = self.stats.cpu().numpy()
-        return {"mean_reward": float(b["reward"].mean().item()), "loss": float(st[0]),
-                "entropy": float(st[3]), "updates": self.t}
+            for e in range(self.epochs):
+                for i in range(self.n_mb):
+                    self._update(self.perm[e, i * self.mb:(i + 1) * self.mb], self.mb)
 
 
 def evaluate(cfg: dict, mode: str, horizon: int, seed: int, policy=None, warm: int = 1) -> dict:
@@ -153,6 +177,7 @@ def main(argv=None):
     ap.add_argument("--lr", type=float, default=1e-3)
     ap.add_argument("--seed", type=int, default=1)
     ap.add_argument("--every", type=int, default=10)
+    ap.add_argument("--no-graph", action="store_true", help="launch every kernel from Python")
     a = ap.parse_args(argv)
     import torch
     cfg = W.CONFIGS[a.workload](a.envs)
@@ -160,7 +185,7 @@ def main(argv=None):
     Ws, bs = W.policy_weights(a.workload, dims, a.seed)
     mask = W.param_mask(a.workload, dims)
     tr = Trainer(cfg, dims, hv, W.mlp_acts(a.workload), (Ws, bs), mask, algo=a.algo,
-                 horizon=a.horizon, lr=a.lr, seed=a.seed)
+                 horizon=a.horizon, lr=a.lr, seed=a.seed, graph=not a.no_graph)
     t0 = time.perf_counter()
     hist = []
     for i in range(a.iters):

@@ -76,6 +76,27 @@ def test_iteration_runs_and_moves_the_policy(name, algo):
         assert not moved[mask == 0].any() and moved[mask != 0].mean() > 0.5
 
 
+@pytest.mark.parametrize("algo", ["ppo", "reinforce"])
+def test_graph_replay_equals_eager_iterations(algo):
+    """Four iterations replayed from one captured CUDA graph give the eager iterations'
+    parameters bit for bit (same kernels, same minibatch draws, device step counter)."""
+    train = _train()
+    name = "c3s"
+    cfg = W.CONFIGS[name](96)
+    dims, hv = W.mlp_dims(name)
+    out = []
+    for graph in (False, True):
+        tr = train.Trainer(cfg, dims, hv, None, W.policy_weights(name, dims, 2),
+                           W.param_mask(name, dims), algo=algo, horizon=64, minibatch=2048,
+                           epochs=2, lr=1e-3, graph=graph)
+        for _ in range(4):
+            s = tr.iteration()
+        torch.cuda.synchronize()
+        out.append((tr.params.cpu().numpy(), tr.t_dev.item(), s["updates"], tr.graph is not None))
+    (pe, te, ue, ge), (pg, tg, ug, gg) = out
+    assert np.array_equal(pe, pg) and te == tg == ue == ug and gg and not ge
+
+
 def test_training_beats_round_robin_on_heterogeneous_routing():
     """The segregation result in miniature (Sec. 5): 40 PPO iterations on the two-server
     fast/slow router lift the mean reward per decision well above its start and the
