@@ -258,12 +258,30 @@ struct FusedLossArgs {
   int dz_rows;                       // rows of each dZ buffer
   int poff[SIMX_MAX_LAYERS];         // offset of layer l's dW in the flat gradient
   int n_params;
+  int wst_off;                       // float offset of the weight staging buffer (WS kernels)
   float* part;                       // [gridDim.x][n_params]
   double* spart;                     // [gridDim.x][4]
   int64_t ntiles;
 };
 
-template <int R>
+// One layer's packed weights (n floats, n % 4 == 0, both ends 16-byte aligned) copied
+// into shared memory by asynchronous 16-byte copies, all in flight at once; the caller
+// runs stage_wait() and a block barrier before reading them.
+__device__ __forceinline__ void stage_weights(float* dst, const float* __restrict__ src, int n) {
+  for (int i = threadIdx.x; i < n / 4; i += blockDim.x) {
+    const unsigned d = static_cast<unsigned>(__cvta_generic_to_shared(dst + 4 * i));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(src + 4 * i)
+                 : "memory");
+  }
+  asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+
+__device__ __forceinline__ void stage_wait() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
+// WS: each layer's weights are staged in shared memory before its product (policies
+// whose weights do not stay in L1 beside one block's shared memory); the products read
+// the same values in the same order either way.
+template <int R, bool WS>
 __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant__ FusedLossArgs F) {
   constexpr int kLR = R, kLld = R + 4, kLanes = kLThreads / R;  // lanes per row in the head
   extern __shared__ float sm[];
@@ -273,6 +291,7 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
   float* dzA = acts + (size_t)F.act_off[L + 1] * kLld;     // two dZ buffers
   float* dzB = dzA + (size_t)F.dz_rows * kLld;
   float* gacc = dzB + (size_t)F.dz_rows * kLld;            // dW/db accumulators [n_params]
+  float* wst = sm + F.wst_off;                             // WS: one layer's weights
   for (int i = threadIdx.x; i < F.n_params; i += blockDim.x) gacc[i] = 0.0f;
   double st_pg = 0.0, st_v = 0.0, st_h = 0.0, st_cf = 0.0;
   const int D = a.dims[0];
@@ -282,6 +301,7 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
   for (int64_t tile = blockIdx.x; tile < F.ntiles; tile += gridDim.x) {
     const int64_t r0 = tile * kLR;
     __syncthreads();
+    if (WS) stage_weights(wst, F.Wt[0], a.dims[0] * F.npad[1]);  // lands during the gather
     // gather X [D][R]: thread (r, dq) reads features dq, dq + kLanes, ... of row r
     // (rows past n are zero and have zero dZ); consecutive threads take consecutive
     // rows, so for a fixed feature the reads are coalesced along the env axis
@@ -300,7 +320,14 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
     }
     __syncthreads();
     for (int l = 0; l < L; ++l) {
-      tile_gemm<R>(F.Wt[l], F.npad[l + 1], a.dims[l], a.dims[l + 1],
+      const float* Wf = F.Wt[l];
+      if (WS) {
+        if (l > 0) stage_weights(wst, F.Wt[l], a.dims[l] * F.npad[l + 1]);
+        stage_wait();
+        __syncthreads();
+        Wf = wst;
+      }
+      tile_gemm<R>(Wf, F.npad[l + 1], a.dims[l], a.dims[l + 1],
                    acts + (size_t)F.act_off[l] * kLld, acts + (size_t)F.act_off[l + 1] * kLld, 0,
                    a.b[l], a.act[l], nullptr,
                    F.dact_off[l + 1] >= 0 ? acts + (size_t)F.dact_off[l + 1] * kLld : nullptr);
@@ -379,6 +406,7 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
       const float* Hl = acts + (size_t)F.act_off[l] * kLld;
       float* gW = gacc + F.poff[l];
       float* gb = gW + (size_t)N * K;
+      if (WS && l > 0) stage_weights(wst, F.Wn[l], N * F.kpad[l]);  // lands during dW, db
       // dW += dZ^T H: 4 x 4 blocks of (j, k); the tile's rows are split over S
       // adjacent lanes (S > 1 for thin layers) whose partial sums are combined before
       // the block's accumulator is updated
@@ -411,7 +439,11 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
         float* dzn = (dz == dzA) ? dzB : dzA;
         // dZ_{l-1}[k][r] = sum_j W_l[j][k] dZ_l[j][r] * (1 - H_l[k][r]^2)
         const int pa = a.act[l - 1];  // activation whose derivative applies
-        tile_gemm<R>(F.Wn[l], F.kpad[l], N, K, dz, dzn, 1, nullptr, pa,
+        if (WS) {
+          stage_wait();
+          __syncthreads();
+        }
+        tile_gemm<R>(WS ? wst : F.Wn[l], F.kpad[l], N, K, dz, dzn, 1, nullptr, pa,
                      pa == 2 ? acts + (size_t)F.dact_off[l] * kLld : Hl, nullptr);
         __syncthreads();
         dz = dzn;
@@ -489,6 +521,8 @@ struct FusedPlan {
   int npad[SIMX_MAX_LAYERS + 1], kpad[SIMX_MAX_LAYERS + 1], act_off[SIMX_MAX_LAYERS + 2];
   int dact_off[SIMX_MAX_LAYERS + 1];
   int dz_rows, poff[SIMX_MAX_LAYERS], n_params, grid;
+  bool stage;
+  int wst_off;
   size_t smem, w_off[SIMX_MAX_LAYERS][2], part_off, spart_off, total;
 };
 
@@ -546,11 +580,30 @@ FusedPlan plan_r(const LossArgs& a, int R) {
   return p;
 }
 
-// 64-row tiles when two blocks of them fit in shared memory, else 32-row tiles.
+// 64-row tiles when two blocks of them fit in shared memory, else 32-row tiles.  A
+// plan with one block per SM stages each layer's weights in shared memory when the
+// largest layer fits beside it (then the weights no longer compete with the block's
+// shared memory for L1, where they missed on 128-wide layers).
 FusedPlan plan(const LossArgs& a) {
   const FusedPlan p64 = plan_r(a, 64);
   if (p64.ok && p64.smem <= 110 * 1024) return p64;
-  return plan_r(a, 32);
+  FusedPlan p = plan_r(a, 32);
+  if (!p.ok || p.smem <= 110 * 1024) return p;
+  int wmax = 0;
+  for (int l = 0; l < a.n_layers; ++l) {
+    const int f = a.dims[l] * p.npad[l + 1];
+    const int b = a.dims[l + 1] * p.kpad[l];
+    wmax = f > wmax ? f : wmax;
+    if (l > 0) wmax = b > wmax ? b : wmax;
+  }
+  const size_t off = (p.smem / 16) * 16 + (p.smem % 16 ? 16 : 0);  // 16-byte aligned
+  const size_t with = off + (size_t)wmax * sizeof(float);
+  if (with + 2 * 1024 <= 227 * 1024) {  // + the static statistics buffer and a margin
+    p.stage = true;
+    p.wst_off = (int)(off / sizeof(float));
+    p.smem = with;
+  }
+  return p;
 }
 }  // namespace
 
@@ -583,16 +636,14 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
   F.dz_rows = p.dz_rows;
   for (int l = 0; l < a.n_layers; ++l) F.poff[l] = p.poff[l];
   F.n_params = p.n_params;
+  F.wst_off = p.wst_off;
   F.part = reinterpret_cast<float*>(base + p.part_off);
   F.spart = reinterpret_cast<double*>(base + p.spart_off);
   F.ntiles = (a.n + p.R - 1) / p.R;
-  if (p.R == 64) {
-    cudaFuncSetAttribute(k_loss_fused<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
-    k_loss_fused<64><<<p.grid, kLThreads, p.smem, s>>>(F);
-  } else {
-    cudaFuncSetAttribute(k_loss_fused<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
-    k_loss_fused<32><<<p.grid, kLThreads, p.smem, s>>>(F);
-  }
+  auto k = p.R == 64 ? k_loss_fused<64, false>
+                     : (p.stage ? k_loss_fused<32, true> : k_loss_fused<32, false>);
+  cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+  k<<<p.grid, kLThreads, p.smem, s>>>(F);
   launch_loss_reduce(F.part, p.grid, p.n_params, F.spart, a, s);
   count_launches(a.n_layers + 1);
   return cudaGetLastError();
