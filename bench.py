@@ -50,6 +50,9 @@ def _args():
     p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
                    help="loss-gradient products: tf32 tensor cores (parity 1e-2) or fp32 (1e-5)")
     p.add_argument("--cpu-child", default=None, help=argparse.SUPPRESS)
+    p.add_argument("--minibatch-loss", default=None, metavar="WORKLOAD",
+                   help="time the PPO loss gradient on 8192-row minibatches of a workload's "
+                        "rollout (both precisions) and exit")
     return p.parse_args()
 
 
@@ -367,7 +370,7 @@ class Clocks:
 # DRAM bytes (read + write) of one k_rollout launch of the benchmark workload, from an
 # ncu capture of the current kernel; to be re-measured (or set to None) whenever the
 # rollout kernel changes.
-ROLLOUT_DRAM_BYTES = 116.2e6
+ROLLOUT_DRAM_BYTES = 114.7e6
 
 
 def _peaks():
@@ -430,6 +433,54 @@ def hbm_step_measure(simx, W, torch, E=65536, steps=100, warm=10) -> dict:
             "bytes_per_env_step": per, "achieved": gbs, "peak": hbm, "unit": "GB/s",
             "frac": gbs / hbm, "peak_source": "%s hbm_gbs" % src, "l2": l2,
             "timing": "CUDA graph of %d steps, replayed %d times, CUDA events" % (steps, reps)}
+
+
+def run_minibatch_loss(name: str, E: int = 256, steps: int = 20) -> None:
+    """The PPO loss gradient (Sec. 4.3) on 8192-row minibatches drawn from a rollout of
+    `name` (E envs x its horizon): median of `steps` timed calls per precision after 3
+    warm-up calls, CUDA events on the stream; one JSON line."""
+    import numpy as np
+    import torch
+
+    from paper_2607_05272_gb300 import build as B
+    from paper_2607_05272_gb300 import workloads as W
+    B.build()
+    from paper_2607_05272_gb300 import simx
+    cfg = W.CONFIGS[name](E)
+    H = W.HORIZON[name]
+    dims, hv = W.mlp_dims(name)
+    Ws, bs = W.policy_weights(name, dims, 1)
+    pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws],
+                      [torch.from_numpy(b).cuda() for b in bs], hv, W.mlp_acts(name))
+    sim = simx.Sim(cfg)
+    sim.reset(W.SEED[name])
+    buf = simx.alloc_rollout(E, sim.D, H, has_value=hv)
+    sim.rollout("sample", H, buf, pol)
+    n = E * H
+    rng = np.random.default_rng(1)
+    ret = torch.from_numpy(rng.standard_normal((H, E)).astype(np.float32)).cuda()
+    adv = torch.from_numpy(rng.standard_normal((H, E)).astype(np.float32)).cuda()
+    idx = torch.from_numpy(rng.permutation(n)[:8192].astype(np.int64)).cuda()
+    grad = torch.empty(pol.n_params, device="cuda")
+    stats = torch.empty(5, device="cuda")
+    ws = torch.empty(simx.ppo_loss_grad_workspace_size(pol, 8192), dtype=torch.uint8, device="cuda")
+    P = sum(w.size for w in Ws)
+    flop = 8192 * (6.0 * P - 2.0 * dims[0] * dims[1])
+    line = {"workload": name, "rows": 8192, "mlp": dims, "flop_per_call": flop}
+    for prec in ("fp32", "tf32"):
+        ts = []
+        for i in range(3 + steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            simx.ppo_loss_grad(pol, buf, ret, adv, idx, 8192, "ppo", 0.2, 0.5, 0.01, grad, stats,
+                               ws, precision=prec)
+            e1.record()
+            torch.cuda.synchronize()
+            if i >= 3:
+                ts.append(e0.elapsed_time(e1))
+        ms = statistics.median(ts)
+        line[prec] = {"ms": ms, "minibatches_per_s": 1e3 / ms, "tflops": flop / (ms * 1e-3) / 1e12}
+    print(json.dumps(line), flush=True)
 
 
 # --- replicas (N > 1): every rank simulates its own envs, no data-path collective -------
@@ -631,7 +682,7 @@ def run_gpu(a) -> None:
                 "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak,
                 "traffic": ROLLOUT_DRAM_BYTES,
                 "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one "
-                                  "k_rollout launch of this workload (5.8 MB + 110.4 MB)",
+                                  "k_rollout launch of this workload (5.0 MB + 109.7 MB)",
                 "peak_source": fp32_src}
     elif dom == 3:
         roof = roof_loss
@@ -680,6 +731,9 @@ def main():
         return
     if a.sweep_child:
         _sweep_child(a.sweep_child)
+        return
+    if a.minibatch_loss:
+        run_minibatch_loss(a.minibatch_loss)
         return
     if a.sweep:
         run_sweep(a)

@@ -356,6 +356,7 @@ static void base_args(simx_ctx* c, RolloutArgs& a) {
   a.G = choose_lanes(c->cfg.n_envs);
   a.threads = choose_threads(c->cfg.n_envs, a.G);
   act_layout((int)c->cfg.obs_dim, (int)a.n_actions, a.maxd4, a.apad);
+  a.bs_pad = 4;
   a.tr_gap = c->trace.gap;
   a.tr_type = c->trace.type;
   a.tr_cost = c->trace.cost;
@@ -417,6 +418,7 @@ static simx_status prepare_policy(simx_ctx* c, const simx_mlp* pol, int mode, Ro
       v = pack_mlp(pol, c->pack, a.mlp, s);
       if (v != SIMX_OK) return v;
       act_layout(mlp_maxdim(pol), (int)a.n_actions, a.maxd4, a.apad);
+      a.bs_pad = act_stride_pad(a.mlp, a.threads / a.G, a.threads);
       break;
     }
     case SIMX_POLICY_STATIC:

@@ -36,6 +36,7 @@ struct RolloutArgs {
   int apad;         // softmax scratch floats per env (multiple of 4)
   int G;            // lanes per env (8, 16 or 32)
   int threads;      // threads per block (64, 128 or 256)
+  int bs_pad;       // activation row stride = envs per block + bs_pad (see act_stride_pad)
   // trace replay (arrival_kind TRACE): gaps, types (or null), costs (or null), length
   const uint32_t* tr_gap;
   const uint8_t* tr_type;
@@ -56,6 +57,12 @@ struct PolicyArgs {
   int maxd4, apad;
   int G, threads;
 };
+
+// Padding of the block's activation rows: 4 (16-byte rows) when some layer takes the
+// 4-env tiles of mlp_tiles, else 1.  With 4 envs per block a stride of 8 floats put
+// every output group of a warp's stores in one bank (an 8-way conflict); an odd stride
+// spreads them over all 32.
+int act_stride_pad(const DevMlp& m, int B, int threads);
 
 cudaError_t launch_rollout(const RolloutArgs& a, cudaStream_t s);
 // step_thread.cu: one thread per env for the policy-free modes

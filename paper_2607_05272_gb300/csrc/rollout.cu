@@ -658,7 +658,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
   const Grp<G> g;
   const int B = (int)blockDim.x / G;
-  const int Bs = B + 4;  // row stride of the activation buffers
+  const int Bs = B + A.bs_pad;  // row stride of the activation buffers
   const uint32_t slot = threadIdx.x / G;
   const uint32_t env_raw = blockIdx.x * (uint32_t)B + slot;
   const bool live = env_raw < A.st.E;
@@ -933,12 +933,12 @@ __global__ void __launch_bounds__(kMaxThreads) k_observe(const __grid_constant__
   Srv L{0u, 0u, Pair{0u, 0u}, Pair{0u, 0u}};
   if (ROUTE) {
     if (g.gl < K) load_srv(A.st, env, g.gl, L);
-    observe_route<G>(c, g, s, L, ocol, B + 4);
+    observe_route<G>(c, g, s, L, ocol, B + A.bs_pad);
   } else {
     load_srv(A.st, env, 0, L);
-    observe_single<G>(c, g, s, L, ringb, ocol, B + 4);
+    observe_single<G>(c, g, s, L, ringb, ocol, B + A.bs_pad);
   }
-  write_obs<G>(g, ocol, B + 4, A.obs_dim, A.next_obs, A.next_ld, env);
+  write_obs<G>(g, ocol, B + A.bs_pad, A.obs_dim, A.next_obs, A.next_ld, env);
 }
 
 // Canonical state image of each env (header, servers, queue lengths, FIFO contents
@@ -1077,8 +1077,14 @@ static unsigned grid_for(int64_t n, int envs_per_block) {
   return (unsigned)((n + envs_per_block - 1) / envs_per_block);
 }
 
+int act_stride_pad(const DevMlp& m, int B, int threads) {
+  for (int l = 0; l < m.n_layers; ++l)
+    if ((B / 4) * ((m.dims[l + 1] + 3) / 4) >= threads) return 4;  // mlp_forward_block's test
+  return 1;
+}
+
 static size_t env_smem(const RolloutArgs& a, int B) {
-  return ((size_t)2 * a.maxd4 * (B + 4) + (size_t)a.apad * B) * sizeof(float);
+  return ((size_t)2 * a.maxd4 * (B + a.bs_pad) + (size_t)a.apad * B) * sizeof(float);
 }
 
 template <bool ROUTE, int G>
