@@ -256,11 +256,20 @@ __global__ void k_colsum(const float* __restrict__ dZ, int64_t n, int N, int64_t
 
 struct WsLayout {
   size_t X, H[SIMX_MAX_LAYERS], Dg[SIMX_MAX_LAYERS], Z, part, statp, total;
-  int splits, head_blocks;
+  int splits[SIMX_MAX_LAYERS], head_blocks;
 };
 
-static int dw_splits(int64_t n) {
-  int64_t s = (n + 2047) / 2048;  // >= 2048 rows per split
+// Row splits of layer l's dW product (output N x K tiles of 64 x 64, reduction over the
+// n rows): one per 2048 rows, and at least enough that the product launches two blocks
+// per SM, without going below 64 rows per split or above 512 splits.  A fixed function
+// of the sizes, so the summation order is the same on every run.
+static int dw_splits(int64_t n, int N, int K) {
+  const int64_t tiles = (int64_t)((N + kBM - 1) / kBM) * ((K + kBN - 1) / kBN);
+  int64_t s = (n + 2047) / 2048;
+  const int64_t fill = (2 * 152 + tiles - 1) / tiles;
+  if (s < fill) s = fill;
+  const int64_t most = (n + 63) / 64;
+  if (s > most) s = most;
   if (s > 512) s = 512;
   if (s < 1) s = 1;
   return (int)s;
@@ -280,13 +289,13 @@ static WsLayout layout(const LossArgs& a) {
   for (int l = 1; l < a.n_layers; ++l)  // GELU derivative of layer l's input
     w.Dg[l] = a.act[l - 1] == 2 ? take((size_t)n * a.dims[l] * sizeof(float)) : 0;
   w.Z = take((size_t)n * a.dims[a.n_layers] * sizeof(float));
-  w.splits = dw_splits(n);
-  size_t maxw = 0;
+  size_t maxw = 0;  // the largest split-partial buffer: splits x N x K floats
   for (int l = 0; l < a.n_layers; ++l) {
-    const size_t sz = (size_t)a.dims[l + 1] * a.dims[l];
+    w.splits[l] = dw_splits(n, a.dims[l + 1], a.dims[l]);
+    const size_t sz = (size_t)w.splits[l] * a.dims[l + 1] * a.dims[l];
     if (sz > maxw) maxw = sz;
   }
-  w.part = take((size_t)w.splits * maxw * sizeof(float));
+  w.part = take(maxw * sizeof(float));
   w.head_blocks = (int)((n + kHeadThreads - 1) / kHeadThreads);
   w.statp = take((size_t)w.head_blocks * 4 * sizeof(double));
   w.total = off;
@@ -370,7 +379,7 @@ cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
   const float* dZ = Z;
   for (int l = L - 1; l >= 0; --l) {
     const int K = a.dims[l], N = a.dims[l + 1];
-    const int splits = w.splits;
+    const int splits = w.splits[l];
     const int64_t kps = (n + splits - 1) / splits;
     // dW = dZ^T H_in : M = N, N = K, reduction over rows
     Gemm g{};
