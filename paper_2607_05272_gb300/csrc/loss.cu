@@ -39,11 +39,66 @@ struct Gemm {
   float* D;           // GELU derivative, D(i, j) = D[i * ldc + j]: written by EPI_BIAS_ACT, read by EPI_DACT
   int epi;
   int act;
+  int mode_a, mode_b;  // operand load modes (load_tile), set by gemm()
 };
 
+// One operand's 64 x 16 tile X(r, k) = X[r * sr + k * sk], r in [r0, r0 + 64) (rows of
+// A or columns of B), k in [k0, k0 + 16), four values per thread.  mode 1: 16-byte loads
+// along k (sk == 1, sr % 4 == 0, 16-byte base, k0 % 4 == 0); mode 2: 16-byte loads along
+// r (sr == 1, sk % 4 == 0, 16-byte base); they serve full tiles, element loads with
+// bounds serve the rest and modes 0 and 3 (consecutive threads walking r, or k when the
+// operand is contiguous along k).  v[c] goes to shared (kk[c], rr[c]).
+struct TileLoad {
+  float v[4];
+  int kk[4], rr[4];
+};
+
+__device__ __forceinline__ void load_tile(const float* __restrict__ X, int64_t sr, int64_t sk,
+                                          int mode, int64_t r0, int64_t rlim, int64_t k0,
+                                          int64_t ke, TileLoad& t) {
+  const int tid = threadIdx.x;
+  const bool full = r0 + kBM <= rlim && k0 + kBK <= ke;
+  if (full && mode == 1) {
+    const int r = tid / 4, kq = tid % 4;
+    const float4 q = *reinterpret_cast<const float4*>(X + (r0 + r) * sr + k0 + 4 * kq);
+    t.v[0] = q.x, t.v[1] = q.y, t.v[2] = q.z, t.v[3] = q.w;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) t.kk[c] = 4 * kq + c, t.rr[c] = r;
+  } else if (full && mode == 2) {
+    const int k = tid / 16, rq = tid % 16;
+    const float4 q = *reinterpret_cast<const float4*>(X + r0 + 4 * rq + (k0 + k) * sk);
+    t.v[0] = q.x, t.v[1] = q.y, t.v[2] = q.z, t.v[3] = q.w;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) t.kk[c] = k, t.rr[c] = 4 * rq + c;
+  } else {
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int e = tid + kGemmThreads * c;
+      int k, r;
+      if (mode == 1 || mode == 3) {  // consecutive threads walk k
+        k = e % kBK;
+        r = e / kBK;
+      } else {
+        r = e % kBM;
+        k = e / kBM;
+      }
+      const int64_t rg = r0 + r, kg = k0 + k;
+      t.v[c] = (rg < rlim && kg < ke) ? X[rg * sr + kg * sk] : 0.0f;
+      t.kk[c] = k;
+      t.rr[c] = r;
+    }
+  }
+}
+
+// C(i, j) = sum over k in [kb, ke) of A(i, k) B(k, j), k in increasing order (one fma
+// chain per output), then the epilogue.  64 x 64 output tile per block, each thread a
+// contiguous 4 x 4 block read from shared memory as 16-byte rows; the next k tile is
+// loaded into registers while the current one is multiplied (two shared buffers, one
+// barrier per tile).
 __global__ void __launch_bounds__(kGemmThreads) k_gemm(const __grid_constant__ Gemm g) {
-  __shared__ float As[kBK][kBM + 4];
-  __shared__ float Bs[kBK][kBN + 4];
+  constexpr int kLd = kBM + 4;
+  __shared__ __align__(16) float As[2][kBK][kLd];
+  __shared__ __align__(16) float Bs[2][kBK][kLd];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int64_t i0 = (int64_t)blockIdx.y * kBM, j0 = (int64_t)blockIdx.x * kBN;
   const int64_t kb = (int64_t)blockIdx.z * g.k_per_split;
@@ -53,54 +108,52 @@ __global__ void __launch_bounds__(kGemmThreads) k_gemm(const __grid_constant__ G
   for (int a = 0; a < 4; ++a)
 #pragma unroll
     for (int b = 0; b < 4; ++b) acc[a][b] = 0.0f;
+  TileLoad ta, tb;
+  int cur = 0;
+  if (kb < ke) {
+    load_tile(g.A, g.sai, g.sak, g.mode_a, i0, g.M, kb, ke, ta);
+    load_tile(g.B, g.sbj, g.sbk, g.mode_b, j0, g.N, kb, ke, tb);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      As[0][ta.kk[c]][ta.rr[c]] = ta.v[c];
+      Bs[0][tb.kk[c]][tb.rr[c]] = tb.v[c];
+    }
+  }
+  __syncthreads();
   for (int64_t k0 = kb; k0 < ke; k0 += kBK) {
-    for (int q = threadIdx.x; q < kBK * kBM; q += kGemmThreads) {
-      int kk, ii;
-      if (g.sak == 1) {  // contiguous along k: consecutive threads walk k
-        kk = q % kBK;
-        ii = q / kBK;
-      } else {
-        ii = q % kBM;
-        kk = q / kBM;
-      }
-      const int64_t i = i0 + ii, k = k0 + kk;
-      As[kk][ii] = (i < g.M && k < ke) ? g.A[i * g.sai + k * g.sak] : 0.0f;
+    const bool more = k0 + kBK < ke;
+    if (more) {
+      load_tile(g.A, g.sai, g.sak, g.mode_a, i0, g.M, k0 + kBK, ke, ta);
+      load_tile(g.B, g.sbj, g.sbk, g.mode_b, j0, g.N, k0 + kBK, ke, tb);
     }
-    for (int q = threadIdx.x; q < kBK * kBN; q += kGemmThreads) {
-      int kk, jj;
-      if (g.sbk == 1) {
-        kk = q % kBK;
-        jj = q / kBK;
-      } else {
-        jj = q % kBN;
-        kk = q / kBN;
-      }
-      const int64_t j = j0 + jj, k = k0 + kk;
-      Bs[kk][jj] = (j < g.N && k < ke) ? g.B[k * g.sbk + j * g.sbj] : 0.0f;
-    }
-    __syncthreads();
 #pragma unroll
     for (int kk = 0; kk < kBK; ++kk) {
-      float av[4], bv[4];
-#pragma unroll
-      for (int a = 0; a < 4; ++a) av[a] = As[kk][ty + 16 * a];
-#pragma unroll
-      for (int b = 0; b < 4; ++b) bv[b] = Bs[kk][tx + 16 * b];
+      const float4 av = *reinterpret_cast<const float4*>(&As[cur][kk][4 * ty]);
+      const float4 bv = *reinterpret_cast<const float4*>(&Bs[cur][kk][4 * tx]);
+      const float a4[4] = {av.x, av.y, av.z, av.w}, b4[4] = {bv.x, bv.y, bv.z, bv.w};
 #pragma unroll
       for (int a = 0; a < 4; ++a)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) acc[a][b] = __fmaf_rn(av[a], bv[b], acc[a][b]);
+        for (int b = 0; b < 4; ++b) acc[a][b] = __fmaf_rn(a4[a], b4[b], acc[a][b]);
+    }
+    if (more) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        As[cur ^ 1][ta.kk[c]][ta.rr[c]] = ta.v[c];
+        Bs[cur ^ 1][tb.kk[c]][tb.rr[c]] = tb.v[c];
+      }
     }
     __syncthreads();
+    cur ^= 1;
   }
   float* C = g.C + (int64_t)blockIdx.z * g.split_stride;
 #pragma unroll
   for (int a = 0; a < 4; ++a) {
-    const int64_t i = i0 + ty + 16 * a;
+    const int64_t i = i0 + 4 * ty + a;
     if (i >= g.M) continue;
 #pragma unroll
     for (int b = 0; b < 4; ++b) {
-      const int64_t j = j0 + tx + 16 * b;
+      const int64_t j = j0 + 4 * tx + b;
       if (j >= g.N) continue;
       float v = acc[a][b];
       if (g.epi == EPI_BIAS || g.epi == EPI_BIAS_ACT) v = __fadd_rn(v, g.bias[j]);
@@ -121,7 +174,21 @@ __global__ void __launch_bounds__(kGemmThreads) k_gemm(const __grid_constant__ G
   }
 }
 
-static cudaError_t gemm(const Gemm& g, int splits, cudaStream_t s) {
+// Load mode of an operand X(r, k) = X[r * sr + k * sk] for load_tile: 16-byte loads need
+// a 16-byte base, the other stride a multiple of 4, and (along k) tiles starting on a
+// multiple of 4, which k_per_split % 16 == 0 (or a single split from k = 0) provides.
+static int load_mode(const float* X, int64_t sr, int64_t sk, int64_t k_per_split, int splits) {
+  const bool aligned = (reinterpret_cast<uintptr_t>(X) & 15) == 0;
+  const bool k_ok = splits == 1 || k_per_split % 16 == 0;
+  if (aligned && sk == 1 && sr % 4 == 0 && k_ok) return 1;
+  if (aligned && sr == 1 && sk % 4 == 0) return 2;
+  return sk == 1 ? 3 : 0;  // element loads, walking the contiguous direction
+}
+
+static cudaError_t gemm(const Gemm& g0, int splits, cudaStream_t s) {
+  Gemm g = g0;
+  g.mode_a = load_mode(g.A, g.sai, g.sak, g.k_per_split, splits);
+  g.mode_b = load_mode(g.B, g.sbj, g.sbk, g.k_per_split, splits);
   const dim3 grid((unsigned)((g.N + kBN - 1) / kBN), (unsigned)((g.M + kBM - 1) / kBM), (unsigned)splits);
   k_gemm<<<grid, kGemmThreads, 0, s>>>(g);
   count_launches(1);
