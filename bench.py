@@ -44,7 +44,7 @@ def _args():
     p.add_argument("--no-hbm-step", action="store_true")
     p.add_argument("--sweep", action="store_true",
                    help="every configuration (c1-c5, c5 at every env count): one JSON line each")
-    p.add_argument("--sweep-configs", default="c1,c2,c3,c4,c5,c1p",
+    p.add_argument("--sweep-configs", default="c1,c2,c3,c4,c5,c1p,c3s,c3t",
                    help="comma-separated subset of the sweep's configurations")
     p.add_argument("--sweep-child", default=None, help=argparse.SUPPRESS)
     p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
@@ -233,7 +233,8 @@ def run_sweep(a) -> None:
     print(json.dumps({"fp32_fma_probe_tflops": fp["tflops"], "sms": fp["sms"], "hbm_gbs": hbm,
                       "hbm_source": src}), flush=True)
     cases = [("c1", 64, 10000, "sample"), ("c2", 4096, 512, "sample"), ("c3", 16384, 256, "sample"),
-             ("c4", 65536, 512, "sample"), ("c1p", 4096, 2000, "sample")]
+             ("c4", 65536, 512, "sample"), ("c1p", 4096, 2000, "sample"),
+             ("c3s", 4096, 256, "sample"), ("c3t", 16384, 256, "sample")]
     cases += [("c5", e, 1024, "argmax") for e in (1024, 4096, 16384, 65536, 262144, 1048576)]
     keep = set(a.sweep_configs.split(","))
     cases = [c for c in cases if c[0] in keep]
