@@ -471,9 +471,21 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
   }
 }
 
-// Transposed (forward) and row-major padded (backward) copies of each W_l.
-__global__ void k_pack_loss_w(const float* __restrict__ W, int N, int K, int npad, int kpad,
-                              float* __restrict__ Wt, float* __restrict__ Wn) {
+// Transposed (forward) and row-major padded (backward) copies of each W_l; blockIdx.y
+// is the layer, so one launch packs them all.
+struct PackArgs {
+  const float* W[SIMX_MAX_LAYERS];
+  float* Wt[SIMX_MAX_LAYERS];
+  float* Wn[SIMX_MAX_LAYERS];
+  int N[SIMX_MAX_LAYERS], K[SIMX_MAX_LAYERS], npad[SIMX_MAX_LAYERS], kpad[SIMX_MAX_LAYERS];
+};
+
+__global__ void k_pack_loss_w(const __grid_constant__ PackArgs P) {
+  const int l = blockIdx.y;
+  const float* __restrict__ W = P.W[l];
+  float* __restrict__ Wt = P.Wt[l];
+  float* __restrict__ Wn = P.Wn[l];
+  const int N = P.N[l], K = P.K[l], npad = P.npad[l], kpad = P.kpad[l];
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < K * npad) {
     const int k = i / npad, j = i % npad;
@@ -616,16 +628,25 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
   char* base = static_cast<char*>(ws);
   FusedLossArgs F{};
   F.a = a;
+  PackArgs pk{};
+  int nmax = 0;
   for (int l = 0; l < a.n_layers; ++l) {
     float* Wt = reinterpret_cast<float*>(base + p.w_off[l][0]);
     float* Wn = reinterpret_cast<float*>(base + p.w_off[l][1]);
     const int n = a.dims[l] * p.npad[l + 1] > a.dims[l + 1] * p.kpad[l] ? a.dims[l] * p.npad[l + 1]
                                                                          : a.dims[l + 1] * p.kpad[l];
-    k_pack_loss_w<<<(n + 255) / 256, 256, 0, s>>>(a.W[l], a.dims[l + 1], a.dims[l], p.npad[l + 1],
-                                                  p.kpad[l], Wt, Wn);
+    nmax = n > nmax ? n : nmax;
+    pk.W[l] = a.W[l];
+    pk.Wt[l] = Wt;
+    pk.Wn[l] = Wn;
+    pk.N[l] = a.dims[l + 1];
+    pk.K[l] = a.dims[l];
+    pk.npad[l] = p.npad[l + 1];
+    pk.kpad[l] = p.kpad[l];
     F.Wt[l] = Wt;
     F.Wn[l] = Wn;
   }
+  k_pack_loss_w<<<dim3((unsigned)((nmax + 255) / 256), (unsigned)a.n_layers), 256, 0, s>>>(pk);
   for (int l = 0; l <= a.n_layers; ++l) {
     F.npad[l] = p.npad[l];
     F.kpad[l] = p.kpad[l];
@@ -645,7 +666,7 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
   k<<<p.grid, kLThreads, p.smem, s>>>(F);
   launch_loss_reduce(F.part, p.grid, p.n_params, F.spart, a, s);
-  count_launches(a.n_layers + 1);
+  count_launches(2);
   return cudaGetLastError();
 }
 
