@@ -418,7 +418,7 @@ static simx_status prepare_policy(simx_ctx* c, const simx_mlp* pol, int mode, Ro
       v = pack_mlp(pol, c->pack, a.mlp, s);
       if (v != SIMX_OK) return v;
       act_layout(mlp_maxdim(pol), (int)a.n_actions, a.maxd4, a.apad);
-      a.bs_pad = act_stride_pad(a.mlp, a.threads / a.G, a.threads);
+      a.bs_pad = act_stride_pad(a.mlp, 32 / a.G, 32);  // k_rollout's warp-local forward
       break;
     }
     case SIMX_POLICY_STATIC:

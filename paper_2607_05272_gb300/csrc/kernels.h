@@ -59,7 +59,7 @@ struct PolicyArgs {
 };
 
 // Padding of the block's activation rows: 4 (16-byte rows) when some layer takes the
-// 4-env tiles of mlp_tiles, else 1.  With 4 envs per block a stride of 8 floats put
+// 4-env tiles of mlp_tiles (B envs shared by `threads` threads), else 1.  With 4 envs per block a stride of 8 floats put
 // every output group of a warp's stores in one bank (an 8-way conflict); an odd stride
 // spreads them over all 32.
 int act_stride_pad(const DevMlp& m, int B, int threads);

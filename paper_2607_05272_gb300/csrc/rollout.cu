@@ -700,7 +700,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
     float logp = 0.0f, value = 0.0f;
     int a = 0;
     if (use_mlp) {
-      const float* Z = mlp_forward_block(A.mlp, X0, X1, B, Bs);
+      const float* Z = mlp_forward_warp(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G));
       if (live)
         a = sample_action<G>(A.mlp, Z + slot, Bs, scratch, A.policy_mode, A.key0, A.key1, s.tg,
                              env, logp, value, g);
@@ -1079,7 +1079,7 @@ static unsigned grid_for(int64_t n, int envs_per_block) {
 
 int act_stride_pad(const DevMlp& m, int B, int threads) {
   for (int l = 0; l < m.n_layers; ++l)
-    if ((B / 4) * ((m.dims[l + 1] + 3) / 4) >= threads) return 4;  // mlp_forward_block's test
+    if ((B / 4) * ((m.dims[l + 1] + 3) / 4) >= threads) return 4;  // the forward's TE test
   return 1;
 }
 

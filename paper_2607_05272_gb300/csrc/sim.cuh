@@ -114,13 +114,15 @@ static __device__ __noinline__ void gelu_tile(float* Y, int ld, int j0, int N, i
 
 // act: the activation after this layer: -1 none (output layer), 0 tanh, 1 identity,
 // 2 GELU (det_gelu).
+// Threads tid, tid + nthr, ... of the cooperating group take the tiles.
 template <int TE>
 __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
                                           const float* __restrict__ bias, int K, int N, int Npad,
-                                          const float* X, float* Y, int B, int ld, int act) {
+                                          const float* X, float* Y, int B, int ld, int act,
+                                          int tid, int nthr) {
   const int neb = B / TE, nob = (N + 3) / 4;
   const int ntiles = neb * nob;
-  for (int tile = threadIdx.x; tile < ntiles; tile += blockDim.x) {
+  for (int tile = tid; tile < ntiles; tile += nthr) {
     const int eb = tile % neb, ob = tile / neb;
     float acc[TE][4];
 #pragma unroll
@@ -187,9 +189,36 @@ __device__ __forceinline__ float* mlp_forward_block(const DevMlp& m, float* X0, 
     const int K = m.dims[l], N = m.dims[l + 1], Np = m.npad[l + 1];
     const int th = m.act[l];
     // 4-env tiles when they keep every thread busy, otherwise 1-env tiles
-    if ((B / 4) * ((N + 3) / 4) >= (int)blockDim.x) mlp_tiles<4>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th);
-    else mlp_tiles<1>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th);
+    if ((B / 4) * ((N + 3) / 4) >= (int)blockDim.x)
+      mlp_tiles<4>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th, threadIdx.x, blockDim.x);
+    else
+      mlp_tiles<1>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th, threadIdx.x, blockDim.x);
     __syncthreads();
+    float* t = in;
+    in = out;
+    out = t;
+  }
+  return in;
+}
+
+// The same forward for the Bw envs (columns col0 .. col0 + Bw - 1) whose lanes form this
+// warp: only the warp's own lanes take its tiles, so warp barriers replace block
+// barriers.  Every output is still the K-ordered fma chain.  Returns the buffer (not
+// offset by col0) holding the last layer.
+__device__ __forceinline__ float* mlp_forward_warp(const DevMlp& m, float* X0, float* X1, int Bw,
+                                                  int ld, int col0) {
+  float* in = X0;
+  float* out = X1;
+  const int lane = (int)(threadIdx.x & 31u);
+  __syncwarp();
+  for (int l = 0; l < m.n_layers; ++l) {
+    const int K = m.dims[l], N = m.dims[l + 1], Np = m.npad[l + 1];
+    const int th = m.act[l];
+    if ((Bw / 4) * ((N + 3) / 4) >= 32)
+      mlp_tiles<4>(m.Wt[l], m.bias[l], K, N, Np, in + col0, out + col0, Bw, ld, th, lane, 32);
+    else
+      mlp_tiles<1>(m.Wt[l], m.bias[l], K, N, Np, in + col0, out + col0, Bw, ld, th, lane, 32);
+    __syncwarp();
     float* t = in;
     in = out;
     out = t;
