@@ -346,41 +346,42 @@ __device__ void next_arrival(const RolloutArgs& A, const Grp<G>& g, uint32_t env
         return;
       }
     }
-  }
-  // DIURNAL: constant rate inside a 500 ms epoch; a gap crossing the epoch end is
-  // discarded and redrawn from the epoch end at the next epoch's rate.  Every lane
-  // of the group computes the same values.
-  for (;;) {
-    if (++s.events > kEventCap) {
-      s.status |= kStEvent;
-      return;
+  } else {
+    // DIURNAL: constant rate inside a 500 ms epoch; a gap crossing the epoch end is
+    // discarded and redrawn from the epoch end at the next epoch's rate.  Every lane
+    // of the group computes the same values.
+    for (;;) {
+      if (++s.events > kEventCap) {
+        s.status |= kStEvent;
+        return;
+      }
+      if (s.ep_cached != s.ep) {
+        const U4 we = philox(s.ep, env, kStreamEpoch, 0u, A.key0, A.key1);
+        s.ep_factor = det_exp(__fmul_rn(c.burst_sigma, normal01(we.x, we.y)));
+        s.ep_cached = s.ep;
+      }
+      const float rate = __fmul_rn(c.diurnal_rate[(s.ep + s.epo) % c.diurnal_len], s.ep_factor);
+      const float mean = __fdiv_rn(1.0e6f, rate);
+      const U4 w = philox(s.cj, env, kStreamArrival, 0u, A.key0, A.key1);
+      const uint32_t gap = duration_us(__fmul_rn(mean, expo1(w.x)));
+      s.cj += 1u;
+      const uint64_t end = (uint64_t)(s.ep + 1u) * (uint64_t)c.epoch_us;
+      if ((uint64_t)s.cT + gap < end) {
+        s.cT = add_time(s.cT, gap, s.status);
+        s.pt = s.cT;
+        s.pty = req_type(c, w.y);
+        s.pc = ((int32_t)s.pty == c.cost_type) ? req_cost(c, w.w) : 0u;
+        s.narr += 1u;
+        return;
+      }
+      if (end >= kTimeLimit) {
+        s.status |= kStTime;
+        s.cT = kTimeLimit;
+      } else {
+        s.cT = (uint32_t)end;
+      }
+      s.ep += 1u;
     }
-    if (s.ep_cached != s.ep) {
-      const U4 we = philox(s.ep, env, kStreamEpoch, 0u, A.key0, A.key1);
-      s.ep_factor = det_exp(__fmul_rn(c.burst_sigma, normal01(we.x, we.y)));
-      s.ep_cached = s.ep;
-    }
-    const float rate = __fmul_rn(c.diurnal_rate[(s.ep + s.epo) % c.diurnal_len], s.ep_factor);
-    const float mean = __fdiv_rn(1.0e6f, rate);
-    const U4 w = philox(s.cj, env, kStreamArrival, 0u, A.key0, A.key1);
-    const uint32_t gap = duration_us(__fmul_rn(mean, expo1(w.x)));
-    s.cj += 1u;
-    const uint64_t end = (uint64_t)(s.ep + 1u) * (uint64_t)c.epoch_us;
-    if ((uint64_t)s.cT + gap < end) {
-      s.cT = add_time(s.cT, gap, s.status);
-      s.pt = s.cT;
-      s.pty = req_type(c, w.y);
-      s.pc = ((int32_t)s.pty == c.cost_type) ? req_cost(c, w.w) : 0u;
-      s.narr += 1u;
-      return;
-    }
-    if (end >= kTimeLimit) {
-      s.status |= kStTime;
-      s.cT = kTimeLimit;
-    } else {
-      s.cT = (uint32_t)end;
-    }
-    s.ep += 1u;
   }
 }
 
