@@ -418,7 +418,12 @@ static simx_status prepare_policy(simx_ctx* c, const simx_mlp* pol, int mode, Ro
       v = pack_mlp(pol, c->pack, a.mlp, s);
       if (v != SIMX_OK) return v;
       act_layout(mlp_maxdim(pol), (int)a.n_actions, a.maxd4, a.apad);
-      a.bs_pad = act_stride_pad(a.mlp, 32 / a.G, 32);  // k_rollout's warp-local forward
+      // k_rollout's forward: warp-local for narrow policies at 16 or 32 lanes per env in
+      // SINGLE mode (each warp then loads every weight row, which wide layers cannot
+      // afford); the kernel has that variant only there
+      a.mlp_warp = (!route && a.G >= 16 && mlp_maxdim(pol) <= 64) ? 1 : 0;
+      a.bs_pad = a.mlp_warp ? act_stride_pad(a.mlp, 32 / a.G, 32)
+                            : act_stride_pad(a.mlp, a.threads / a.G, a.threads);
       break;
     }
     case SIMX_POLICY_STATIC:

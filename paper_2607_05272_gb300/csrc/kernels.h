@@ -37,6 +37,7 @@ struct RolloutArgs {
   int G;            // lanes per env (8, 16 or 32)
   int threads;      // threads per block (64, 128 or 256)
   int bs_pad;       // activation row stride = envs per block + bs_pad (see act_stride_pad)
+  int mlp_warp;     // 1: each warp runs the policy for its own envs (see mlp_forward_warp)
   // trace replay (arrival_kind TRACE): gaps, types (or null), costs (or null), length
   const uint32_t* tr_gap;
   const uint8_t* tr_type;

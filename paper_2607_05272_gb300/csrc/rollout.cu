@@ -653,7 +653,7 @@ __device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int B
 // maxd4 x B floats (feature-major) and a softmax scratch of apad floats per env.
 // Every lane stays alive to the end (groups past the last env do no work) so that
 // warps reconverge at each phase and the block can run the MLP together.
-template <bool ROUTE, int G, bool TR>
+template <bool ROUTE, int G, bool TR, bool WARP>
 __global__ void __launch_bounds__(kMaxThreads, min_blocks<G>())
 k_rollout(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
@@ -701,7 +701,11 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
     float logp = 0.0f, value = 0.0f;
     int a = 0;
     if (use_mlp) {
-      const float* Z = mlp_forward_warp(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G));
+      // WARP: each warp runs the policy for its own 1-2 envs (narrow policies); else
+      // block-wide, whose warps share each weight row instead of each loading it.  A
+      // template parameter: both forwards in one kernel slowed the narrow case by 16 %.
+      const float* Z = WARP ? mlp_forward_warp(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G))
+                            : mlp_forward_block(A.mlp, X0, X1, B, Bs);
       if (live)
         a = sample_action<G>(A.mlp, Z + slot, Bs, scratch, A.policy_mode, A.key0, A.key1, s.tg,
                              env, logp, value, g);
@@ -1092,7 +1096,10 @@ template <bool ROUTE, int G>
 static cudaError_t rollout_t(const RolloutArgs& a, cudaStream_t s) {
   const int B = a.threads / G;
   const size_t sh = env_smem(a, B);
-  auto k = a.cfg.arrival_kind == SIMX_ARR_TRACE ? k_rollout<ROUTE, G, true> : k_rollout<ROUTE, G, false>;
+  const bool tr = a.cfg.arrival_kind == SIMX_ARR_TRACE;
+  auto k = tr ? k_rollout<ROUTE, G, true, false> : k_rollout<ROUTE, G, false, false>;
+  if constexpr (!ROUTE && G >= 16)  // the warp-local forward is instantiated where it applies
+    if (a.mlp_warp) k = tr ? k_rollout<ROUTE, G, true, true> : k_rollout<ROUTE, G, false, true>;
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
   k<<<grid_for(a.st.E, B), a.threads, sh, s>>>(a);
   count_launches(1);
