@@ -371,7 +371,7 @@ class Clocks:
 # DRAM bytes (read + write) of one k_rollout launch of the benchmark workload, from an
 # ncu capture of the current kernel; to be re-measured (or set to None) whenever the
 # rollout kernel changes.
-ROLLOUT_DRAM_BYTES = 114.7e6
+ROLLOUT_DRAM_BYTES = 123.8e6
 
 
 def _peaks():
@@ -683,7 +683,7 @@ def run_gpu(a) -> None:
                 "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak,
                 "traffic": ROLLOUT_DRAM_BYTES,
                 "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one "
-                                  "k_rollout launch of this workload (5.0 MB + 109.7 MB)",
+                                  "k_rollout launch of this workload (10.0 MB + 113.8 MB)",
                 "peak_source": fp32_src}
     elif dom == 3:
         roof = roof_loss
