@@ -280,7 +280,9 @@ simx_status sim_step_batched(simx_ctx* ctx, const int32_t* d_actions, const simx
 /*
  * Collect `horizon` decision steps of every env into `out` in one persistent launch:
  * observation, fused policy forward, action, reward, done (Sec. 4.1, Sec. 4.2).
- * Equivalent, bit for bit, to `horizon` calls of sim_step_batched.
+ * Equivalent, bit for bit, to `horizon` calls of sim_step_batched.  The context repacks
+ * the policy into a buffer of its own, grown when a larger policy is passed: a CUDA graph
+ * that captured a call stays valid while no larger policy is passed to the context.
  */
 simx_status rollout_collect(simx_ctx* ctx, const simx_mlp* pol, int policy_mode,
                             int32_t horizon, const simx_rollout* out, void* stream);
@@ -291,11 +293,25 @@ simx_status rollout_collect(simx_ctx* ctx, const simx_mlp* pol, int policy_mode,
  * POLICY Philox counter, so this reproduces the actions the rollout drew.
  * Outputs (any may be NULL): d_logits [n_actions][ld], d_value [ld], d_action [ld] u8,
  * d_logp [ld].  policy_mode: SAMPLE or ARGMAX.
+ * The policy is repacked into a buffer the library keeps per device: calls on one device
+ * must not overlap on the GPU, and a call with a larger policy replaces the buffer (a
+ * CUDA graph that captured an earlier call would then use freed memory).  For concurrent
+ * streams or graph capture use policy_forward_ws.
  */
 simx_status policy_forward(const simx_mlp* pol, const float* d_obs, int64_t ld, int64_t n,
                            int policy_mode, uint64_t seed, uint32_t step, uint32_t env_base,
                            float* d_logits, float* d_value, uint8_t* d_action, float* d_logp,
                            void* stream);
+
+/* policy_forward with a caller-owned device workspace of policy_forward_workspace_size(pol)
+   bytes (16-byte aligned) for the repacked policy: no state shared between calls, so calls
+   may run on concurrent streams and inside captured CUDA graphs (the workspace must
+   outlive the graph).  SIMX_EINVAL for a short, misaligned or NULL workspace. */
+size_t policy_forward_workspace_size(const simx_mlp* pol);
+simx_status policy_forward_ws(const simx_mlp* pol, const float* d_obs, int64_t ld, int64_t n,
+                              int policy_mode, uint64_t seed, uint32_t step, uint32_t env_base,
+                              float* d_logits, float* d_value, uint8_t* d_action, float* d_logp,
+                              void* d_workspace, size_t workspace_bytes, void* stream);
 
 /*
  * Returns and advantages over a [T][E] buffer (Sec. 4.3):

@@ -507,28 +507,27 @@ simx_status rollout_collect(simx_ctx* c, const simx_mlp* pol, int policy_mode, i
   return SIMX_OK;
 }
 
-simx_status policy_forward(const simx_mlp* pol, const float* d_obs, int64_t ld, int64_t n,
-                           int policy_mode, uint64_t seed, uint32_t step, uint32_t env_base,
-                           float* d_logits, float* d_value, uint8_t* d_action, float* d_logp,
-                           void* stream) {
-  if (!d_obs) return fail(SIMX_EINVAL, "d_obs is NULL");
-  if (n < 0 || ld < n) return fail(SIMX_EINVAL, "n %lld, ld %lld", (long long)n, (long long)ld);
-  if (policy_mode != SIMX_POLICY_SAMPLE && policy_mode != SIMX_POLICY_ARGMAX)
-    return fail(SIMX_EINVAL, "policy_forward supports SAMPLE and ARGMAX");
-  simx_status v = validate_mlp(pol, 0, 0);
-  if (v != SIMX_OK) return v;
-  if (d_value && !pol->has_value) return fail(SIMX_EINVAL, "d_value given but the policy has no value row");
-  if (n == 0) return SIMX_OK;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev < 0 || dev >= 64) return fail(SIMX_EINVAL, "device %d", dev);
-  std::lock_guard<std::mutex> lk(g_pf_mu);
+// Floats of a policy repacked in the kernels' layout (pack_mlp).
+static size_t packed_floats(const simx_mlp* m) {
+  size_t need = 0;
+  for (int l = 0; l < m->n_layers; ++l) {
+    const int np = round_up(m->dims[l + 1], 4);
+    need += (size_t)m->dims[l] * np + np;
+  }
+  return need;
+}
+
+// policy_forward with the repack buffer P (the library's per-device one, or a caller's).
+static simx_status policy_forward_into(Packed& P, const simx_mlp* pol, const float* d_obs,
+                                       int64_t ld, int64_t n, int policy_mode, uint64_t seed,
+                                       uint32_t step, uint32_t env_base, float* d_logits,
+                                       float* d_value, uint8_t* d_action, float* d_logp,
+                                       cudaStream_t s) {
   PolicyArgs p;
   std::memset(&p, 0, sizeof(p));
-  const cudaStream_t s = (cudaStream_t)stream;
   p.G = choose_lanes(n);
   p.threads = choose_threads(n, p.G);
-  v = pack_mlp(pol, g_pf_pack[dev], p.mlp, s);
+  simx_status v = pack_mlp(pol, P, p.mlp, s);
   if (v != SIMX_OK) return v;
   act_layout(mlp_maxdim(pol), p.mlp.n_actions, p.maxd4, p.apad);
   p.obs = d_obs;
@@ -546,6 +545,54 @@ simx_status policy_forward(const simx_mlp* pol, const float* d_obs, int64_t ld, 
   cudaError_t e = launch_policy_forward(p, s);
   if (e != cudaSuccess) return cuda_fail(e, "policy_forward launch");
   return SIMX_OK;
+}
+
+static simx_status policy_forward_check(const simx_mlp* pol, const float* d_obs, int64_t ld,
+                                        int64_t n, int policy_mode, const float* d_value) {
+  if (!d_obs) return fail(SIMX_EINVAL, "d_obs is NULL");
+  if (n < 0 || ld < n) return fail(SIMX_EINVAL, "n %lld, ld %lld", (long long)n, (long long)ld);
+  if (policy_mode != SIMX_POLICY_SAMPLE && policy_mode != SIMX_POLICY_ARGMAX)
+    return fail(SIMX_EINVAL, "policy_forward supports SAMPLE and ARGMAX");
+  simx_status v = validate_mlp(pol, 0, 0);
+  if (v != SIMX_OK) return v;
+  if (d_value && !pol->has_value) return fail(SIMX_EINVAL, "d_value given but the policy has no value row");
+  return SIMX_OK;
+}
+
+simx_status policy_forward(const simx_mlp* pol, const float* d_obs, int64_t ld, int64_t n,
+                           int policy_mode, uint64_t seed, uint32_t step, uint32_t env_base,
+                           float* d_logits, float* d_value, uint8_t* d_action, float* d_logp,
+                           void* stream) {
+  simx_status v = policy_forward_check(pol, d_obs, ld, n, policy_mode, d_value);
+  if (v != SIMX_OK || n == 0) return v;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) return fail(SIMX_EINVAL, "device %d", dev);
+  std::lock_guard<std::mutex> lk(g_pf_mu);
+  return policy_forward_into(g_pf_pack[dev], pol, d_obs, ld, n, policy_mode, seed, step, env_base,
+                             d_logits, d_value, d_action, d_logp, (cudaStream_t)stream);
+}
+
+size_t policy_forward_workspace_size(const simx_mlp* pol) {
+  if (!pol || pol->n_layers < 1 || pol->n_layers > SIMX_MAX_LAYERS) return 0;
+  return packed_floats(pol) * sizeof(float);
+}
+
+simx_status policy_forward_ws(const simx_mlp* pol, const float* d_obs, int64_t ld, int64_t n,
+                              int policy_mode, uint64_t seed, uint32_t step, uint32_t env_base,
+                              float* d_logits, float* d_value, uint8_t* d_action, float* d_logp,
+                              void* d_workspace, size_t workspace_bytes, void* stream) {
+  simx_status v = policy_forward_check(pol, d_obs, ld, n, policy_mode, d_value);
+  if (v != SIMX_OK || n == 0) return v;
+  const size_t need = packed_floats(pol) * sizeof(float);
+  if (!d_workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(d_workspace) & 15))
+    return fail(SIMX_EINVAL, "workspace of %zu bytes (16-byte aligned) needed, %zu given", need,
+                workspace_bytes);
+  Packed P;  // the caller's buffer: large enough, so pack_mlp neither frees nor allocates
+  P.buf = static_cast<float*>(d_workspace);
+  P.cap = workspace_bytes / sizeof(float);
+  return policy_forward_into(P, pol, d_obs, ld, n, policy_mode, seed, step, env_base, d_logits,
+                             d_value, d_action, d_logp, (cudaStream_t)stream);
 }
 
 simx_status compute_returns_gae(const float* d_rew, const float* d_val, const uint8_t* d_done,

@@ -97,6 +97,8 @@ SIGNATURES = [
     ("sim_step_batched", C.c_int, [P, P, P, C.c_int, P, I64, P, P, P, P, P]),
     ("rollout_collect", C.c_int, [P, P, C.c_int, I32, P, P]),
     ("policy_forward", C.c_int, [P, P, I64, I64, C.c_int, U64, U32, U32, P, P, P, P, P]),
+    ("policy_forward_workspace_size", SZ, [P]),
+    ("policy_forward_ws", C.c_int, [P, P, I64, I64, C.c_int, U64, U32, U32, P, P, P, P, P, SZ, P]),
     ("compute_returns_gae", C.c_int, [P, P, P, P, I64, I64, I64, F, F, P, P, P]),
     ("returns_baseline_workspace_size", SZ, [I64]),
     ("returns_baseline", C.c_int, [P, I64, P, P, P, SZ, P]),
@@ -327,12 +329,25 @@ def alloc_rollout(E: int, D: int, H: int, has_value: bool = False, trace: bool =
     return buf
 
 
+def policy_forward_workspace_size(policy: Policy) -> int:
+    return lib().policy_forward_workspace_size(C.byref(policy.c))
+
+
 def policy_forward(policy: Policy, obs, n: int, policy_mode: str, seed: int, step: int,
                    env_base: int = 0, logits=None, value=None, action=None, logp=None,
-                   stream=None):
-    _check(lib().policy_forward(C.byref(policy.c), _ptr(obs), obs.shape[-1], n,
-                                POLICY[policy_mode], seed, step, env_base, _ptr(logits),
-                                _ptr(value), _ptr(action), _ptr(logp), _stream(stream)))
+                   stream=None, workspace=None):
+    """policy_forward, or policy_forward_ws when a device workspace (uint8 tensor of
+    policy_forward_workspace_size bytes) is given: needed for concurrent streams and for
+    CUDA-graph capture."""
+    if workspace is None:
+        _check(lib().policy_forward(C.byref(policy.c), _ptr(obs), obs.shape[-1], n,
+                                    POLICY[policy_mode], seed, step, env_base, _ptr(logits),
+                                    _ptr(value), _ptr(action), _ptr(logp), _stream(stream)))
+        return
+    _check(lib().policy_forward_ws(C.byref(policy.c), _ptr(obs), obs.shape[-1], n,
+                                   POLICY[policy_mode], seed, step, env_base, _ptr(logits),
+                                   _ptr(value), _ptr(action), _ptr(logp), _ptr(workspace),
+                                   workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def compute_returns_gae(rew, done, gamma: float, lam: float, ret, adv=None, val=None,

@@ -64,6 +64,9 @@ class Trainer:
         self.adv = torch.empty((horizon, E), device="cuda")
         self.last = torch.zeros(E, device="cuda")  # V of the state after the rollout
         self.obs_next = torch.empty((self.sim.D, E), device="cuda")
+        # the bootstrap forward's own repack buffer (captured graphs keep its address)
+        self.pf_ws = torch.empty(simx.policy_forward_workspace_size(self.policy),
+                                 dtype=torch.uint8, device="cuda")
         self.n_rows = E * horizon
         rows = self.n_rows if algo == "reinforce" else min(minibatch, self.n_rows)
         self.loss_ws = torch.empty(simx.ppo_loss_grad_workspace_size(self.policy, rows),
@@ -116,7 +119,7 @@ class Trainer:
         if self.has_value:  # bootstrap value of each env's current state
             self.sim.observe(self.obs_next)
             simx.policy_forward(self.policy, self.obs_next, self.E, "argmax", 0, 0,
-                                value=self.last)
+                                value=self.last, workspace=self.pf_ws)
         if self.algo == "reinforce":
             if self.has_value:  # learned baseline: A = G - V (GAE with lambda = 1)
                 simx.compute_returns_gae(b["reward"], b["done"], self.gamma, 1.0, self.ret,

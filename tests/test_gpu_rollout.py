@@ -288,7 +288,9 @@ def test_trace_call_order_and_arguments():
     sim.close()
 
 
-def test_policy_forward_matches_oracle():
+@pytest.mark.parametrize("with_ws", [False, True])
+def test_policy_forward_matches_oracle(with_ws):
+    """Both entries (the library's repack buffer, or a caller workspace) against the oracle."""
     simx = _simx()
     for name, mode in (("c3", "sample"), ("c4", "argmax"), ("c2", "sample"), ("c1p", "sample")):
         pol, host = _policy(simx, name, seed=3)
@@ -301,8 +303,16 @@ def test_policy_forward_matches_oracle():
         act = torch.empty(n, dtype=torch.uint8, device="cuda")
         lp = torch.empty(n, device="cuda")
         val = torch.empty(n, device="cuda") if host[2] else None
+        ws = None
+        if with_ws:
+            ws = torch.empty(simx.policy_forward_workspace_size(pol), dtype=torch.uint8,
+                             device="cuda")
+            with pytest.raises(simx.SimxError) as e:   # one byte short
+                simx.policy_forward(pol, torch.from_numpy(obs).cuda(), n, mode, 99, 5,
+                                    env_base=100, logits=logits, workspace=ws[:-1])
+            assert e.value.status == simx.EINVAL
         simx.policy_forward(pol, torch.from_numpy(obs).cuda(), n, mode, 99, 5, env_base=100,
-                            logits=logits, value=val, action=act, logp=lp)
+                            logits=logits, value=val, action=act, logp=lp, workspace=ws)
         torch.cuda.synchronize()
         for i in range(n):
             lg, v, a, l = oracle.policy(host, obs[:, i], ORC_MODE[mode], 99, 5, 100 + i)
