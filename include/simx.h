@@ -319,7 +319,8 @@ simx_status policy_forward_ws(const simx_mlp* pol, const float* d_obs, int64_t l
  *             (d_ret gets G; d_adv may be NULL);
  *   lam >= 0: GAE  delta_t = r_t + gamma (1 - d_t) V_{t+1} - V_t, V_T = last_value,
  *             A_t = delta_t + gamma lam (1 - d_t) A_{t+1}, R_t = A_t + V_t.
- * d_val is required for GAE; d_last_val [E] may be NULL (zeros).  ld >= E.
+ * d_val is required for GAE; d_last_val [E] may be NULL (zeros).  ld >= E.  T == 0 or
+ * E == 0 is an empty problem: SIMX_OK, nothing touched (its buffers may be NULL).
  */
 simx_status compute_returns_gae(const float* d_rew, const float* d_val, const uint8_t* d_done,
                                 const float* d_last_val, int64_t T, int64_t E, int64_t ld,

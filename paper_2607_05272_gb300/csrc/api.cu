@@ -598,8 +598,9 @@ simx_status policy_forward_ws(const simx_mlp* pol, const float* d_obs, int64_t l
 simx_status compute_returns_gae(const float* d_rew, const float* d_val, const uint8_t* d_done,
                                 const float* d_last_val, int64_t T, int64_t E, int64_t ld,
                                 float gamma, float lam, float* d_ret, float* d_adv, void* stream) {
-  if (!d_rew || !d_done || !d_ret) return fail(SIMX_EINVAL, "rewards, dones and returns are required");
   if (T < 0 || E < 0 || ld < E) return fail(SIMX_EINVAL, "T %lld, E %lld, ld %lld", (long long)T, (long long)E, (long long)ld);
+  if (T == 0 || E == 0) return SIMX_OK;  // nothing to compute (empty buffers may be NULL)
+  if (!d_rew || !d_done || !d_ret) return fail(SIMX_EINVAL, "rewards, dones and returns are required");
   if (!std::isfinite(gamma)) return fail(SIMX_EINVAL, "gamma");
   if (lam >= 0.0f && (!d_val || !d_adv)) return fail(SIMX_EINVAL, "GAE needs values and an advantage buffer");
   cudaError_t e = launch_returns_gae(d_rew, d_val, d_done, d_last_val, T, E, ld, gamma, lam, d_ret,

@@ -258,3 +258,40 @@ def test_adam_rejects_bad_arguments():
         with pytest.raises(simx.SimxError) as e:   # the last: clipping without a workspace
             simx.adam_step(x, x, x, x, **kw)
         assert e.value.status == simx.EINVAL
+
+
+def test_empty_inputs():
+    """Empty inputs: returns over T = 0 or E = 0 and a policy forward of 0 columns are
+    no-ops; a loss over 0 rows, a baseline over 0 returns and an Adam step over 0
+    parameters are refused with EINVAL."""
+    simx = _simx()
+    ret = torch.full((4, 8), 7.0, device="cuda")
+    simx.compute_returns_gae(torch.zeros((0, 8), device="cuda"),
+                             torch.zeros((0, 8), dtype=torch.uint8, device="cuda"), 0.99, -1.0,
+                             ret[:0])
+    simx.compute_returns_gae(torch.zeros((4, 0), device="cuda"),
+                             torch.zeros((4, 0), dtype=torch.uint8, device="cuda"), 0.99, -1.0,
+                             ret[:, :0])
+    torch.cuda.synchronize()
+    assert torch.all(ret == 7.0)
+    ws = torch.empty(64, dtype=torch.uint8, device="cuda")
+    with pytest.raises(simx.SimxError) as e:
+        simx.returns_baseline(torch.zeros(0, device="cuda"), torch.zeros(0, device="cuda"),
+                              torch.zeros(1, device="cuda"), ws)
+    assert e.value.status == simx.EINVAL
+    x = torch.zeros(0, device="cuda")
+    with pytest.raises(simx.SimxError) as e:
+        simx.adam_step(x, x, x, x, 1, 1e-3)
+    assert e.value.status == simx.EINVAL
+    cfg, pol, host, buf = _rollout_for_loss(simx, "c2", 5, 4)
+    grad = torch.empty(pol.n_params, device="cuda")
+    stats = torch.empty(5, device="cuda")
+    lws = torch.empty(simx.ppo_loss_grad_workspace_size(pol, 1), dtype=torch.uint8, device="cuda")
+    with pytest.raises(simx.SimxError) as e:
+        simx.ppo_loss_grad(pol, buf, torch.zeros((4, 5), device="cuda"),
+                           torch.zeros((4, 5), device="cuda"), None, 0, "reinforce", 0.2, 0.0, 0.0,
+                           grad, stats, lws)
+    assert e.value.status == simx.EINVAL
+    obs = torch.zeros((pol.Ws[0].shape[1], 4), device="cuda")
+    simx.policy_forward(pol, obs, 0, "argmax", 1, 0)
+    torch.cuda.synchronize()
