@@ -205,6 +205,57 @@ def synthetic_trace(n: int, seed: int, mean_gap_us: float = 300.0, cv: float = 2
     return gap, typ, cost
 
 
+def trace_from_timestamps(t_us, types=None, costs_us=None, wrap_gap_us=None):
+    """The trace format of sim_set_trace from absolute request timestamps (sorted, in us):
+    gap_i = t_i - t_{i-1} for i >= 1 and gap_0 = the gap taken when the replay wraps from
+    the last entry to the first (default: the mean gap).  Types (values >= n_types count as
+    the last type) and per-request costs in us pass through; rounding to whole us and
+    clamping to u32 / u8 are the only changes."""
+    t = np.asarray(t_us, dtype=np.float64)
+    if t.ndim != 1 or len(t) < 1:
+        raise ValueError("need a non-empty 1-D array of timestamps")
+    if np.any(np.diff(t) < 0):
+        raise ValueError("timestamps must be sorted")
+    t = np.rint(t - t[0])
+    gap = np.empty(len(t), np.float64)
+    gap[1:] = np.diff(t)
+    if wrap_gap_us is None:
+        wrap_gap_us = t[-1] / (len(t) - 1) if len(t) > 1 else 1.0
+    gap[0] = np.rint(wrap_gap_us)
+    gap = np.clip(gap, 0, 2 ** 32 - 1).astype(np.uint32)
+    typ = None if types is None else np.clip(np.asarray(types), 0, 255).astype(np.uint8)
+    cost = None if costs_us is None else np.clip(np.rint(np.asarray(costs_us, np.float64)), 0,
+                                                 2 ** 32 - 1).astype(np.uint32)
+    for a in (typ, cost):
+        if a is not None and len(a) != len(gap):
+            raise ValueError("types and costs need one entry per timestamp")
+    return gap, typ, cost
+
+
+def trace_from_csv(path, time_col, time_unit_us=1.0, type_col=None, type_map=None,
+                   cost_col=None, cost_unit_us=1.0, wrap_gap_us=None, delimiter=","):
+    """A trace from a CSV request log with a header row (for instance a user's copy of a
+    serving log): the timestamp column (seconds -> time_unit_us = 1e6), an optional type
+    column mapped through `type_map` (a dict from the column's strings to type numbers, or
+    numeric types when None) and an optional cost column (scaled by cost_unit_us, e.g. a
+    token count times the us per token).  Rows are sorted by time."""
+    import csv
+    with open(path, newline="") as f:
+        rows = list(csv.DictReader(f, delimiter=delimiter))
+    if not rows:
+        raise ValueError("no rows in %s" % path)
+    t = np.array([float(r[time_col]) * time_unit_us for r in rows])
+    order = np.argsort(t, kind="stable")
+    typ = None
+    if type_col is not None:
+        raw = [rows[i][type_col] for i in order]
+        typ = [type_map[v] if type_map is not None else int(float(v)) for v in raw]
+    cost = None
+    if cost_col is not None:
+        cost = [float(rows[i][cost_col]) * cost_unit_us for i in order]
+    return trace_from_timestamps(t[order], typ, cost, wrap_gap_us)
+
+
 def c2t(n_envs: int = 4096) -> dict:
     """Trace replay (Sec. 3.2 real-world traces) on c2's server: every arrival, its gap
     and its type come from a 100,000-entry synthetic BurstGPT-shaped trace (mean gap

@@ -13,6 +13,7 @@
 workloads' in the queueing pins.)
 """
 import numpy as np
+import pytest
 
 import oracle
 from paper_2607_05272_gb300 import workloads as W
@@ -120,3 +121,31 @@ def test_dd1_overloaded_waits_grow_linearly():
     assert np.all(tr[:, 1] == 1)
     assert np.array_equal(tr[:, 2], 1100 * (k - 1))
     assert out["state"][0][13] == 0   # nothing dropped
+
+
+def test_trace_from_timestamps_round_trip():
+    t = np.array([1000.0, 1000.0, 1250.4, 1300.0, 9000.0])
+    gap, typ, cost = W.trace_from_timestamps(t, [0, 1, 3, 1, 0], [5.0, 6.4, 7.5, 0.0, 1e3])
+    assert list(gap[1:]) == [0, 250, 50, 7700]            # t rounded to us, then differenced
+    assert gap[0] == 2000                                   # wrap gap: the mean gap (8000 / 4)
+    assert np.array_equal(np.cumsum(gap[1:]), np.rint(t[1:] - t[0]))
+    assert list(typ) == [0, 1, 3, 1, 0] and list(cost) == [5, 6, 8, 0, 1000]
+    g2, _, _ = W.trace_from_timestamps(t, wrap_gap_us=123)
+    assert g2[0] == 123
+    with pytest.raises(ValueError):
+        W.trace_from_timestamps([3.0, 1.0])
+
+
+def test_trace_from_csv(tmp_path):
+    p = tmp_path / "log.csv"
+    p.write_text("ts,model,out_tokens\n0.5,big,10\n0.1,small,3\n0.25,small,4\n")
+    gap, typ, cost = W.trace_from_csv(p, "ts", 1e6, "model", {"small": 0, "big": 1},
+                                      "out_tokens", 20000.0)
+    assert list(gap[1:]) == [150000, 250000] and gap[0] == 200000
+    assert list(typ) == [0, 0, 1] and list(cost) == [60000, 80000, 200000]
+    # the oracle replays it: the first pending request is entry o's gap away
+    cfg = _route_cfg((gap, typ, cost))
+    e = oracle.OracleEnv(cfg, 0, 3)
+    e.reset()
+    o = _start(0, 3, 3)
+    assert e.export()[9] == gap[o]
