@@ -367,6 +367,11 @@ __device__ int t_action(const Ctx& x, TEnv<K>& s) {
 // threads over that latency: more residency beats more registers.
 template <bool ROUTE, int K, int MINB, bool TR>
 __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant__ RolloutArgs A) {
+  // Programmatic dependent launch: the next step's blocks may be scheduled as soon as every
+  // block of this one has started; each waits here until the previous grid has completed
+  // and its stores are visible, before it reads or writes any state.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const uint32_t env = blockIdx.x * blockDim.x + threadIdx.x;
   if (env >= A.st.E) return;
   const DevState& st = A.st;
@@ -586,14 +591,26 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
 }
 
 // 4 resident blocks per SM (128 registers): one wave of 77,824 envs; fewer registers
-// spill the server state of the router.
+// spill the server state of the router.  Launched with programmatic stream serialization
+// so that back-to-back steps (a graph of sim_step_batched calls) overlap one step's block
+// launch with the previous step's tail; the kernel's griddepcontrol.wait keeps the order.
 template <bool ROUTE, int K>
 cudaError_t step_thread_t(const RolloutArgs& a, cudaStream_t s) {
-  if (a.cfg.arrival_kind == SIMX_ARR_TRACE)
-    k_step_thread<ROUTE, K, 4, true><<<(a.st.E + 127) / 128, 128, 0, s>>>(a);
-  else
-    k_step_thread<ROUTE, K, 4, false><<<(a.st.E + 127) / 128, 128, 0, s>>>(a);
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3((a.st.E + 127) / 128);
+  lc.blockDim = dim3(128);
+  lc.dynamicSmemBytes = 0;
+  lc.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = at;
+  lc.numAttrs = 1;
+  cudaError_t e = a.cfg.arrival_kind == SIMX_ARR_TRACE
+                      ? cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 4, true>, a)
+                      : cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 4, false>, a);
   count_launches(1);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
