@@ -214,26 +214,57 @@ __device__ __forceinline__ uint64_t t_speed(const simx_config& c, int k, uint64_
   return (L * s + 8u) >> 4;
 }
 
-// ROUTE mode: server i starts a batch at time st (the oldest-head type, tie: type 0).
+// ROUTE mode: one server's queue state, selected out of the register arrays by unrolled
+// selects so that the batch start below is emitted once per call site instead of once per
+// server (the K-fold copies made the kernel's instruction fetch its largest stall).
+struct Srv {
+  uint32_t busy, bsize, qh0, qc0, qh1, qc1;
+};
+
 template <int K>
-__device__ __forceinline__ void t_start(const Ctx& x, TEnv<K>& s, int i, uint32_t st,
+__device__ __forceinline__ Srv srv_get(const TEnv<K>& s, int i) {
+  Srv r{s.busy[0], s.bsize[0], s.qh0[0], s.qc0[0], s.qh1[0], s.qc1[0]};
+#pragma unroll
+  for (int k = 1; k < K; ++k)
+    if (i == k) r = Srv{s.busy[k], s.bsize[k], s.qh0[k], s.qc0[k], s.qh1[k], s.qc1[k]};
+  return r;
+}
+
+template <int K>
+__device__ __forceinline__ void srv_put(TEnv<K>& s, int i, const Srv& r) {
+#pragma unroll
+  for (int k = 0; k < K; ++k)
+    if (i == k) {
+      s.busy[k] = r.busy;
+      s.bsize[k] = r.bsize;
+      s.qh0[k] = r.qh0;
+      s.qc0[k] = r.qc0;
+      s.qh1[k] = r.qh1;
+      s.qc1[k] = r.qc1;
+    }
+}
+
+// ROUTE mode: server i (state r) starts a batch at time st (the oldest-head type, tie:
+// type 0).
+template <int K>
+__device__ __forceinline__ void t_start(const Ctx& x, TEnv<K>& s, Srv& r, int i, uint32_t st,
                                         uint32_t& stn, uint64_t& w0, uint64_t& w1) {
   const simx_config& c = x.A.cfg;
   const uint32_t cap = c.queue_cap, T = c.n_types;
   uint32_t* rs = x.ring + (size_t)i * T * cap;
   uint32_t h;
-  if (s.qc0[i] > 0u && s.qc1[i] > 0u) {
-    h = rs[cap + s.qh1[i]] < rs[s.qh0[i]] ? 1u : 0u;
-  } else if (s.qc0[i] > 0u) {
+  if (r.qc0 > 0u && r.qc1 > 0u) {
+    h = rs[cap + r.qh1] < rs[r.qh0] ? 1u : 0u;
+  } else if (r.qc0 > 0u) {
     h = 0u;
-  } else if (s.qc1[i] > 0u) {
+  } else if (r.qc1 > 0u) {
     h = 1u;
   } else {
     return;
   }
-  const uint32_t qn = h ? s.qc1[i] : s.qc0[i];
-  const uint32_t head = h ? s.qh1[i] : s.qh0[i];
-  const uint32_t n = s.bsize[i] < qn ? s.bsize[i] : qn;
+  const uint32_t qn = h ? r.qc1 : r.qc0;
+  const uint32_t head = h ? r.qh1 : r.qh0;
+  const uint32_t n = r.bsize < qn ? r.bsize : qn;
   const bool costed = (int32_t)h == c.cost_type;
   uint64_t W = 0, csum = 0;
   for (uint32_t j = 0; j < n; ++j) {
@@ -242,15 +273,15 @@ __device__ __forceinline__ void t_start(const Ctx& x, TEnv<K>& s, int i, uint32_
     if (costed) csum += x.cost[(size_t)i * cap + slot];
   }
   if (h) {
-    s.qh1[i] = (head + n) & (cap - 1u);
-    s.qc1[i] -= n;
+    r.qh1 = (head + n) & (cap - 1u);
+    r.qc1 -= n;
   } else {
-    s.qh0[i] = (head + n) & (cap - 1u);
-    s.qc0[i] -= n;
+    r.qh0 = (head + n) & (cap - 1u);
+    r.qc0 -= n;
   }
   const uint64_t L = costed ? (uint64_t)c.alpha_us[h] + csum
                             : (uint64_t)c.alpha_us[h] + (uint64_t)c.beta_us[h] * n;
-  s.busy[i] = t_add(st, t_speed(c, i, L), s.status);
+  r.busy = t_add(st, t_speed(c, i, L), s.status);
   stn += n;
   if (h) w1 += W; else w0 += W;
   s.ndisp += n;
@@ -494,6 +525,7 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
       uint64_t w0 = 0, w1 = 0;
       if (!frozen) {
         s.events = 0;
+        bool go = false;
 #pragma unroll
         for (int k = 0; k < K; ++k) {
           if ((uint32_t)k != kk) continue;
@@ -508,7 +540,12 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
             if (mt) s.nd1 += 1u; else s.nd0 += 1u;
           }
           s.bsize[k] = b;
-          if (s.busy[k] <= now) t_start<K>(x, s, k, now, stn, w0, w1);
+          go = s.busy[k] <= now;
+        }
+        if (go) {  // the routed-to server is free: it starts a batch now
+          Srv r = srv_get<K>(s, (int)kk);
+          t_start<K>(x, s, r, (int)kk, now, stn, w0, w1);
+          srv_put<K>(s, (int)kk, r);
         }
         qafter = t_queued(s);
         t_next_arrival<K, TR>(x, s);
@@ -516,9 +553,18 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
         if (gap < 1u) gap = 1u;
         const float inst = __fdiv_rn(1.0e6f, __uint2float_rn(gap));
         s.rate = __fadd_rn(s.rate, __fmul_rn(0.0625f, __fsub_rn(inst, s.rate)));
+        // every server free by the next arrival starts batches, server by server in
+        // index order (one copy of the batch start for all servers)
+        for (;;) {
+          int k = -1;  // the lowest-index server free by then with requests queued
 #pragma unroll
-        for (int k = 0; k < K; ++k)
-          while (s.busy[k] <= s.pt && (s.qc0[k] + s.qc1[k]) > 0u) t_start<K>(x, s, k, s.busy[k], stn, w0, w1);
+          for (int j = K - 1; j >= 0; --j)
+            if (s.busy[j] <= s.pt && (s.qc0[j] + s.qc1[j]) > 0u) k = j;
+          if (k < 0) break;
+          Srv r = srv_get<K>(s, k);
+          t_start<K>(x, s, r, k, r.busy, stn, w0, w1);
+          srv_put<K>(s, k, r);
+        }
         s.now = s.pt;
       } else {
         qafter = t_queued(s);
