@@ -15,6 +15,7 @@ from .binding import (  # noqa: F401
     detlog,
     dettanh,
     duration,
+    gridq,
     lib,
     make_config,
     map_fn,

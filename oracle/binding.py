@@ -60,7 +60,8 @@ _TRACE_FIELDS = ("trace_gap", "trace_type", "trace_cost", "trace_len")
 class OrcMlp(C.Structure):
     _fields_ = [("n_layers", C.c_int32), ("dims", C.c_int32 * (MAX_LAYERS + 1)),
                 ("W", C.c_void_p * MAX_LAYERS), ("b", C.c_void_p * MAX_LAYERS),
-                ("has_value", C.c_int32), ("act", C.c_int32 * MAX_LAYERS)]
+                ("has_value", C.c_int32), ("act", C.c_int32 * MAX_LAYERS),
+                ("grid", C.c_int32), ("gx", C.c_int32 * MAX_LAYERS)]
 
 
 class OrcStepOut(C.Structure):
@@ -104,6 +105,7 @@ def lib():
             L.orc_map.argtypes = [C.c_int, P, P, I64]
             L.orc_philox_n.argtypes = [U32, U32, U32, U64, I64, P]
             L.orc_samplers.argtypes = [P, C.c_int, F, P, I64, P]
+            L.orc_gridq_n.argtypes = [P, I64, I32, P]
             _lib = L
     return _lib
 
@@ -138,7 +140,7 @@ def make_config(cfg: dict) -> OrcConfig:
 class _Mlp:
     """Keeps the numpy weight arrays alive while the C struct points at them."""
 
-    def __init__(self, Ws, bs, has_value, acts=None):
+    def __init__(self, Ws, bs, has_value, acts=None, grid=None):
         self.Ws = [np.ascontiguousarray(w, dtype=np.float32) for w in Ws]
         self.bs = [np.ascontiguousarray(b, dtype=np.float32) for b in bs]
         m = OrcMlp()
@@ -151,6 +153,10 @@ class _Mlp:
         m.has_value = int(bool(has_value))
         for l, a in enumerate(acts or []):
             m.act[l] = {"tanh": 0, "identity": 1, "gelu": 2}.get(a, a)
+        if grid is not None:          # the input grid exponent of every layer
+            m.grid = 1
+            for l, e in enumerate(grid):
+                m.gx[l] = int(e)
         self.c = m
 
 
@@ -158,7 +164,7 @@ def _mlp(mlp):
     if mlp is None:
         return None, None
     Ws, bs, hv = mlp[:3]
-    m = _Mlp(Ws, bs, hv, mlp[3] if len(mlp) > 3 else None)
+    m = _Mlp(Ws, bs, hv, mlp[3] if len(mlp) > 3 else None, mlp[4] if len(mlp) > 4 else None)
     return m, C.byref(m.c)
 
 
@@ -196,6 +202,14 @@ def samplers(cfg: dict, kind: int, words, scale: float = 1.0) -> np.ndarray:
     w = np.ascontiguousarray(words, dtype=np.uint32)
     out = np.empty(w.shape[0], np.float32)
     lib().orc_samplers(C.byref(c), kind, scale, w.ctypes.data, w.shape[0], out.ctypes.data)
+    return out
+
+
+def gridq(v, e: int) -> np.ndarray:
+    """The grid policy's rounding Q(v, e) = clamp(rint(v 2^e), -255, 255) 2^-e (fp32)."""
+    v = np.ascontiguousarray(v, dtype=np.float32)
+    out = np.empty_like(v)
+    lib().orc_gridq_n(v.ctypes.data, v.size, int(e), out.ctypes.data)
     return out
 
 

@@ -669,22 +669,50 @@ void orc_env_observe(const orc_env* ec, float* obs) {
 
 /* Policy (Sec. 4.2): tanh MLP; categorical sampling by inversion of the cumulative
    softmax with a POLICY-stream uniform, or argmax.  All fp32, sums in index order. */
+/* Grid rounding of the grid policy: v 2^e is an exact power-of-two scaling in fp64,
+   nearbyint rounds to nearest with ties to even (the default mode), and the clamped
+   integer times 2^-e is exact in fp32. */
+float orc_gridq(float v, int32_t e) {
+  double r = nearbyint(ldexp((double)v, e));
+  if (r > 255.0) r = 255.0;
+  if (r < -255.0) r = -255.0;
+  return (float)ldexp(r, -e);
+}
+
+void orc_gridq_n(const float* v, int64_t n, int32_t e, float* out) {
+  for (int64_t i = 0; i < n; ++i) out[i] = orc_gridq(v[i], e);
+}
+
 void orc_policy(const orc_mlp* m, const float* obs, int mode, uint64_t seed, uint32_t step,
                 uint32_t env_id, float* logits, float* value, int32_t* action, float* logp) {
-  float bufa[512], bufb[512];
+  float bufa[512], bufb[512], bufq[512];
   const float* x = obs;
   float* y = bufa;
+  if (m->grid) {
+    for (int k = 0; k < m->dims[0]; ++k) bufq[k] = orc_gridq(obs[k], m->gx[0]);
+    x = bufq;
+  }
   for (int l = 0; l < m->n_layers; ++l) {
     int K = m->dims[l], N = m->dims[l + 1];
     const float* W = m->W[l];
     for (int j = 0; j < N; ++j) {
-      float acc = 0.0f;
-      for (int k = 0; k < K; ++k) acc = fmaf(W[(size_t)j * K + k], x[k], acc);
-      float z = acc + m->b[l][j];
+      float z;
+      if (m->grid) {
+        /* the exact dot product: each fp64 product of two floats is exact, and so is the
+           fp64 sum of grid products; one rounding to fp32 at the end */
+        double acc = 0.0;
+        for (int k = 0; k < K; ++k) acc += (double)W[(size_t)j * K + k] * (double)x[k];
+        z = (float)(acc + (double)m->b[l][j]);
+      } else {
+        float acc = 0.0f;
+        for (int k = 0; k < K; ++k) acc = fmaf(W[(size_t)j * K + k], x[k], acc);
+        z = acc + m->b[l][j];
+      }
       if (l + 1 < m->n_layers) {
         if (m->act[l] == 1) y[j] = z;
         else if (m->act[l] == 2) y[j] = orc_detgelu(z);
         else y[j] = orc_dettanh(z);
+        if (m->grid) y[j] = orc_gridq(y[j], m->gx[l + 1]);
       } else {
         y[j] = z;
       }

@@ -70,6 +70,14 @@ typedef struct {
   const float* b[ORC_MAX_LAYERS];
   int32_t has_value;
   int32_t act[ORC_MAX_LAYERS];   /* after layer l < n_layers - 1: 0 tanh, 1 identity, 2 GELU */
+  /* Grid policy (the exact policy forward; Sec. 4.2 network on a fixed-point grid): when
+     grid != 0 the input of layer l is put on the grid 2^-gx[l] by orc_gridq (the
+     observation for l = 0, the activated hidden output otherwise) and every pre-activation
+     is the exact dot product plus bias, rounded once to fp32.  With weights on a grid
+     2^-e_w (|mantissa| <= 255), biases on 2^-(gx[l] + e_w) (|mantissa| <= 2^16) and
+     dims[l] <= 256 that value is exact, so any summation order reproduces it. */
+  int32_t grid;
+  int32_t gx[ORC_MAX_LAYERS];
 } orc_mlp;
 
 typedef struct orc_env orc_env;
@@ -93,6 +101,9 @@ float orc_detlog(float x);
 float orc_detexp(float x);
 float orc_dettanh(float x);
 float orc_detgelu(float x);
+/* Grid rounding Q(v, e) = clamp(rint(v 2^e), -255, 255) 2^-e, ties to even. */
+float orc_gridq(float v, int32_t e);
+void orc_gridq_n(const float* v, int64_t n, int32_t e, float* out);
 float orc_detcos2pi(float u);
 float orc_normal(uint32_t w0, uint32_t w1);
 uint32_t orc_duration(float x);

@@ -362,6 +362,44 @@ def mlp_weights(dims, seed: int, sigma: float = 0.1):
     return Ws, bs
 
 
+# Grid policy (the exact policy forward): layer l's input lives on the grid 2^-gx[l] with
+# integer mantissas |m| <= GRID_M, its weights on 2^-ew[l] with |m| <= GRID_M, its biases
+# on the product grid 2^-(gx[l] + ew[l]) with |m| <= GRID_MB, and dims[l] <= GRID_MAX_K,
+# so that every pre-activation is an integer number of product units below 2^24.
+GRID_M, GRID_MB, GRID_MAX_K = 255, 1 << 16, 256
+
+
+def grid_weights(dims, seed: int, gx, ew, sigma: float = 1.0):
+    """Weights and biases of a grid policy: integer mantissas drawn from a rounded
+    Gaussian of sd sigma * 2^ew / sqrt(fan-in) (clipped to the mantissa range) times the
+    layer's grid units; biases small multiples of the product unit."""
+    rng = np.random.default_rng(seed)
+    Ws, bs = [], []
+    for l, (k, n) in enumerate(zip(dims[:-1], dims[1:])):
+        sd = sigma * 2.0 ** ew[l] / math.sqrt(k)
+        m = np.clip(np.rint(rng.standard_normal((n, k)) * sd), -GRID_M, GRID_M)
+        Ws.append(np.ldexp(m, -int(ew[l])).astype(np.float32))
+        mb = rng.integers(-GRID_M, GRID_M + 1, n)
+        bs.append(np.ldexp(mb.astype(np.float64), -int(gx[l] + ew[l])).astype(np.float32))
+    return Ws, bs
+
+
+def grid_check(Ws, bs, gx, ew) -> None:
+    """Raise ValueError unless the weights satisfy the grid policy's premise (each
+    pre-activation an exact fp32 value in any summation order)."""
+    for l, (w, b) in enumerate(zip(Ws, bs)):
+        w = np.asarray(w, np.float64)
+        b = np.asarray(b, np.float64)
+        if w.shape[1] > GRID_MAX_K:
+            raise ValueError("layer %d: fan-in %d above %d" % (l, w.shape[1], GRID_MAX_K))
+        mw = np.ldexp(w, int(ew[l]))
+        mb = np.ldexp(b, int(gx[l] + ew[l]))
+        if np.any(mw != np.rint(mw)) or np.any(np.abs(mw) > GRID_M):
+            raise ValueError("layer %d: weights off the grid 2^-%d or above %d units" % (l, ew[l], GRID_M))
+        if np.any(mb != np.rint(mb)) or np.any(np.abs(mb) > GRID_MB):
+            raise ValueError("layer %d: biases off the product grid or above 2^16 units" % l)
+
+
 def mlp_acts(name: str) -> list:
     """The activation after each hidden layer of `name`'s policy."""
     n_hidden = len(MLP_SHAPES[name][0]) - 2
