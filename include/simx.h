@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define SIMX_ABI_VERSION 4u
+#define SIMX_ABI_VERSION 5u
 #define SIMX_MAX_TYPES 2
 #define SIMX_MAX_SERVERS 8
 #define SIMX_MAX_BSIZES 8
@@ -173,6 +173,16 @@ typedef enum { SIMX_ACT_TANH = 0, SIMX_ACT_IDENTITY = 1, SIMX_ACT_GELU = 2 } sim
  * attention over one token is a linear map, and separate heads are one hidden layer with
  * zero blocks in the output layer.  W_l is row-major [dims[l+1]][dims[l]] fp32, device
  * memory.
+ *
+ * Grid policy (grid != 0; the exact policy forward): the input of layer l is first put
+ * on the grid 2^-gx[l] (0 <= gx[l] <= 24) by Q(v, e) = clamp(rint(v 2^e), -255, 255) 2^-e,
+ * ties to even: the observation for l = 0, the activated hidden output of layer l - 1
+ * otherwise; the output layer is not rounded.  When the caller's weights lie on a grid
+ * 2^-e_w with integer mantissas |m| <= 255, the biases on 2^-(gx[l] + e_w) with |m| <=
+ * 2^16, and every fan-in is <= 256, each pre-activation is an exact fp32 value (the exact
+ * dot product plus bias), identical under any summation order; the library does not read
+ * the weights back to check this.  Grid policies run in rollout_collect, sim_step_batched
+ * and policy_forward; the loss-gradient entry points reject them (SIMX_EINVAL).
  */
 typedef struct simx_mlp {
   int32_t n_layers;                     /* 1 .. SIMX_MAX_LAYERS */
@@ -181,6 +191,8 @@ typedef struct simx_mlp {
   const float* b[SIMX_MAX_LAYERS];
   int32_t has_value;
   int32_t act[SIMX_MAX_LAYERS];         /* simx_act after layer l < n_layers - 1 */
+  int32_t grid;                         /* 0: plain fp32 policy; 1: grid policy */
+  int32_t gx[SIMX_MAX_LAYERS];          /* grid policy: input grid exponent of layer l */
 } simx_mlp;
 
 /* Rollout buffer (device memory, caller-owned).  ld >= n_envs is the env stride. */

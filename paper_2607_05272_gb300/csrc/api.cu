@@ -136,6 +136,12 @@ simx_status validate_mlp(const simx_mlp* m, uint32_t obs_dim, uint32_t n_actions
     if (!m->W[l] || !m->b[l]) return fail(SIMX_EINVAL, "layer %d weights are NULL", l);
   for (int l = 0; l + 1 < m->n_layers; ++l)
     if (m->act[l] < SIMX_ACT_TANH || m->act[l] > SIMX_ACT_GELU) return fail(SIMX_EINVAL, "act[%d] = %d", l, m->act[l]);
+  if (m->grid != 0 && m->grid != 1) return fail(SIMX_EINVAL, "grid = %d", m->grid);
+  if (m->grid)
+    for (int l = 0; l < m->n_layers; ++l) {
+      if (m->gx[l] < 0 || m->gx[l] > 24) return fail(SIMX_EINVAL, "gx[%d] = %d (0 .. 24)", l, m->gx[l]);
+      if (m->dims[l] > 256) return fail(SIMX_EINVAL, "grid policy fan-in %d above 256", m->dims[l]);
+    }
   return SIMX_OK;
 }
 
@@ -180,6 +186,8 @@ simx_status pack_mlp(const simx_mlp* m, Packed& P, DevMlp& out, cudaStream_t s) 
   }
   out.n_layers = m->n_layers;
   out.has_value = m->has_value ? 1 : 0;
+  out.grid = m->grid ? 1 : 0;
+  for (int l = 0; l < m->n_layers; ++l) out.gx[l] = m->grid ? m->gx[l] : 0;
   out.n_actions = m->dims[m->n_layers] - out.has_value;
   return SIMX_OK;
 }
@@ -639,6 +647,7 @@ static simx_status loss_args(const simx_mlp* pol, const simx_rollout* buf, int64
   if (p->precision != SIMX_PREC_FP32 && p->precision != SIMX_PREC_TF32)
     return fail(SIMX_EINVAL, "precision %d", p->precision);
   if (!d_adv || !d_grad || !d_stats) return fail(SIMX_EINVAL, "adv, grad and stats are required");
+  if (pol->grid) return fail(SIMX_EINVAL, "grid policies have no loss-gradient path");
   if (pol->has_value && !d_ret) return fail(SIMX_EINVAL, "a value row needs return targets");
   if (E < 1 || buf->ld != E) return fail(SIMX_EINVAL, "n_rows_per_step %lld must equal the rollout ld %lld", (long long)E, (long long)buf->ld);
   std::memset(&a, 0, sizeof(a));

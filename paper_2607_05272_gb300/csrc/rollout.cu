@@ -653,7 +653,7 @@ __device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int B
 // maxd4 x B floats (feature-major) and a softmax scratch of apad floats per env.
 // Every lane stays alive to the end (groups past the last env do no work) so that
 // warps reconverge at each phase and the block can run the MLP together.
-template <bool ROUTE, int G, bool TR, bool WARP>
+template <bool ROUTE, int G, bool TR, bool WARP, bool GRID>
 __global__ void __launch_bounds__(kMaxThreads, min_blocks<G>())
 k_rollout(const __grid_constant__ RolloutArgs A) {
   extern __shared__ float smem[];
@@ -704,8 +704,8 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
       // WARP: each warp runs the policy for its own 1-2 envs (narrow policies); else
       // block-wide, whose warps share each weight row instead of each loading it.  A
       // template parameter: both forwards in one kernel slowed the narrow case by 16 %.
-      const float* Z = WARP ? mlp_forward_warp(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G))
-                            : mlp_forward_block(A.mlp, X0, X1, B, Bs);
+      const float* Z = WARP ? mlp_forward_warp<GRID>(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G))
+                            : mlp_forward_block<GRID>(A.mlp, X0, X1, B, Bs);
       if (live)
         a = sample_action<G>(A.mlp, Z + slot, Bs, scratch, A.policy_mode, A.key0, A.key1, s.tg,
                              env, logp, value, g);
@@ -1060,7 +1060,8 @@ k_policy_forward(const __grid_constant__ PolicyArgs P) {
   float* scratch = smem + (size_t)2 * P.maxd4 * Bs + (size_t)slot * P.apad;
   const int D = P.mlp.dims[0];
   for (int d = (int)g.gl; d < D; d += G) X0[d * Bs + slot] = live ? P.obs[(int64_t)d * P.ld + i] : 0.0f;
-  const float* Z = mlp_forward_block(P.mlp, X0, X1, B, Bs);
+  const float* Z = P.mlp.grid ? mlp_forward_block<true>(P.mlp, X0, X1, B, Bs)
+                              : mlp_forward_block<false>(P.mlp, X0, X1, B, Bs);
   if (!live) return;
   float logp, value;
   const uint32_t env = P.env_base + (uint32_t)i;
@@ -1097,9 +1098,14 @@ static cudaError_t rollout_t(const RolloutArgs& a, cudaStream_t s) {
   const int B = a.threads / G;
   const size_t sh = env_smem(a, B);
   const bool tr = a.cfg.arrival_kind == SIMX_ARR_TRACE;
-  auto k = tr ? k_rollout<ROUTE, G, true, false> : k_rollout<ROUTE, G, false, false>;
+  // GRID: the grid policy's instantiations (a.mlp.grid is 0 without a policy)
+  const bool gr = a.mlp.grid != 0;
+  auto k = tr ? (gr ? k_rollout<ROUTE, G, true, false, true> : k_rollout<ROUTE, G, true, false, false>)
+              : (gr ? k_rollout<ROUTE, G, false, false, true> : k_rollout<ROUTE, G, false, false, false>);
   if constexpr (!ROUTE && G >= 16)  // the warp-local forward is instantiated where it applies
-    if (a.mlp_warp) k = tr ? k_rollout<ROUTE, G, true, true> : k_rollout<ROUTE, G, false, true>;
+    if (a.mlp_warp)
+      k = tr ? (gr ? k_rollout<ROUTE, G, true, true, true> : k_rollout<ROUTE, G, true, true, false>)
+             : (gr ? k_rollout<ROUTE, G, false, true, true> : k_rollout<ROUTE, G, false, true, false>);
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
   k<<<grid_for(a.st.E, B), a.threads, sh, s>>>(a);
   count_launches(1);

@@ -43,6 +43,8 @@ struct DevMlp {
   int npad[SIMX_MAX_LAYERS + 1];
   int n_layers, has_value, n_actions;
   int act[SIMX_MAX_LAYERS];  // simx_act after layer l, -1 for the output layer
+  int grid;                  // grid policy: layer l's input on the grid 2^-gx[l]
+  int gx[SIMX_MAX_LAYERS];
 };
 
 template <int G>
@@ -112,14 +114,42 @@ static __device__ __noinline__ void gelu_tile(float* Y, int ld, int j0, int N, i
     for (int e = 0; e < te; ++e) Y[j * ld + e] = det_gelu(Y[j * ld + e]);
 }
 
+// Grid rounding of the grid policy (the exact policy forward): Q(v, e) = clamp(rint(v 2^e),
+// -255, 255) 2^-e with ties to even, 0 <= e <= 24.  Both scalings are by exact powers of
+// two, so the only rounding is rintf's.
+__device__ __forceinline__ float grid_q(float v, int e) {
+  const float up = __int_as_float((127 + e) << 23), down = __int_as_float((127 - e) << 23);
+  const float r = fminf(fmaxf(rintf(__fmul_rn(v, up)), -255.0f), 255.0f);
+  return __fmul_rn(r, down);
+}
+
+// Grid rounding of rows j0 .. min(j0 + 4, N) - 1, columns 0 .. te - 1 of Y (after the
+// activation).  Out of line, like gelu_tile, so the other policies' loop stays small.
+static __device__ __noinline__ void grid_tile(float* Y, int ld, int j0, int N, int te, int e) {
+  for (int j = j0; j < j0 + 4 && j < N; ++j)
+    for (int c = 0; c < te; ++c) Y[j * ld + c] = grid_q(Y[j * ld + c], e);
+}
+
+// The observation of a grid policy on its input grid: rows 0 .. D-1, columns 0 .. B-1 of
+// X (row stride ld), split over threads tid, tid + nthr, ...
+static __device__ __noinline__ void grid_rows(float* X, int D, int B, int ld, int e, int tid,
+                                              int nthr) {
+  for (int i = tid; i < D * B; i += nthr) {
+    float* x = X + (i / B) * ld + i % B;
+    *x = grid_q(*x, e);
+  }
+}
+
 // act: the activation after this layer: -1 none (output layer), 0 tanh, 1 identity,
-// 2 GELU (det_gelu).
+// 2 GELU (det_gelu); GRID and gq >= 0: the grid policy's rounding of the activated
+// output.  GRID is a template parameter so that the fp32 policies' instantiations carry
+// no trace of it (an untaken runtime check here slowed the narrow rollout by about 5 %).
 // Threads tid, tid + nthr, ... of the cooperating group take the tiles.
-template <int TE>
+template <int TE, bool GRID>
 __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
                                           const float* __restrict__ bias, int K, int N, int Npad,
                                           const float* X, float* Y, int B, int ld, int act,
-                                          int tid, int nthr) {
+                                          int gq, int tid, int nthr) {
   const int neb = B / TE, nob = (N + 3) / 4;
   const int ntiles = neb * nob;
   for (int tile = tid; tile < ntiles; tile += nthr) {
@@ -174,25 +204,33 @@ __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
     } else if (act == 2) {
       gelu_tile(Y + TE * eb, ld, 4 * ob, N, TE);
     }
+    if (GRID && gq >= 0) grid_tile(Y + TE * eb, ld, 4 * ob, N, TE, gq);
   }
 }
 
 // Forward through every layer for the block's envs: the observation is in X0,
 // layers alternate X0 -> X1 -> X0 ...; returns the buffer holding the last layer
-// (logits rows 0..A-1, value row A).  Contains the block barriers.
+// (logits rows 0..A-1, value row A).  Contains the block barriers.  GRID: the grid
+// policy (m.grid set), whose inputs and hidden outputs are rounded to their grids.
+template <bool GRID>
 __device__ __forceinline__ float* mlp_forward_block(const DevMlp& m, float* X0, float* X1, int B,
                                                    int ld) {
   float* in = X0;
   float* out = X1;
   __syncthreads();
+  if (GRID) {
+    grid_rows(X0, m.dims[0], B, ld, m.gx[0], threadIdx.x, blockDim.x);
+    __syncthreads();
+  }
   for (int l = 0; l < m.n_layers; ++l) {
     const int K = m.dims[l], N = m.dims[l + 1], Np = m.npad[l + 1];
     const int th = m.act[l];
+    const int gq = (GRID && l + 1 < m.n_layers) ? m.gx[l + 1] : -1;
     // 4-env tiles when they keep every thread busy, otherwise 1-env tiles
     if ((B / 4) * ((N + 3) / 4) >= (int)blockDim.x)
-      mlp_tiles<4>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th, threadIdx.x, blockDim.x);
+      mlp_tiles<4, GRID>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th, gq, threadIdx.x, blockDim.x);
     else
-      mlp_tiles<1>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th, threadIdx.x, blockDim.x);
+      mlp_tiles<1, GRID>(m.Wt[l], m.bias[l], K, N, Np, in, out, B, ld, th, gq, threadIdx.x, blockDim.x);
     __syncthreads();
     float* t = in;
     in = out;
@@ -205,19 +243,25 @@ __device__ __forceinline__ float* mlp_forward_block(const DevMlp& m, float* X0, 
 // warp: only the warp's own lanes take its tiles, so warp barriers replace block
 // barriers.  Every output is still the K-ordered fma chain.  Returns the buffer (not
 // offset by col0) holding the last layer.
+template <bool GRID>
 __device__ __forceinline__ float* mlp_forward_warp(const DevMlp& m, float* X0, float* X1, int Bw,
                                                   int ld, int col0) {
   float* in = X0;
   float* out = X1;
   const int lane = (int)(threadIdx.x & 31u);
   __syncwarp();
+  if (GRID) {
+    grid_rows(X0 + col0, m.dims[0], Bw, ld, m.gx[0], lane, 32);
+    __syncwarp();
+  }
   for (int l = 0; l < m.n_layers; ++l) {
     const int K = m.dims[l], N = m.dims[l + 1], Np = m.npad[l + 1];
     const int th = m.act[l];
+    const int gq = (GRID && l + 1 < m.n_layers) ? m.gx[l + 1] : -1;
     if ((Bw / 4) * ((N + 3) / 4) >= 32)
-      mlp_tiles<4>(m.Wt[l], m.bias[l], K, N, Np, in + col0, out + col0, Bw, ld, th, lane, 32);
+      mlp_tiles<4, GRID>(m.Wt[l], m.bias[l], K, N, Np, in + col0, out + col0, Bw, ld, th, gq, lane, 32);
     else
-      mlp_tiles<1>(m.Wt[l], m.bias[l], K, N, Np, in + col0, out + col0, Bw, ld, th, lane, 32);
+      mlp_tiles<1, GRID>(m.Wt[l], m.bias[l], K, N, Np, in + col0, out + col0, Bw, ld, th, gq, lane, 32);
     __syncwarp();
     float* t = in;
     in = out;

@@ -55,7 +55,8 @@ class Config(C.Structure):
 class Mlp(C.Structure):
     _fields_ = [("n_layers", C.c_int32), ("dims", C.c_int32 * (MAX_LAYERS + 1)),
                 ("W", C.c_void_p * MAX_LAYERS), ("b", C.c_void_p * MAX_LAYERS),
-                ("has_value", C.c_int32), ("act", C.c_int32 * MAX_LAYERS)]
+                ("has_value", C.c_int32), ("act", C.c_int32 * MAX_LAYERS),
+                ("grid", C.c_int32), ("gx", C.c_int32 * MAX_LAYERS)]
 
 
 ACT = {"tanh": 0, "identity": 1, "gelu": 2}
@@ -166,9 +167,10 @@ def _stream(stream=None):
 class Policy:
     """A simx_mlp over device tensors W_l [out, in] and b_l [out] (fp32, contiguous);
     acts: the activation after each hidden layer ("tanh", "identity" or "gelu"; default
-    tanh)."""
+    tanh); grid: for a grid policy (the exact policy forward), the input grid exponent of
+    every layer (its weights must lie on the grid that workloads.grid_check checks)."""
 
-    def __init__(self, Ws, bs, has_value: bool, acts=None):
+    def __init__(self, Ws, bs, has_value: bool, acts=None, grid=None):
         self.Ws = [w.contiguous() for w in Ws]
         self.bs = [b.contiguous() for b in bs]
         self.has_value = bool(has_value)
@@ -183,6 +185,10 @@ class Policy:
         m.has_value = int(self.has_value)
         for l, a in enumerate(acts or []):
             m.act[l] = ACT[a] if isinstance(a, str) else int(a)
+        if grid is not None:
+            m.grid = 1
+            for l, e in enumerate(grid):
+                m.gx[l] = int(e)
         self.c = m
 
     flat = None  # the flat parameter vector when built by from_flat

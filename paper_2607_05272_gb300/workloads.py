@@ -30,7 +30,7 @@ import math
 
 import numpy as np
 
-ABI_VERSION = 4
+ABI_VERSION = 5
 MODE_SINGLE, MODE_ROUTE = 0, 1
 ARR_THINNED, ARR_DIURNAL, ARR_TRACE = 0, 1, 2
 POLICY = {"sample": 0, "argmax": 1, "static": 2, "rr": 3, "sq": 4, "random": 5, "external": 6}
