@@ -81,27 +81,55 @@ def act_grad(kind, z):
     return 1.0 - np.tanh(z) ** 2
 
 
-def _forward(Ws, bs, X, acts=None):
-    h = np.asarray(X, np.float64)
+def _grid_act(kind, z, e):
+    """A grid policy's hidden output: the activation of the fp32 pre-activation by the
+    simulator oracle's deterministic fp32 functions, then the grid rounding Q(., e).  The
+    rounding turns values into integers, so it is taken in the kernels' precision; the
+    fp64 pre-activation of a grid policy is an exact fp32 value, so the cast is exact."""
+    from .binding import gridq, map_fn
+    kind = ACT_NAMES.get(kind, kind)
+    z32 = np.asarray(z, np.float32)
+    if kind == IDENTITY:
+        a = z32
+    else:
+        a = map_fn("gelu" if kind == GELU else "tanh", z32.ravel()).reshape(z32.shape)
+    return gridq(a.ravel(), e).reshape(z32.shape).astype(np.float64)
+
+
+def _forward(Ws, bs, X, acts=None, grid=None):
+    """grid: the input grid exponent of every layer of a grid policy (the exact policy
+    forward): its layer inputs are rounded to their grids, and the backward pass lets the
+    gradient through the rounding unchanged (the straight-through estimator)."""
+    if grid is None:
+        h = np.asarray(X, np.float64)
+    else:
+        from .binding import gridq
+        X32 = np.asarray(X, np.float32)
+        h = gridq(X32.ravel(), grid[0]).reshape(X32.shape).astype(np.float64)
     inputs, zs = [], []
     L = len(Ws)
     for l in range(L):
         inputs.append(h)
         z = h @ np.asarray(Ws[l], np.float64).T + np.asarray(bs[l], np.float64)
         zs.append(z)
-        h = act_fn(acts[l] if acts else TANH, z) if l + 1 < L else z
+        if l + 1 == L:
+            h = z
+        elif grid is None:
+            h = act_fn(acts[l] if acts else TANH, z)
+        else:
+            h = _grid_act(acts[l] if acts else TANH, z, grid[l + 1])
     return inputs, zs, h
 
 
-def forward(Ws, bs, X, acts=None):
+def forward(Ws, bs, X, acts=None, grid=None):
     """MLP forward in fp64 (tanh hidden layers unless acts says otherwise); returns the
     list of layer inputs and the last layer's output."""
-    inputs, _, h = _forward(Ws, bs, X, acts)
+    inputs, _, h = _forward(Ws, bs, X, acts, grid)
     return inputs, h
 
 
 def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=0.2,
-              c_value=0.5, c_entropy=0.01, acts=None):
+              c_value=0.5, c_entropy=0.01, acts=None, grid=None):
     """Loss, statistics and the gradient with respect to every W_l, b_l (fp64).
 
     pi = softmax(logits); policy term REINFORCE -mean(adv log pi(a)) or PPO
@@ -109,7 +137,7 @@ def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=
     plus c_value mean((V - ret)^2) when a value row exists, minus c_entropy mean(H[pi]).
     Returns (grads [(gW, gb) per layer], stats [L, pg, v, H, clipfrac]).
     """
-    inputs, zs, Z = _forward(Ws, bs, X, acts)
+    inputs, zs, Z = _forward(Ws, bs, X, acts, grid)
     n = Z.shape[0]
     A = Z.shape[1] - (1 if has_value else 0)
     logits = Z[:, :A]

@@ -125,3 +125,78 @@ def test_premise_check():
     bb[0][0] = np.float32(np.ldexp(float((1 << 16) + 1), -(gx[0] + ew[0])))
     with pytest.raises(ValueError):
         W.grid_check(Ws, bb, gx, ew)
+
+
+def _grid_problem(name, seed, n=24):
+    dims, hv = W.mlp_dims(name)
+    acts = W.mlp_acts(name)
+    gx = [5] + [7] * (len(dims) - 2)
+    ew = [8] * (len(dims) - 1)
+    Ws, bs = W.grid_weights(dims, seed, gx, ew)
+    rng = np.random.default_rng(seed)
+    X = (rng.standard_normal((n, dims[0])) * 1.5).astype(np.float32)
+    return Ws, bs, hv, acts, gx, X
+
+
+@pytest.mark.parametrize("name", ["c3", "c1p"])
+def test_loss_oracle_grid_forward_is_the_policy(name):
+    """The loss oracle's grid forward (fp64 sums, fp32 activations and rounding) gives the
+    simulator oracle's logits and value bit for bit (the rounding decisions agree)."""
+    from oracle import rl
+    Ws, bs, hv, acts, gx, X = _grid_problem(name, 5)
+    _, Z = rl.forward(Ws, bs, X, acts, gx)
+    for i in range(len(X)):
+        lg, v, _, _ = oracle.policy((Ws, bs, hv, acts, gx), X[i], ARGMAX, 1, 0, 0)
+        A = len(lg)
+        assert np.array_equal(Z[i, :A].astype(np.float32).view(np.uint32), lg.view(np.uint32))
+        assert np.all(Z[i, :A].astype(np.float32) == Z[i, :A])     # exact in fp32
+        if hv:
+            assert np.float32(Z[i, A]) == np.float32(v)
+
+
+@pytest.mark.parametrize("name,algo", [("c3", 1), ("c1p", 0), ("c1p", 1)])
+def test_grid_straight_through_gradient_matches_autograd(name, algo):
+    """The grid policy's gradient passes the rounding straight through: PyTorch autograd of
+    the same forward written as h = a + (q - a).detach() (q the rounded values) agrees."""
+    torch = pytest.importorskip("torch")
+    from oracle import rl
+    Ws, bs, hv, acts, gx, X = _grid_problem(name, 9)
+    n = len(X)
+    rng = np.random.default_rng(3)
+    inputs, Z = rl.forward(Ws, bs, X, acts, gx)
+    A = Z.shape[1] - (1 if hv else 0)
+    a = rng.integers(0, A, n)
+    adv = rng.standard_normal(n)
+    ret = rng.standard_normal(n)
+    lpo = rng.standard_normal(n) * 0.3 - 1.4
+    grads, stats = rl.loss_grad(Ws, bs, hv, X, a, lpo, adv, ret, algo, 0.2, 0.5, 0.01,
+                                acts=acts, grid=gx)
+    tW = [torch.tensor(w, dtype=torch.float64, requires_grad=True) for w in Ws]
+    tb = [torch.tensor(b, dtype=torch.float64, requires_grad=True) for b in bs]
+    fns = {rl.TANH: torch.tanh, rl.IDENTITY: lambda z: z,
+           rl.GELU: lambda z: torch.nn.functional.gelu(z, approximate="tanh")}
+    h = torch.tensor(inputs[0])
+    for l in range(len(Ws)):
+        z = h @ tW[l].T + tb[l]
+        if l + 1 < len(Ws):
+            act = fns[rl.ACT_NAMES.get(acts[l], acts[l])](z)
+            h = act + (torch.tensor(inputs[l + 1]) - act).detach()
+        else:
+            h = z
+    assert np.array_equal(h.detach().numpy(), Z)
+    logpi = torch.log_softmax(h[:, :A], dim=1)
+    lpa = logpi[torch.arange(n), torch.tensor(a)]
+    advt = torch.tensor(adv)
+    if algo == rl.REINFORCE:
+        pg = -(advt * lpa).mean()
+    else:
+        rho = torch.exp(lpa - torch.tensor(lpo))
+        pg = -torch.minimum(rho * advt, torch.clamp(rho, 0.8, 1.2) * advt).mean()
+    loss = pg - 0.01 * (-(logpi.exp() * logpi).sum(1).mean())
+    if hv:
+        loss = loss + 0.5 * ((h[:, A] - torch.tensor(ret)) ** 2).mean()
+    loss.backward()
+    assert stats[0] == pytest.approx(loss.item(), rel=1e-12, abs=1e-12)
+    for (gW, gb), w, b in zip(grads, tW, tb):
+        assert np.allclose(gW, w.grad.numpy(), rtol=1e-10, atol=1e-12)
+        assert np.allclose(gb, b.grad.numpy(), rtol=1e-10, atol=1e-12)
