@@ -152,3 +152,37 @@ def test_single_long_batch_reward_weight():
     assert s2[HDR] == now + 20_000 + 2_000 * 2        # long: alpha 20 ms + 2 ms per request
     assert s2[21] == 1 and s2[20] == 2
     assert s2[22] == f32(10_000.0).view(np.uint32)    # last mean wait 20,000 / 2
+
+
+def test_route_reward_counts_every_batch_until_the_next_arrival():
+    """c3 router, Sec. 4.1 reward r = n - sum_type w_type W_type over the batches started
+    between this decision and the next: a one-entry trace (gap 30 ms) fixes the next
+    arrival at 80 ms.  The long request routed to idle server 1 (b = 1) starts at once
+    (wait 0); server 0 frees at 60 ms and starts its two queued short requests (waits 20
+    and 15 ms).  r = 3 - 0.001 * 35,000 - 0.0001 * 0."""
+    cfg = W.c3(1)
+    cfg.update(arrival_kind=W.ARR_TRACE, n_mod_states=1, accept_thr=[W.TWO24, W.TWO24],
+               trace=(np.array([30_000], np.uint32), None, None), queue_cap=256)
+    e, s = _env(cfg)
+    K = 4
+    now = 50_000
+    s[0], s[9], s[10] = now, now, 1                    # pending: a long request at 50 ms
+    s[2], s[3] = 5, now                                # next candidate: 50 ms + 30 ms
+    s[23] = f32(4000.0).view(np.uint32)
+    for k in range(K):
+        s[HDR + 2 * k + 1] = 4
+    s[HDR + 0] = 60_000                                # server 0 busy until 60 ms
+    _rings(cfg, s, {(0, 0): [40_000, 45_000]})
+    s[12] = 3
+    e.load(s)
+    o = e.step(6, None, action=1 * 4 + 0)              # server 1, b = bsizes[0] = 1
+    assert o["trace"] == [now, 3, 35_000, 2]           # qafter: server 0's two, before 60 ms
+    want = f32(3.0) - (f32(0.001) * f32(35_000.0) + f32(0.0001) * f32(0.0))
+    assert o["reward"] == want
+    s2 = e.export()
+    assert s2[0] == 80_000 and s2[9] == 80_000         # the next decision: the next arrival
+    assert s2[HDR + 0] == 60_000 + 1_000 + 50 * 2      # short batch of 2: alpha_0 + 2 beta_0
+    assert s2[HDR + 2] == now + 20_000 + 2_000 * 1     # long batch of 1: alpha_1 + beta_1
+    cnt = HDR + 2 * K
+    assert list(s2[cnt: cnt + 2 * K]) == [0] * (2 * K)  # every queue empty
+    assert s2[14] == 3                                 # dispatched
