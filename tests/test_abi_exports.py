@@ -56,10 +56,44 @@ def _struct_fields(name):
     return out
 
 
-@pytest.mark.parametrize("name,cls", [("simx_config", simx.Config), ("simx_rollout", simx.Rollout),
+@pytest.mark.parametrize("name,cls", [("simx_config", simx.Config), ("simx_mlp", simx.Mlp),
+                                      ("simx_rollout", simx.Rollout),
                                       ("simx_loss_params", simx.LossParams)])
 def test_struct_layouts_match_header(name, cls):
     assert _struct_fields(name) == [f[0] for f in cls._fields_]
+
+
+STRUCTS = [("simx_config", simx.Config), ("simx_mlp", simx.Mlp), ("simx_rollout", simx.Rollout),
+           ("simx_loss_params", simx.LossParams), ("simx_counters", simx.Counters),
+           ("simx_adam_params", simx.AdamParams)]
+
+
+def test_struct_offsets_match_the_c_compiler(tmp_path):
+    """Every ctypes struct of the binding has the C compiler's size and field offsets
+    (gcc on include/simx.h), so no field drifts between the header and the binding."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("no gcc")
+    lines = ["#include <stdio.h>", "#include <stddef.h>", '#include "simx.h"', "int main(void) {"]
+    for name, cls in STRUCTS:
+        lines.append('  printf("%s size %%zu\\n", sizeof(%s));' % (name, name))
+        for f in cls._fields_:
+            lines.append('  printf("%s %s %%zu\\n", offsetof(%s, %s));' % (name, f[0], name, f[0]))
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.check_call(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), "-o", str(exe),
+                           str(src)])
+    got = {}
+    for ln in subprocess.check_output([str(exe)]).decode().splitlines():
+        s_name, field, val = ln.split()
+        got[(s_name, field)] = int(val)
+    for name, cls in STRUCTS:
+        assert got[(name, "size")] == C.sizeof(cls), name
+        for f in cls._fields_:
+            assert got[(name, f[0])] == getattr(cls, f[0]).offset, (name, f[0])
 
 
 def test_host_entry_points(lib):
