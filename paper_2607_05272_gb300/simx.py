@@ -194,7 +194,7 @@ class Policy:
     flat = None  # the flat parameter vector when built by from_flat
 
     @classmethod
-    def from_flat(cls, flat, dims, has_value: bool, acts=None):
+    def from_flat(cls, flat, dims, has_value: bool, acts=None, grid=None):
         """A policy whose W_l, b_l are views into one flat fp32 device vector in the
         gradient's order (W0, b0, W1, b1, ...): the optimiser updates it in place."""
         Ws, bs, off = [], [], 0
@@ -204,7 +204,7 @@ class Policy:
             bs.append(flat[off:off + n])
             off += n
         assert off == flat.numel()
-        pol = cls(Ws, bs, has_value, acts)
+        pol = cls(Ws, bs, has_value, acts, grid)
         pol.flat = flat
         return pol
 
