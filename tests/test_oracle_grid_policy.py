@@ -200,3 +200,19 @@ def test_grid_straight_through_gradient_matches_autograd(name, algo):
     for (gW, gb), w, b in zip(grads, tW, tb):
         assert np.allclose(gW, w.grad.numpy(), rtol=1e-10, atol=1e-12)
         assert np.allclose(gb, b.grad.numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_gridq_over_all_finite_floats():
+    """Q against its definition in fp64 (exact there) over every finite fp32 input and grid
+    exponent 0 .. 24: huge values, subnormals and signed zeros included."""
+    hyp = pytest.importorskip("hypothesis")
+    st = pytest.importorskip("hypothesis.strategies")
+
+    @hyp.settings(max_examples=3000, deadline=None)
+    @hyp.given(st.floats(width=32, allow_nan=False, allow_infinity=False), st.integers(0, 24))
+    def check(v, e):
+        got = oracle.gridq(np.float32([v]), e)[0]
+        want = np.float32(np.ldexp(min(max(np.rint(np.ldexp(np.float64(v), e)), -255.0), 255.0), -e))
+        assert got.view(np.uint32) == want.view(np.uint32), (v, e, got, want)
+
+    check()
