@@ -176,8 +176,9 @@ typedef enum { SIMX_ACT_TANH = 0, SIMX_ACT_IDENTITY = 1, SIMX_ACT_GELU = 2 } sim
  *
  * Grid policy (grid != 0; the exact policy forward): the input of layer l is first put
  * on the grid 2^-gx[l] (0 <= gx[l] <= 24) by Q(v, e) = clamp(rint(v 2^e), -255, 255) 2^-e,
- * ties to even, for finite v (infinities clamp; NaN is not an input): the observation for l = 0, the activated hidden output of layer l - 1
- * otherwise; the output layer is not rounded.  When the caller's weights lie on a grid
+ * ties to even, for finite v (infinities clamp; NaN is not an input): the observation
+ * for l = 0, the activated hidden output of layer l - 1 otherwise; the output layer is
+ * not rounded.  When the caller's weights lie on a grid
  * 2^-e_w with integer mantissas |m| <= 255, the biases on 2^-(gx[l] + e_w) with |m| <=
  * 2^16, and every fan-in is <= 256, each pre-activation is an exact fp32 value (the exact
  * dot product plus bias), identical under any summation order; the library does not read
