@@ -301,6 +301,20 @@ simx_status rollout_collect(simx_ctx* ctx, const simx_mlp* pol, int policy_mode,
                             int32_t horizon, const simx_rollout* out, void* stream);
 
 /*
+ * The launch that rollout_collect and sim_step_batched take for this context, policy and
+ * mode (host only: no device work; the lane and block choice follows the device's SM
+ * count).  host_out[4] receives: [0] kernel, 0 = the fused step with the policy forward
+ * (one group of lanes per env), 1 = the thread-per-env step of the policy-free modes;
+ * [1] lanes per env (1 for the thread-per-env step); [2] threads per block; [3] 1 when
+ * each warp runs the policy forward for its own envs, 0 for the block-wide forward.
+ * It exists so that tests and benchmarks can state which instantiation they exercise.
+ * SIMX_EINVAL for a NULL argument, an unknown mode or a policy that rollout_collect
+ * would refuse.
+ */
+simx_status simx_launch_shape(simx_ctx* ctx, const simx_mlp* pol, int policy_mode,
+                              int32_t* host_out);
+
+/*
  * Batched policy forward (Sec. 4.2) for n observation columns d_obs [dims[0]][ld].
  * Column i is env (env_base + i) at global decision step `step`, which fixes its
  * POLICY Philox counter, so this reproduces the actions the rollout drew.
@@ -379,12 +393,16 @@ simx_status ppo_loss_grad(const simx_mlp* pol, const simx_rollout* buf, int64_t 
  *   - Arguments and results are those of ppo_loss_grad.
  *   - A minibatch whose workspace (ppo_loss_grad_workspace_size) exceeds the buffer is
  *     rejected with SIMX_EINVAL and a message giving both sizes.
- *   - The first call on a device looks up the buffer's device address (once per
- *     device, with that device current); make that first call before any stream
- *     capture.
- *   - Every call shares the one buffer: calls that overlap on the GPU (different
- *     streams, or devices sharing a call in flight) race and must be ordered by the
- *     caller.  Nothing needs to start at zero: each call writes all scratch it reads.
+ *   - The first call on a device looks up the buffer's device address (with that
+ *     device current) and keeps it for the device's context; make that first call
+ *     before any stream capture.  A device reset (cudaDeviceReset) ends the context
+ *     and may move the buffer: the first call in the new context looks the address
+ *     up again, so after a reset that call, too, belongs before any capture.
+ *   - Each device has its own copy of the buffer, and every call on that device uses
+ *     it: calls on the same device that overlap on the GPU (different streams, or
+ *     host threads without ordering between them) race and must be ordered by the
+ *     caller.  Calls on different devices do not share scratch.  Nothing needs to
+ *     start at zero: each call writes all scratch it reads.
  */
 #define SIMX_NOALLOC_SCRATCH_BYTES (16u << 20)
 simx_status ppo_loss_grad_noalloc(const simx_mlp* pol, const simx_rollout* buf,

@@ -1,5 +1,6 @@
 // api.cu — the C ABI of libsimx.so (declared in include/simx.h): argument
 // validation on the host, device state ownership, and kernel launches.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -17,6 +18,22 @@ using namespace simx;
 
 static std::atomic<uint64_t> g_launches{0};
 void simx::count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+// SM count of the current device, looked up once per device (152 on a GB300).  Without a
+// usable device (a host that only builds or sizes workspaces) the GB300's count is taken.
+static std::atomic<int> g_sms[64];
+int simx::sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+  int n = g_sms[dev].load(std::memory_order_relaxed);
+  if (n > 0) return n;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return 152;
+  }
+  g_sms[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
 
 namespace {
 
@@ -415,6 +432,13 @@ simx_status sim_observe(simx_ctx* c, float* d_obs, int64_t ld, void* stream) {
   return SIMX_OK;
 }
 
+// k_rollout's forward: warp-local for narrow policies at 16 or 32 lanes per env in SINGLE
+// mode (each warp then loads every weight row, which wide layers cannot afford); the
+// kernel has that variant only there.
+static int mlp_warp_of(bool route, int G, const simx_mlp* pol) {
+  return (!route && G >= 16 && mlp_maxdim(pol) <= 64) ? 1 : 0;
+}
+
 static simx_status prepare_policy(simx_ctx* c, const simx_mlp* pol, int mode, RolloutArgs& a,
                                   cudaStream_t s) {
   const bool route = c->cfg.mode == SIMX_MODE_ROUTE;
@@ -426,10 +450,7 @@ static simx_status prepare_policy(simx_ctx* c, const simx_mlp* pol, int mode, Ro
       v = pack_mlp(pol, c->pack, a.mlp, s);
       if (v != SIMX_OK) return v;
       act_layout(mlp_maxdim(pol), (int)a.n_actions, a.maxd4, a.apad);
-      // k_rollout's forward: warp-local for narrow policies at 16 or 32 lanes per env in
-      // SINGLE mode (each warp then loads every weight row, which wide layers cannot
-      // afford); the kernel has that variant only there
-      a.mlp_warp = (!route && a.G >= 16 && mlp_maxdim(pol) <= 64) ? 1 : 0;
+      a.mlp_warp = mlp_warp_of(route, a.G, pol);
       a.bs_pad = a.mlp_warp ? act_stride_pad(a.mlp, 32 / a.G, 32)
                             : act_stride_pad(a.mlp, a.threads / a.G, a.threads);
       break;
@@ -512,6 +533,28 @@ simx_status rollout_collect(simx_ctx* c, const simx_mlp* pol, int policy_mode, i
   cudaError_t e = step_thread_supported(a) ? launch_step_thread(a, s) : launch_rollout(a, s);
   if (e != cudaSuccess) return cuda_fail(e, "rollout launch");
   c->last = s;
+  return SIMX_OK;
+}
+
+simx_status simx_launch_shape(simx_ctx* c, const simx_mlp* pol, int policy_mode,
+                              int32_t* host_out) {
+  if (!c || !host_out) return fail(SIMX_EINVAL, "ctx or host_out is NULL");
+  const bool route = c->cfg.mode == SIMX_MODE_ROUTE;
+  const bool net = policy_mode == SIMX_POLICY_SAMPLE || policy_mode == SIMX_POLICY_ARGMAX;
+  if (policy_mode < 0 || policy_mode > SIMX_POLICY_EXTERNAL) return fail(SIMX_EINVAL, "policy_mode %d", policy_mode);
+  if (net) {
+    simx_status v = validate_mlp(pol, c->cfg.obs_dim, n_actions_of(c->cfg));
+    if (v != SIMX_OK) return v;
+  }
+  cudaSetDevice(c->device);
+  RolloutArgs a;
+  base_args(c, a);
+  a.policy_mode = policy_mode;
+  const bool thread = step_thread_supported(a);
+  host_out[0] = thread ? 1 : 0;
+  host_out[1] = thread ? 1 : a.G;
+  host_out[2] = thread ? 128 : a.threads;
+  host_out[3] = (!thread && net) ? mlp_warp_of(route, a.G, pol) : 0;
   return SIMX_OK;
 }
 
@@ -708,11 +751,42 @@ simx_status ppo_loss_grad(const simx_mlp* pol, const simx_rollout* buf, int64_t 
 // ---------------------------------------------------------------------------
 // Allocation-free loss gradient: the scratch is this file-scope device array.  Host
 // code may not use its name as a device address (it is a host-side stand-in), so the
-// address is looked up once per device with cudaGetSymbolAddress.
+// address is looked up with cudaGetSymbolAddress, with the device current, on the first
+// call on each device.  The address belongs to the device's context: after a device
+// reset the module is loaded again and the array may move, so the cached address is
+// kept together with the context's unique id and looked up again when that id changes.
 // ---------------------------------------------------------------------------
 static __device__ __align__(256) unsigned char g_noalloc_scratch[SIMX_NOALLOC_SCRATCH_BYTES];
 static std::mutex g_noalloc_mu;
-static void* g_noalloc_ptr[64] = {};
+struct NoallocSlot {
+  unsigned long long ctx_id;  // unique id of the context the address was found in
+  void* ptr;
+};
+static NoallocSlot g_noalloc[64] = {};
+
+// Unique id of the current context (cuCtxGetId, reached through the runtime's driver
+// entry points so that the library links no driver library); false when there is no
+// current context or the driver lacks the call.  Called with g_noalloc_mu held.
+static bool current_ctx_id(unsigned long long* id) {
+  static bool tried = false;
+  static void* get_cur = nullptr;
+  static void* get_id = nullptr;
+  if (!tried) {
+    tried = true;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &get_cur, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess || q != cudaDriverEntryPointSuccess)
+      get_cur = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &get_id, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess || q != cudaDriverEntryPointSuccess)
+      get_id = nullptr;
+    cudaGetLastError();
+  }
+  if (!get_cur || !get_id) return false;
+  CUcontext ctx = nullptr;
+  if (reinterpret_cast<CUresult (*)(CUcontext*)>(get_cur)(&ctx) != CUDA_SUCCESS || !ctx) return false;
+  return reinterpret_cast<CUresult (*)(CUcontext, unsigned long long*)>(get_id)(ctx, id) == CUDA_SUCCESS;
+}
 
 static simx_status noalloc_scratch(void** out) {
   int dev = 0;
@@ -720,13 +794,17 @@ static simx_status noalloc_scratch(void** out) {
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
   if (dev < 0 || dev >= 64) return fail(SIMX_EINVAL, "device %d", dev);
   std::lock_guard<std::mutex> lk(g_noalloc_mu);
-  if (!g_noalloc_ptr[dev]) {
+  NoallocSlot& slot = g_noalloc[dev];
+  unsigned long long id = 0;
+  const bool known = current_ctx_id(&id);
+  if (!slot.ptr || !known || id != slot.ctx_id) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess || !p) return cuda_fail(e, "cudaGetSymbolAddress(scratch)");
-    g_noalloc_ptr[dev] = p;
+    slot.ptr = p;
+    slot.ctx_id = current_ctx_id(&id) ? id : 0;
   }
-  *out = g_noalloc_ptr[dev];
+  *out = slot.ptr;
   return SIMX_OK;
 }
 

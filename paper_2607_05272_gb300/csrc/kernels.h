@@ -11,6 +11,8 @@ namespace simx {
 
 // Host-side count of kernel launches (every launcher adds its launches).
 void count_launches(int n);
+// SM count of the current device (grid sizes and lane choices scale with it).
+int sm_count();
 
 struct RolloutArgs {
   simx_config cfg;

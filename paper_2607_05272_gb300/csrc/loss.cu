@@ -333,7 +333,7 @@ struct WsLayout {
 static int dw_splits(int64_t n, int N, int K) {
   const int64_t tiles = (int64_t)((N + kBM - 1) / kBM) * ((K + kBN - 1) / kBN);
   int64_t s = (n + 2047) / 2048;
-  const int64_t fill = (2 * 152 + tiles - 1) / tiles;
+  const int64_t fill = (2 * (int64_t)sm_count() + tiles - 1) / tiles;
   if (s < fill) s = fill;
   const int64_t most = (n + 63) / 64;
   if (s > most) s = most;

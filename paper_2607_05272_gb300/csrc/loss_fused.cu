@@ -573,7 +573,7 @@ FusedPlan plan_r(const LossArgs& a, int R) {
   const int64_t ntiles = (a.n + R - 1) / R;
   // resident blocks per SM: 128 registers x 256 threads allow two; shared memory may allow fewer
   const int per_sm = p.smem <= 110 * 1024 ? 2 : 1;
-  int64_t grid = (int64_t)152 * per_sm;
+  int64_t grid = (int64_t)sm_count() * per_sm;
   if (grid > ntiles) grid = ntiles;
   p.grid = (int)(grid < 1 ? 1 : grid);
   size_t off = 0;

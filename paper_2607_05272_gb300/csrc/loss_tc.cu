@@ -675,7 +675,8 @@ struct Ws {
 Ws ws_layout(const LossArgs& a, const Plan& p) {
   Ws w{};
   const int64_t ntiles = (a.n + kR - 1) / kR;
-  w.grid = (int)(ntiles < 152 ? ntiles : 152);
+  const int64_t sms = sm_count();
+  w.grid = (int)(ntiles < sms ? ntiles : sms);
   if (w.grid < 1) w.grid = 1;
   w.part = 0;
   w.spart = ((size_t)w.grid * p.n_params * sizeof(float) + 255) & ~(size_t)255;

@@ -11,7 +11,7 @@ namespace simx {
 namespace {
 
 constexpr int kAdamThreads = 256;
-constexpr int kNormBlocks = 304;  // two per SM
+constexpr int kNormBlocks = 304;  // fixed (two per GB300 SM): the same sum order on any device
 
 __global__ void __launch_bounds__(kAdamThreads) k_sumsq(const float* __restrict__ g,
                                                         const uint8_t* __restrict__ mask,
@@ -111,7 +111,7 @@ cudaError_t launch_adam(float* p, const float* g, float* m, float* v, const uint
     count_launches(1);
   }
   int64_t blocks = (n + kAdamThreads - 1) / kAdamThreads;
-  if (blocks > 152 * 8) blocks = 152 * 8;
+  if (blocks > (int64_t)sm_count() * 8) blocks = (int64_t)sm_count() * 8;
   k_adam<<<(unsigned)blocks, kAdamThreads, 0, s>>>(p, g, m, v, mask, n, scal, d_t != nullptr,
                                                    step_size, inv_sqrt_c2, b1, b2, eps);
   count_launches(1);

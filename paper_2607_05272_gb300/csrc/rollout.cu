@@ -1200,23 +1200,24 @@ int choose_lanes(int64_t envs) {
     const int v = atoi(f);
     if (v == 8 || v == 16 || v == 32) return v;
   }
-  const int64_t target_warps = 152 * 16;
+  const int64_t target_warps = (int64_t)sm_count() * 16;
   if (envs <= target_warps) return 32;
   if (envs * 16 / 32 <= target_warps) return 16;
   return 8;
 }
 
 // Threads per block: the largest of 256, 128, 64 that still gives at least four
-// blocks per SM (two for 64), so small env counts spread over all 152 SMs.
+// blocks per SM (two for 64), so small env counts spread over every SM.
 // The environment variable SIMX_THREADS (64, 128 or 256) overrides the choice.
 int choose_threads(int64_t envs, int G) {
   if (const char* f = getenv("SIMX_THREADS")) {
     const int v = atoi(f);
     if ((v == 64 || v == 128 || v == 256) && v >= G) return v;
   }
+  const int64_t sms = sm_count();
   for (int t = 256; t >= 64; t /= 2) {
     const int64_t blocks = (envs + t / G - 1) / (t / G);
-    if (blocks >= (t == 64 ? 2 : 4) * 152 || t == 64) return t;
+    if (blocks >= (t == 64 ? 2 : 4) * sms || t == 64) return t;
   }
   return 64;
 }

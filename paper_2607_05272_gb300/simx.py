@@ -97,6 +97,7 @@ SIGNATURES = [
     ("sim_observe", C.c_int, [P, P, I64, P]),
     ("sim_step_batched", C.c_int, [P, P, P, C.c_int, P, I64, P, P, P, P, P]),
     ("rollout_collect", C.c_int, [P, P, C.c_int, I32, P, P]),
+    ("simx_launch_shape", C.c_int, [P, P, C.c_int, P]),
     ("policy_forward", C.c_int, [P, P, I64, I64, C.c_int, U64, U32, U32, P, P, P, P, P]),
     ("policy_forward_workspace_size", SZ, [P]),
     ("policy_forward_ws", C.c_int, [P, P, I64, I64, C.c_int, U64, U32, U32, P, P, P, P, P, SZ, P]),
@@ -294,6 +295,15 @@ class Sim:
             setattr(r, k, None if t is None else t.data_ptr())
         _check(lib().rollout_collect(self._h, C.byref(policy.c) if policy else None,
                                      POLICY[policy_mode], horizon, C.byref(r), _stream(stream)))
+
+    def launch_shape(self, policy_mode: str, policy: Policy = None) -> dict:
+        """The launch rollout_collect takes (simx_launch_shape): kernel ("fused" or
+        "thread"), lanes per env, threads per block, warp-local policy forward."""
+        out = (C.c_int32 * 4)()
+        _check(lib().simx_launch_shape(self._h, C.byref(policy.c) if policy else None,
+                                       POLICY[policy_mode], out))
+        return dict(kernel="thread" if out[0] else "fused", lanes=out[1], threads=out[2],
+                    mlp_warp=bool(out[3]))
 
     def stats(self) -> dict:
         c = Counters()

@@ -8,10 +8,11 @@ order, so these compare within tolerances derived from the arithmetic:
 * loss gradients, per tensor: ||g - g_ref|| <= 1e-5 ||g_ref||, per element:
   |g - g_ref| <= 1e-5 (|g_ref| + rms(g_ref)); the tensor-core (TF32-input) path is held
   to 1e-2 under the same definitions.
-Sizes span several blocks with ragged tails, plus the full c1 returns shape; env counts
-from 65,536 that are a multiple of 4 take the one-pass four-envs-per-thread kernel (with
-horizons that are not a multiple of its 8-step lookahead), the rest the chunked two-pass
-one (262,145 envs among them).
+Sizes span several blocks with ragged tails, plus the full c1 returns shape; every env
+count here (up to 40,000) takes the chunked two-pass returns kernel.  Env counts from
+65,536 that are a multiple of 4 take the one-pass four-envs-per-thread kernel instead;
+test_gpu_launch_shapes.py covers it at 65,536 and 262,144 envs (and 262,145, which
+falls back to the chunked one).
 """
 import numpy as np
 import pytest
