@@ -99,6 +99,9 @@ def lib():
             L.orc_env_status.argtypes = [P]
             L.orc_env_status.restype = U32
             L.orc_env_little.argtypes = [P, U32, P, P]
+            L.orc_env_switch_log.argtypes = [P, P, U32]
+            L.orc_env_switch_log_count.argtypes = [P]
+            L.orc_env_switch_log_count.restype = U32
             L.orc_policy.argtypes = [P, P, C.c_int, U64, U32, U32, P, P, P, P]
             L.orc_rollout.argtypes = [P, P, U64, C.c_int, P, I64, I32, P, P, P, P, P, P, P, P]
             L.orc_rollout.restype = C.c_int
@@ -333,6 +336,16 @@ class OracleEnv:
 
     def status(self) -> int:
         return lib().orc_env_status(self._e)
+
+    def attach_switch_log(self, cap: int) -> None:
+        """Record the modulating chain from the next reset on: (time, state) at time 0
+        and at every switch processed, up to cap pairs (see switch_log)."""
+        self._swlog = np.zeros((cap, 2), np.uint32)
+        lib().orc_env_switch_log(self._e, self._swlog.ctypes.data, cap)
+
+    def switch_log(self) -> np.ndarray:
+        n = lib().orc_env_switch_log_count(self._e)
+        return self._swlog[:n].copy()
 
     def little(self, t_end: int):
         a = C.c_uint64()

@@ -242,6 +242,8 @@ struct orc_env {
   uint32_t q_last[ORC_MAX_SERVERS][2]; /* time of that queue's last change */
   uint32_t step_n;
   uint64_t step_w[2];
+  uint32_t* swlog;   /* optional log of the modulating chain: (time, state) pairs */
+  uint32_t swlog_cap, swlog_n;
 };
 
 uint32_t orc_obs_dim(const orc_config* c) {
@@ -365,6 +367,16 @@ static uint32_t dwell_us(orc_env* e, uint32_t i) {
   return orc_duration(e->c.dwell_mean_us * expo1(w[0]));
 }
 
+/* Test hook: record (time, state) of the modulating chain, at reset and at every switch
+   processed, when the caller attached a log (orc_env_switch_log).  Records nothing
+   that the simulation reads. */
+static void swlog_push(orc_env* e, uint32_t t, uint32_t state) {
+  if (!e->swlog || e->swlog_n >= e->swlog_cap) return;
+  e->swlog[2 * e->swlog_n] = t;
+  e->swlog[2 * e->swlog_n + 1] = state;
+  e->swlog_n += 1u;
+}
+
 /* Modulating chain: switch i >= 1 at S_i = S_{i-1} + dwell_i, S_0 = 0.
    All switches at times <= limit take effect. */
 static void process_switches(orc_env* e, uint32_t limit) {
@@ -372,6 +384,7 @@ static void process_switches(orc_env* e, uint32_t limit) {
   while (e->sw_T <= limit) {
     if (count_event(e)) return;
     e->mstate ^= 1u;
+    swlog_push(e, e->sw_T, e->mstate);
     e->sw_i += 1u;
     e->sw_T = add_time(e, e->sw_T, dwell_us(e, e->sw_i));
   }
@@ -560,6 +573,14 @@ void orc_env_free(orc_env* e) {
 
 uint32_t orc_env_status(const orc_env* e) { return e->status; }
 
+void orc_env_switch_log(orc_env* e, uint32_t* pairs, uint32_t cap) {
+  e->swlog = pairs;
+  e->swlog_cap = pairs ? cap : 0u;
+  e->swlog_n = 0;
+}
+
+uint32_t orc_env_switch_log_count(const orc_env* e) { return e->swlog_n; }
+
 void orc_env_little(const orc_env* ec, uint32_t t_end, uint64_t* area, uint64_t* waits) {
   orc_env* e = (orc_env*)ec;
   uint64_t a = 0, w = e->sum_wait;
@@ -579,7 +600,11 @@ void orc_env_reset(orc_env* e) {
   uint32_t* qa = e->qarr;
   uint32_t* qc = e->qcost;
   uint32_t K = e->K, T = e->T, cap = e->cap, A = e->A;
+  uint32_t* swlog = e->swlog;
+  const uint32_t swlog_cap = e->swlog_cap;
   memset(e, 0, sizeof(*e));
+  e->swlog = swlog;
+  e->swlog_cap = swlog_cap;
   e->c = c;
   e->id = id;
   e->key[0] = key0;
@@ -600,6 +625,7 @@ void orc_env_reset(orc_env* e) {
   draw(e, 0, ORC_STREAM_INIT, w);
   if (c.n_mod_states == 2) {
     e->mstate = w[0] >> 31;
+    swlog_push(e, 0, e->mstate);
     e->sw_i = 1;
     e->sw_T = add_time(e, 0, dwell_us(e, 1));
   } else {

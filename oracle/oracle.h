@@ -120,6 +120,12 @@ void orc_env_step(orc_env* e, const orc_mlp* m, int mode, int32_t ext_action, or
 void orc_env_export(const orc_env* e, uint32_t* words);
 void orc_env_import(orc_env* e, const uint32_t* words);
 uint32_t orc_env_status(const orc_env* e);
+/* Test hook: attach a host array of cap (time, state) pairs that the env fills, from its
+   next reset on, with the modulating chain's state at time 0 and the time and new state
+   of every switch it processes (n_mod_states = 2 only); NULL detaches.  The count of
+   pairs written is orc_env_switch_log_count.  The simulation does not read the log. */
+void orc_env_switch_log(orc_env* e, uint32_t* pairs, uint32_t cap);
+uint32_t orc_env_switch_log_count(const orc_env* e);
 /* Exact finite-horizon Little identity pieces up to time t_end (>= every event):
    *area = integral of the total queue length over [0, t_end] accumulated event by
    event; *waits = summed queueing time of dispatched requests plus (t_end - arrival)
