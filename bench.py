@@ -1,12 +1,16 @@
 #!/usr/bin/env python
 """Throughput benchmark of the batched rollout engine (one JSON line on rank 0).
 
-Workload: the single-server bursty heterogeneous environment (4096 envs x 512
-decision steps, two-state MMPP 300/3000 req/s, 80/20 short/long requests, per-type
-queues of 256, MLP 16-64-64-12, REINFORCE with a mean-return baseline), inputs
-synthetic and seeded.  One step is one pass of the whole hot path over one batch:
-rollout_collect (simulation + fused policy) -> REINFORCE returns -> mean baseline
--> loss gradient over all 2,097,152 rows, every stage a kernel of libsimx.so.
+Workload: the trace-shaped multi-server environment (65,536 envs x 512 decision steps
+per GPU, 8 simulated servers, diurnal 1000-8000 req/s x lognormal(0, 1) burst factors
+per 500 ms, Pareto(1.5, 10 ms) long-request costs, 85/15 short/long, action = server x
+batch size (48), MLP 28-256-256-48 plus a value row, PPO with GAE(0.99, 0.95)), the
+largest configuration that fits one GPU, inputs synthetic and seeded.  One step is one
+pass of the whole hot path over one batch, every numeric stage a kernel of libsimx.so:
+rollout_collect (simulation + fused policy) -> bootstrap value -> GAE -> one PPO epoch
+over the 33,554,432 rows in 4096 minibatches of 8192 (loss gradient + Adam update
+each, replayed from a CUDA graph).  --epochs 4 runs the four epochs of the full PPO
+update.  The minibatch permutation is drawn on the device by torch.randperm.
 
 metric: simulated decision steps per second (envs x horizon x ranks / step time).
 --impl reference times the oracle (the plain CPU reference) on a bounded sample of
@@ -27,21 +31,29 @@ sys.path.insert(0, ROOT)
 
 METRIC = "simulated decision steps/sec"
 UNIT = "steps/s"
-WORKLOAD = "c2"
-SEED_BASE = 0x5EED0002
-GAMMA = 0.99
+WORKLOAD = "c4"
+ENVS, HORIZON, MINIBATCH = 65536, 512, 8192
+SEED_BASE = 0x5EED0004
+GAMMA, LAMBDA = 0.99, 0.95
+CLIP, C_VALUE, C_ENTROPY, LR, MAX_NORM = 0.2, 0.5, 0.01, 3e-4, 0.5
 L2_FLUSH_BYTES = 256 << 20
+WORKLOAD_TEXT = ("c4: 65,536 envs x 512 steps per GPU, 8 servers, diurnal 1000-8000 req/s x "
+                 "lognormal(0,1) per 500 ms, Pareto(1.5, 10 ms) long costs, 85/15 short/long, "
+                 "MLP 28-256-256-48+V, PPO (GAE 0.99/0.95, clip 0.2, minibatches of 8192, Adam)")
 
 
 def _args():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=100)
-    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--epochs", type=int, default=1,
+                   help="PPO epochs per step (passes of minibatches over the rollout buffer)")
     p.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-hbm-step", action="store_true")
+    p.add_argument("--no-extras", action="store_true", help="skip the c2 and 1M-env c5 extra lines")
     p.add_argument("--sweep", action="store_true",
                    help="every configuration (c1-c5, c5 at every env count): one JSON line each")
     p.add_argument("--sweep-configs", default="c1,c2,c3,c4,c5,c1p,c3s,c3t",
@@ -59,61 +71,82 @@ def _args():
 # --------------------------------------------------------------------------- #
 # CPU reference (the oracle), run in a child process with single-threaded BLAS
 # --------------------------------------------------------------------------- #
-def _oracle_step(n_envs: int, env0: int, H: int):
-    """One oracle pass of the hot path over envs [env0, env0 + n_envs): rollout,
-    returns, mean baseline, REINFORCE loss gradient (fp64).  Returns seconds."""
+def _oracle_step(n_envs: int, env0: int, H: int, epochs: int):
+    """One oracle pass of the hot path over envs [env0, env0 + n_envs) of the workload:
+    rollout, bootstrap value, GAE, then `epochs` PPO epochs over the sample's rows in
+    minibatches of up to 8192 (fp64 loss gradient and Adam on each).  Returns seconds."""
     import numpy as np
 
     import oracle
     from oracle import rl
     from paper_2607_05272_gb300 import workloads as W
-    cfg = W.c2(n_envs)
+    cfg = W.CONFIGS[WORKLOAD](ENVS)
     dims, hv = W.mlp_dims(WORKLOAD)
-    Ws, bs = W.mlp_weights(dims, 1)
+    Ws, bs = W.policy_weights(WORKLOAD, dims, 1)
     t0 = time.perf_counter()
-    out = oracle.rollout(cfg, (Ws, bs, hv), SEED_BASE, 0, list(range(env0, env0 + n_envs)), H)
-    G = rl.returns(out["reward"], out["done"], GAMMA)
-    adv, _ = rl.baseline(G)
-    X = out["obs"].transpose(0, 2, 1).reshape(-1, dims[0])
-    rl.loss_grad(Ws, bs, hv, X, out["action"].ravel(), out["logp"].ravel(), adv.ravel(),
-                 G.ravel(), rl.REINFORCE, 0.2, 0.0, 0.0)
+    ids = list(range(env0, env0 + n_envs))
+    # H + 1 decisions: the first H are the rollout, the last one's observation is each
+    # env's state after it, whose value row bootstraps GAE
+    full = oracle.rollout(cfg, (Ws, bs, hv), SEED_BASE, 0, ids, H + 1)
+    out = {k: full[k][:H] for k in ("obs", "action", "logp", "value", "reward", "done")}
+    _, Z = rl.forward(Ws, bs, full["obs"][H].T)
+    last = Z[:, -1].astype(np.float32)
+    A, R = rl.gae(out["reward"], out["value"], out["done"], GAMMA, LAMBDA, last)
+    n = n_envs * H
+    flat = np.concatenate([np.concatenate([w.ravel(), b.ravel()]) for w, b in zip(Ws, bs)])
+    p, m, v = flat.astype(np.float64), np.zeros(flat.size), np.zeros(flat.size)
+    rng = np.random.default_rng(env0)
+    t = 0
+    for _ in range(epochs):
+        perm = rng.permutation(n)
+        for i in range(0, n, MINIBATCH):
+            rows = perm[i:i + MINIBATCH]
+            X, a, lpo = rl.gather_rows(out["obs"], out["action"], out["logp"], rows, n_envs)
+            tt, ee = rows // n_envs, rows % n_envs
+            g, _ = rl.loss_grad(Ws, bs, hv, X, a, lpo, A[tt, ee], R[tt, ee], rl.PPO, CLIP, C_VALUE,
+                                C_ENTROPY)
+            t += 1
+            p, m, v = rl.adam_step(p, rl.flat(g), m, v, t, LR, max_grad_norm=MAX_NORM)
     return time.perf_counter() - t0
 
 
 def _cpu_child(spec: str):
-    kind, n_envs, steps, warm = spec.split(",")
-    n_envs, steps, warm = int(n_envs), int(steps), int(warm)
-    H = 512
+    kind, n_envs, steps, warm, epochs = spec.split(",")
+    n_envs, steps, warm, epochs = int(n_envs), int(steps), int(warm), int(epochs)
     times = []
     for i in range(warm + steps):
-        dt = _oracle_step(n_envs, (i * n_envs) % 4096, H)
+        dt = _oracle_step(n_envs, (i * n_envs) % ENVS, HORIZON, epochs)
         if i >= warm:
             times.append(dt)
-    print(json.dumps({"times": times, "env_steps": n_envs * H}))
+    print(json.dumps({"times": times, "env_steps": n_envs * HORIZON}))
 
 
-def _run_cpu(n_envs: int, steps: int, warm: int) -> dict:
+def _run_cpu(n_envs: int, steps: int, warm: int, epochs: int) -> dict:
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
     r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-child",
-                        "x,%d,%d,%d" % (n_envs, steps, warm)], capture_output=True, text=True,
-                       env=env, cwd=ROOT)
+                        "x,%d,%d,%d,%d" % (n_envs, steps, warm, epochs)], capture_output=True,
+                       text=True, env=env, cwd=ROOT)
     if r.returncode != 0:
         raise RuntimeError("oracle child failed:\n" + r.stderr[-2000:])
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-def cpu_baseline() -> dict:
+def _sample_text(n: int, epochs: int) -> str:
+    return ("%d envs x %d steps of the same workload (rollout, bootstrap value, GAE, %d PPO "
+            "epoch(s) of loss gradient + Adam over those rows), single-threaded"
+            % (n, HORIZON, epochs))
+
+
+def cpu_baseline(epochs: int) -> dict:
     """The oracle as it stands, single-threaded, on a bounded sample (~10-20 s)."""
     import oracle
     oracle.build()
-    probe = _run_cpu(16, 1, 0)
-    per_env = probe["times"][0] / 16.0
-    n = int(max(16, min(4096, 12.0 / max(per_env, 1e-6))))
-    res = _run_cpu(n, 1, 0)
+    probe = _run_cpu(2, 1, 0, epochs)
+    per_env = probe["times"][0] / 2.0
+    n = int(max(2, min(4096, 12.0 / max(per_env, 1e-6))))
+    res = _run_cpu(n, 1, 0, epochs)
     v = res["env_steps"] / res["times"][0]
-    return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": "%d envs x 512 steps of the same workload (rollout + returns + baseline + "
-                      "loss gradient), single-threaded" % n}
+    return {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": _sample_text(n, epochs)}
 
 
 def run_reference(a) -> None:
@@ -122,23 +155,20 @@ def run_reference(a) -> None:
         return
     import oracle
     oracle.build()
-    probe = _run_cpu(16, 1, 0)
-    per_env = probe["times"][0] / 16.0
+    probe = _run_cpu(2, 1, 0, a.epochs)
+    per_env = probe["times"][0] / 2.0
     budget = min(6.0, 150.0 / max(1, a.steps + a.warmup))  # whole run within a few minutes
-    n = int(max(4, min(4096, budget / max(per_env, 1e-6))))
-    res = _run_cpu(n, a.steps, a.warmup)
+    n = int(max(2, min(4096, budget / max(per_env, 1e-6))))
+    res = _run_cpu(n, a.steps, a.warmup, a.epochs)
     t = statistics.mean(res["times"])
     v = res["env_steps"] / t
-    sample = ("%d envs x 512 steps per step (rollout + returns + baseline + loss gradient), "
-              "single-threaded" % n)
     line = {
         "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": a.gpus,
         "steps": a.steps, "warmup": a.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": "c2: 4096 envs x 512 steps, MMPP 300/3000 req/s, 80/20 short/long, "
-                               "MLP 16-64-64-12, REINFORCE + mean baseline",
-                   "sample_envs": n},
-        "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD_TEXT, "ppo_epochs_per_step": a.epochs, "sample_envs": n},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": _sample_text(n, a.epochs)},
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -369,9 +399,10 @@ class Clocks:
 
 
 # DRAM bytes (read + write) of one k_rollout launch of the benchmark workload, from an
-# ncu capture of the current kernel; to be re-measured (or set to None) whenever the
-# rollout kernel changes.
-ROLLOUT_DRAM_BYTES = 123.8e6
+# ncu capture of the current kernel; None until one is taken, and to be re-measured (or
+# set back to None) whenever the rollout kernel changes.
+ROLLOUT_DRAM_BYTES = None
+ROLLOUT_DRAM_SOURCE = None
 
 
 def _peaks():
@@ -507,6 +538,191 @@ def job_value(world: int, units_per_rank: int, ms: float) -> float:
     return world * units_per_rank / (ms * 1e-3)
 
 
+class PPOStep:
+    """One step of the benchmark on this GPU: rollout -> bootstrap value -> GAE -> PPO
+    epochs (loss gradient + Adam per minibatch, the minibatch loop replayed from a CUDA
+    graph captured on the first call after a warm eager one)."""
+
+    def __init__(self, simx, W, torch, seed: int, epochs: int, precision: str, device: int):
+        import numpy as np
+        self.simx, self.torch = simx, torch
+        self.E, self.H, self.mb, self.epochs, self.precision = ENVS, HORIZON, MINIBATCH, epochs, precision
+        cfg = W.CONFIGS[WORKLOAD](self.E)
+        self.dims, hv = W.mlp_dims(WORKLOAD)
+        Ws, bs = W.policy_weights(WORKLOAD, self.dims, 1)
+        self.host_params = np.concatenate([np.concatenate([w.ravel(), b.ravel()])
+                                           for w, b in zip(Ws, bs)]).astype(np.float32)
+        self.params = torch.from_numpy(self.host_params.copy()).cuda()
+        self.policy = simx.Policy.from_flat(self.params, self.dims, hv)
+        n = self.params.numel()
+        self.m = torch.zeros(n, device="cuda")
+        self.v = torch.zeros(n, device="cuda")
+        self.grad = torch.empty(n, device="cuda")
+        self.stats = torch.empty(5, device="cuda")
+        self.adam_ws = torch.empty(simx.adam_workspace_size(n), dtype=torch.uint8, device="cuda")
+        self.t_dev = torch.zeros(1, dtype=torch.int64, device="cuda")
+        self.sim = simx.Sim(cfg, device=device)
+        self.sim.reset(seed)
+        self.D = self.sim.D
+        self.buf = simx.alloc_rollout(self.E, self.D, self.H, has_value=True)
+        self.ret = torch.empty((self.H, self.E), device="cuda")
+        self.adv = torch.empty((self.H, self.E), device="cuda")
+        self.last = torch.empty(self.E, device="cuda")
+        self.obs_next = torch.empty((self.D, self.E), device="cuda")
+        self.pf_ws = torch.empty(simx.policy_forward_workspace_size(self.policy),
+                                 dtype=torch.uint8, device="cuda")
+        self.n_rows = self.E * self.H
+        self.n_mb = self.n_rows // self.mb
+        self.loss_ws = torch.empty(simx.ppo_loss_grad_workspace_size(self.policy, self.mb),
+                                   dtype=torch.uint8, device="cuda")
+        self.perm = torch.empty((epochs, self.n_rows), dtype=torch.int64, device="cuda")
+        self.gen = torch.Generator(device="cuda")
+        self.gen.manual_seed(seed)
+        self.graph = None
+        self.graph_launches = 0
+        self.replays = 0
+
+    def _updates(self):
+        s = self.simx
+        for e in range(self.epochs):
+            for i in range(self.n_mb):
+                s.ppo_loss_grad(self.policy, self.buf, self.ret, self.adv,
+                                self.perm[e, i * self.mb:(i + 1) * self.mb], self.mb, "ppo", CLIP,
+                                C_VALUE, C_ENTROPY, self.grad, self.stats, self.loss_ws,
+                                precision=self.precision)
+                s.adam_step(self.params, self.grad, self.m, self.v, self.t_dev, LR,
+                            max_grad_norm=MAX_NORM, workspace=self.adam_ws)
+
+    def run(self, ev=None):
+        """One step; ev: five CUDA events bracketing the permutation draw, the rollout, the
+        bootstrap + GAE and the PPO updates."""
+        torch, s, stream = self.torch, self.simx, self.torch.cuda.current_stream()
+
+        def mark(i):
+            if ev:
+                ev[i].record(stream)
+        mark(0)
+        for e in range(self.epochs):
+            self.perm[e] = torch.randperm(self.n_rows, device="cuda", generator=self.gen)
+        mark(1)
+        self.sim.rollout("sample", self.H, self.buf, self.policy)
+        mark(2)
+        self.sim.observe(self.obs_next)
+        s.policy_forward(self.policy, self.obs_next, self.E, "argmax", 0, 0, value=self.last,
+                         workspace=self.pf_ws)
+        s.compute_returns_gae(self.buf["reward"], self.buf["done"], GAMMA, LAMBDA, self.ret,
+                              adv=self.adv, val=self.buf["value"], last_val=self.last)
+        mark(3)
+        if self.graph is None:
+            self._updates()          # eager: sizes every library-side buffer first
+            self.graph = torch.cuda.CUDAGraph()
+            l0 = s.launches()
+            with torch.cuda.graph(self.graph, capture_error_mode="relaxed"):
+                self._updates()
+            self.graph_launches = s.launches() - l0   # library kernels in one replay
+        else:
+            self.graph.replay()
+            self.replays += 1
+        mark(4)
+
+    def close(self):
+        self.sim.close()
+
+
+def _minibatch_loss_ms(st, torch, reps: int = 20) -> dict:
+    """Average duration of one loss-gradient call and one Adam call of the step's update
+    loop, each timed alone (CUDA events on the stream, after the timed region)."""
+    s = st.simx
+    idx = st.perm[0, :st.mb]
+    out = {}
+    for name, fn in (("loss", lambda: s.ppo_loss_grad(st.policy, st.buf, st.ret, st.adv, idx, st.mb,
+                                                      "ppo", CLIP, C_VALUE, C_ENTROPY, st.grad,
+                                                      st.stats, st.loss_ws,
+                                                      precision=st.precision)),
+                     ("adam", lambda: s.adam_step(st.params, st.grad, st.m, st.v, st.t_dev, LR,
+                                                  max_grad_norm=MAX_NORM, workspace=st.adam_ws))):
+        fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        out[name] = e0.elapsed_time(e1) / reps
+    return out
+
+
+def _c2_extra(simx, W, torch, reps: int = 5) -> dict:
+    """The single-server workload (4096 envs x 512, MMPP, MLP 16-64-64-12, REINFORCE with
+    a mean baseline): rollout + returns + baseline + loss gradient over all rows."""
+    E, H = 4096, W.HORIZON["c2"]
+    dims, hv = W.mlp_dims("c2")
+    Ws, bs = W.mlp_weights(dims, 1)
+    pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws], [torch.from_numpy(b).cuda() for b in bs], hv)
+    sim = simx.Sim(W.c2(E))
+    sim.reset(0x5EED0002)
+    n = E * H
+    buf = simx.alloc_rollout(E, sim.D, H)
+    ret = torch.empty((H, E), device="cuda")
+    adv = torch.empty((H, E), device="cuda")
+    mean = torch.empty(1, device="cuda")
+    ws_b = torch.empty(simx.returns_baseline_workspace_size(n), dtype=torch.uint8, device="cuda")
+    grad = torch.empty(pol.n_params, device="cuda")
+    stats = torch.empty(5, device="cuda")
+    ws_l = torch.empty(simx.ppo_loss_grad_workspace_size(pol, n), dtype=torch.uint8, device="cuda")
+
+    def step():
+        sim.rollout("sample", H, buf, pol)
+        simx.compute_returns_gae(buf["reward"], buf["done"], GAMMA, -1.0, ret)
+        simx.returns_baseline(ret, adv, mean, ws_b)
+        simx.ppo_loss_grad(pol, buf, ret, adv, None, n, "reinforce", 0.2, 0.0, 0.0, grad, stats,
+                           ws_l, precision="tf32")
+    for _ in range(3):
+        step()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    sim.close()
+    return {"workload": "c2: 4096 envs x 512, MMPP 300/3000 req/s, MLP 16-64-64-12, REINFORCE + "
+                        "mean baseline, loss over all rows (tf32)",
+            "ms_per_step": ms, "decision_steps_per_s": n / (ms * 1e-3), "steps": reps}
+
+
+def _c5_extra(simx, W, torch, E: int = 1048576) -> dict:
+    """c5 at its largest size: the argmax rollout of 1,048,576 envs x 1024 steps and GAE."""
+    H = W.HORIZON["c5"]
+    dims, hv = W.mlp_dims("c5")
+    Ws, bs = W.policy_weights("c5", dims, 1)
+    pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws], [torch.from_numpy(b).cuda() for b in bs], hv)
+    sim = simx.Sim(W.c5(E))
+    sim.reset(W.SEED["c5"])
+    buf = simx.alloc_rollout(E, sim.D, H, has_value=True)
+    sim.rollout("argmax", 8, buf, pol)
+    adv = torch.empty((H, E), device="cuda")
+    ret = torch.empty((H, E), device="cuda")
+    last = torch.zeros(E, device="cuda")
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    e[0].record()
+    sim.rollout("argmax", H, buf, pol)
+    e[1].record()
+    simx.compute_returns_gae(buf["reward"], buf["done"], GAMMA, LAMBDA, ret, adv=adv,
+                             val=buf["value"], last_val=last)
+    e[2].record()
+    torch.cuda.synchronize()
+    r_ms, g_ms = e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2])
+    st, _ = sim.last_status()
+    sim.close()
+    del buf, adv, ret
+    torch.cuda.empty_cache()
+    return {"workload": "c5: %d envs x %d, argmax, MLP 13-128-128-16+V" % (E, H), "status": st,
+            "rollout_ms": r_ms, "decision_steps_per_s": E * H / (r_ms * 1e-3),
+            "gae_ms": g_ms, "gae_samples_per_s": E * H / (g_ms * 1e-3)}
+
+
 def run_gpu(a) -> None:
     import numpy as np
     import torch
@@ -525,72 +741,38 @@ def run_gpu(a) -> None:
         import torch.distributed as dist
         dist.init_process_group("nccl")
 
-    # Replicas: every rank simulates its own 4096 envs (seed offset by rank); no
-    # data-path collective, only the timing barrier and max-reduction.
-    E, H = 4096, W.HORIZON[WORKLOAD]
-    cfg = W.c2(E)
-    dims, hv = W.mlp_dims(WORKLOAD)
-    Ws, bs = W.mlp_weights(dims, 1)
-    dWs = [torch.from_numpy(w).cuda() for w in Ws]
-    dbs = [torch.from_numpy(b).cuda() for b in bs]
-    pol = simx.Policy(dWs, dbs, hv)
-    sim = simx.Sim(cfg, device=local)
-    sim.reset(replica_seed(rank))
-    D = sim.D
-    n = E * H
-    buf = simx.alloc_rollout(E, D, H)
-    ret = torch.empty((H, E), device="cuda")
-    adv = torch.empty((H, E), device="cuda")
-    mean = torch.empty(1, device="cuda")
-    ws_b = torch.empty(simx.returns_baseline_workspace_size(n), dtype=torch.uint8, device="cuda")
-    grad = torch.empty(pol.n_params, device="cuda")
-    stats = torch.empty(5, device="cuda")
-    ws_l = torch.empty(simx.ppo_loss_grad_workspace_size(pol, n), dtype=torch.uint8, device="cuda")
+    # Replicas: every rank simulates and trains on its own 65,536 envs (seed offset by
+    # rank); no data-path collective, only the timing barrier and max-reduction.
+    st = PPOStep(simx, W, torch, replica_seed(rank), a.epochs, a.loss_precision, local)
+    E, H, n = st.E, st.H, st.n_rows
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
-    fp = measure_fp32_peak(simx, torch)  # FP32 roofline denominator, measured on this GPU
-    stream = torch.cuda.current_stream()
-
-    def step(ev=None):
-        if ev:
-            ev[0].record(stream)
-        sim.rollout("sample", H, buf, pol)
-        if ev:
-            ev[1].record(stream)
-        simx.compute_returns_gae(buf["reward"], buf["done"], GAMMA, -1.0, ret)
-        if ev:
-            ev[2].record(stream)
-        simx.returns_baseline(ret, adv, mean, ws_b)
-        if ev:
-            ev[3].record(stream)
-        simx.ppo_loss_grad(pol, buf, ret, adv, None, n, "reinforce", 0.2, 0.0, 0.0, grad, stats,
-                           ws_l, precision=a.loss_precision)
-        if ev:
-            ev[4].record(stream)
+    fp = measure_fp32_peak(simx, torch)
 
     for _ in range(a.warmup):
-        step()
+        st.run()
     torch.cuda.synchronize()
 
-    # candidates generated per rollout launch (for the algorithmic FLOP count)
-    cj0 = sim.save()[:, 2].astype(np.int64)
+    cj0 = st.sim.save()[:, 2].astype(np.int64)   # arrival candidates drawn so far
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(a.steps)]
     clocks = Clocks(local) if rank == 0 else None
-    l0 = simx.launches()
+    l0, r0 = simx.launches(), st.replays
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
     t_wall = time.perf_counter()
     for k in range(a.steps):
         flush.zero_()  # evict L2 between steps (outside the timed events)
-        step(evs[k])
+        st.run(evs[k])
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     t_wall = time.perf_counter() - t_wall
-    launches = simx.launches() - l0
+    # launches made from the host plus the library kernels inside every graph replay
+    launches = simx.launches() - l0 + (st.replays - r0) * st.graph_launches
     clk = clocks.stop() if clocks else None
-    cj1 = sim.save()[:, 2].astype(np.int64)
+    cj1 = st.sim.save()[:, 2].astype(np.int64)
     cand_per_launch = float((cj1 - cj0).sum()) / a.steps
+    state_status = st.sim.last_status()
 
     phase_ms = [[evs[k][i].elapsed_time(evs[k][i + 1]) for i in range(4)] for k in range(a.steps)]
     step_ms = [evs[k][0].elapsed_time(evs[k][4]) for k in range(a.steps)]
@@ -598,102 +780,79 @@ def run_gpu(a) -> None:
     ph = [statistics.mean(p[i] for p in phase_ms) for i in range(4)]
     ms = max_over_ranks(ms, dist, "cuda")
     value = job_value(world, n, ms)
-    st, code = sim.last_status()
-    if st != 0:
-        raise RuntimeError("device status 0x%x after the timed region" % code)
+    if state_status[0] != 0:
+        raise RuntimeError("device status 0x%x after the timed region" % state_status[1])
 
-    # end to end through the public API: policy in from pinned host memory, gradient and
-    # statistics back to the host, every step
+    # end to end through the public API: the policy's parameters in from pinned host
+    # memory, the updated parameters and the last update's statistics back, every step
     e2e = None
     if not a.no_e2e:
-        hW = [torch.from_numpy(w).pin_memory() for w in Ws]
-        hb = [torch.from_numpy(b).pin_memory() for b in bs]
-        hg = torch.empty(pol.n_params, dtype=torch.float32).pin_memory()
+        hp = torch.from_numpy(st.host_params.copy()).pin_memory()
+        hout = torch.empty_like(hp).pin_memory()
         hs = torch.empty(5, dtype=torch.float32).pin_memory()
-        h2d = sum(w.numel() * 4 for w in hW) + sum(b.numel() * 4 for b in hb)
-        d2h = hg.numel() * 4 + hs.numel() * 4
-        k_e2e = max(3, min(a.steps, 50))
+        k_e2e = max(3, min(a.steps, 10))
         if dist:
             dist.barrier()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         for _ in range(k_e2e):
-            for d, h in zip(dWs + dbs, hW + hb):
-                d.copy_(h, non_blocking=True)
-            step()
-            hg.copy_(grad, non_blocking=True)
-            hs.copy_(stats, non_blocking=True)
+            st.params.copy_(hp, non_blocking=True)
+            st.run()
+            hout.copy_(st.params, non_blocking=True)
+            hs.copy_(st.stats, non_blocking=True)
             torch.cuda.synchronize()
         t_e2e = (time.perf_counter() - t0) / k_e2e
         t_e2e = max_over_ranks(t_e2e, dist, "cuda")
-        e2e = {"value": job_value(world, n, t_e2e * 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h}
+        e2e = {"value": job_value(world, n, t_e2e * 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": hp.numel() * 4,
+               "d2h_bytes_per_step": hout.numel() * 4 + hs.numel() * 4}
 
-    # the loss gradient in the other precision, on the same buffer, for comparison
-    other = "fp32" if a.loss_precision == "tf32" else "tf32"
-    lo_ms = []
-    for _ in range(5):
-        flush.zero_()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        simx.ppo_loss_grad(pol, buf, ret, adv, None, n, "reinforce", 0.2, 0.0, 0.0, grad, stats,
-                           ws_l, precision=other)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        lo_ms.append(e0.elapsed_time(e1))
-    loss_other_ms = statistics.median(lo_ms[1:])
+    mb_ms = _minibatch_loss_ms(st, torch)
 
     # the policy-free batched step (Sec. 5.1 Shortest-Queue router) of the multi-server
-    # environment at 65,536 envs: state read and written every step, HBM-bound
+    # environment: state read and written every step, HBM-bound
     hbm_step = None if a.no_hbm_step else [hbm_step_measure(simx, W, torch, E=e)
                                             for e in (65536, 1048576)]
+    extras = None
+    if rank == 0 and not a.no_extras:
+        extras = {"c2": _c2_extra(simx, W, torch), "c5_1m": _c5_extra(simx, W, torch)}
 
     # roofline of the dominant kernel
     peaks, src = _peaks()
     sm_mhz = float(peaks.get("sm_max_mhz", 2070.0))
-    fp32_nominal = fp["sms"] * 128 * 2 * sm_mhz * 1e6 / 1e12  # FMA lanes x clock
-    fp32_peak = fp["tflops"]
-    fp32_src = ("measured FMA probe (libsimx k_fma_probe, best of 5): %.1f TFLOP/s; nominal "
-                "%d SMs x 128 lanes x 2 x %.0f MHz = %.1f" % (fp32_peak, fp["sms"], sm_mhz,
-                                                            fp32_nominal))
+    fp32_nominal = fp["sms"] * 128 * 2 * sm_mhz * 1e6 / 1e12  # FMA lanes x maximum clock
+    fp32_src = ("%d SMs x 128 FP32 lanes x 2 flops x %.0f MHz (unit counts and maximum clock); "
+                "the library's FMA probe measures %.1f TFLOP/s" % (fp["sms"], sm_mhz, fp["tflops"]))
+    dims = st.dims
     P = sum(dims[l] * dims[l + 1] for l in range(len(dims) - 1))
     hidden = sum(dims[1:-1])
-    A = dims[-1] - (1 if hv else 0)
+    A = dims[-1] - 1
     flop_rollout = n * (2.0 * P + 20.0 * hidden + 20.0 * A) + 15.0 * cand_per_launch
-    flop_loss = n * (6.0 * P - 2.0 * dims[0] * dims[1])
-    phases = {"rollout_ms": ph[0], "returns_ms": ph[1], "baseline_ms": ph[2], "loss_grad_ms": ph[3],
-              "loss_grad_%s_ms" % other: loss_other_ms}
-    # the loss kernel against its own bound: FP32 lanes, or the TF32 tensor pipe (nominally
-    # half the bf16 rate; the measured bf16 GEMM peak x 0.5)
+    flop_mb = st.mb * (6.0 * P - 2.0 * dims[0] * dims[1])
+    update_ms = ph[3]
+    phases = {"permutation_ms": ph[0], "rollout_ms": ph[1], "bootstrap_gae_ms": ph[2],
+              "ppo_update_ms": update_ms, "minibatches_per_step": st.n_mb * st.epochs,
+              "loss_grad_call_ms": mb_ms["loss"], "adam_call_ms": mb_ms["adam"]}
+    tf32_peak = float(peaks.get("bf16_tflops", 1900.0)) * 0.5
+    loss_share = mb_ms["loss"] / max(mb_ms["loss"] + mb_ms["adam"], 1e-9)
+    loss_live_ms = update_ms * loss_share / (st.n_mb * st.epochs)
+    ach_l = flop_mb / (loss_live_ms * 1e-3) / 1e12
     if a.loss_precision == "tf32":
-        tf32_peak = float(peaks.get("bf16_tflops", 1900.0)) * 0.5
-        ach_l = flop_loss / (ph[3] * 1e-3) / 1e12
-        roof_loss = {"kernel": "k_loss_tc (tcgen05 kind::tf32)", "bound": "tensor", "achieved": ach_l,
-                     "peak": tf32_peak, "unit": "TFLOP/s", "frac": ach_l / tf32_peak, "traffic": None,
-                     "peak_source": "%s bf16_tflops x 0.5 (nominal tf32 / bf16 rate)" % src}
+        roof_loss = {"kernel": "loss gradient (tensor-core tf32 kernels)", "bound": "tensor",
+                     "achieved": ach_l, "peak": tf32_peak, "unit": "TFLOP/s", "frac": ach_l / tf32_peak,
+                     "traffic": None, "peak_source": "%s bf16_tflops x 0.5 (nominal tf32 / bf16 rate)" % src,
+                     "ms_per_call": loss_live_ms}
     else:
-        ach_l = flop_loss / (ph[3] * 1e-3) / 1e12
-        roof_loss = {"kernel": "k_loss_fused (FP32 SIMT)", "bound": "alu", "achieved": ach_l,
-                     "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach_l / fp32_peak, "traffic": None,
-                     "peak_source": fp32_src}
-    dom = max(range(4), key=lambda i: ph[i])
-    if dom == 0:
-        ach = flop_rollout / (ph[0] * 1e-3) / 1e12
-        roof = {"kernel": "k_rollout (simulation + fused policy)", "bound": "alu", "achieved": ach,
-                "peak": fp32_peak, "unit": "TFLOP/s", "frac": ach / fp32_peak,
-                "traffic": ROLLOUT_DRAM_BYTES,
-                "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one "
-                                  "k_rollout launch of this workload (10.0 MB + 113.8 MB)",
-                "peak_source": fp32_src}
-    elif dom == 3:
-        roof = roof_loss
-    else:
-        hbm = float(peaks.get("hbm_gbs", 6800.0))
-        byts = n * 13.0 if dom == 1 else n * 12.0
-        ach = byts / (ph[dom] * 1e-3) / 1e9
-        roof = {"kernel": "returns" if dom == 1 else "baseline", "bound": "hbm", "achieved": ach,
-                "peak": hbm, "unit": "GB/s", "frac": ach / hbm, "traffic": None,
-                "peak_source": "%s hbm_gbs" % src}
+        roof_loss = {"kernel": "loss gradient (FP32 SIMT kernels)", "bound": "alu", "achieved": ach_l,
+                     "peak": fp32_nominal, "unit": "TFLOP/s", "frac": ach_l / fp32_nominal,
+                     "traffic": None, "peak_source": fp32_src, "ms_per_call": loss_live_ms}
+    ach_r = flop_rollout / (ph[1] * 1e-3) / 1e12
+    roof_rollout = {"kernel": "k_rollout (simulation + fused policy)", "bound": "alu",
+                    "achieved": ach_r, "peak": fp32_nominal, "unit": "TFLOP/s",
+                    "frac": ach_r / fp32_nominal, "traffic": ROLLOUT_DRAM_BYTES,
+                    "traffic_source": ROLLOUT_DRAM_SOURCE, "peak_source": fp32_src,
+                    "flop_per_launch": flop_rollout}
+    roof = roof_rollout if ph[1] >= update_ms * loss_share else roof_loss
 
     if rank == 0:
         line = {
@@ -701,26 +860,27 @@ def run_gpu(a) -> None:
             "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32+tf32" if a.loss_precision == "tf32" else "f32",
             "data": "synthetic",
-            "config": {"workload": "c2: 4096 envs x 512 steps per GPU, MMPP 300/3000 req/s, "
-                                   "80/20 short/long, MLP 16-64-64-12, REINFORCE + mean baseline",
-                       "envs_per_gpu": E, "horizon": H, "l2": "flushed (256 MB write) before every "
-                       "timed step", "parallelism": "replicas" if world > 1 else "single GPU",
-                       "loss_precision": "tf32 tensor cores, split tf32 first layer, fp32 "
-                       "accumulation (parity 1e-2)" if a.loss_precision == "tf32" else
-                       "fp32 (parity 1e-5)"},
+            "config": {"workload": WORKLOAD_TEXT, "envs_per_gpu": E, "horizon": H,
+                       "ppo_epochs_per_step": st.epochs, "minibatch": st.mb,
+                       "l2": "flushed (256 MB write) before every timed step",
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "loss_precision": "tf32 tensor cores, fp32 accumulation (parity 1e-2)"
+                       if a.loss_precision == "tf32" else "fp32 (parity 1e-5)"},
             "phases_ms": phases,
             "roofline": roof,
+            "roofline_rollout": roof_rollout,
             "roofline_loss": roof_loss,
             "e2e": e2e,
             "hbm_step": hbm_step,
+            "extras": extras,
             "gpu_launches": launches,
             "clocks": clk,
             "wall_s": t_wall,
         }
         if world == 1 and not a.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_baseline()
+            line["cpu_baseline"] = cpu_baseline(a.epochs)
         print(json.dumps(line), flush=True)
-    sim.close()
+    st.close()
     if dist:
         dist.destroy_process_group()
 
