@@ -404,7 +404,7 @@ simx_status ppo_loss_grad(const simx_mlp* pol, const simx_rollout* buf, int64_t 
  *     caller.  Calls on different devices do not share scratch.  Nothing needs to
  *     start at zero: each call writes all scratch it reads.
  */
-#define SIMX_NOALLOC_SCRATCH_BYTES (16u << 20)
+#define SIMX_NOALLOC_SCRATCH_BYTES (64u << 20)
 simx_status ppo_loss_grad_noalloc(const simx_mlp* pol, const simx_rollout* buf,
                                   int64_t n_rows_per_step, const float* d_ret, const float* d_adv,
                                   const int64_t* d_idx, int64_t n, const simx_loss_params* params,

@@ -117,6 +117,9 @@ size_t loss_fused_workspace(const LossArgs& a);
 cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 void launch_loss_reduce(const float* part, int nb, int n_params, const double* spart,
                         const LossArgs& a, cudaStream_t s);
+// the same with nbs statistics partials (nb gradient partials summed in order)
+void launch_loss_reduce_n(const float* part, int nb, int n_params, const double* spart, int nbs,
+                          const LossArgs& a, cudaStream_t s);
 // fma_probe.cu
 cudaError_t launch_fma_probe(int64_t iters, float* sink, double* flops, cudaStream_t s);
 
@@ -130,6 +133,10 @@ size_t fma_probe_sink_floats();
 bool loss_tc_fits(const LossArgs& a);
 size_t loss_tc_workspace(const LossArgs& a);
 cudaError_t launch_loss_tc(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
+// loss_wide.cu
+bool loss_wide_fits(const LossArgs& a);
+size_t loss_wide_workspace(const LossArgs& a);
+cudaError_t launch_loss_wide(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s);
 
 }  // namespace simx

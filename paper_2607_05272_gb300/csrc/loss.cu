@@ -372,15 +372,18 @@ static WsLayout layout(const LossArgs& a) {
 // Large enough for every path, so that the size does not depend on the precision.
 size_t loss_workspace_bytes(const LossArgs& a) {
   const size_t f = loss_fused_fits(a) ? loss_fused_workspace(a) : layout(a).total;
-  const size_t t = loss_tc_workspace(a);
+  const bool tc = loss_tc_fits(a);
+  const size_t t = tc ? loss_tc_workspace(a) : loss_wide_workspace(a);
   return f > t ? f : t;
 }
 
-// TF32 requests whose policy fits the tensor-core kernel take it (loss_tc.cu); otherwise
-// policies whose parameters and per-tile activations fit in shared memory take the fused
-// FP32 one-kernel path (loss_fused.cu), and wider ones the GEMM pipeline below.
+// TF32 requests whose policy fits the one-SM tensor-core kernel take it (loss_tc.cu), and
+// wider tanh policies (layers up to 256) the streamed tensor-core kernels (loss_wide.cu);
+// otherwise policies whose parameters and per-tile activations fit in shared memory take
+// the fused FP32 one-kernel path (loss_fused.cu), and wider ones the GEMM pipeline below.
 cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s) {
   if (a.precision == SIMX_PREC_TF32 && loss_tc_fits(a)) return launch_loss_tc(a, ws, ws_bytes, s);
+  if (a.precision == SIMX_PREC_TF32 && loss_wide_fits(a)) return launch_loss_wide(a, ws, ws_bytes, s);
   if (loss_fused_fits(a)) return launch_loss_fused(a, ws, ws_bytes, s);
   const WsLayout w = layout(a);
   if (ws_bytes < w.total) return cudaErrorInvalidValue;

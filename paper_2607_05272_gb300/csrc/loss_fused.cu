@@ -674,8 +674,13 @@ cudaError_t launch_loss_fused(const LossArgs& a, void* ws, size_t ws_bytes, cuda
 // fp64 statistics into a.stats.
 void launch_loss_reduce(const float* part, int nb, int n_params, const double* spart,
                         const LossArgs& a, cudaStream_t s) {
+  launch_loss_reduce_n(part, nb, n_params, spart, nb, a, s);
+}
+
+void launch_loss_reduce_n(const float* part, int nb, int n_params, const double* spart, int nbs,
+                          const LossArgs& a, cudaStream_t s) {
   k_reduce_blocks<<<(n_params + 255) / 256, 256, 0, s>>>(part, nb, n_params, a.grad);
-  k_fused_stats<<<1, 128, 0, s>>>(spart, nb, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
+  k_fused_stats<<<1, 128, 0, s>>>(spart, nbs, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
   count_launches(2);
 }
 

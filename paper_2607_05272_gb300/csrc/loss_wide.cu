@@ -1,0 +1,777 @@
+// loss_wide.cu — REINFORCE / PPO loss gradient (Sec. 4.3) on the tensor cores for tanh
+// policies whose layers are up to 256 wide (c3 / c5: 13-128-128-17, c4: 28-256-256-49),
+// too wide for loss_tc.cu's kernel, which holds every operand of a policy in one SM.
+//
+// Notation: L layers, H_0 = X (the minibatch's observations), Z_l = H_l W_l^T + b_l,
+// H_{l+1} = tanh(Z_l); G_l = dL/dZ_l.  Backward: dH_l = G_l W_l and
+// G_{l-1} = dH_l * (1 - H_l^2); dW_l = G_l^T H_l, db_l = sum over rows of G_l.
+// Every matrix product is a chain of tcgen05.mma kind::tf32 (TF32 inputs, FP32
+// accumulation in tensor memory) with M = 128.  Three kernels per call:
+//
+//   k_lw_prep  the policy's weights as MMA operand images in global memory: W_l (the
+//              forward B operand) and W_l^T (the backward one) cut into chunks of 32 K
+//              values, each chunk laid out exactly as the shared-memory operand so that
+//              one bulk copy moves it; TF32 rounded.  The first layer's image is
+//              [W_hi | W_lo | W_hi], the split-TF32 product x_hi w_hi + x_hi w_lo +
+//              x_lo w_hi as one GEMM against [x_hi | x_hi | x_lo] (raw observations reach
+//              magnitudes in the hundreds; one TF32 pass there moves saturated tanh units'
+//              derivatives by percents).
+//   k_lw_rows  one CTA per 128-row tile: the whole forward pass, the loss head and the
+//              backward pass down to G_0 for its rows.  The A operand (the tile's
+//              activations, or G) stays resident in shared memory, written by the
+//              epilogue of the previous product; the weight chunks stream through a ring
+//              of shared-memory stages by bulk copies, the MMAs of chunk c queued before
+//              the stage of chunk c - 1 is refilled.  H_l and G_l go to global memory as
+//              feature-major images (the layout of the weight-gradient products).
+//   k_lw_dw    [dW_l | db_l] = G_l^T [H_l | 1] with K = the rows, split over CTAs by
+//              (layer, block of 128 outputs, row range); each CTA writes its slice of
+//              one full-length partial gradient per row range, which the block reduction
+//              shared with the other loss paths sums in range order (deterministic).
+//
+// Elementwise work between the products (bias, tanh, the loss head, 1 - h^2) is done
+// in FP32 by threads reading the accumulators with tcgen05.ld: thread = TMEM lane =
+// tile row, the two warps of a lane quarter splitting the columns.  Accuracy is that of
+// TF32 inputs (about 1e-3 relative per product), held to 1e-2 by the tests; the FP32 SIMT
+// kernels are the exact alternative.
+#include <cstdint>
+
+#include "kernels.h"
+#include "tc_common.cuh"
+
+namespace simx {
+namespace lw {
+
+using namespace tcx;
+
+constexpr int kR = 128;            // rows per tile (MMA M)
+constexpr int kThreads = 256;      // 8 warps: 2 per TMEM lane quarter
+constexpr int kKC = 32;            // K values per streamed chunk
+constexpr int kMaxStages = 3;
+constexpr long long kWaitCycles = 2000000000LL;  // bound on any wait (about 1 s)
+
+int r16(int x) { return (x + 15) / 16 * 16; }
+int r32(int x) { return (x + 31) / 32 * 32; }
+
+struct Plan {
+  bool ok;
+  int L, n_params;
+  int K[SIMX_MAX_LAYERS], N[SIMX_MAX_LAYERS];
+  int Ka[SIMX_MAX_LAYERS];   // forward A width (GEMM K): 3 r32(K_0) for layer 0, r32(K_l) after
+  int Nf[SIMX_MAX_LAYERS];   // forward MMA N: r16(N_l)
+  int Gk[SIMX_MAX_LAYERS];   // backward A width (GEMM K of dH_l = G_l W_l): r32(N_l)
+  int Kb[SIMX_MAX_LAYERS];   // backward MMA N: r16(K_l)
+  int Fh[SIMX_MAX_LAYERS];   // features of the H_l image: r16(K_l)
+  int Fg[SIMX_MAX_LAYERS];   // features of the G_l image: r16(N_l)
+  int poff[SIMX_MAX_LAYERS];
+  // k_lw_rows
+  int a_bytes, stage_bytes, nstages, smem, tcols;
+  // k_lw_dw
+  int mt0[SIMX_MAX_LAYERS];  // first work item of layer l (blocks of 128 outputs)
+  int mt_total, S, dw_stage_bytes, dw_nstages, dw_smem, dw_tcols;
+  int64_t n_pad, ntiles, nchunks;
+  // workspace byte offsets
+  size_t wf[SIMX_MAX_LAYERS], wb[SIMX_MAX_LAYERS], img_h[SIMX_MAX_LAYERS], img_g[SIMX_MAX_LAYERS];
+  size_t part, spart, total;
+  int64_t wf_elems[SIMX_MAX_LAYERS], wb_elems[SIMX_MAX_LAYERS];
+};
+
+struct Args {
+  LossArgs a;
+  Plan p;
+  unsigned char* ws;
+};
+
+// Byte offset of (feature f, row r) in a feature-major image of F features: blocks of
+// 32 rows, in each block the feature groups of 8 one after another, each group the
+// K-major operand of 8 features x 32 rows (8 core matrices of 4 rows).
+__device__ __forceinline__ size_t img_off(int f, int64_t r, int F) {
+  return (size_t)((r >> 5) * (F >> 3) + (f >> 3)) * 1024 + (size_t)(((r & 31) >> 2) * 128 + (f & 7) * 16 + (r & 3) * 4);
+}
+
+// Byte offset of (row j, value kk) inside one 32-value chunk of a weight image.
+__device__ __forceinline__ uint32_t chunk_off(int j, int kk) {
+  return (uint32_t)((j >> 3) * 1024 + (kk >> 2) * 128 + (j & 7) * 16 + (kk & 3) * 4);
+}
+
+// ---------------------------------------------------------------------------------
+// k_lw_prep: the weight operand images of every layer (TF32 rounded, zero padded).
+// ---------------------------------------------------------------------------------
+__global__ void k_lw_prep(const __grid_constant__ Args A) {
+  const LossArgs& a = A.a;
+  const Plan& P = A.p;
+  int64_t total = 0;
+  for (int l = 0; l < P.L; ++l) total += P.wf_elems[l] + P.wb_elems[l];
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    int64_t q = i;
+    int l = 0;
+    bool fwd = true;
+    for (; l < P.L; ++l) {
+      if (q < P.wf_elems[l]) { fwd = true; break; }
+      q -= P.wf_elems[l];
+      if (q < P.wb_elems[l]) { fwd = false; break; }
+      q -= P.wb_elems[l];
+    }
+    const int K = P.K[l], N = P.N[l];
+    const float* W = a.W[l];
+    if (fwd) {
+      // chunk c of Nf rows x 32 values; element (row j = output, kk)
+      const int Nf = P.Nf[l];
+      const int c = (int)(q / (Nf * kKC)), rem = (int)(q % (Nf * kKC));
+      const int j = rem / kKC, kk = rem % kKC;
+      float v;
+      if (l == 0) {
+        const int per = P.Ka[0] / 3 / kKC;  // chunks of one copy of K_0
+        const int part = c / per, k = kKC * (c % per) + kk;
+        const float w = (j < N && k < K) ? W[(size_t)j * K + k] : 0.0f;
+        const float hi = to_tf32(w);
+        v = part == 1 ? to_tf32(w - hi) : hi;
+      } else {
+        const int k = kKC * c + kk;
+        v = (j < N && k < K) ? to_tf32(W[(size_t)j * K + k]) : 0.0f;
+      }
+      float* dst = reinterpret_cast<float*>(A.ws + P.wf[l] + (size_t)c * Nf * kKC * 4 + chunk_off(j, kk));
+      *dst = v;
+    } else {
+      // chunk c of Kb rows (input units k) x 32 values (outputs j = 32 c + jj)
+      const int Kb = P.Kb[l];
+      const int c = (int)(q / (Kb * kKC)), rem = (int)(q % (Kb * kKC));
+      const int k = rem / kKC, jj = rem % kKC;
+      const int j = kKC * c + jj;
+      const float v = (k < K && j < N) ? to_tf32(W[(size_t)j * K + k]) : 0.0f;
+      float* dst = reinterpret_cast<float*>(A.ws + P.wb[l] + (size_t)c * Kb * kKC * 4 + chunk_off(k, jj));
+      *dst = v;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// k_lw_rows: forward, loss head and backward of one 128-row tile.
+// ---------------------------------------------------------------------------------
+__device__ __forceinline__ float tanh_fast(float x) {
+  return 1.0f - __fdividef(2.0f, __expf(2.0f * x) + 1.0f);
+}
+
+struct Smem {
+  unsigned char* abuf;     // the resident A operand (activations or G of the tile)
+  unsigned char* stages;   // ring of weight chunks
+  uint64_t* full;          // [kMaxStages] chunk landed (bulk copy transactions)
+  uint64_t* mmab;          // [kMaxStages] MMAs reading the stage completed
+  uint64_t* drain;         // every MMA of the CTA completed (end of kernel)
+  uint32_t* tbase;         // tensor memory base address
+  int* abort_flag;         // a wait timed out: stop issuing work
+  double* dstat;           // [4 warps][4] statistics
+};
+
+__device__ __forceinline__ Smem carve(unsigned char* sm, const Plan& P, int stage_bytes, int nstages,
+                                      int a_bytes) {
+  Smem s;
+  s.abuf = sm;
+  s.stages = sm + a_bytes;
+  unsigned char* m = sm + a_bytes + (size_t)nstages * stage_bytes;
+  s.full = reinterpret_cast<uint64_t*>(m);
+  s.mmab = s.full + kMaxStages;
+  s.drain = s.mmab + kMaxStages;
+  s.tbase = reinterpret_cast<uint32_t*>(s.drain + 1);
+  s.abort_flag = reinterpret_cast<int*>(s.tbase + 1);
+  s.dstat = reinterpret_cast<double*>(m + 128);
+  (void)P;
+  return s;
+}
+
+// Thread 0's side of one GEMM  D = A B^T  over nc chunks of 32 K values: A resident at
+// a_addr (row-group stride a_sbo), B chunks of bbytes streamed from bsrc through the
+// stage ring.  `next` counts the chunks of every earlier GEMM of the kernel (stage and
+// barrier parity follow from it); issued / consumed track this thread's loads and MMAs.
+__device__ void gemm_issue(const Smem& s, int S, int stage_bytes, int next, int& issued,
+                           int& consumed, uint32_t a_addr, uint32_t a_sbo, const unsigned char* bsrc,
+                           uint32_t bbytes, int nc, int Nmma, uint32_t dtm) {
+  const uint32_t id = idesc_tf32(kR, Nmma);
+  auto load = [&](int c) -> bool {
+    const int k = next + c, st = k % S;
+    if (k >= S && !mbar_wait(&s.mmab[st], (uint32_t)(((k - S) / S) & 1), kWaitCycles)) return false;
+    mbar_arrive_expect_tx(&s.full[st], bbytes);
+    bulk_g2s(s.stages + (size_t)st * stage_bytes, bsrc + (size_t)c * bbytes, bbytes, &s.full[st]);
+    issued = k + 1;
+    return true;
+  };
+  const int pre = nc < S - 1 ? nc : S - 1;
+  for (int c = 0; c < pre; ++c)
+    if (!load(c)) {
+      *s.abort_flag = 1;
+      return;
+    }
+  for (int c = 0; c < nc; ++c) {
+    const int k = next + c, st = k % S;
+    if (!mbar_wait(&s.full[st], (uint32_t)((k / S) & 1), kWaitCycles)) {
+      *s.abort_flag = 1;
+      return;
+    }
+    fence_after();
+    const uint32_t bs = su32(s.stages + (size_t)st * stage_bytes);
+#pragma unroll
+    for (int ks = 0; ks < kKC / 8; ++ks)
+      mma_tf32(dtm, sdesc(a_addr + (uint32_t)c * 1024u + (uint32_t)ks * 256u, 128, a_sbo),
+               sdesc(bs + (uint32_t)ks * 256u, 128, 1024), id, (c | ks) ? 1u : 0u);
+    commit(&s.mmab[st]);
+    consumed = k + 1;
+    if (c + S - 1 < nc && !load(c + S - 1)) {
+      *s.abort_flag = 1;
+      return;
+    }
+  }
+}
+
+// Thread 0 at the end of a kernel: waits (bounded) for loads it issued that no MMA
+// consumed, then for every MMA it issued, so nothing is in flight when the CTA's
+// shared and tensor memory are released.
+__device__ void drain_all(const Smem& s, int S, int issued, int consumed) {
+  for (int k = consumed; k < issued; ++k) mbar_wait(&s.full[k % S], (uint32_t)((k / S) & 1), kWaitCycles);
+  commit(s.drain);
+  mbar_wait(s.drain, 0u, kWaitCycles);
+}
+
+__global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__ Args A) {
+  extern __shared__ __align__(1024) unsigned char sm[];
+  const LossArgs& a = A.a;
+  const Plan& P = A.p;
+  const int L = P.L, S = P.nstages;
+  const Smem s = carve(sm, P, P.stage_bytes, S, P.a_bytes);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int quarter = warp & 3, cq = warp >> 2;
+  const int r = 32 * quarter + lane;
+  const int64_t grow = (int64_t)blockIdx.x * kR + r;   // row of the padded minibatch
+  const bool live = grow < a.n;
+
+  if (tid == 0) {
+    for (int i = 0; i < kMaxStages; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.mmab[i], 1);
+    }
+    mbar_init(s.drain, 1);
+    mbar_fence_init();
+    *s.abort_flag = 0;
+  }
+  if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.tcols);
+
+  // the tile's observations: x_hi, x_hi, x_lo side by side in the A buffer (split TF32)
+  // and the FP32 values in the H_0 image; the head thread's per-row inputs
+  int64_t row = 0;
+  if (live) row = a.idx ? a.idx[grow] : grow;
+  const int64_t t = row / a.E, e = row % a.E;
+  const int D = P.K[0];
+  {
+    const int Kc = P.Ka[0] / 3, W0 = P.Ka[0], F0 = P.Fh[0];
+    unsigned char* img = A.ws + P.img_h[0];
+    for (int cb = cq; cb < Kc / 4; cb += 2) {
+      float hi[4], lo[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int f = 4 * cb + i;
+        const float x = (live && f < D) ? a.obs[(t * D + f) * a.E + e] : 0.0f;
+        hi[i] = to_tf32(x);
+        lo[i] = to_tf32(x - hi[i]);
+        if (f < F0) *reinterpret_cast<float*>(img + img_off(f, grow, F0)) = x;
+      }
+      const float4 h4 = make_float4(hi[0], hi[1], hi[2], hi[3]);
+      *reinterpret_cast<float4*>(s.abuf + rm_off(r, 4 * cb, W0)) = h4;
+      *reinterpret_cast<float4*>(s.abuf + rm_off(r, Kc + 4 * cb, W0)) = h4;
+      *reinterpret_cast<float4*>(s.abuf + rm_off(r, 2 * Kc + 4 * cb, W0)) =
+          make_float4(lo[0], lo[1], lo[2], lo[3]);
+    }
+  }
+  int ac = 0;
+  float adv = 0.0f, lpo = 0.0f, ret = 0.0f;
+  if (cq == 0 && live) {
+    ac = a.action[row];
+    adv = a.adv[row];
+    lpo = a.algo == SIMX_ALGO_PPO ? a.logp_old[row] : 0.0f;
+    ret = a.has_value ? a.ret[row] : 0.0f;
+  }
+
+  auto stage_sync = [&]() -> bool {
+    fence_async_smem();
+    fence_before();
+    __syncthreads();
+    fence_after();
+    return *s.abort_flag == 0;
+  };
+  stage_sync();
+  const uint32_t tmem = *s.tbase;
+  const uint32_t tl = tmem + ((uint32_t)(32 * quarter) << 16);   // this warp's lane quarter
+  const uint32_t abuf_addr = su32(s.abuf);
+  int next = 0, issued = 0, consumed = 0;
+  double st_pg = 0.0, st_v = 0.0, st_h = 0.0, st_cf = 0.0;
+  const float inv_n = 1.0f / (float)a.n;
+
+  // one GEMM: thread 0 streams and issues, every thread then waits for its last commit
+  auto gemm = [&](int a_width, const unsigned char* bsrc, uint32_t bbytes, int nc, int Nmma) -> bool {
+    if (tid == 0 && *s.abort_flag == 0)
+      gemm_issue(s, S, P.stage_bytes, next, issued, consumed, abuf_addr, (uint32_t)(a_width / 4) * 128u,
+                 bsrc, bbytes, nc, Nmma, tmem);
+    const int klast = next + nc - 1;
+    next += nc;
+    if (!mbar_wait(&s.mmab[klast % S], (uint32_t)((klast / S) & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
+    __syncwarp();
+    fence_after();
+    return *s.abort_flag == 0;
+  };
+
+  // Loads columns c0 .. c0 + 15 of this thread's accumulator row (only those < ncols;
+  // the rest read as 0); every thread of the warp takes part (the loads are warp-wide).
+  auto ld16 = [&](int c0, int ncols, float (&z)[16]) {
+    uint32_t u[4][4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (c0 + 4 * q < ncols) tm_ld4_nw(tl + (uint32_t)(c0 + 4 * q), u[q]);
+      else u[q][0] = u[q][1] = u[q][2] = u[q][3] = 0u;
+    }
+    tm_wait();
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      reg_fence(u[q]);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) z[4 * q + i] = __uint_as_float(u[q][i]);
+    }
+  };
+
+  bool ok = true;
+  // ---- forward
+  for (int l = 0; l < L && ok; ++l) {
+    const int Nf = P.Nf[l];
+    ok = gemm(P.Ka[l], A.ws + P.wf[l], (uint32_t)Nf * kKC * 4u, P.Ka[l] / kKC, Nf);
+    if (!ok) break;
+    const int Nl = P.N[l];
+    const float* bias = a.b[l];
+    if (l + 1 < L) {
+      // H_{l+1} = tanh(Z_l + b_l): TF32 into the A buffer (width Ka[l+1], zero padded),
+      // FP32 into the H_{l+1} image; the two warps of a quarter take alternate 16-column
+      // blocks
+      const int Wn = P.Ka[l + 1], Fn = P.Fh[l + 1];
+      unsigned char* img = A.ws + P.img_h[l + 1];
+      for (int c0 = 16 * cq; c0 < Wn; c0 += 32) {
+        float z[16];
+        ld16(c0, Nl, z);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int j0 = c0 + 4 * q;
+          if (j0 >= Wn) break;
+          float h[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int j = j0 + i;
+            h[i] = j < Nl ? tanh_fast(z[4 * q + i] + bias[j]) : 0.0f;
+            if (j < Fn) *reinterpret_cast<float*>(img + img_off(j, grow, Fn)) = h[i];
+          }
+          *reinterpret_cast<float4*>(s.abuf + rm_off(r, j0, Wn)) =
+              make_float4(to_tf32(h[0]), to_tf32(h[1]), to_tf32(h[2]), to_tf32(h[3]));
+        }
+      }
+    } else if (cq == 0) {
+      // loss head for row r: G = dL/dZ over the logits (and the value row)
+      const int NA = a.n_actions;
+      float m = -__uint_as_float(0x7F800000u);
+      for (int c0 = 0; c0 < NA; c0 += 16) {
+        float z[16];
+        ld16(c0, Nl, z);
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if (c0 + i < NA) m = fmaxf(m, z[i] + bias[c0 + i]);
+      }
+      float Ssum = 0.0f;
+      for (int c0 = 0; c0 < NA; c0 += 16) {
+        float z[16];
+        ld16(c0, Nl, z);
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if (c0 + i < NA) Ssum += __expf(z[i] + bias[c0 + i] - m);
+      }
+      const float lse = m + __logf(Ssum);
+      float Hent = 0.0f, lpa = 0.0f, zv = 0.0f;
+      for (int c0 = 0; c0 < Nl; c0 += 16) {
+        float z[16];
+        ld16(c0, Nl, z);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int j = c0 + i;
+          if (j < NA) {
+            const float lp = z[i] + bias[j] - lse;
+            Hent -= __expf(lp) * lp;
+            if (j == ac) lpa = lp;
+          } else if (j == NA && j < Nl) {
+            zv = z[i] + bias[j];
+          }
+        }
+      }
+      float coef = 0.0f, dv = 0.0f;
+      if (live) {
+        float pg;
+        if (a.algo == SIMX_ALGO_REINFORCE) {
+          coef = adv;
+          pg = -adv * lpa;
+        } else {
+          const float rho = __expf(lpa - lpo);
+          const float s1 = rho * adv;
+          const float s2 = fminf(fmaxf(rho, 1.0f - a.clip_eps), 1.0f + a.clip_eps) * adv;
+          pg = -fminf(s1, s2);
+          coef = (s1 <= s2 ? adv : 0.0f) * rho;
+          st_cf += fabsf(rho - 1.0f) > a.clip_eps ? 1.0 : 0.0;
+        }
+        if (a.has_value) {
+          dv = zv - ret;
+          st_v += (double)dv * (double)dv;
+        }
+        st_pg += pg;
+        st_h += Hent;
+      }
+      // G_{L-1}: TF32 into the A buffer (width Gk), FP32 into the G image
+      const int Wg = P.Gk[l], Fg = P.Fg[l];
+      unsigned char* img = A.ws + P.img_g[l];
+      for (int c0 = 0; c0 < Wg; c0 += 16) {
+        float z[16];
+        ld16(c0, Nl, z);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int j0 = c0 + 4 * q;
+          float g[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int j = j0 + i;
+            float v = 0.0f;
+            if (live && j < NA) {
+              const float lp = z[4 * q + i] + bias[j] - lse;
+              const float p = __expf(lp);
+              const float onehot = (j == ac) ? 1.0f : 0.0f;
+              v = (-coef * (onehot - p) + a.c_entropy * p * (lp + Hent)) * inv_n;
+            } else if (live && a.has_value && j == NA) {
+              v = 2.0f * a.c_value * dv * inv_n;
+            }
+            g[i] = v;
+            if (j < Fg) *reinterpret_cast<float*>(img + img_off(j, grow, Fg)) = v;
+          }
+          *reinterpret_cast<float4*>(s.abuf + rm_off(r, j0, Wg)) =
+              make_float4(to_tf32(g[0]), to_tf32(g[1]), to_tf32(g[2]), to_tf32(g[3]));
+        }
+      }
+    }
+    ok = stage_sync();
+  }
+  // ---- backward: dH_l = G_l W_l, G_{l-1} = dH_l (1 - H_l^2)
+  for (int l = L - 1; l >= 1 && ok; --l) {
+    const int Kb = P.Kb[l];
+    ok = gemm(P.Gk[l], A.ws + P.wb[l], (uint32_t)Kb * kKC * 4u, P.Gk[l] / kKC, Kb);
+    if (!ok) break;
+    const int Kl = P.K[l], Fh = P.Fh[l], Fg = P.Fg[l - 1];
+    const int Wg = l - 1 >= 1 ? P.Gk[l - 1] : 0;
+    const int width = Wg > Fg ? Wg : Fg;
+    const unsigned char* himg = A.ws + P.img_h[l];
+    unsigned char* gimg = A.ws + P.img_g[l - 1];
+    for (int c0 = 16 * cq; c0 < width; c0 += 32) {
+      float z[16];
+      ld16(c0, Kl, z);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int j0 = c0 + 4 * q;
+        if (j0 >= width) break;
+        float g[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int j = j0 + i;
+          float v = 0.0f;
+          if (j < Kl) {
+            const float h = *reinterpret_cast<const float*>(himg + img_off(j, grow, Fh));
+            v = z[4 * q + i] * (1.0f - h * h);
+          }
+          g[i] = v;
+          if (j < Fg) *reinterpret_cast<float*>(gimg + img_off(j, grow, Fg)) = v;
+        }
+        if (j0 < Wg)
+          *reinterpret_cast<float4*>(s.abuf + rm_off(r, j0, Wg)) =
+              make_float4(to_tf32(g[0]), to_tf32(g[1]), to_tf32(g[2]), to_tf32(g[3]));
+      }
+    }
+    ok = stage_sync();
+  }
+
+  // ---- end: nothing in flight, statistics of the tile's rows, tensor memory released
+  if (tid == 0) drain_all(s, S, issued, consumed);
+  if (cq == 0) {
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) {
+      st_pg += __shfl_xor_sync(0xFFFFFFFFu, st_pg, d);
+      st_v += __shfl_xor_sync(0xFFFFFFFFu, st_v, d);
+      st_h += __shfl_xor_sync(0xFFFFFFFFu, st_h, d);
+      st_cf += __shfl_xor_sync(0xFFFFFFFFu, st_cf, d);
+    }
+    if (lane == 0) {
+      s.dstat[4 * warp + 0] = st_pg;
+      s.dstat[4 * warp + 1] = st_v;
+      s.dstat[4 * warp + 2] = st_h;
+      s.dstat[4 * warp + 3] = st_cf;
+    }
+  }
+  fence_before();
+  __syncthreads();
+  if (tid < 4) {
+    const double v = s.dstat[tid] + s.dstat[4 + tid] + s.dstat[8 + tid] + s.dstat[12 + tid];
+    double* sp = reinterpret_cast<double*>(A.ws + P.spart);
+    sp[(size_t)blockIdx.x * 4 + tid] = *s.abort_flag == 0 ? v : __longlong_as_double(0x7FF8000000000000LL);
+  }
+  if (warp == 0) {
+    fence_after();
+    tm_dealloc(tmem, (uint32_t)P.tcols);
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// k_lw_dw: [dW_l | db_l] of one block of 128 outputs of layer l over one row range.
+// ---------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, 1) k_lw_dw(const __grid_constant__ Args A) {
+  extern __shared__ __align__(1024) unsigned char sm[];
+  const Plan& P = A.p;
+  const int S = P.dw_nstages, SB = P.dw_stage_bytes;
+  // the first 2 KB hold the ones operand of db (feature 0 = 1, features 1..15 = 0)
+  const Smem s = carve(sm, P, SB, S, 2048);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int quarter = warp & 3, cq = warp >> 2;
+  const int item = blockIdx.x % P.mt_total, split = blockIdx.x / P.mt_total;
+  int l = 0;
+  while (l + 1 < P.L && P.mt0[l + 1] <= item) ++l;
+  const int mt = item - P.mt0[l];
+  const int64_t c_lo = (int64_t)split * P.nchunks / P.S, c_hi = (int64_t)(split + 1) * P.nchunks / P.S;
+  const int nc = (int)(c_hi - c_lo);
+  const int Fh = P.Fh[l], Fg = P.Fg[l];
+  const int ng = (Fg >> 3) - 16 * mt < 16 ? (Fg >> 3) - 16 * mt : 16;   // feature groups of G
+  const uint32_t aA = (uint32_t)ng * 1024u, bB = (uint32_t)Fh * 128u;
+
+  if (tid == 0) {
+    for (int i = 0; i < kMaxStages; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.mmab[i], 1);
+    }
+    mbar_init(s.drain, 1);
+    mbar_fence_init();
+    *s.abort_flag = 0;
+  }
+  for (int i = tid; i < 512; i += kThreads)
+    reinterpret_cast<float*>(sm)[i] = (i < 256 && ((i >> 2) & 7) == 0) ? 1.0f : 0.0f;
+  if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.dw_tcols);
+  fence_async_smem();
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *s.tbase;
+  int issued = 0, consumed = 0;
+
+  if (tid == 0 && nc > 0) {
+    const unsigned char* gsrc = A.ws + P.img_g[l];
+    const unsigned char* hsrc = A.ws + P.img_h[l];
+    const uint32_t idw = idesc_tf32(kR, Fh), idb = idesc_tf32(kR, 16);
+    const uint32_t ones = su32(sm);
+    auto load = [&](int c) -> bool {
+      const int st = c % S;
+      if (c >= S && !mbar_wait(&s.mmab[st], (uint32_t)(((c - S) / S) & 1), kWaitCycles)) return false;
+      const int64_t rc = c_lo + c;
+      unsigned char* dst = s.stages + (size_t)st * SB;
+      mbar_arrive_expect_tx(&s.full[st], aA + bB);
+      bulk_g2s(dst, gsrc + (size_t)(rc * (Fg >> 3) + 16 * mt) * 1024, aA, &s.full[st]);
+      bulk_g2s(dst + 16384, hsrc + (size_t)rc * (Fh >> 3) * 1024, bB, &s.full[st]);
+      issued = c + 1;
+      return true;
+    };
+    const int pre = nc < S - 1 ? nc : S - 1;
+    bool fine = true;
+    for (int c = 0; c < pre && fine; ++c) fine = load(c);
+    for (int c = 0; c < nc && fine; ++c) {
+      const int st = c % S;
+      if (!mbar_wait(&s.full[st], (uint32_t)((c / S) & 1), kWaitCycles)) {
+        fine = false;
+        break;
+      }
+      fence_after();
+      const uint32_t sa = su32(s.stages + (size_t)st * SB), sb = sa + 16384;
+#pragma unroll
+      for (int ks = 0; ks < kKC / 8; ++ks) {
+        const uint64_t ad = sdesc(sa + (uint32_t)ks * 256u, 128, 1024);
+        const uint32_t acc = (c | ks) ? 1u : 0u;
+        mma_tf32(tmem, ad, sdesc(sb + (uint32_t)ks * 256u, 128, 1024), idw, acc);
+        mma_tf32(tmem + (uint32_t)Fh, ad, sdesc(ones + (uint32_t)ks * 256u, 128, 1024), idb, acc);
+      }
+      commit(&s.mmab[st]);
+      consumed = c + 1;
+      if (c + S - 1 < nc) fine = load(c + S - 1);
+    }
+    if (!fine) *s.abort_flag = 1;
+  }
+  if (nc > 0 && !mbar_wait(&s.mmab[(nc - 1) % S], (uint32_t)(((nc - 1) / S) & 1), kWaitCycles))
+    atomicOr(s.abort_flag, 1);
+  fence_after();
+  __syncthreads();
+  const bool ok = *s.abort_flag == 0;
+
+  // read out: lane m = output j = 128 mt + m; columns k < K_l of dW, column Fh of db
+  const int Kl = P.K[l], Nl = P.N[l];
+  const int j = 128 * mt + 32 * quarter + lane;
+  float* out = reinterpret_cast<float*>(A.ws + P.part) + (size_t)split * P.n_params + P.poff[l];
+  const uint32_t tl = tmem + ((uint32_t)(32 * quarter) << 16);
+  const float nanv = __uint_as_float(0x7FC00000u);
+  for (int c0 = 16 * cq; c0 < Fh; c0 += 32) {
+    uint32_t u[4][4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) tm_ld4_nw(tl + (uint32_t)(c0 + 4 * q), u[q]);
+    tm_wait();
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      reg_fence(u[q]);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int k = c0 + 4 * q + i;
+        if (j < Nl && k < Kl)
+          out[(size_t)j * Kl + k] = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[q][i]) : nanv);
+      }
+    }
+  }
+  if (cq == 0) {
+    uint32_t u[4];
+    tm_ld4_nw(tl + (uint32_t)Fh, u);
+    tm_wait();
+    reg_fence(u);
+    if (j < Nl) out[(size_t)Nl * Kl + j] = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[0]) : nanv);
+  }
+  if (tid == 0) drain_all(s, S, issued, consumed);
+  fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    fence_after();
+    tm_dealloc(tmem, (uint32_t)P.dw_tcols);
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------------
+size_t al256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+int pow2_cols(int need) {
+  int c = 32;
+  while (c < need) c *= 2;
+  return c;
+}
+
+Plan plan(const LossArgs& a) {
+  Plan p{};
+  p.ok = false;
+  const int L = a.n_layers;
+  if (L < 2 || L > SIMX_MAX_LAYERS || a.n < 1) return p;
+  for (int l = 0; l + 1 < L; ++l)
+    if (a.act[l] != 0) return p;  // tanh hidden layers only
+  p.L = L;
+  int P = 0, maxA = 0, maxB = 0, maxFh = 0, tneed = 0;
+  for (int l = 0; l < L; ++l) {
+    const int K = a.dims[l], N = a.dims[l + 1];
+    if (K < 1 || N < 1 || K > 256 || N > 256) return p;
+    p.K[l] = K;
+    p.N[l] = N;
+    p.Ka[l] = l == 0 ? 3 * r32(K) : r32(K);
+    p.Nf[l] = r16(N);
+    p.Gk[l] = r32(N);
+    p.Kb[l] = r16(K);
+    p.Fh[l] = r16(K);
+    p.Fg[l] = r16(N);
+    p.poff[l] = P;
+    P += N * K + N;
+    maxA = maxA > p.Ka[l] ? maxA : p.Ka[l];
+    if (l >= 1) maxA = maxA > p.Gk[l] ? maxA : p.Gk[l];
+    maxB = maxB > p.Nf[l] ? maxB : p.Nf[l];
+    if (l >= 1) maxB = maxB > p.Kb[l] ? maxB : p.Kb[l];
+    maxFh = maxFh > p.Fh[l] ? maxFh : p.Fh[l];
+    tneed = tneed > p.Nf[l] ? tneed : p.Nf[l];
+    if (l >= 1) tneed = tneed > p.Kb[l] ? tneed : p.Kb[l];
+  }
+  p.n_params = P;
+  const int limit = 227 * 1024, misc = 256;
+  p.a_bytes = kR * maxA * 4;
+  p.stage_bytes = maxB * kKC * 4;
+  p.nstages = kMaxStages;
+  while (p.nstages > 2 && p.a_bytes + p.nstages * p.stage_bytes + misc > limit) --p.nstages;
+  p.smem = p.a_bytes + p.nstages * p.stage_bytes + misc;
+  if (p.smem > limit) return p;
+  p.tcols = pow2_cols(tneed);
+  if (p.tcols > 512) return p;
+  // weight-gradient products
+  p.mt_total = 0;
+  for (int l = 0; l < L; ++l) {
+    p.mt0[l] = p.mt_total;
+    p.mt_total += (p.N[l] + 127) / 128;
+  }
+  p.n_pad = (a.n + kR - 1) / kR * kR;
+  p.ntiles = p.n_pad / kR;
+  p.nchunks = p.n_pad / kKC;
+  int64_t S = sm_count() / p.mt_total;
+  if (S < 1) S = 1;
+  if (S > p.nchunks) S = p.nchunks;
+  p.S = (int)S;
+  p.dw_stage_bytes = 16384 + maxFh * 128;
+  p.dw_nstages = kMaxStages;
+  p.dw_smem = 2048 + p.dw_nstages * p.dw_stage_bytes + misc;
+  if (p.dw_smem > limit) return p;
+  p.dw_tcols = pow2_cols(maxFh + 16);
+  if (p.dw_tcols > 512) return p;
+  // workspace
+  size_t off = 0;
+  for (int l = 0; l < L; ++l) {
+    p.wf_elems[l] = (int64_t)(p.Ka[l] / kKC) * p.Nf[l] * kKC;
+    p.wb_elems[l] = l >= 1 ? (int64_t)(p.Gk[l] / kKC) * p.Kb[l] * kKC : 0;
+    p.wf[l] = off;
+    off = al256(off + (size_t)p.wf_elems[l] * 4);
+    p.wb[l] = off;
+    off = al256(off + (size_t)p.wb_elems[l] * 4);
+  }
+  for (int l = 0; l < L; ++l) {
+    p.img_h[l] = off;
+    off = al256(off + (size_t)p.n_pad * p.Fh[l] * 4);
+    p.img_g[l] = off;
+    off = al256(off + (size_t)p.n_pad * p.Fg[l] * 4);
+  }
+  p.part = off;
+  off = al256(off + (size_t)p.S * p.n_params * 4);
+  p.spart = off;
+  off = al256(off + (size_t)p.ntiles * 4 * sizeof(double));
+  p.total = off;
+  p.ok = true;
+  return p;
+}
+
+}  // namespace lw
+
+bool loss_wide_fits(const LossArgs& a) { return lw::plan(a).ok; }
+
+size_t loss_wide_workspace(const LossArgs& a) {
+  const lw::Plan p = lw::plan(a);
+  return p.ok ? p.total : 0;
+}
+
+cudaError_t launch_loss_wide(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s) {
+  const lw::Plan p = lw::plan(a);
+  if (!p.ok || ws_bytes < p.total) return cudaErrorInvalidValue;
+  lw::Args A{};
+  A.a = a;
+  A.p = p;
+  A.ws = static_cast<unsigned char*>(ws);
+  int64_t elems = 0;
+  for (int l = 0; l < p.L; ++l) elems += p.wf_elems[l] + p.wb_elems[l];
+  int64_t blocks = (elems + 255) / 256;
+  const int64_t cap = (int64_t)sm_count() * 4;
+  if (blocks > cap) blocks = cap;
+  lw::k_lw_prep<<<(unsigned)blocks, 256, 0, s>>>(A);
+  cudaFuncSetAttribute(lw::k_lw_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
+  lw::k_lw_rows<<<(unsigned)p.ntiles, lw::kThreads, p.smem, s>>>(A);
+  cudaFuncSetAttribute(lw::k_lw_dw, cudaFuncAttributeMaxDynamicSharedMemorySize, p.dw_smem);
+  lw::k_lw_dw<<<(unsigned)(p.mt_total * p.S), lw::kThreads, p.dw_smem, s>>>(A);
+  count_launches(3);
+  launch_loss_reduce_n(reinterpret_cast<const float*>(A.ws + p.part), p.S, p.n_params,
+                       reinterpret_cast<const double*>(A.ws + p.spart), (int)p.ntiles, a, s);
+  return cudaGetLastError();
+}
+
+}  // namespace simx

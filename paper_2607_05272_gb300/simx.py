@@ -424,7 +424,7 @@ def adam_step(params, grad, m, v, t, lr: float, beta1: float = 0.9, beta2: float
                                 C.byref(p), _ptr(workspace), ws_bytes, _stream(stream)))
 
 
-NOALLOC_SCRATCH_BYTES = 16 << 20
+NOALLOC_SCRATCH_BYTES = 64 << 20
 
 
 def ppo_loss_grad_noalloc(policy: Policy, buf: dict, ret, adv, idx, n: int, algo: str,

@@ -187,6 +187,13 @@ def test_loss_gradient_matches_oracle(name, algo, E, H, nmb):
     ("c2", "ppo", 37, 300, 9001, None),
     ("c3", "ppo", 64, 256, 8192, 64),           # value head, 13-64-64-17
     ("c3", "reinforce", 21, 50, None, 32),
+    # the streamed kernels of wide policies (layers up to 256)
+    ("c3", "ppo", 64, 256, 8192, None),         # 13-128-128-17, a full minibatch
+    ("c3", "ppo", 8, 64, 333, None),            # three tiles, the last ragged
+    ("c4", "ppo", 33, 128, 3000, None),         # 28-256-256-49
+    ("c4", "reinforce", 9, 100, None, None),    # every row, 8 tiles
+    ("c3", "ppo", 16, 256, 4001, 100),          # 13-100-100-17: widths off the 16 / 32 grid
+    ("c3s", "ppo", 32, 256, 8192, None),        # 10-128-128-9, two-tower policy
 ])
 def test_tensor_core_loss_gradient_matches_oracle(name, algo, E, H, nmb, hidden):
     """TF32 tensor-core loss gradient against the fp64 oracle, within 1e-2."""
@@ -197,10 +204,10 @@ def test_tensor_core_loss_gradient_matches_oracle(name, algo, E, H, nmb, hidden)
     assert abs(s[4] - st[4]) <= 1.0 / n
 
 
-@pytest.mark.parametrize("name,hidden", [("c3", None), ("c1p", None)])
+@pytest.mark.parametrize("name,hidden", [("c1p", None), ("c1p", 256)])
 def test_tensor_core_request_falls_back(name, hidden):
-    """A policy the tensor-core kernel does not take (too wide, or with identity / GELU
-    layers) gives the FP32 path's exact bits."""
+    """A policy the tensor-core kernels do not take (identity / GELU layers) gives the
+    FP32 path's exact bits."""
     simx = _simx()
     a = _loss_case(simx, name, "ppo", 16, 64, 700, "tf32", hidden)
     b = _loss_case(simx, name, "ppo", 16, 64, 700, "fp32", hidden)

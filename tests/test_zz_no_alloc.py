@@ -35,14 +35,16 @@ def _setup(name, E, H, seed=21, hidden=None):
 
 
 # (workload, algorithm, envs, steps, minibatch rows or None, hidden width, precision):
-# the fused FP32 kernel (c3, c2), the TF32 tensor-core kernel (c2; c3 with 64-wide
-# hidden layers and a value row), and the GEMM pipeline of policies too wide for one SM
-# (c4's 28-256-256-49 on a minibatch whose workspace still fits the built-in buffer).
+# the fused FP32 kernel (c3, c2), the one-SM TF32 tensor-core kernel (c2; c3 with 64-wide
+# hidden layers and a value row), and for c4's 28-256-256-49 on a minibatch whose
+# workspace still fits the built-in buffer the FP32 GEMM pipeline and the streamed TF32
+# tensor-core kernels.
 CASES = [("c3", "ppo", 64, 256, 8192, None, "fp32"),
          ("c2", "reinforce", 40, 512, None, None, "fp32"),
          ("c2", "reinforce", 40, 512, None, None, "tf32"),
          ("c3", "ppo", 64, 256, 8192, 64, "tf32"),
-         ("c4", "ppo", 33, 128, 1500, None, "fp32")]
+         ("c4", "ppo", 33, 128, 1500, None, "fp32"),
+         ("c4", "ppo", 33, 128, 1500, None, "tf32")]
 
 
 @pytest.mark.parametrize("name,algo,E,H,nmb,hidden,prec", CASES)
@@ -76,12 +78,12 @@ def test_noalloc_matches_workspace_entry_point_twice(name, algo, E, H, nmb, hidd
 
 
 def test_noalloc_rejects_a_minibatch_beyond_its_scratch():
-    simx, pol, buf = _setup("c4", 33, 256)
-    n = 33 * 256
+    simx, pol, buf = _setup("c4", 33, 512)
+    n = 33 * 512
     need = simx.ppo_loss_grad_workspace_size(pol, n)
     assert need > simx.NOALLOC_SCRATCH_BYTES
-    adv = torch.zeros((256, 33), device="cuda")
-    ret = torch.zeros((256, 33), device="cuda")
+    adv = torch.zeros((512, 33), device="cuda")
+    ret = torch.zeros((512, 33), device="cuda")
     g = torch.empty(pol.n_params, device="cuda")
     st = torch.empty(5, device="cuda")
     with pytest.raises(simx.SimxError) as ei:
