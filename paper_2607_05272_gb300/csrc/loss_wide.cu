@@ -158,6 +158,7 @@ struct Smem {
   uint64_t* full;          // [kMaxStages] chunk landed (bulk copy transactions)
   uint64_t* mmab;          // [kMaxStages] MMAs reading the stage completed
   uint64_t* drain;         // every MMA of the CTA completed (end of kernel)
+  uint64_t* accb;          // the accumulator of the current GEMM is complete
   uint32_t* tbase;         // tensor memory base address
   int* abort_flag;         // a wait timed out: stop issuing work
   double* dstat;           // [4 warps][4] statistics
@@ -172,7 +173,8 @@ __device__ __forceinline__ Smem carve(unsigned char* sm, const Plan& P, int stag
   s.full = reinterpret_cast<uint64_t*>(m);
   s.mmab = s.full + kMaxStages;
   s.drain = s.mmab + kMaxStages;
-  s.tbase = reinterpret_cast<uint32_t*>(s.drain + 1);
+  s.accb = s.drain + 1;
+  s.tbase = reinterpret_cast<uint32_t*>(s.accb + 1);
   s.abort_flag = reinterpret_cast<int*>(s.tbase + 1);
   s.dstat = reinterpret_cast<double*>(m + 128);
   (void)P;
@@ -183,6 +185,9 @@ __device__ __forceinline__ Smem carve(unsigned char* sm, const Plan& P, int stag
 // a_addr (row-group stride a_sbo), B chunks of bbytes streamed from bsrc through the
 // stage ring.  `next` counts the chunks of every earlier GEMM of the kernel (stage and
 // barrier parity follow from it); issued / consumed track this thread's loads and MMAs.
+// A stage barrier is waited on only once the use before has completed (so a parity names
+// one phase); the accumulator's completion is announced on its own barrier, accb, with
+// one phase per GEMM, which the other threads wait on.
 __device__ void gemm_issue(const Smem& s, int S, int stage_bytes, int next, int& issued,
                            int& consumed, uint32_t a_addr, uint32_t a_sbo, const unsigned char* bsrc,
                            uint32_t bbytes, int nc, int Nmma, uint32_t dtm) {
@@ -220,6 +225,7 @@ __device__ void gemm_issue(const Smem& s, int S, int stage_bytes, int next, int&
       return;
     }
   }
+  commit(s.accb);
 }
 
 // Thread 0 at the end of a kernel: waits (bounded) for loads it issued that no MMA
@@ -249,6 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
       mbar_init(&s.mmab[i], 1);
     }
     mbar_init(s.drain, 1);
+    mbar_init(s.accb, 1);
     mbar_fence_init();
     *s.abort_flag = 0;
   }
@@ -300,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   const uint32_t tmem = *s.tbase;
   const uint32_t tl = tmem + ((uint32_t)(32 * quarter) << 16);   // this warp's lane quarter
   const uint32_t abuf_addr = su32(s.abuf);
-  int next = 0, issued = 0, consumed = 0;
+  int next = 0, issued = 0, consumed = 0, ngemm = 0;
   double st_pg = 0.0, st_v = 0.0, st_h = 0.0, st_cf = 0.0;
   const float inv_n = 1.0f / (float)a.n;
 
@@ -309,9 +316,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     if (tid == 0 && *s.abort_flag == 0)
       gemm_issue(s, S, P.stage_bytes, next, issued, consumed, abuf_addr, (uint32_t)(a_width / 4) * 128u,
                  bsrc, bbytes, nc, Nmma, tmem);
-    const int klast = next + nc - 1;
     next += nc;
-    if (!mbar_wait(&s.mmab[klast % S], (uint32_t)((klast / S) & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
+    if (!mbar_wait(s.accb, (uint32_t)(ngemm & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
+    ++ngemm;
     __syncwarp();
     fence_after();
     return *s.abort_flag == 0;
@@ -550,6 +557,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_dw(const __grid_constant__ A
       mbar_init(&s.mmab[i], 1);
     }
     mbar_init(s.drain, 1);
+    mbar_init(s.accb, 1);
     mbar_fence_init();
     *s.abort_flag = 0;
   }
@@ -601,10 +609,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_dw(const __grid_constant__ A
       consumed = c + 1;
       if (c + S - 1 < nc) fine = load(c + S - 1);
     }
-    if (!fine) *s.abort_flag = 1;
+    if (fine) commit(s.accb);
+    else *s.abort_flag = 1;
   }
-  if (nc > 0 && !mbar_wait(&s.mmab[(nc - 1) % S], (uint32_t)(((nc - 1) / S) & 1), kWaitCycles))
-    atomicOr(s.abort_flag, 1);
+  if (nc > 0 && !mbar_wait(s.accb, 0u, kWaitCycles)) atomicOr(s.abort_flag, 1);
   fence_after();
   __syncthreads();
   const bool ok = *s.abort_flag == 0;
