@@ -44,7 +44,8 @@ namespace lw {
 using namespace tcx;
 
 constexpr int kR = 128;            // rows per tile (MMA M)
-constexpr int kThreads = 256;      // 8 warps: 2 per TMEM lane quarter
+constexpr int kThreads = 512;      // k_lw_rows: 16 warps, 4 per TMEM lane quarter
+constexpr int kDwThreads = 256;    // k_lw_dw: 8 warps, 2 per lane quarter
 constexpr int kKC = 32;            // K values per streamed chunk
 constexpr int kMaxStages = 3;
 constexpr long long kWaitCycles = 2000000000LL;  // bound on any wait (about 1 s)
@@ -81,11 +82,63 @@ struct Args {
   unsigned char* ws;
 };
 
-// Byte offset of (feature f, row r) in a feature-major image of F features: blocks of
-// 32 rows, in each block the feature groups of 8 one after another, each group the
-// K-major operand of 8 features x 32 rows (8 core matrices of 4 rows).
-__device__ __forceinline__ size_t img_off(int f, int64_t r, int F) {
-  return (size_t)((r >> 5) * (F >> 3) + (f >> 3)) * 1024 + (size_t)(((r & 31) >> 2) * 128 + (f & 7) * 16 + (r & 3) * 4);
+// Byte offset of feature f inside a 32-row block of a feature-major image: blocks of 32
+// rows, in each block the feature groups of 8 one after another, each group the K-major
+// operand of 8 features x 32 rows (8 core matrices of 4 rows, 128 bytes apart); so
+// (feature f, row r) is at block (r / 32) + img_col(f) + ((r % 32) / 4) * 128 + (r % 4) * 4.
+__device__ __forceinline__ uint32_t img_col(int f) { return (uint32_t)((f >> 3) * 1024 + (f & 7) * 16); }
+
+// 4 x 4 transposes inside each group of 4 lanes: afterwards lane 4m + j holds, at
+// v[4a + i], what lane 4m + i held at v[4a + j] (applied twice it is the identity).
+__device__ __forceinline__ void quad_transpose(float (&v)[16], int j) {
+#pragma unroll
+  for (int a = 0; a < 4; ++a) {
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      const float send = (j & 2) ? v[4 * a + b] : v[4 * a + b + 2];
+      const float recv = __shfl_xor_sync(0xFFFFFFFFu, send, 2);
+      if (j & 2) v[4 * a + b] = recv;
+      else v[4 * a + b + 2] = recv;
+    }
+#pragma unroll
+    for (int b = 0; b < 4; b += 2) {
+      const float send = (j & 1) ? v[4 * a + b] : v[4 * a + b + 1];
+      const float recv = __shfl_xor_sync(0xFFFFFFFFu, send, 1);
+      if (j & 1) v[4 * a + b] = recv;
+      else v[4 * a + b + 1] = recv;
+    }
+  }
+}
+
+// The 32-row block of an image of F features that holds this warp's rows.
+__device__ __forceinline__ size_t img_blk(int64_t grow, int F) {
+  return (size_t)((grow >> 5) * (F >> 3)) * 1024;
+}
+
+// This warp's 32 rows x features c0 .. c0 + 15 (v: the lane's row) into an image block:
+// after the transpose each lane stores whole 16-byte segments (one feature, 4 rows), so
+// the warp writes contiguous runs.  v is transposed in place.
+__device__ __forceinline__ void img_store16(unsigned char* blk, int c0, float (&v)[16], int lane) {
+  quad_transpose(v, lane & 3);
+  const int m = lane >> 2, j = lane & 3;
+#pragma unroll
+  for (int a = 0; a < 4; ++a)
+    *reinterpret_cast<float4*>(blk + img_col(c0 + 4 * a + j) + m * 128) =
+        make_float4(v[4 * a], v[4 * a + 1], v[4 * a + 2], v[4 * a + 3]);
+}
+
+// The inverse: features c0 .. c0 + 15 of the lane's row from an image block.
+__device__ __forceinline__ void img_load16(const unsigned char* blk, int c0, float (&v)[16], int lane) {
+  const int m = lane >> 2, j = lane & 3;
+#pragma unroll
+  for (int a = 0; a < 4; ++a) {
+    const float4 t = *reinterpret_cast<const float4*>(blk + img_col(c0 + 4 * a + j) + m * 128);
+    v[4 * a] = t.x;
+    v[4 * a + 1] = t.y;
+    v[4 * a + 2] = t.z;
+    v[4 * a + 3] = t.w;
+  }
+  quad_transpose(v, j);
 }
 
 // Byte offset of (row j, value kk) inside one 32-value chunk of a weight image.
@@ -181,33 +234,63 @@ __device__ __forceinline__ Smem carve(unsigned char* sm, const Plan& P, int stag
   return s;
 }
 
-// Thread 0's side of one GEMM  D = A B^T  over nc chunks of 32 K values: A resident at
-// a_addr (row-group stride a_sbo), B chunks of bbytes streamed from bsrc through the
-// stage ring.  `next` counts the chunks of every earlier GEMM of the kernel (stage and
-// barrier parity follow from it); issued / consumed track this thread's loads and MMAs.
-// A stage barrier is waited on only once the use before has completed (so a parity names
-// one phase); the accumulator's completion is announced on its own barrier, accb, with
-// one phase per GEMM, which the other threads wait on.
-__device__ void gemm_issue(const Smem& s, int S, int stage_bytes, int next, int& issued,
-                           int& consumed, uint32_t a_addr, uint32_t a_sbo, const unsigned char* bsrc,
-                           uint32_t bbytes, int nc, int Nmma, uint32_t dtm) {
-  const uint32_t id = idesc_tf32(kR, Nmma);
-  auto load = [&](int c) -> bool {
-    const int k = next + c, st = k % S;
-    if (k >= S && !mbar_wait(&s.mmab[st], (uint32_t)(((k - S) / S) & 1), kWaitCycles)) return false;
-    mbar_arrive_expect_tx(&s.full[st], bbytes);
-    bulk_g2s(s.stages + (size_t)st * stage_bytes, bsrc + (size_t)c * bbytes, bbytes, &s.full[st]);
-    issued = k + 1;
-    return true;
-  };
-  const int pre = nc < S - 1 ? nc : S - 1;
-  for (int c = 0; c < pre; ++c)
-    if (!load(c)) {
-      *s.abort_flag = 1;
-      return;
+// The weight chunks of k_lw_rows in the order its GEMMs consume them (forward layers
+// 0 .. L-1, then the backward products of layers L-1 .. 1): GEMM g takes the global
+// chunks k0[g] .. k0[g + 1] - 1; chunk k goes through stage k % S.
+struct Sched {
+  int ng, total;
+  int k0[2 * SIMX_MAX_LAYERS];
+  const unsigned char* src[2 * SIMX_MAX_LAYERS];
+  uint32_t bytes[2 * SIMX_MAX_LAYERS];
+};
+
+__device__ Sched make_sched(const Plan& P, unsigned char* ws) {
+  Sched q;
+  q.ng = 2 * P.L - 1;
+  int k = 0;
+  for (int g = 0; g < q.ng; ++g) {
+    q.k0[g] = k;
+    if (g < P.L) {
+      q.src[g] = ws + P.wf[g];
+      q.bytes[g] = (uint32_t)P.Nf[g] * kKC * 4u;
+      k += P.Ka[g] / kKC;
+    } else {
+      const int l = 2 * P.L - 1 - g;
+      q.src[g] = ws + P.wb[l];
+      q.bytes[g] = (uint32_t)P.Kb[l] * kKC * 4u;
+      k += P.Gk[l] / kKC;
     }
-  for (int c = 0; c < nc; ++c) {
-    const int k = next + c, st = k % S;
+  }
+  q.k0[q.ng] = k;
+  q.total = k;
+  return q;
+}
+
+// Thread 0: the bulk copy of global chunk k into its stage, once the MMAs that read the
+// stage's previous chunk have completed (each stage barrier is waited on only after the
+// use before it completed, so a parity names one phase).
+__device__ bool load_chunk(const Smem& s, const Sched& q, int S, int stage_bytes, int k) {
+  const int st = k % S;
+  if (k >= S && !mbar_wait(&s.mmab[st], (uint32_t)(((k - S) / S) & 1), kWaitCycles)) return false;
+  int g = 0;
+  while (q.k0[g + 1] <= k) ++g;
+  const uint32_t b = q.bytes[g];
+  mbar_arrive_expect_tx(&s.full[st], b);
+  bulk_g2s(s.stages + (size_t)st * stage_bytes, q.src[g] + (size_t)(k - q.k0[g]) * b, b, &s.full[st]);
+  return true;
+}
+
+// Thread 0's side of GEMM g  D = A B^T: A resident at a_addr (row-group stride a_sbo),
+// the B chunks through the stage ring.  After the MMAs of chunk k are queued, copies are
+// issued up to chunk k + S - 1, running on into the next GEMMs' chunks, so that those
+// arrive while the other threads work on this GEMM's result.  The accumulator's
+// completion is announced on accb (one phase per GEMM), which every thread waits on.
+__device__ void gemm_issue(const Smem& s, const Sched& q, int S, int stage_bytes, int g,
+                           int& issued, int& consumed, uint32_t a_addr, uint32_t a_sbo, int Nmma,
+                           uint32_t dtm) {
+  const uint32_t id = idesc_tf32(kR, Nmma);
+  for (int k = q.k0[g]; k < q.k0[g + 1]; ++k) {
+    const int st = k % S, c = k - q.k0[g];
     if (!mbar_wait(&s.full[st], (uint32_t)((k / S) & 1), kWaitCycles)) {
       *s.abort_flag = 1;
       return;
@@ -220,9 +303,13 @@ __device__ void gemm_issue(const Smem& s, int S, int stage_bytes, int next, int&
                sdesc(bs + (uint32_t)ks * 256u, 128, 1024), id, (c | ks) ? 1u : 0u);
     commit(&s.mmab[st]);
     consumed = k + 1;
-    if (c + S - 1 < nc && !load(c + S - 1)) {
-      *s.abort_flag = 1;
-      return;
+    const int upto = k + S < q.total ? k + S : q.total;
+    while (issued < upto) {
+      if (!load_chunk(s, q, S, stage_bytes, issued)) {
+        *s.abort_flag = 1;
+        return;
+      }
+      ++issued;
     }
   }
   commit(s.accb);
@@ -244,11 +331,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   const int L = P.L, S = P.nstages;
   const Smem s = carve(sm, P, P.stage_bytes, S, P.a_bytes);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int quarter = warp & 3, cq = warp >> 2;
+  const int quarter = warp & 3, cq = warp >> 2;   // lane quarter; column share 0..3
   const int r = 32 * quarter + lane;
   const int64_t grow = (int64_t)blockIdx.x * kR + r;   // row of the padded minibatch
   const bool live = grow < a.n;
 
+  // thread 0: barriers, then the first weight chunks on their way before anything else
+  Sched sch;
+  int issued = 0, consumed = 0;
   if (tid == 0) {
     for (int i = 0; i < kMaxStages; ++i) {
       mbar_init(&s.full[i], 1);
@@ -258,42 +348,53 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     mbar_init(s.accb, 1);
     mbar_fence_init();
     *s.abort_flag = 0;
+    sch = make_sched(P, A.ws);
+    const int upto = S - 1 < sch.total ? S - 1 : sch.total;
+    for (; issued < upto; ++issued) load_chunk(s, sch, S, P.stage_bytes, issued);
   }
   if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.tcols);
 
   // the tile's observations: x_hi, x_hi, x_lo side by side in the A buffer (split TF32)
   // and the FP32 values in the H_0 image; the head thread's per-row inputs
   int64_t row = 0;
-  if (live) row = a.idx ? a.idx[grow] : grow;
+  if (live) row = a.idx ? __ldg(a.idx + grow) : grow;
   const int64_t t = row / a.E, e = row % a.E;
   const int D = P.K[0];
   {
     const int Kc = P.Ka[0] / 3, W0 = P.Ka[0], F0 = P.Fh[0];
-    unsigned char* img = A.ws + P.img_h[0];
-    for (int cb = cq; cb < Kc / 4; cb += 2) {
-      float hi[4], lo[4];
+    unsigned char* img = A.ws + P.img_h[0] + img_blk(grow, F0);
+    // 16 features per pass: every gather load issued before any store
+    for (int c0 = 16 * cq; c0 < Kc; c0 += 64) {
+      float x[16];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int f = 4 * cb + i;
-        const float x = (live && f < D) ? a.obs[(t * D + f) * a.E + e] : 0.0f;
-        hi[i] = to_tf32(x);
-        lo[i] = to_tf32(x - hi[i]);
-        if (f < F0) *reinterpret_cast<float*>(img + img_off(f, grow, F0)) = x;
+      for (int i = 0; i < 16; ++i) {
+        const int f = c0 + i;
+        x[i] = (live && f < D) ? __ldg(a.obs + (t * D + f) * a.E + e) : 0.0f;
       }
-      const float4 h4 = make_float4(hi[0], hi[1], hi[2], hi[3]);
-      *reinterpret_cast<float4*>(s.abuf + rm_off(r, 4 * cb, W0)) = h4;
-      *reinterpret_cast<float4*>(s.abuf + rm_off(r, Kc + 4 * cb, W0)) = h4;
-      *reinterpret_cast<float4*>(s.abuf + rm_off(r, 2 * Kc + 4 * cb, W0)) =
-          make_float4(lo[0], lo[1], lo[2], lo[3]);
+#pragma unroll
+      for (int qq = 0; qq < 4; ++qq) {
+        float hi[4], lo[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          hi[i] = to_tf32(x[4 * qq + i]);
+          lo[i] = to_tf32(x[4 * qq + i] - hi[i]);
+        }
+        const int k = c0 + 4 * qq;
+        const float4 h4 = make_float4(hi[0], hi[1], hi[2], hi[3]);
+        *reinterpret_cast<float4*>(s.abuf + rm_off(r, k, W0)) = h4;
+        *reinterpret_cast<float4*>(s.abuf + rm_off(r, Kc + k, W0)) = h4;
+        *reinterpret_cast<float4*>(s.abuf + rm_off(r, 2 * Kc + k, W0)) = make_float4(lo[0], lo[1], lo[2], lo[3]);
+      }
+      if (c0 < F0) img_store16(img, c0, x, lane);
     }
   }
   int ac = 0;
   float adv = 0.0f, lpo = 0.0f, ret = 0.0f;
   if (cq == 0 && live) {
-    ac = a.action[row];
-    adv = a.adv[row];
-    lpo = a.algo == SIMX_ALGO_PPO ? a.logp_old[row] : 0.0f;
-    ret = a.has_value ? a.ret[row] : 0.0f;
+    ac = __ldg(a.action + row);
+    adv = __ldg(a.adv + row);
+    lpo = a.algo == SIMX_ALGO_PPO ? __ldg(a.logp_old + row) : 0.0f;
+    ret = a.has_value ? __ldg(a.ret + row) : 0.0f;
   }
 
   auto stage_sync = [&]() -> bool {
@@ -307,46 +408,43 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   const uint32_t tmem = *s.tbase;
   const uint32_t tl = tmem + ((uint32_t)(32 * quarter) << 16);   // this warp's lane quarter
   const uint32_t abuf_addr = su32(s.abuf);
-  int next = 0, issued = 0, consumed = 0, ngemm = 0;
+  int ngemm = 0;
   double st_pg = 0.0, st_v = 0.0, st_h = 0.0, st_cf = 0.0;
   const float inv_n = 1.0f / (float)a.n;
 
-  // one GEMM: thread 0 streams and issues, every thread then waits for its last commit
-  auto gemm = [&](int a_width, const unsigned char* bsrc, uint32_t bbytes, int nc, int Nmma) -> bool {
-    if (tid == 0 && *s.abort_flag == 0)
-      gemm_issue(s, S, P.stage_bytes, next, issued, consumed, abuf_addr, (uint32_t)(a_width / 4) * 128u,
-                 bsrc, bbytes, nc, Nmma, tmem);
-    next += nc;
-    if (!mbar_wait(s.accb, (uint32_t)(ngemm & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
+  // GEMM g: thread 0 issues it, every thread then waits for the accumulator
+  auto gemm = [&](int g, int a_width, int Nmma) -> bool {
+    // warp 0's other lanes wait at the warp barrier, not polling beside the issuing lane
+    if (warp == 0) {
+      if (lane == 0 && *s.abort_flag == 0)
+        gemm_issue(s, sch, S, P.stage_bytes, g, issued, consumed, abuf_addr,
+                   (uint32_t)(a_width / 4) * 128u, Nmma, tmem);
+      __syncwarp();
+    }
+    if (!mbar_wait_idle(s.accb, (uint32_t)(ngemm & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
     ++ngemm;
     __syncwarp();
     fence_after();
     return *s.abort_flag == 0;
   };
 
-  // Loads columns c0 .. c0 + 15 of this thread's accumulator row (only those < ncols;
-  // the rest read as 0); every thread of the warp takes part (the loads are warp-wide).
+  // Columns c0 .. c0 + 15 of this thread's accumulator row (one warp-wide load; columns
+  // from ncols on read as 0).  The allocation covers them: tcols is a power of two at
+  // least as large as every 32-rounded width read here.
   auto ld16 = [&](int c0, int ncols, float (&z)[16]) {
-    uint32_t u[4][4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      if (c0 + 4 * q < ncols) tm_ld4_nw(tl + (uint32_t)(c0 + 4 * q), u[q]);
-      else u[q][0] = u[q][1] = u[q][2] = u[q][3] = 0u;
-    }
+    uint32_t u[16];
+    tm_ld16_nw(tl + (uint32_t)c0, u);
     tm_wait();
+    reg_fence16(u);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      reg_fence(u[q]);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) z[4 * q + i] = __uint_as_float(u[q][i]);
-    }
+    for (int i = 0; i < 16; ++i) z[i] = c0 + i < ncols ? __uint_as_float(u[i]) : 0.0f;
   };
 
   bool ok = true;
   // ---- forward
   for (int l = 0; l < L && ok; ++l) {
     const int Nf = P.Nf[l];
-    ok = gemm(P.Ka[l], A.ws + P.wf[l], (uint32_t)Nf * kKC * 4u, P.Ka[l] / kKC, Nf);
+    ok = gemm(l, P.Ka[l], Nf);
     if (!ok) break;
     const int Nl = P.N[l];
     const float* bias = a.b[l];
@@ -355,24 +453,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
       // FP32 into the H_{l+1} image; the two warps of a quarter take alternate 16-column
       // blocks
       const int Wn = P.Ka[l + 1], Fn = P.Fh[l + 1];
-      unsigned char* img = A.ws + P.img_h[l + 1];
-      for (int c0 = 16 * cq; c0 < Wn; c0 += 32) {
-        float z[16];
+      unsigned char* img = A.ws + P.img_h[l + 1] + img_blk(grow, Fn);
+      for (int c0 = 16 * cq; c0 < Wn; c0 += 64) {
+        float z[16], bv[16], h[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) bv[i] = c0 + i < Nl ? __ldg(bias + c0 + i) : 0.0f;
         ld16(c0, Nl, z);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int j0 = c0 + 4 * q;
-          if (j0 >= Wn) break;
-          float h[4];
+        for (int i = 0; i < 16; ++i) h[i] = c0 + i < Nl ? tanh_fast(z[i] + bv[i]) : 0.0f;
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int j = j0 + i;
-            h[i] = j < Nl ? tanh_fast(z[4 * q + i] + bias[j]) : 0.0f;
-            if (j < Fn) *reinterpret_cast<float*>(img + img_off(j, grow, Fn)) = h[i];
-          }
-          *reinterpret_cast<float4*>(s.abuf + rm_off(r, j0, Wn)) =
-              make_float4(to_tf32(h[0]), to_tf32(h[1]), to_tf32(h[2]), to_tf32(h[3]));
-        }
+        for (int qq = 0; qq < 4; ++qq)
+          *reinterpret_cast<float4*>(s.abuf + rm_off(r, c0 + 4 * qq, Wn)) =
+              make_float4(to_tf32(h[4 * qq]), to_tf32(h[4 * qq + 1]), to_tf32(h[4 * qq + 2]),
+                          to_tf32(h[4 * qq + 3]));
+        if (c0 < Fn) img_store16(img, c0, h, lane);
       }
     } else if (cq == 0) {
       // loss head for row r: G = dL/dZ over the logits (and the value row)
@@ -383,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         ld16(c0, Nl, z);
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          if (c0 + i < NA) m = fmaxf(m, z[i] + bias[c0 + i]);
+          if (c0 + i < NA) m = fmaxf(m, z[i] + __ldg(bias + c0 + i));
       }
       float Ssum = 0.0f;
       for (int c0 = 0; c0 < NA; c0 += 16) {
@@ -391,7 +485,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         ld16(c0, Nl, z);
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          if (c0 + i < NA) Ssum += __expf(z[i] + bias[c0 + i] - m);
+          if (c0 + i < NA) Ssum += __expf(z[i] + __ldg(bias + c0 + i) - m);
       }
       const float lse = m + __logf(Ssum);
       float Hent = 0.0f, lpa = 0.0f, zv = 0.0f;
@@ -402,11 +496,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         for (int i = 0; i < 16; ++i) {
           const int j = c0 + i;
           if (j < NA) {
-            const float lp = z[i] + bias[j] - lse;
+            const float lp = z[i] + __ldg(bias + j) - lse;
             Hent -= __expf(lp) * lp;
             if (j == ac) lpa = lp;
           } else if (j == NA && j < Nl) {
-            zv = z[i] + bias[j];
+            zv = z[i] + __ldg(bias + j);
           }
         }
       }
@@ -433,32 +527,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
       }
       // G_{L-1}: TF32 into the A buffer (width Gk), FP32 into the G image
       const int Wg = P.Gk[l], Fg = P.Fg[l];
-      unsigned char* img = A.ws + P.img_g[l];
+      unsigned char* img = A.ws + P.img_g[l] + img_blk(grow, Fg);
       for (int c0 = 0; c0 < Wg; c0 += 16) {
-        float z[16];
+        float z[16], bv[16], g[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) bv[i] = c0 + i < NA ? __ldg(bias + c0 + i) : 0.0f;
         ld16(c0, Nl, z);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int j0 = c0 + 4 * q;
-          float g[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int j = j0 + i;
-            float v = 0.0f;
-            if (live && j < NA) {
-              const float lp = z[4 * q + i] + bias[j] - lse;
-              const float p = __expf(lp);
-              const float onehot = (j == ac) ? 1.0f : 0.0f;
-              v = (-coef * (onehot - p) + a.c_entropy * p * (lp + Hent)) * inv_n;
-            } else if (live && a.has_value && j == NA) {
-              v = 2.0f * a.c_value * dv * inv_n;
-            }
-            g[i] = v;
-            if (j < Fg) *reinterpret_cast<float*>(img + img_off(j, grow, Fg)) = v;
+        for (int i = 0; i < 16; ++i) {
+          const int j = c0 + i;
+          float v = 0.0f;
+          if (live && j < NA) {
+            const float lp = z[i] + bv[i] - lse;
+            const float p = __expf(lp);
+            const float onehot = (j == ac) ? 1.0f : 0.0f;
+            v = (-coef * (onehot - p) + a.c_entropy * p * (lp + Hent)) * inv_n;
+          } else if (live && a.has_value && j == NA) {
+            v = 2.0f * a.c_value * dv * inv_n;
           }
-          *reinterpret_cast<float4*>(s.abuf + rm_off(r, j0, Wg)) =
-              make_float4(to_tf32(g[0]), to_tf32(g[1]), to_tf32(g[2]), to_tf32(g[3]));
+          g[i] = v;
         }
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq)
+          *reinterpret_cast<float4*>(s.abuf + rm_off(r, c0 + 4 * qq, Wg)) =
+              make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
+                          to_tf32(g[4 * qq + 3]));
+        if (c0 < Fg) img_store16(img, c0, g, lane);
       }
     }
     ok = stage_sync();
@@ -466,36 +560,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   // ---- backward: dH_l = G_l W_l, G_{l-1} = dH_l (1 - H_l^2)
   for (int l = L - 1; l >= 1 && ok; --l) {
     const int Kb = P.Kb[l];
-    ok = gemm(P.Gk[l], A.ws + P.wb[l], (uint32_t)Kb * kKC * 4u, P.Gk[l] / kKC, Kb);
+    ok = gemm(2 * L - 1 - l, P.Gk[l], Kb);
     if (!ok) break;
     const int Kl = P.K[l], Fh = P.Fh[l], Fg = P.Fg[l - 1];
     const int Wg = l - 1 >= 1 ? P.Gk[l - 1] : 0;
     const int width = Wg > Fg ? Wg : Fg;
-    const unsigned char* himg = A.ws + P.img_h[l];
-    unsigned char* gimg = A.ws + P.img_g[l - 1];
-    for (int c0 = 16 * cq; c0 < width; c0 += 32) {
-      float z[16];
+    const unsigned char* himg = A.ws + P.img_h[l] + img_blk(grow, Fh);
+    unsigned char* gimg = A.ws + P.img_g[l - 1] + img_blk(grow, Fg);
+    for (int c0 = 16 * cq; c0 < width; c0 += 64) {
+      float z[16], hv[16], g[16];
+      if (c0 < Fh) img_load16(himg, c0, hv, lane);
+      else
+#pragma unroll
+        for (int i = 0; i < 16; ++i) hv[i] = 0.0f;
       ld16(c0, Kl, z);
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int j0 = c0 + 4 * q;
-        if (j0 >= width) break;
-        float g[4];
+      for (int i = 0; i < 16; ++i) g[i] = c0 + i < Kl ? z[i] * (1.0f - hv[i] * hv[i]) : 0.0f;
+      if (c0 < Wg)
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int j = j0 + i;
-          float v = 0.0f;
-          if (j < Kl) {
-            const float h = *reinterpret_cast<const float*>(himg + img_off(j, grow, Fh));
-            v = z[4 * q + i] * (1.0f - h * h);
-          }
-          g[i] = v;
-          if (j < Fg) *reinterpret_cast<float*>(gimg + img_off(j, grow, Fg)) = v;
-        }
-        if (j0 < Wg)
-          *reinterpret_cast<float4*>(s.abuf + rm_off(r, j0, Wg)) =
-              make_float4(to_tf32(g[0]), to_tf32(g[1]), to_tf32(g[2]), to_tf32(g[3]));
-      }
+        for (int qq = 0; qq < 4; ++qq)
+          *reinterpret_cast<float4*>(s.abuf + rm_off(r, c0 + 4 * qq, Wg)) =
+              make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
+                          to_tf32(g[4 * qq + 3]));
+      if (c0 < Fg) img_store16(gimg, c0, g, lane);
     }
     ok = stage_sync();
   }
@@ -533,7 +620,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
 // ---------------------------------------------------------------------------------
 // k_lw_dw: [dW_l | db_l] of one block of 128 outputs of layer l over one row range.
 // ---------------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, 1) k_lw_dw(const __grid_constant__ Args A) {
+__global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__ Args A) {
   extern __shared__ __align__(1024) unsigned char sm[];
   const Plan& P = A.p;
   const int S = P.dw_nstages, SB = P.dw_stage_bytes;
@@ -561,7 +648,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_dw(const __grid_constant__ A
     mbar_fence_init();
     *s.abort_flag = 0;
   }
-  for (int i = tid; i < 512; i += kThreads)
+  for (int i = tid; i < 512; i += kDwThreads)
     reinterpret_cast<float*>(sm)[i] = (i < 256 && ((i >> 2) & 7) == 0) ? 1.0f : 0.0f;
   if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.dw_tcols);
   fence_async_smem();
@@ -571,7 +658,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_dw(const __grid_constant__ A
   const uint32_t tmem = *s.tbase;
   int issued = 0, consumed = 0;
 
-  if (tid == 0 && nc > 0) {
+  if (warp == 0 && lane == 0 && nc > 0) {
     const unsigned char* gsrc = A.ws + P.img_g[l];
     const unsigned char* hsrc = A.ws + P.img_h[l];
     const uint32_t idw = idesc_tf32(kR, Fh), idb = idesc_tf32(kR, 16);
@@ -612,7 +699,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_dw(const __grid_constant__ A
     if (fine) commit(s.accb);
     else *s.abort_flag = 1;
   }
-  if (nc > 0 && !mbar_wait(s.accb, 0u, kWaitCycles)) atomicOr(s.abort_flag, 1);
+  __syncwarp();
+  if (nc > 0 && !mbar_wait_idle(s.accb, 0u, kWaitCycles)) atomicOr(s.abort_flag, 1);
   fence_after();
   __syncthreads();
   const bool ok = *s.abort_flag == 0;
@@ -775,7 +863,7 @@ cudaError_t launch_loss_wide(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
   cudaFuncSetAttribute(lw::k_lw_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
   lw::k_lw_rows<<<(unsigned)p.ntiles, lw::kThreads, p.smem, s>>>(A);
   cudaFuncSetAttribute(lw::k_lw_dw, cudaFuncAttributeMaxDynamicSharedMemorySize, p.dw_smem);
-  lw::k_lw_dw<<<(unsigned)(p.mt_total * p.S), lw::kThreads, p.dw_smem, s>>>(A);
+  lw::k_lw_dw<<<(unsigned)(p.mt_total * p.S), lw::kDwThreads, p.dw_smem, s>>>(A);
   count_launches(3);
   launch_loss_reduce_n(reinterpret_cast<const float*>(A.ws + p.part), p.S, p.n_params,
                        reinterpret_cast<const double*>(A.ws + p.spart), (int)p.ntiles, a, s);

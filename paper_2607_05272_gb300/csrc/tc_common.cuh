@@ -82,6 +82,17 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* mbar, uint32_t parity, long 
   }
 }
 
+// The same for threads that only wait for a result: they back off between polls so that
+// the thread issuing the work keeps the issue slots of its scheduler.
+__device__ __forceinline__ bool mbar_wait_idle(uint64_t* mbar, uint32_t parity, long long limit) {
+  const long long t0 = clock64();
+  for (;;) {
+    if (mbar_test(mbar, parity)) return true;
+    if (clock64() - t0 > limit) return false;
+    __nanosleep(64);
+  }
+}
+
 // One arrival that also announces `bytes` of transactions the phase must receive.
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* mbar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(mbar)), "r"(bytes)
@@ -111,6 +122,22 @@ __device__ __forceinline__ void tm_ld4_nw(uint32_t taddr, uint32_t (&u)[4]) {
                : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3])
                : "r"(taddr)
                : "memory");
+}
+// Sixteen consecutive accumulator columns of this thread's lane, without the wait.
+__device__ __forceinline__ void tm_ld16_nw(uint32_t taddr, uint32_t (&u)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15}, [%16];"
+      : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]),
+        "=r"(u[7]), "=r"(u[8]), "=r"(u[9]), "=r"(u[10]), "=r"(u[11]), "=r"(u[12]), "=r"(u[13]),
+        "=r"(u[14]), "=r"(u[15])
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void reg_fence16(uint32_t (&u)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; i += 4)
+    asm volatile("" : "+r"(u[i]), "+r"(u[i + 1]), "+r"(u[i + 2]), "+r"(u[i + 3]));
 }
 __device__ __forceinline__ void tm_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void reg_fence(uint32_t (&u)[4]) {
