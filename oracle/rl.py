@@ -129,13 +129,16 @@ def forward(Ws, bs, X, acts=None, grid=None):
 
 
 def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=0.2,
-              c_value=0.5, c_entropy=0.01, acts=None, grid=None):
+              c_value=0.5, c_entropy=0.01, acts=None, grid=None, abs_terms=False):
     """Loss, statistics and the gradient with respect to every W_l, b_l (fp64).
 
     pi = softmax(logits); policy term REINFORCE -mean(adv log pi(a)) or PPO
     -mean(min(rho adv, clip(rho, 1-eps, 1+eps) adv)) with rho = exp(log pi(a) - logp_old);
     plus c_value mean((V - ret)^2) when a value row exists, minus c_entropy mean(H[pi]).
-    Returns (grads [(gW, gb) per layer], stats [L, pg, v, H, clipfrac]).
+    Returns (grads [(gW, gb) per layer], stats [L, pg, v, H, clipfrac]); with abs_terms
+    also, per layer, the sums over rows of the absolute addends of each gradient entry,
+    (|dz|^T |h_in|, sum |dz|): the scale of the rounding error any summation of those
+    addends can make (the condition of the sum).
     """
     inputs, zs, Z = _forward(Ws, bs, X, acts, grid)
     n = Z.shape[0]
@@ -176,14 +179,19 @@ def loss_grad(Ws, bs, has_value, X, actions, logp_old, adv, ret, algo, clip_eps=
         loss += c_value * vloss
         dZ[:, A] = 2.0 * c_value * (v - r) / n
     grads = [None] * len(Ws)
+    absg = [None] * len(Ws)
     dz = dZ
     for l in range(len(Ws) - 1, -1, -1):
         h_in = inputs[l]
         grads[l] = (dz.T @ h_in, dz.sum(axis=0))
+        if abs_terms:
+            absg[l] = (np.abs(dz).T @ np.abs(h_in), np.abs(dz).sum(axis=0))
         if l > 0:
             dh = dz @ np.asarray(Ws[l], np.float64)
             dz = dh * act_grad(acts[l - 1] if acts else TANH, zs[l - 1])
     stats = np.array([loss, pg, vloss, H.mean(), clipfrac])
+    if abs_terms:
+        return grads, stats, absg
     return grads, stats
 
 

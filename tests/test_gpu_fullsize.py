@@ -6,8 +6,10 @@
 * The benchmark step's returns and mean baseline over all 2,097,152 rows against the fp64
   recurrence (within 1e-5 of the recurrence on absolute values), and its REINFORCE loss
   gradient and loss value against the fp64 oracle (computed in row chunks) on the same
-  advantages and returns: TF32 within 1e-2, FP32 within 1e-5, per tensor in norm and per
-  element (|g - g_ref| <= tol (|g_ref| + rms(g_ref))).
+  advantages and returns: TF32 within 1e-2, FP32 within 1e-5 per tensor in norm, and per
+  element against the condition of each entry's sum over the rows: |g - g_ref| <=
+  tol |g_ref| + eps_sum (sum of the absolute values of its per-row addends), eps_sum the
+  rounding bound of such a sum (1e-2 TF32, 1e-3 FP32).
 * The policy-free router step at 65,536 envs (the thread-per-env kernel's
   configuration): sampled envs' records and final state bit for bit.
 """
@@ -72,20 +74,21 @@ def test_c2_benchmark_rollout_sampled_envs_bit_exact():
 
 def _oracle_loss_chunked(Ws, bs, obs, act, logp, adv, G, n, chunk=262144):
     """REINFORCE loss gradient over all n rows, in row chunks (each chunk's mean weighted
-    by its share of the rows)."""
+    by its share of the rows), with the sum of absolute addends of every entry."""
     E = obs.shape[2]
-    total, stats = None, np.zeros(5)
+    total, scale, stats = None, None, np.zeros(5)
     for r0 in range(0, n, chunk):
         rows = np.arange(r0, min(n, r0 + chunk))
         X, a, lpo = rl.gather_rows(obs, act, logp, rows, E)
         t, e = rows // E, rows % E
-        g, st = rl.loss_grad(Ws, bs, False, X, a, lpo, adv[t, e], G[t, e], rl.REINFORCE,
-                             0.2, 0.0, 0.0)
+        g, st, ab = rl.loss_grad(Ws, bs, False, X, a, lpo, adv[t, e], G[t, e], rl.REINFORCE,
+                                 0.2, 0.0, 0.0, abs_terms=True)
         w = len(rows) / n
-        f = rl.flat(g) * w
+        f, fa = rl.flat(g) * w, rl.flat(ab) * w
         total = f if total is None else total + f
+        scale = fa if scale is None else scale + fa
         stats += np.asarray(st, np.float64) * w
-    return total, stats
+    return total, scale, stats
 
 
 def test_c2_benchmark_step_full_size_loss_gradient():
@@ -121,10 +124,14 @@ def test_c2_benchmark_step_full_size_loss_gradient():
     # the loss on the advantages and returns both sides are given (the GPU's fp32 values)
     A_gpu = adv.cpu().numpy().astype(np.float64)
     Ws, bs, _ = host
-    g_ref, st_ref = _oracle_loss_chunked(Ws, bs, buf["obs"].cpu().numpy(),
+    g_ref, g_abs, st_ref = _oracle_loss_chunked(Ws, bs, buf["obs"].cpu().numpy(),
                                          buf["action"].cpu().numpy(), buf["logp"].cpu().numpy(),
                                          A_gpu, G_gpu, n)
-    for prec, tol in (("tf32", 1e-2), ("fp32", 1e-5)):
+    # per element: tol |g_ref| + eps_sum (sum of |addends|).  eps_sum bounds the rounding
+    # of a sum over the rows: TF32 inputs (2^-11 relative each) within 1e-2; FP32
+    # accumulation of depth below 16,384 (rows per block plus blocks) within
+    # 16,384 x 2^-24 < 1e-3 of the absolute sum
+    for prec, tol, eps_sum in (("tf32", 1e-2, 1e-2), ("fp32", 1e-5, 1e-3)):
         g, st = grads[prec]
         off = 0
         for w, b in zip(Ws, bs):
@@ -132,8 +139,12 @@ def test_c2_benchmark_step_full_size_loss_gradient():
                 gg, rr = g[off:off + size], g_ref[off:off + size]
                 off += size
                 assert np.linalg.norm(gg - rr) <= tol * np.linalg.norm(rr) + 1e-12, prec
-                rms = np.sqrt(np.mean(rr ** 2))
-                assert np.all(np.abs(gg - rr) <= tol * (np.abs(rr) + rms) + 1e-12), prec
+                # per element, against the condition of the sum over 2M rows: the sum
+                # of its absolute addends
+                sc = g_abs[off - size:off]
+                ratio = np.abs(gg - rr) / (tol * np.abs(rr) + eps_sum * sc + 1e-12)
+                worst = int(np.argmax(ratio))
+                assert ratio[worst] <= 1.0, (prec, off - size, worst, gg[worst], rr[worst], sc[worst])
         assert abs(st[0] - st_ref[0]) <= tol * (abs(st_ref[0]) + 1.0), prec
 
 
