@@ -33,6 +33,18 @@ __global__ void __launch_bounds__(kAdamThreads) k_sumsq(const float* __restrict_
   if (threadIdx.x == 0) part[blockIdx.x] = red[0];
 }
 
+// b^t for t >= 1 by binary powering in fp64 (a few dependent multiplies: a general pow
+// is a long fp64 chain, and fp64 is slow on this GPU).
+__device__ double pow_int(double b, int64_t t) {
+  double r = 1.0;
+  while (t > 0) {
+    if (t & 1) r *= b;
+    b *= b;
+    t >>= 1;
+  }
+  return r;
+}
+
 // scal[0] = min(1, max_norm / ||g||) (1 for a zero gradient, or without clipping);
 // with a device step counter also t = ++*d_t, scal[1] = lr / (1 - b1^t) and
 // scal[2] = 1 / sqrt(1 - b2^t), the bias corrections the host computes otherwise.
@@ -52,8 +64,8 @@ __global__ void k_adam_scalars(const double* part, int nb, float max_norm, int64
   if (d_t) {
     const int64_t t = *d_t + 1;
     *d_t = t;
-    scal[1] = (float)((double)lr / (1.0 - pow((double)b1, (double)t)));
-    scal[2] = (float)(1.0 / sqrt(1.0 - pow((double)b2, (double)t)));
+    scal[1] = (float)((double)lr / (1.0 - pow_int((double)b1, t)));
+    scal[2] = (float)(1.0 / sqrt(1.0 - pow_int((double)b2, t)));
   }
 }
 
