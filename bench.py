@@ -852,7 +852,14 @@ def run_gpu(a) -> None:
                     "frac": ach_r / fp32_nominal, "traffic": ROLLOUT_DRAM_BYTES,
                     "traffic_source": ROLLOUT_DRAM_SOURCE, "peak_source": fp32_src,
                     "flop_per_launch": flop_rollout}
-    roof = roof_rollout if ph[1] >= update_ms * loss_share else roof_loss
+    # the dominant single kernel: the loss-gradient call is five kernels (weight images,
+    # per-tile forward/backward, weight-gradient products, two reductions), the largest
+    # about two thirds of the call (profiles/), so k_rollout leads unless the whole call
+    # outweighs it by more than that
+    loss_total_ms = update_ms * loss_share
+    roof = roof_rollout if ph[1] >= 0.7 * loss_total_ms else roof_loss
+    roof_rollout["dominance"] = ("k_rollout %.1f ms per step; the loss-gradient calls %.1f ms per "
+                                 "step over five kernels" % (ph[1], loss_total_ms))
 
     if rank == 0:
         line = {

@@ -66,6 +66,7 @@ struct Plan {
   int poff[SIMX_MAX_LAYERS];
   // k_lw_rows
   int a_bytes, stage_bytes, nstages, smem, tcols;
+  int hs_off;                // the loss head's scratch inside the A buffer (3 KB)
   // k_lw_dw
   int mt0[SIMX_MAX_LAYERS];  // first work item of layer l (blocks of 128 outputs)
   int mt_total, S, dw_stage_bytes, dw_nstages, dw_smem, dw_tcols;
@@ -390,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   }
   int ac = 0;
   float adv = 0.0f, lpo = 0.0f, ret = 0.0f;
-  if (cq == 0 && live) {
+  if (live) {
     ac = __ldg(a.action + row);
     adv = __ldg(a.adv + row);
     lpo = a.algo == SIMX_ALGO_PPO ? __ldg(a.logp_old + row) : 0.0f;
@@ -454,11 +455,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
       // blocks
       const int Wn = P.Ka[l + 1], Fn = P.Fh[l + 1];
       unsigned char* img = A.ws + P.img_h[l + 1] + img_blk(grow, Fn);
+      // the next block's accumulator load is in flight while this block is computed
+      uint32_t u[16];
+      if (16 * cq < Wn) tm_ld16_nw(tl + (uint32_t)(16 * cq), u);
       for (int c0 = 16 * cq; c0 < Wn; c0 += 64) {
         float z[16], bv[16], h[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) bv[i] = c0 + i < Nl ? __ldg(bias + c0 + i) : 0.0f;
-        ld16(c0, Nl, z);
+        tm_wait();
+        reg_fence16(u);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) z[i] = c0 + i < Nl ? __uint_as_float(u[i]) : 0.0f;
+        if (c0 + 64 < Wn) tm_ld16_nw(tl + (uint32_t)(c0 + 64), u);
 #pragma unroll
         for (int i = 0; i < 16; ++i) h[i] = c0 + i < Nl ? tanh_fast(z[i] + bv[i]) : 0.0f;
 #pragma unroll
@@ -468,28 +476,42 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
                           to_tf32(h[4 * qq + 3]));
         if (c0 < Fn) img_store16(img, c0, h, lane);
       }
-    } else if (cq == 0) {
-      // loss head for row r: G = dL/dZ over the logits (and the value row)
+    } else {
+      // loss head: G = dL/dZ over the logits (and the value row).  The four warps of a
+      // lane quarter share each row, one 16-column block in four each; the row's max,
+      // sum, entropy, chosen log-probability and value meet in a shared scratch (the A
+      // buffer past G's columns, free at this point), combined in a fixed order.
       const int NA = a.n_actions;
-      float m = -__uint_as_float(0x7F800000u);
-      for (int c0 = 0; c0 < NA; c0 += 16) {
+      const int Wg = P.Gk[l], Fg = P.Fg[l];
+      float* red = reinterpret_cast<float*>(s.abuf + P.hs_off);   // [4][128]
+      float* lz = red + 4 * kR;                                     // [2][128]
+      float mloc = -__uint_as_float(0x7F800000u);
+      for (int c0 = 16 * cq; c0 < NA; c0 += 64) {
         float z[16];
         ld16(c0, Nl, z);
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          if (c0 + i < NA) m = fmaxf(m, z[i] + __ldg(bias + c0 + i));
+          if (c0 + i < NA) mloc = fmaxf(mloc, z[i] + __ldg(bias + c0 + i));
       }
-      float Ssum = 0.0f;
-      for (int c0 = 0; c0 < NA; c0 += 16) {
+      red[cq * kR + r] = mloc;
+      __syncthreads();
+      const float m = fmaxf(fmaxf(red[r], red[kR + r]), fmaxf(red[2 * kR + r], red[3 * kR + r]));
+      __syncthreads();
+      float sloc = 0.0f;
+      for (int c0 = 16 * cq; c0 < NA; c0 += 64) {
         float z[16];
         ld16(c0, Nl, z);
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          if (c0 + i < NA) Ssum += __expf(z[i] + __ldg(bias + c0 + i) - m);
+          if (c0 + i < NA) sloc += __expf(z[i] + __ldg(bias + c0 + i) - m);
       }
+      red[cq * kR + r] = sloc;
+      __syncthreads();
+      const float Ssum = ((red[r] + red[kR + r]) + red[2 * kR + r]) + red[3 * kR + r];
       const float lse = m + __logf(Ssum);
-      float Hent = 0.0f, lpa = 0.0f, zv = 0.0f;
-      for (int c0 = 0; c0 < Nl; c0 += 16) {
+      __syncthreads();
+      float hloc = 0.0f;
+      for (int c0 = 16 * cq; c0 < Nl; c0 += 64) {
         float z[16];
         ld16(c0, Nl, z);
 #pragma unroll
@@ -497,16 +519,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
           const int j = c0 + i;
           if (j < NA) {
             const float lp = z[i] + __ldg(bias + j) - lse;
-            Hent -= __expf(lp) * lp;
-            if (j == ac) lpa = lp;
+            hloc -= __expf(lp) * lp;
+            if (j == ac) lz[r] = lp;
           } else if (j == NA && j < Nl) {
-            zv = z[i] + __ldg(bias + j);
+            lz[kR + r] = z[i] + __ldg(bias + j);
           }
         }
       }
+      red[cq * kR + r] = hloc;
+      __syncthreads();
+      const float Hent = ((red[r] + red[kR + r]) + red[2 * kR + r]) + red[3 * kR + r];
+      const float lpa = lz[r];
+      const float zv = Nl > NA ? lz[kR + r] : 0.0f;
       float coef = 0.0f, dv = 0.0f;
       if (live) {
         float pg;
+        double cf = 0.0;
         if (a.algo == SIMX_ALGO_REINFORCE) {
           coef = adv;
           pg = -adv * lpa;
@@ -516,19 +544,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
           const float s2 = fminf(fmaxf(rho, 1.0f - a.clip_eps), 1.0f + a.clip_eps) * adv;
           pg = -fminf(s1, s2);
           coef = (s1 <= s2 ? adv : 0.0f) * rho;
-          st_cf += fabsf(rho - 1.0f) > a.clip_eps ? 1.0 : 0.0;
+          cf = fabsf(rho - 1.0f) > a.clip_eps ? 1.0 : 0.0;
         }
-        if (a.has_value) {
-          dv = zv - ret;
+        if (a.has_value) dv = zv - ret;
+        if (cq == 0) {   // one thread per row keeps the row's statistics
+          st_cf += cf;
           st_v += (double)dv * (double)dv;
+          st_pg += pg;
+          st_h += Hent;
         }
-        st_pg += pg;
-        st_h += Hent;
       }
       // G_{L-1}: TF32 into the A buffer (width Gk), FP32 into the G image
-      const int Wg = P.Gk[l], Fg = P.Fg[l];
       unsigned char* img = A.ws + P.img_g[l] + img_blk(grow, Fg);
-      for (int c0 = 0; c0 < Wg; c0 += 16) {
+      for (int c0 = 16 * cq; c0 < Wg; c0 += 64) {
         float z[16], bv[16], g[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) bv[i] = c0 + i < NA ? __ldg(bias + c0 + i) : 0.0f;
@@ -567,13 +595,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     const int width = Wg > Fg ? Wg : Fg;
     const unsigned char* himg = A.ws + P.img_h[l] + img_blk(grow, Fh);
     unsigned char* gimg = A.ws + P.img_g[l - 1] + img_blk(grow, Fg);
+    uint32_t u[16];
+    if (16 * cq < width) tm_ld16_nw(tl + (uint32_t)(16 * cq), u);
     for (int c0 = 16 * cq; c0 < width; c0 += 64) {
       float z[16], hv[16], g[16];
       if (c0 < Fh) img_load16(himg, c0, hv, lane);
       else
 #pragma unroll
         for (int i = 0; i < 16; ++i) hv[i] = 0.0f;
-      ld16(c0, Kl, z);
+      tm_wait();
+      reg_fence16(u);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) z[i] = c0 + i < Kl ? __uint_as_float(u[i]) : 0.0f;
+      if (c0 + 64 < width) tm_ld16_nw(tl + (uint32_t)(c0 + 64), u);
 #pragma unroll
       for (int i = 0; i < 16; ++i) g[i] = c0 + i < Kl ? z[i] * (1.0f - hv[i] * hv[i]) : 0.0f;
       if (c0 < Wg)
@@ -786,6 +820,9 @@ Plan plan(const LossArgs& a) {
   }
   p.n_params = P;
   const int limit = 227 * 1024, misc = 256;
+  // the head's scratch follows G_{L-1} in the A buffer: make the buffer long enough
+  p.hs_off = kR * p.Gk[L - 1] * 4;
+  if (maxA < p.Gk[L - 1] + 6) maxA = (p.Gk[L - 1] + 6 + 31) / 32 * 32;
   p.a_bytes = kR * maxA * 4;
   p.stage_bytes = maxB * kKC * 4;
   p.nstages = kMaxStages;
