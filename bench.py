@@ -62,6 +62,8 @@ def _args():
     p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
                    help="loss-gradient products: tf32 tensor cores (parity 1e-2) or fp32 (1e-5)")
     p.add_argument("--cpu-child", default=None, help=argparse.SUPPRESS)
+    p.add_argument("--hbm-step-only", type=int, default=None, metavar="ENVS",
+                   help="time only the policy-free batched step at this env count and exit")
     p.add_argument("--minibatch-loss", default=None, metavar="WORKLOAD",
                    help="time the PPO loss gradient on 8192-row minibatches of a workload's "
                         "rollout (both precisions) and exit")
@@ -902,6 +904,15 @@ def main():
         return
     if a.minibatch_loss:
         run_minibatch_loss(a.minibatch_loss)
+        return
+    if a.hbm_step_only:
+        import torch
+
+        from paper_2607_05272_gb300 import build as B
+        from paper_2607_05272_gb300 import workloads as W
+        B.build()
+        from paper_2607_05272_gb300 import simx
+        print(json.dumps(hbm_step_measure(simx, W, torch, E=a.hbm_step_only)), flush=True)
         return
     if a.sweep:
         run_sweep(a)

@@ -555,6 +555,15 @@ simx_status simx_launch_shape(simx_ctx* c, const simx_mlp* pol, int policy_mode,
   host_out[1] = thread ? 1 : a.G;
   host_out[2] = thread ? 128 : a.threads;
   host_out[3] = (!thread && net) ? mlp_warp_of(route, a.G, pol) : 0;
+  host_out[4] = 0;
+  if (!thread && net) {  // the launch's plan for the grid forward (no repack needed)
+    a.mlp_warp = host_out[3];
+    a.mlp.n_layers = pol->n_layers;
+    for (int l = 0; l <= pol->n_layers; ++l) a.mlp.dims[l] = pol->dims[l];
+    a.mlp.grid = pol->grid;
+    plan_tc_forward(a, a.threads / a.G);
+    host_out[4] = a.tc.on;
+  }
   return SIMX_OK;
 }
 

@@ -14,6 +14,21 @@ void count_launches(int n);
 // SM count of the current device (grid sizes and lane choices scale with it).
 int sm_count();
 
+// The grid policy's forward on the tensor cores inside the fused step (rollout.cu): per
+// layer l the weights as bf16 A operands of nmt[l] tiles of 128 outputs x Kp[l] inputs,
+// the block's envs (padded to Bn columns) as the bf16 B operand, an FP32 accumulator in
+// tensor memory.  Byte offsets are inside the kernel's dynamic shared memory.
+struct TcPlan {
+  int on;                     // 1: this launch runs the grid forward on the tensor cores
+  int Bn;                     // MMA N: the block's envs rounded up to 16
+  int Kp[SIMX_MAX_LAYERS];    // layer inputs rounded up to 16
+  int nmt[SIMX_MAX_LAYERS];   // tiles of 128 outputs
+  uint32_t w_off[SIMX_MAX_LAYERS];
+  uint32_t x_off[2];          // the two activation operand buffers (Bn x Kx bf16)
+  uint32_t bar_off;           // mbarrier (8 B) and tensor-memory base (4 B)
+  int tcols;                  // tensor-memory columns allocated per block
+};
+
 struct RolloutArgs {
   simx_config cfg;
   DevState st;
@@ -40,6 +55,7 @@ struct RolloutArgs {
   int threads;      // threads per block (64, 128 or 256)
   int bs_pad;       // activation row stride = envs per block + bs_pad (see act_stride_pad)
   int mlp_warp;     // 1: each warp runs the policy for its own envs (see mlp_forward_warp)
+  TcPlan tc;        // grid policies: the tensor-core forward (tc.on = 0 otherwise)
   // trace replay (arrival_kind TRACE): gaps, types (or null), costs (or null), length
   const uint32_t* tr_gap;
   const uint8_t* tr_type;
@@ -78,6 +94,9 @@ cudaError_t launch_load(const DevState& st, int32_t cost_type, uint64_t words, c
 cudaError_t launch_stats(const DevState& st, unsigned long long* out, cudaStream_t s);
 cudaError_t launch_repack(const float* W, const float* b, int N, int K, int Npad, float* Wt, float* bias, cudaStream_t s);
 cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s);
+// Sets a.tc (and the activation rows a.maxd4 it needs) when the grid forward of this
+// launch can run on the tensor cores; returns the dynamic shared memory of the launch.
+size_t plan_tc_forward(RolloutArgs& a, int B);
 int choose_lanes(int64_t envs);
 int choose_threads(int64_t envs, int G);
 

@@ -7,9 +7,11 @@
 // rollout_collect uses H = horizon; sim_step_batched uses H = 1.
 #include <cstdint>
 #include <cstdlib>
+#include <cstring>
 
 #include "kernels.h"
 #include "sim.cuh"
+#include "tc_common.cuh"
 
 namespace simx {
 
@@ -648,6 +650,154 @@ __device__ __forceinline__ void write_obs(const Grp<G>& g, const float* o, int B
   for (int d = (int)g.gl; d < D; d += G) dst[(int64_t)d * ld + e] = o[d * B];
 }
 
+// ---------------------------------------------------------------------------------
+// The grid policy's forward on the tensor cores (the exact policy forward).  On the
+// grid every input, weight and hidden output is an integer multiple of its grid unit
+// with a mantissa of at most 255, so each is exact in bf16, every product is exact in
+// fp32, and every partial sum of a pre-activation stays below 2^24 product units: the
+// tensor core's FP32 accumulation gives the exact dot product, the bits the FP32 FMA
+// chains give.  Per layer: the block's envs are the N columns of one tcgen05.mma chain
+// per tile of 128 outputs (kind::f16, bf16 operands, K = 16 per instruction), the
+// weights the A operand resident in shared memory for the launch; threads then read the
+// accumulator (lane = output, column = env), add the bias in FP32, apply the activation
+// and the grid rounding, and write the next layer's operand, or the logits and value
+// into the activation buffer the sampler reads.
+// ---------------------------------------------------------------------------------
+namespace tcf {
+
+using namespace tcx;
+
+constexpr long long kWaitCycles = 2000000000LL;  // bound on the MMA wait (about 1 s)
+
+// Byte offset of (row i, k) in a K-major bf16 operand whose rows hold Kp values: core
+// matrices of 8 rows x 8 values (16 bytes), K-adjacent ones 128 bytes apart.
+__device__ __forceinline__ uint32_t boff(int i, int k, int Kp) {
+  return (uint32_t)(((i >> 3) * (Kp >> 3) + (k >> 3)) * 128 + (i & 7) * 16 + (k & 7) * 2);
+}
+
+// bf16 bits of a value exact in bf16 (on the grid), which is its fp32 bits' upper half.
+__device__ __forceinline__ uint16_t bf16_bits(float v) { return (uint16_t)(__float_as_uint(v) >> 16); }
+
+// Once per launch: the weights of every layer into shared memory as bf16 A tiles (zero
+// padded), the mbarrier, and (warp 0) the tensor memory of the block.
+__device__ void setup(const RolloutArgs& A, unsigned char* sm, uint32_t* tbase) {
+  const DevMlp& m = A.mlp;
+  const TcPlan& P = A.tc;
+  for (int l = 0; l < m.n_layers; ++l) {
+    const int K = m.dims[l], N = m.dims[l + 1], Kp = P.Kp[l], Np = m.npad[l + 1];
+    const int rows = 128 * P.nmt[l];
+    uint16_t* w = reinterpret_cast<uint16_t*>(sm + P.w_off[l]);
+    for (int i = threadIdx.x; i < rows * Kp; i += blockDim.x) {
+      const int j = i / Kp, k = i % Kp;
+      const float v = (j < N && k < K) ? m.Wt[l][(size_t)k * Np + j] : 0.0f;
+      w[boff(j, k, Kp) / 2] = bf16_bits(v);
+    }
+  }
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sm + P.bar_off);
+  if (threadIdx.x == 0) {
+    mbar_init(bar, 1);
+    mbar_fence_init();
+  }
+  if (threadIdx.x < 32) tm_alloc(tbase, (uint32_t)P.tcols);
+  fence_async_smem();
+  fence_before();
+  __syncthreads();
+  fence_after();
+}
+
+__device__ void teardown(const RolloutArgs& A, uint32_t tmem) {
+  fence_before();
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    fence_after();
+    tm_dealloc(tmem, (uint32_t)A.tc.tcols);
+  }
+}
+
+// Returns the buffer holding the last layer (X1: logits rows 0..A-1, value row A) with
+// row stride ld, or sets *timed_out when an MMA wait ran out (the result is then void).
+__device__ float* forward(const RolloutArgs& A, unsigned char* sm, uint32_t tmem, float* X0,
+                          float* X1, int B, int ld, uint32_t& phase, bool& timed_out) {
+  const DevMlp& m = A.mlp;
+  const TcPlan& P = A.tc;
+  const int tid = threadIdx.x, nthr = blockDim.x, warp = tid >> 5, lane = tid & 31;
+  const int Bn = P.Bn, L = m.n_layers;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sm + P.bar_off);
+  // the observation on its grid as the first B operand (padding columns and rows zero)
+  __syncthreads();
+  {
+    const int D = m.dims[0], Kp = P.Kp[0];
+    uint16_t* xb = reinterpret_cast<uint16_t*>(sm + P.x_off[0]);
+    for (int i = tid; i < Bn * Kp; i += nthr) {
+      const int e = i % Bn, k = i / Bn;
+      const float v = (e < B && k < D) ? grid_q(X0[k * ld + e], m.gx[0]) : 0.0f;
+      xb[boff(e, k, Kp) / 2] = bf16_bits(v);
+    }
+  }
+  const int quarter = warp & 3, part = warp >> 2, nsplit = nthr >> 7;   // warps per lane quarter
+  for (int l = 0; l < L; ++l) {
+    const int Kp = P.Kp[l], N = m.dims[l + 1];
+    const bool last = l + 1 == L;
+    fence_async_smem();
+    fence_before();
+    __syncthreads();
+    fence_after();
+    if (tid == 0) {
+      const uint32_t id = idesc_bf16(128, Bn);
+      const uint32_t xa = su32(sm + P.x_off[l & 1]);
+      const uint32_t sbo = (uint32_t)(Kp >> 3) * 128u;
+      for (int mt = 0; mt < P.nmt[l]; ++mt) {
+        const uint32_t wa = su32(sm + P.w_off[l]) + (uint32_t)mt * 128u * (uint32_t)Kp * 2u;
+        for (int ks = 0; ks < Kp / 16; ++ks)
+          mma_bf16(tmem + (uint32_t)(mt * Bn), sdesc(wa + (uint32_t)ks * 256u, 128, sbo),
+                   sdesc(xa + (uint32_t)ks * 256u, 128, sbo), id, ks > 0 ? 1u : 0u);
+      }
+      commit(bar);
+    }
+    if (!mbar_wait(bar, phase, kWaitCycles)) timed_out = true;
+    phase ^= 1u;
+    __syncwarp();
+    fence_after();
+    // epilogue: lane = output j of tile mt, 16 env columns per warp
+    const int Kn = last ? 0 : P.Kp[l + 1];
+    const int gq = last ? -1 : m.gx[l + 1];
+    const int act = last ? -1 : m.act[l];
+    const float* bias = m.bias[l];
+    uint16_t* xn = reinterpret_cast<uint16_t*>(sm + P.x_off[(l + 1) & 1]);
+    for (int mt = 0; mt < P.nmt[l]; ++mt) {
+      const int j = 128 * mt + 32 * quarter + lane;
+      for (int c0 = 16 * part; c0 < Bn; c0 += 16 * nsplit) {
+        uint32_t u[16];
+        tm_ld16_nw(tmem + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(mt * Bn + c0), u);
+        tm_wait();
+        reg_fence16(u);
+        const float bj = j < N ? bias[j] : 0.0f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int e = c0 + i;
+          const float z = __fadd_rn(__uint_as_float(u[i]), bj);
+          if (last) {
+            if (j < N && e < B) X1[j * ld + e] = z;
+          } else if (j < Kn) {
+            float y = 0.0f;
+            if (j < N && e < B) {
+              y = z;
+              if (act == 0) y = det_tanh(y);
+              else if (act == 2) y = det_gelu(y);
+              y = grid_q(y, gq);
+            }
+            xn[boff(e, j, Kn) / 2] = bf16_bits(y);
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+  return X1;
+}
+
+}  // namespace tcf
+
 // The rollout / step kernel.  A block of blockDim.x threads owns B = blockDim.x / G
 // envs, one per G-lane group.  Shared memory: two activation buffers X0, X1 of
 // maxd4 x B floats (feature-major) and a softmax scratch of apad floats per env.
@@ -688,6 +838,14 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
   uint32_t* ringS = ROUTE ? ringb + (size_t)(g.gl < K ? g.gl : 0) * T * cap : ringb;
   uint32_t* costS = (ROUTE && costb) ? costb + (size_t)(g.gl < K ? g.gl : 0) * cap : costb;
   const int D = A.obs_dim;
+  // grid policies on the tensor cores: weights, barrier and tensor memory for the launch
+  unsigned char* tsm = reinterpret_cast<unsigned char*>(smem);
+  uint32_t tc_phase = 0u;
+  bool tc_timeout = false;
+  const bool tc = GRID && !WARP && A.tc.on && use_mlp;
+  uint32_t* tc_tbase = reinterpret_cast<uint32_t*>(tsm + A.tc.bar_off + 8);
+  if (tc) tcf::setup(A, tsm, tc_tbase);
+  const uint32_t tc_tmem = tc ? *tc_tbase : 0u;
 
   for (int t = 0; t < A.H; ++t) {
     // phase 1: observation (Sec. 4.1) into column `slot` of X0
@@ -704,8 +862,14 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
       // WARP: each warp runs the policy for its own 1-2 envs (narrow policies); else
       // block-wide, whose warps share each weight row instead of each loading it.  A
       // template parameter: both forwards in one kernel slowed the narrow case by 16 %.
-      const float* Z = WARP ? mlp_forward_warp<GRID>(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G))
-                            : mlp_forward_block<GRID>(A.mlp, X0, X1, B, Bs);
+      const float* Z;
+      if (tc) {
+        Z = tcf::forward(A, tsm, tc_tmem, X0, X1, B, Bs, tc_phase, tc_timeout);
+        if (tc_timeout) s.status |= SIMX_DEV_TC_TIMEOUT;
+      } else {
+        Z = WARP ? mlp_forward_warp<GRID>(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G))
+                 : mlp_forward_block<GRID>(A.mlp, X0, X1, B, Bs);
+      }
       if (live)
         a = sample_action<G>(A.mlp, Z + slot, Bs, scratch, A.policy_mode, A.key0, A.key1, s.tg,
                              env, logp, value, g);
@@ -845,6 +1009,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
     }
     __syncwarp();
   }
+  if (tc) tcf::teardown(A, tc_tmem);
   if (!live) return;
   if (A.next_obs) {
     if (ROUTE) observe_route<G>(c, g, s, L, ocol, Bs);
@@ -1093,10 +1258,53 @@ static size_t env_smem(const RolloutArgs& a, int B) {
   return ((size_t)2 * a.maxd4 * (B + a.bs_pad) + (size_t)a.apad * B) * sizeof(float);
 }
 
+// The tensor-core grid forward applies to block-wide forwards of grid policies in blocks
+// of at least 128 threads (4 warps cover the 128 lanes of a tile) with layers up to 256
+// wide; SIMX_TC_FORWARD=0 turns it off (the FP32 tiles then give the same bits).
+size_t plan_tc_forward(RolloutArgs& a, int B) {
+  std::memset(&a.tc, 0, sizeof(a.tc));
+  const DevMlp& m = a.mlp;
+  const bool net = a.policy_mode == SIMX_POLICY_SAMPLE || a.policy_mode == SIMX_POLICY_ARGMAX;
+  bool ok = net && m.grid && !a.mlp_warp && a.threads >= 128 && B >= 1 && B <= 32;
+  if (const char* f = getenv("SIMX_TC_FORWARD"))
+    if (f[0] == '0') ok = false;
+  for (int l = 0; ok && l < m.n_layers; ++l)
+    if (m.dims[l] > 256 || m.dims[l + 1] > 256) ok = false;
+  if (!ok) return env_smem(a, B);
+  RolloutArgs t = a;
+  const int L = m.n_layers;
+  int rows = m.dims[0] > m.dims[L] ? m.dims[0] : m.dims[L];
+  t.maxd4 = (rows + 3) / 4 * 4;   // X0 holds the observation, X1 the last layer
+  TcPlan& P = t.tc;
+  P.Bn = (B + 15) / 16 * 16;
+  size_t off = (env_smem(t, B) + 127) / 128 * 128;
+  int Kx = 16, cols = 0;
+  for (int l = 0; l < L; ++l) {
+    P.Kp[l] = (m.dims[l] + 15) / 16 * 16;
+    P.nmt[l] = (m.dims[l + 1] + 127) / 128;
+    P.w_off[l] = (uint32_t)off;
+    off += (size_t)P.nmt[l] * 128 * P.Kp[l] * 2;
+    Kx = Kx > P.Kp[l] ? Kx : P.Kp[l];
+    cols = cols > P.nmt[l] * P.Bn ? cols : P.nmt[l] * P.Bn;
+  }
+  for (int b = 0; b < 2; ++b) {
+    P.x_off[b] = (uint32_t)off;
+    off += (size_t)P.Bn * Kx * 2;
+  }
+  P.bar_off = (uint32_t)off;
+  off += 16;
+  P.tcols = cols <= 32 ? 32 : (cols <= 64 ? 64 : 128);
+  if (off > 227 * 1024) return env_smem(a, B);
+  P.on = 1;
+  a = t;
+  return off;
+}
+
 template <bool ROUTE, int G>
-static cudaError_t rollout_t(const RolloutArgs& a, cudaStream_t s) {
-  const int B = a.threads / G;
-  const size_t sh = env_smem(a, B);
+static cudaError_t rollout_t(const RolloutArgs& a0, cudaStream_t s) {
+  const int B = a0.threads / G;
+  RolloutArgs a = a0;
+  const size_t sh = plan_tc_forward(a, B);
   const bool tr = a.cfg.arrival_kind == SIMX_ARR_TRACE;
   // GRID: the grid policy's instantiations (a.mlp.grid is 0 without a policy)
   const bool gr = a.mlp.grid != 0;

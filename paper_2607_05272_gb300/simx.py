@@ -298,12 +298,13 @@ class Sim:
 
     def launch_shape(self, policy_mode: str, policy: Policy = None) -> dict:
         """The launch rollout_collect takes (simx_launch_shape): kernel ("fused" or
-        "thread"), lanes per env, threads per block, warp-local policy forward."""
-        out = (C.c_int32 * 4)()
+        "thread"), lanes per env, threads per block, warp-local policy forward, and
+        whether a grid policy's forward runs on the tensor cores."""
+        out = (C.c_int32 * 5)()
         _check(lib().simx_launch_shape(self._h, C.byref(policy.c) if policy else None,
                                        POLICY[policy_mode], out))
         return dict(kernel="thread" if out[0] else "fused", lanes=out[1], threads=out[2],
-                    mlp_warp=bool(out[3]))
+                    mlp_warp=bool(out[3]), tensor_cores=bool(out[4]))
 
     def stats(self) -> dict:
         c = Counters()

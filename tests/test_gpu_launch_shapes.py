@@ -88,7 +88,7 @@ def _run_sampled(name, E, H, mode, shape, with_state=True):
         assert np.array_equal(state, ref["state"])
 
 
-FUSED = dict(kernel="fused", lanes=8, mlp_warp=False)
+FUSED = dict(kernel="fused", lanes=8, mlp_warp=False, tensor_cores=False)
 
 
 def test_c3_16384_envs_128_thread_blocks():
@@ -109,7 +109,7 @@ def test_c5_argmax_1048576_envs():
                  with_state=False)
 
 
-THREAD = dict(kernel="thread", lanes=1, threads=128, mlp_warp=False)
+THREAD = dict(kernel="thread", lanes=1, threads=128, mlp_warp=False, tensor_cores=False)
 
 
 @pytest.mark.parametrize("E,H,state", [(262144, 256, True), (1048576, 64, False)])
