@@ -62,6 +62,10 @@ def _args():
     p.add_argument("--loss-precision", default="tf32", choices=["tf32", "fp32"],
                    help="loss-gradient products: tf32 tensor cores (parity 1e-2) or fp32 (1e-5)")
     p.add_argument("--cpu-child", default=None, help=argparse.SUPPRESS)
+    p.add_argument("--grid-rollout", default=None, metavar="WORKLOAD",
+                   help="time a grid policy's rollout with the forward on the tensor cores and on "
+                        "the FP32 tiles (the exact policy forward) and exit")
+    p.add_argument("--grid-envs", type=int, default=65536)
     p.add_argument("--hbm-step-only", type=int, default=None, metavar="ENVS",
                    help="time only the policy-free batched step at this env count and exit")
     p.add_argument("--minibatch-loss", default=None, metavar="WORKLOAD",
@@ -467,6 +471,58 @@ def hbm_step_measure(simx, W, torch, E=65536, steps=100, warm=10) -> dict:
             "bytes_per_env_step": per, "achieved": gbs, "peak": hbm, "unit": "GB/s",
             "frac": gbs / hbm, "peak_source": "%s hbm_gbs" % src, "l2": l2,
             "timing": "CUDA graph of %d steps, replayed %d times, CUDA events" % (steps, reps)}
+
+
+def run_grid_rollout(name: str, E: int, reps: int = 3) -> None:
+    """A grid policy (the exact policy forward) on `name`'s env: rollout_collect with the
+    forward on the tensor cores, then on the FP32 tiles (SIMX_TC_FORWARD=0), CUDA events
+    around each launch after a warm-up; the two buffers must be equal bit for bit."""
+    import torch
+
+    from paper_2607_05272_gb300 import build as B
+    from paper_2607_05272_gb300 import workloads as W
+    B.build()
+    from paper_2607_05272_gb300 import simx
+    cfg = W.CONFIGS[name](E)
+    H = W.HORIZON[name]
+    dims, hv = W.mlp_dims(name)
+    gx = [5] + [7] * (len(dims) - 2)
+    ew = [8] * (len(dims) - 1)
+    Ws, bs = W.grid_weights(dims, 21, gx, ew)
+    pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws], [torch.from_numpy(b).cuda() for b in bs],
+                      hv, W.mlp_acts(name), grid=gx)
+    mode = "argmax" if name == "c5" else "sample"
+    line = {"workload": name, "envs": E, "horizon": H, "mlp": dims}
+    bufs = []
+    for tc in ("1", "0"):
+        os.environ["SIMX_TC_FORWARD"] = tc
+        sim = simx.Sim(cfg)
+        shape = sim.launch_shape(mode, pol)
+        sim.reset(W.SEED[name])
+        warm = simx.alloc_rollout(E, sim.D, 4, has_value=hv)
+        sim.rollout(mode, 4, warm, pol)
+        del warm
+        buf = simx.alloc_rollout(E, sim.D, H, has_value=hv)
+        ts = []
+        for _ in range(reps):
+            sim.reset(W.SEED[name])
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            sim.rollout(mode, H, buf, pol)
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        st, _ = sim.last_status()
+        sim.close()
+        ms = statistics.median(ts)
+        key = "tensor_cores" if tc == "1" else "fp32_tiles"
+        line[key] = {"ms": ms, "decision_steps_per_s": E * H / (ms * 1e-3), "status": st,
+                     "launch": shape}
+        bufs.append(buf)
+    os.environ.pop("SIMX_TC_FORWARD", None)
+    line["bit_identical"] = all(torch.equal(bufs[0][k], bufs[1][k]) for k in bufs[0])
+    line["speedup"] = line["fp32_tiles"]["ms"] / line["tensor_cores"]["ms"]
+    print(json.dumps(line), flush=True)
 
 
 def run_minibatch_loss(name: str, E: int = 256, steps: int = 20) -> None:
@@ -904,6 +960,9 @@ def main():
         return
     if a.minibatch_loss:
         run_minibatch_loss(a.minibatch_loss)
+        return
+    if a.grid_rollout:
+        run_grid_rollout(a.grid_rollout, a.grid_envs)
         return
     if a.hbm_step_only:
         import torch
