@@ -16,12 +16,15 @@
 //              x_lo w_hi as one GEMM against [x_hi | x_hi | x_lo] (raw observations reach
 //              magnitudes in the hundreds; one TF32 pass there moves saturated tanh units'
 //              derivatives by percents).
-//   k_lw_rows  one CTA per 128-row tile: the whole forward pass, the loss head and the
-//              backward pass down to G_0 for its rows.  The A operand (the tile's
-//              activations, or G) stays resident in shared memory, written by the
-//              epilogue of the previous product; the weight chunks stream through a ring
-//              of shared-memory stages by bulk copies, the MMAs of chunk c queued before
-//              the stage of chunk c - 1 is refilled.  H_l and G_l go to global memory as
+//   k_lw_rows  a cluster of two CTAs per 128-row tile: the whole forward pass, the loss
+//              head and the backward pass down to G_0 for its rows.  The A operand (the
+//              tile's activations, or G) stays resident in both CTAs' shared memory; each
+//              CTA computes half of the outputs of every product but the last layer's
+//              (its half of the rows of each weight chunk, which stream through a ring of
+//              shared-memory stages by bulk copies, the MMAs of chunk c queued before the
+//              stage of chunk c - 1 is refilled) and writes its half of the next operand
+//              into both A buffers (distributed shared memory, a cluster barrier on each
+//              side); the loss head is split by rows.  H_l and G_l go to global memory as
 //              feature-major images (the layout of the weight-gradient products).
 //   k_lw_dw    [dW_l | db_l] = G_l^T [H_l | 1] with K = the rows, split over CTAs by
 //              (layer, block of 128 outputs, row range); each CTA writes its slice of
@@ -47,7 +50,7 @@ constexpr int kR = 128;            // rows per tile (MMA M)
 constexpr int kThreads = 512;      // k_lw_rows: 16 warps, 4 per TMEM lane quarter
 constexpr int kDwThreads = 256;    // k_lw_dw: 8 warps, 2 per lane quarter
 constexpr int kKC = 32;            // K values per streamed chunk
-constexpr int kMaxStages = 3;
+constexpr int kMaxStages = 6;
 constexpr long long kWaitCycles = 2000000000LL;  // bound on any wait (about 1 s)
 
 int r16(int x) { return (x + 15) / 16 * 16; }
@@ -58,9 +61,11 @@ struct Plan {
   int L, n_params;
   int K[SIMX_MAX_LAYERS], N[SIMX_MAX_LAYERS];
   int Ka[SIMX_MAX_LAYERS];   // forward A width (GEMM K): 3 r32(K_0) for layer 0, r32(K_l) after
-  int Nf[SIMX_MAX_LAYERS];   // forward MMA N: r16(N_l)
+  int Nf[SIMX_MAX_LAYERS];   // forward outputs: r32(N_l) split in two halves, r16 for the last layer
   int Gk[SIMX_MAX_LAYERS];   // backward A width (GEMM K of dH_l = G_l W_l): r32(N_l)
-  int Kb[SIMX_MAX_LAYERS];   // backward MMA N: r16(K_l)
+  int Kb[SIMX_MAX_LAYERS];   // backward products' outputs: r32(K_l), in two halves of hK
+  int hN[SIMX_MAX_LAYERS];   // forward MMA N of one CTA: Nf / 2 (split) or Nf (last layer)
+  int hK[SIMX_MAX_LAYERS];   // backward MMA N of one CTA: Kb / 2
   int Fh[SIMX_MAX_LAYERS];   // features of the H_l image: r16(K_l)
   int Fg[SIMX_MAX_LAYERS];   // features of the G_l image: r16(N_l)
   int poff[SIMX_MAX_LAYERS];
@@ -242,23 +247,27 @@ struct Sched {
   int ng, total;
   int k0[2 * SIMX_MAX_LAYERS];
   const unsigned char* src[2 * SIMX_MAX_LAYERS];
-  uint32_t bytes[2 * SIMX_MAX_LAYERS];
+  uint32_t bytes[2 * SIMX_MAX_LAYERS];    // copied per chunk (this CTA's half of the rows)
+  uint32_t stride[2 * SIMX_MAX_LAYERS];   // between the chunks of the image
 };
 
-__device__ Sched make_sched(const Plan& P, unsigned char* ws) {
+// rank: this CTA's half of the split products (its output rows of each weight chunk).
+__device__ Sched make_sched(const Plan& P, unsigned char* ws, int rank) {
   Sched q;
   q.ng = 2 * P.L - 1;
   int k = 0;
   for (int g = 0; g < q.ng; ++g) {
     q.k0[g] = k;
     if (g < P.L) {
-      q.src[g] = ws + P.wf[g];
-      q.bytes[g] = (uint32_t)P.Nf[g] * kKC * 4u;
+      q.stride[g] = (uint32_t)P.Nf[g] * kKC * 4u;
+      q.bytes[g] = (uint32_t)P.hN[g] * kKC * 4u;
+      q.src[g] = ws + P.wf[g] + (P.hN[g] < P.Nf[g] ? (size_t)rank * q.bytes[g] : 0);
       k += P.Ka[g] / kKC;
     } else {
       const int l = 2 * P.L - 1 - g;
-      q.src[g] = ws + P.wb[l];
-      q.bytes[g] = (uint32_t)P.Kb[l] * kKC * 4u;
+      q.stride[g] = (uint32_t)P.Kb[l] * kKC * 4u;
+      q.bytes[g] = (uint32_t)P.hK[l] * kKC * 4u;
+      q.src[g] = ws + P.wb[l] + (size_t)rank * q.bytes[g];
       k += P.Gk[l] / kKC;
     }
   }
@@ -277,7 +286,8 @@ __device__ bool load_chunk(const Smem& s, const Sched& q, int S, int stage_bytes
   while (q.k0[g + 1] <= k) ++g;
   const uint32_t b = q.bytes[g];
   mbar_arrive_expect_tx(&s.full[st], b);
-  bulk_g2s(s.stages + (size_t)st * stage_bytes, q.src[g] + (size_t)(k - q.k0[g]) * b, b, &s.full[st]);
+  bulk_g2s(s.stages + (size_t)st * stage_bytes, q.src[g] + (size_t)(k - q.k0[g]) * q.stride[g], b,
+           &s.full[st]);
   return true;
 }
 
@@ -325,6 +335,34 @@ __device__ void drain_all(const Smem& s, int S, int issued, int consumed) {
   mbar_wait(s.drain, 0u, kWaitCycles);
 }
 
+// The two CTAs of a cluster share one 128-row tile: each computes half of the outputs of
+// every split product (rank r: rows r * half .. of each weight chunk), and writes its half
+// of the next operand into both CTAs' A buffers (distributed shared memory); the loss head
+// is split by rows instead (the last layer runs whole in both CTAs).
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t peer_addr(uint32_t saddr, uint32_t rank) {
+  uint32_t d;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(saddr), "r"(rank));
+  return d;
+}
+__device__ __forceinline__ void st_peer4(uint32_t addr, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
+               : "memory");
+}
+// Every thread of both CTAs: their shared-memory writes (local and remote) made visible,
+// the tensor cores included, before either goes on.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+  fence_before();
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+  fence_after();
+}
+
 __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__ Args A) {
   extern __shared__ __align__(1024) unsigned char sm[];
   const LossArgs& a = A.a;
@@ -334,7 +372,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, cq = warp >> 2;   // lane quarter; column share 0..3
   const int r = 32 * quarter + lane;
-  const int64_t grow = (int64_t)blockIdx.x * kR + r;   // row of the padded minibatch
+  const int rank = (int)cluster_rank();
+  const int64_t tile = blockIdx.x >> 1;
+  const int64_t grow = tile * kR + r;   // row of the padded minibatch
   const bool live = grow < a.n;
 
   // thread 0: barriers, then the first weight chunks on their way before anything else
@@ -349,14 +389,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     mbar_init(s.accb, 1);
     mbar_fence_init();
     *s.abort_flag = 0;
-    sch = make_sched(P, A.ws);
+    sch = make_sched(P, A.ws, rank);
     const int upto = S - 1 < sch.total ? S - 1 : sch.total;
     for (; issued < upto; ++issued) load_chunk(s, sch, S, P.stage_bytes, issued);
   }
   if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.tcols);
 
-  // the tile's observations: x_hi, x_hi, x_lo side by side in the A buffer (split TF32)
-  // and the FP32 values in the H_0 image; the head thread's per-row inputs
+  // the tile's observations (both CTAs, every row): x_hi, x_hi, x_lo side by side in the A
+  // buffer (split TF32); rank 0 writes the FP32 values to the H_0 image
   int64_t row = 0;
   if (live) row = a.idx ? __ldg(a.idx + grow) : grow;
   const int64_t t = row / a.E, e = row % a.E;
@@ -386,7 +426,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         *reinterpret_cast<float4*>(s.abuf + rm_off(r, Kc + k, W0)) = h4;
         *reinterpret_cast<float4*>(s.abuf + rm_off(r, 2 * Kc + k, W0)) = make_float4(lo[0], lo[1], lo[2], lo[3]);
       }
-      if (c0 < F0) img_store16(img, c0, x, lane);
+      if (rank == 0 && c0 < F0) img_store16(img, c0, x, lane);
     }
   }
   int ac = 0;
@@ -397,36 +437,40 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     lpo = a.algo == SIMX_ALGO_PPO ? __ldg(a.logp_old + row) : 0.0f;
     ret = a.has_value ? __ldg(a.ret + row) : 0.0f;
   }
-
-  auto stage_sync = [&]() -> bool {
-    fence_async_smem();
-    fence_before();
-    __syncthreads();
-    fence_after();
-    return *s.abort_flag == 0;
-  };
-  stage_sync();
+  fence_async_smem();
+  fence_before();
+  __syncthreads();
+  fence_after();
   const uint32_t tmem = *s.tbase;
   const uint32_t tl = tmem + ((uint32_t)(32 * quarter) << 16);   // this warp's lane quarter
   const uint32_t abuf_addr = su32(s.abuf);
+  const uint32_t peer = peer_addr(abuf_addr, (uint32_t)(rank ^ 1));   // the other CTA's A buffer
   int ngemm = 0;
   double st_pg = 0.0, st_v = 0.0, st_h = 0.0, st_cf = 0.0;
   const float inv_n = 1.0f / (float)a.n;
 
-  // GEMM g: thread 0 issues it, every thread then waits for the accumulator
-  auto gemm = [&](int g, int a_width, int Nmma) -> bool {
-    // warp 0's other lanes wait at the warp barrier, not polling beside the issuing lane
+  // a float4 of the next operand into both CTAs' A buffers
+  auto put_both = [&](uint32_t off, float4 v) {
+    *reinterpret_cast<float4*>(s.abuf + off) = v;
+    st_peer4(peer + off, v);
+  };
+
+  // GEMM g: thread 0 issues it, every thread then waits for the accumulator; then both
+  // CTAs meet, so that neither writes into the other's A buffer while its products run.
+  // After an abort no more work is issued, but every cluster barrier is still reached.
+  auto gemm = [&](int g, int a_width, int Nmma) {
+    const bool go = *s.abort_flag == 0;
     if (warp == 0) {
-      if (lane == 0 && *s.abort_flag == 0)
+      if (lane == 0 && go)
         gemm_issue(s, sch, S, P.stage_bytes, g, issued, consumed, abuf_addr,
                    (uint32_t)(a_width / 4) * 128u, Nmma, tmem);
       __syncwarp();
     }
-    if (!mbar_wait_idle(s.accb, (uint32_t)(ngemm & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
+    if (go && !mbar_wait_idle(s.accb, (uint32_t)(ngemm & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
     ++ngemm;
     __syncwarp();
     fence_after();
-    return *s.abort_flag == 0;
+    cluster_sync();
   };
 
   // Columns c0 .. c0 + 15 of this thread's accumulator row (one warp-wide load; columns
@@ -441,52 +485,51 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     for (int i = 0; i < 16; ++i) z[i] = c0 + i < ncols ? __uint_as_float(u[i]) : 0.0f;
   };
 
-  bool ok = true;
   // ---- forward
-  for (int l = 0; l < L && ok; ++l) {
-    const int Nf = P.Nf[l];
-    ok = gemm(l, P.Ka[l], Nf);
-    if (!ok) break;
+  for (int l = 0; l < L; ++l) {
+    const int hN = P.hN[l];
+    gemm(l, P.Ka[l], hN);
+    const bool ok = *s.abort_flag == 0;
     const int Nl = P.N[l];
     const float* bias = a.b[l];
     if (l + 1 < L) {
-      // H_{l+1} = tanh(Z_l + b_l): TF32 into the A buffer (width Ka[l+1], zero padded),
-      // FP32 into the H_{l+1} image; the two warps of a quarter take alternate 16-column
-      // blocks
-      const int Wn = P.Ka[l + 1], Fn = P.Fh[l + 1];
+      // H_{l+1} = tanh(Z_l + b_l) for this CTA's half of the outputs: TF32 into both A
+      // buffers (width Ka[l+1] = Nf[l], zero padded), FP32 into the H_{l+1} image
+      const int Wn = P.Ka[l + 1], Fn = P.Fh[l + 1], j0h = rank * hN;
       unsigned char* img = A.ws + P.img_h[l + 1] + img_blk(grow, Fn);
-      // the next block's accumulator load is in flight while this block is computed
       uint32_t u[16];
-      if (16 * cq < Wn) tm_ld16_nw(tl + (uint32_t)(16 * cq), u);
-      for (int c0 = 16 * cq; c0 < Wn; c0 += 64) {
+      if (ok && 16 * cq < hN) tm_ld16_nw(tl + (uint32_t)(16 * cq), u);
+      for (int c0 = 16 * cq; ok && c0 < hN; c0 += 64) {
+        const int jg = j0h + c0;
         float z[16], bv[16], h[16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) bv[i] = c0 + i < Nl ? __ldg(bias + c0 + i) : 0.0f;
+        for (int i = 0; i < 16; ++i) bv[i] = jg + i < Nl ? __ldg(bias + jg + i) : 0.0f;
         tm_wait();
         reg_fence16(u);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) z[i] = c0 + i < Nl ? __uint_as_float(u[i]) : 0.0f;
-        if (c0 + 64 < Wn) tm_ld16_nw(tl + (uint32_t)(c0 + 64), u);
+        for (int i = 0; i < 16; ++i) z[i] = jg + i < Nl ? __uint_as_float(u[i]) : 0.0f;
+        if (c0 + 64 < hN) tm_ld16_nw(tl + (uint32_t)(c0 + 64), u);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) h[i] = c0 + i < Nl ? tanh_fast(z[i] + bv[i]) : 0.0f;
+        for (int i = 0; i < 16; ++i) h[i] = jg + i < Nl ? tanh_fast(z[i] + bv[i]) : 0.0f;
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq)
-          *reinterpret_cast<float4*>(s.abuf + rm_off(r, c0 + 4 * qq, Wn)) =
-              make_float4(to_tf32(h[4 * qq]), to_tf32(h[4 * qq + 1]), to_tf32(h[4 * qq + 2]),
-                          to_tf32(h[4 * qq + 3]));
-        if (c0 < Fn) img_store16(img, c0, h, lane);
+          put_both(rm_off(r, jg + 4 * qq, Wn),
+                   make_float4(to_tf32(h[4 * qq]), to_tf32(h[4 * qq + 1]), to_tf32(h[4 * qq + 2]),
+                               to_tf32(h[4 * qq + 3])));
+        if (jg < Fn) img_store16(img, jg, h, lane);
       }
     } else {
-      // loss head: G = dL/dZ over the logits (and the value row).  The four warps of a
-      // lane quarter share each row, one 16-column block in four each; the row's max,
-      // sum, entropy, chosen log-probability and value meet in a shared scratch (the A
-      // buffer past G's columns, free at this point), combined in a fixed order.
+      // loss head over the whole last layer (both CTAs hold it): rank r takes lane
+      // quarters 2r and 2r + 1; the four warps of a quarter share each row, one 16-column
+      // block in four each, and the row's max, sum, entropy, chosen log-probability and
+      // value meet in a scratch (the A buffer past G's columns), in a fixed order
+      const bool mine = ok && (quarter >> 1) == rank;
       const int NA = a.n_actions;
       const int Wg = P.Gk[l], Fg = P.Fg[l];
       float* red = reinterpret_cast<float*>(s.abuf + P.hs_off);   // [4][128]
       float* lz = red + 4 * kR;                                     // [2][128]
       float mloc = -__uint_as_float(0x7F800000u);
-      for (int c0 = 16 * cq; c0 < NA; c0 += 64) {
+      for (int c0 = 16 * cq; mine && c0 < NA; c0 += 64) {
         float z[16];
         ld16(c0, Nl, z);
 #pragma unroll
@@ -498,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
       const float m = fmaxf(fmaxf(red[r], red[kR + r]), fmaxf(red[2 * kR + r], red[3 * kR + r]));
       __syncthreads();
       float sloc = 0.0f;
-      for (int c0 = 16 * cq; c0 < NA; c0 += 64) {
+      for (int c0 = 16 * cq; mine && c0 < NA; c0 += 64) {
         float z[16];
         ld16(c0, Nl, z);
 #pragma unroll
@@ -511,7 +554,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
       const float lse = m + __logf(Ssum);
       __syncthreads();
       float hloc = 0.0f;
-      for (int c0 = 16 * cq; c0 < Nl; c0 += 64) {
+      for (int c0 = 16 * cq; mine && c0 < Nl; c0 += 64) {
         float z[16];
         ld16(c0, Nl, z);
 #pragma unroll
@@ -528,100 +571,104 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
       }
       red[cq * kR + r] = hloc;
       __syncthreads();
-      const float Hent = ((red[r] + red[kR + r]) + red[2 * kR + r]) + red[3 * kR + r];
-      const float lpa = lz[r];
-      const float zv = Nl > NA ? lz[kR + r] : 0.0f;
-      float coef = 0.0f, dv = 0.0f;
-      if (live) {
-        float pg;
-        double cf = 0.0;
-        if (a.algo == SIMX_ALGO_REINFORCE) {
-          coef = adv;
-          pg = -adv * lpa;
-        } else {
-          const float rho = __expf(lpa - lpo);
-          const float s1 = rho * adv;
-          const float s2 = fminf(fmaxf(rho, 1.0f - a.clip_eps), 1.0f + a.clip_eps) * adv;
-          pg = -fminf(s1, s2);
-          coef = (s1 <= s2 ? adv : 0.0f) * rho;
-          cf = fabsf(rho - 1.0f) > a.clip_eps ? 1.0 : 0.0;
-        }
-        if (a.has_value) dv = zv - ret;
-        if (cq == 0) {   // one thread per row keeps the row's statistics
-          st_cf += cf;
-          st_v += (double)dv * (double)dv;
-          st_pg += pg;
-          st_h += Hent;
-        }
-      }
-      // G_{L-1}: TF32 into the A buffer (width Gk), FP32 into the G image
-      unsigned char* img = A.ws + P.img_g[l] + img_blk(grow, Fg);
-      for (int c0 = 16 * cq; c0 < Wg; c0 += 64) {
-        float z[16], bv[16], g[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) bv[i] = c0 + i < NA ? __ldg(bias + c0 + i) : 0.0f;
-        ld16(c0, Nl, z);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int j = c0 + i;
-          float v = 0.0f;
-          if (live && j < NA) {
-            const float lp = z[i] + bv[i] - lse;
-            const float p = __expf(lp);
-            const float onehot = (j == ac) ? 1.0f : 0.0f;
-            v = (-coef * (onehot - p) + a.c_entropy * p * (lp + Hent)) * inv_n;
-          } else if (live && a.has_value && j == NA) {
-            v = 2.0f * a.c_value * dv * inv_n;
+      if (mine) {
+        const float Hent = ((red[r] + red[kR + r]) + red[2 * kR + r]) + red[3 * kR + r];
+        const float lpa = lz[r];
+        const float zv = Nl > NA ? lz[kR + r] : 0.0f;
+        float coef = 0.0f, dv = 0.0f;
+        if (live) {
+          float pg;
+          double cf = 0.0;
+          if (a.algo == SIMX_ALGO_REINFORCE) {
+            coef = adv;
+            pg = -adv * lpa;
+          } else {
+            const float rho = __expf(lpa - lpo);
+            const float s1 = rho * adv;
+            const float s2 = fminf(fmaxf(rho, 1.0f - a.clip_eps), 1.0f + a.clip_eps) * adv;
+            pg = -fminf(s1, s2);
+            coef = (s1 <= s2 ? adv : 0.0f) * rho;
+            cf = fabsf(rho - 1.0f) > a.clip_eps ? 1.0 : 0.0;
           }
-          g[i] = v;
+          if (a.has_value) dv = zv - ret;
+          if (cq == 0) {   // one thread per row keeps the row's statistics
+            st_cf += cf;
+            st_v += (double)dv * (double)dv;
+            st_pg += pg;
+            st_h += Hent;
+          }
         }
+        // G_{L-1} of this CTA's rows: TF32 into both A buffers (width Gk), FP32 into the
+        // G image
+        unsigned char* img = A.ws + P.img_g[l] + img_blk(grow, Fg);
+        for (int c0 = 16 * cq; c0 < Wg; c0 += 64) {
+          float z[16], bv[16], g[16];
 #pragma unroll
-        for (int qq = 0; qq < 4; ++qq)
-          *reinterpret_cast<float4*>(s.abuf + rm_off(r, c0 + 4 * qq, Wg)) =
-              make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
-                          to_tf32(g[4 * qq + 3]));
-        if (c0 < Fg) img_store16(img, c0, g, lane);
+          for (int i = 0; i < 16; ++i) bv[i] = c0 + i < NA ? __ldg(bias + c0 + i) : 0.0f;
+          ld16(c0, Nl, z);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const int j = c0 + i;
+            float v = 0.0f;
+            if (live && j < NA) {
+              const float lp = z[i] + bv[i] - lse;
+              const float p = __expf(lp);
+              const float onehot = (j == ac) ? 1.0f : 0.0f;
+              v = (-coef * (onehot - p) + a.c_entropy * p * (lp + Hent)) * inv_n;
+            } else if (live && a.has_value && j == NA) {
+              v = 2.0f * a.c_value * dv * inv_n;
+            }
+            g[i] = v;
+          }
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq)
+            put_both(rm_off(r, c0 + 4 * qq, Wg),
+                     make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
+                                 to_tf32(g[4 * qq + 3])));
+          if (c0 < Fg) img_store16(img, c0, g, lane);
+        }
       }
     }
-    ok = stage_sync();
+    cluster_sync();
   }
-  // ---- backward: dH_l = G_l W_l, G_{l-1} = dH_l (1 - H_l^2)
-  for (int l = L - 1; l >= 1 && ok; --l) {
-    const int Kb = P.Kb[l];
-    ok = gemm(2 * L - 1 - l, P.Gk[l], Kb);
-    if (!ok) break;
+  // ---- backward: dH_l = G_l W_l, G_{l-1} = dH_l (1 - H_l^2), this CTA's half of dH_l
+  for (int l = L - 1; l >= 1; --l) {
+    const int hK = P.hK[l];
+    gemm(2 * L - 1 - l, P.Gk[l], hK);
+    const bool ok = *s.abort_flag == 0;
     const int Kl = P.K[l], Fh = P.Fh[l], Fg = P.Fg[l - 1];
     const int Wg = l - 1 >= 1 ? P.Gk[l - 1] : 0;
-    const int width = Wg > Fg ? Wg : Fg;
+    const int j0h = rank * hK;
     const unsigned char* himg = A.ws + P.img_h[l] + img_blk(grow, Fh);
     unsigned char* gimg = A.ws + P.img_g[l - 1] + img_blk(grow, Fg);
     uint32_t u[16];
-    if (16 * cq < width) tm_ld16_nw(tl + (uint32_t)(16 * cq), u);
-    for (int c0 = 16 * cq; c0 < width; c0 += 64) {
+    if (ok && 16 * cq < hK) tm_ld16_nw(tl + (uint32_t)(16 * cq), u);
+    for (int c0 = 16 * cq; ok && c0 < hK; c0 += 64) {
+      const int jg = j0h + c0;
       float z[16], hv[16], g[16];
-      if (c0 < Fh) img_load16(himg, c0, hv, lane);
+      if (jg < Fh) img_load16(himg, jg, hv, lane);
       else
 #pragma unroll
         for (int i = 0; i < 16; ++i) hv[i] = 0.0f;
       tm_wait();
       reg_fence16(u);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) z[i] = c0 + i < Kl ? __uint_as_float(u[i]) : 0.0f;
-      if (c0 + 64 < width) tm_ld16_nw(tl + (uint32_t)(c0 + 64), u);
+      for (int i = 0; i < 16; ++i) z[i] = jg + i < Kl ? __uint_as_float(u[i]) : 0.0f;
+      if (c0 + 64 < hK) tm_ld16_nw(tl + (uint32_t)(c0 + 64), u);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) g[i] = c0 + i < Kl ? z[i] * (1.0f - hv[i] * hv[i]) : 0.0f;
-      if (c0 < Wg)
+      for (int i = 0; i < 16; ++i) g[i] = jg + i < Kl ? z[i] * (1.0f - hv[i] * hv[i]) : 0.0f;
+      if (jg < Wg)
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq)
-          *reinterpret_cast<float4*>(s.abuf + rm_off(r, c0 + 4 * qq, Wg)) =
-              make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
-                          to_tf32(g[4 * qq + 3]));
-      if (c0 < Fg) img_store16(gimg, c0, g, lane);
+          put_both(rm_off(r, jg + 4 * qq, Wg),
+                   make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
+                               to_tf32(g[4 * qq + 3])));
+      if (jg < Fg) img_store16(gimg, jg, g, lane);
     }
-    ok = stage_sync();
+    cluster_sync();
   }
 
-  // ---- end: nothing in flight, statistics of the tile's rows, tensor memory released
+  // ---- end: nothing in flight, statistics of the CTA's rows, tensor memory released
   if (tid == 0) drain_all(s, S, issued, consumed);
   if (cq == 0) {
 #pragma unroll
@@ -803,20 +850,22 @@ Plan plan(const LossArgs& a) {
     p.K[l] = K;
     p.N[l] = N;
     p.Ka[l] = l == 0 ? 3 * r32(K) : r32(K);
-    p.Nf[l] = r16(N);
+    p.Nf[l] = l + 1 < L ? r32(N) : r16(N);
+    p.hN[l] = l + 1 < L ? p.Nf[l] / 2 : p.Nf[l];
     p.Gk[l] = r32(N);
-    p.Kb[l] = r16(K);
+    p.Kb[l] = r32(K);
+    p.hK[l] = p.Kb[l] / 2;
     p.Fh[l] = r16(K);
     p.Fg[l] = r16(N);
     p.poff[l] = P;
     P += N * K + N;
     maxA = maxA > p.Ka[l] ? maxA : p.Ka[l];
     if (l >= 1) maxA = maxA > p.Gk[l] ? maxA : p.Gk[l];
-    maxB = maxB > p.Nf[l] ? maxB : p.Nf[l];
-    if (l >= 1) maxB = maxB > p.Kb[l] ? maxB : p.Kb[l];
+    maxB = maxB > p.hN[l] ? maxB : p.hN[l];
+    if (l >= 1) maxB = maxB > p.hK[l] ? maxB : p.hK[l];
     maxFh = maxFh > p.Fh[l] ? maxFh : p.Fh[l];
-    tneed = tneed > p.Nf[l] ? tneed : p.Nf[l];
-    if (l >= 1) tneed = tneed > p.Kb[l] ? tneed : p.Kb[l];
+    tneed = tneed > p.hN[l] ? tneed : p.hN[l];
+    if (l >= 1) tneed = tneed > p.hK[l] ? tneed : p.hK[l];
   }
   p.n_params = P;
   const int limit = 227 * 1024, misc = 256;
@@ -845,7 +894,7 @@ Plan plan(const LossArgs& a) {
   if (S > p.nchunks) S = p.nchunks;
   p.S = (int)S;
   p.dw_stage_bytes = 16384 + maxFh * 128;
-  p.dw_nstages = kMaxStages;
+  p.dw_nstages = 3;
   p.dw_smem = 2048 + p.dw_nstages * p.dw_stage_bytes + misc;
   if (p.dw_smem > limit) return p;
   p.dw_tcols = pow2_cols(maxFh + 16);
@@ -869,7 +918,7 @@ Plan plan(const LossArgs& a) {
   p.part = off;
   off = al256(off + (size_t)p.S * p.n_params * 4);
   p.spart = off;
-  off = al256(off + (size_t)p.ntiles * 4 * sizeof(double));
+  off = al256(off + (size_t)2 * p.ntiles * 4 * sizeof(double));   // one entry per CTA
   p.total = off;
   p.ok = true;
   return p;
@@ -897,13 +946,27 @@ cudaError_t launch_loss_wide(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
   const int64_t cap = (int64_t)sm_count() * 4;
   if (blocks > cap) blocks = cap;
   lw::k_lw_prep<<<(unsigned)blocks, 256, 0, s>>>(A);
+  // a cluster of two CTAs per 128-row tile
   cudaFuncSetAttribute(lw::k_lw_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, p.smem);
-  lw::k_lw_rows<<<(unsigned)p.ntiles, lw::kThreads, p.smem, s>>>(A);
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3((unsigned)(2 * p.ntiles));
+  lc.blockDim = dim3(lw::kThreads);
+  lc.dynamicSmemBytes = (size_t)p.smem;
+  lc.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 2;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  lc.attrs = at;
+  lc.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&lc, lw::k_lw_rows, A);
+  if (e != cudaSuccess) return e;
   cudaFuncSetAttribute(lw::k_lw_dw, cudaFuncAttributeMaxDynamicSharedMemorySize, p.dw_smem);
   lw::k_lw_dw<<<(unsigned)(p.mt_total * p.S), lw::kDwThreads, p.dw_smem, s>>>(A);
   count_launches(3);
   launch_loss_reduce_n(reinterpret_cast<const float*>(A.ws + p.part), p.S, p.n_params,
-                       reinterpret_cast<const double*>(A.ws + p.spart), (int)p.ntiles, a, s);
+                       reinterpret_cast<const double*>(A.ws + p.spart), (int)(2 * p.ntiles), a, s);
   return cudaGetLastError();
 }
 
