@@ -636,8 +636,8 @@ __global__ void __launch_bounds__(128, MINB) k_step_thread(const __grid_constant
   }
 }
 
-// 4 resident blocks per SM (128 registers): one wave of 77,824 envs; fewer registers
-// spill the server state of the router.  Launched with programmatic stream serialization
+// 4 resident blocks per SM (128 registers): one wave of 77,824 envs; from 262,144 envs 5
+// (96 registers; 6 would spill the server state of the router).  Launched with programmatic stream serialization
 // so that back-to-back steps (a graph of sim_step_batched calls) overlap one step's block
 // launch with the previous step's tail; the kernel's griddepcontrol.wait keeps the order.
 template <bool ROUTE, int K>
@@ -652,9 +652,17 @@ cudaError_t step_thread_t(const RolloutArgs& a, cudaStream_t s) {
   at[0].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = at;
   lc.numAttrs = 1;
-  cudaError_t e = a.cfg.arrival_kind == SIMX_ARR_TRACE
-                      ? cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 4, true>, a)
-                      : cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 4, false>, a);
+  // from 262,144 envs (several waves) five resident blocks per SM (96 registers, no
+  // spills) beat four: 124.8 against 126.8 us per step at 1,048,576 envs; below that the
+  // single wave of four blocks with 128 registers is faster (8.6 against 10.2 us at 65,536)
+  const bool tr = a.cfg.arrival_kind == SIMX_ARR_TRACE;
+  cudaError_t e;
+  if (a.st.E >= 262144u)
+    e = tr ? cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 5, true>, a)
+           : cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 5, false>, a);
+  else
+    e = tr ? cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 4, true>, a)
+           : cudaLaunchKernelEx(&lc, k_step_thread<ROUTE, K, 4, false>, a);
   count_launches(1);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
