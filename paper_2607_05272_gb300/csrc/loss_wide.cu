@@ -72,6 +72,8 @@ struct Plan {
   // k_lw_rows
   int a_bytes, stage_bytes, nstages, smem, tcols;
   int hs_off;                // the loss head's scratch inside the A buffer (3 KB)
+  int b_off[SIMX_MAX_LAYERS];  // the biases, copied to shared memory after the misc area
+  int b_total;
   // k_lw_dw
   int mt0[SIMX_MAX_LAYERS];  // first work item of layer l (blocks of 128 outputs)
   int mt_total, S, dw_stage_bytes, dw_nstages, dw_smem, dw_tcols;
@@ -394,6 +396,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     for (; issued < upto; ++issued) load_chunk(s, sch, S, P.stage_bytes, issued);
   }
   if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.tcols);
+  // every layer's bias into shared memory (zero past each layer's outputs)
+  float* sbias = reinterpret_cast<float*>(sm + P.a_bytes + (size_t)S * P.stage_bytes + 256);
+  for (int l = 0; l < L; ++l)
+    for (int i = tid; i < (P.N[l] + 15) / 16 * 16; i += kThreads)
+      sbias[P.b_off[l] + i] = i < P.N[l] ? __ldg(a.b[l] + i) : 0.0f;
 
   // the tile's observations (both CTAs, every row): x_hi, x_hi, x_lo side by side in the A
   // buffer (split TF32); rank 0 writes the FP32 values to the H_0 image
@@ -491,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     gemm(l, P.Ka[l], hN);
     const bool ok = *s.abort_flag == 0;
     const int Nl = P.N[l];
-    const float* bias = a.b[l];
+    const float* bias = sbias + P.b_off[l];
     if (l + 1 < L) {
       // H_{l+1} = tanh(Z_l + b_l) for this CTA's half of the outputs: TF32 into both A
       // buffers (width Ka[l+1] = Nf[l], zero padded), FP32 into the H_{l+1} image
@@ -503,7 +510,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         const int jg = j0h + c0;
         float z[16], bv[16], h[16];
 #pragma unroll
-        for (int i = 0; i < 16; ++i) bv[i] = jg + i < Nl ? __ldg(bias + jg + i) : 0.0f;
+        for (int i = 0; i < 16; ++i) bv[i] = jg + i < Nl ? bias[jg + i] : 0.0f;
         tm_wait();
         reg_fence16(u);
 #pragma unroll
@@ -534,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         ld16(c0, Nl, z);
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          if (c0 + i < NA) mloc = fmaxf(mloc, z[i] + __ldg(bias + c0 + i));
+          if (c0 + i < NA) mloc = fmaxf(mloc, z[i] + bias[c0 + i]);
       }
       red[cq * kR + r] = mloc;
       __syncthreads();
@@ -546,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         ld16(c0, Nl, z);
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          if (c0 + i < NA) sloc += __expf(z[i] + __ldg(bias + c0 + i) - m);
+          if (c0 + i < NA) sloc += __expf(z[i] + bias[c0 + i] - m);
       }
       red[cq * kR + r] = sloc;
       __syncthreads();
@@ -561,11 +568,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         for (int i = 0; i < 16; ++i) {
           const int j = c0 + i;
           if (j < NA) {
-            const float lp = z[i] + __ldg(bias + j) - lse;
+            const float lp = z[i] + bias[j] - lse;
             hloc -= __expf(lp) * lp;
             if (j == ac) lz[r] = lp;
           } else if (j == NA && j < Nl) {
-            lz[kR + r] = z[i] + __ldg(bias + j);
+            lz[kR + r] = z[i] + bias[j];
           }
         }
       }
@@ -604,7 +611,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         for (int c0 = 16 * cq; c0 < Wg; c0 += 64) {
           float z[16], bv[16], g[16];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) bv[i] = c0 + i < NA ? __ldg(bias + c0 + i) : 0.0f;
+          for (int i = 0; i < 16; ++i) bv[i] = c0 + i < NA ? bias[c0 + i] : 0.0f;
           ld16(c0, Nl, z);
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
@@ -665,7 +672,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
                                to_tf32(g[4 * qq + 3])));
       if (jg < Fg) img_store16(gimg, jg, g, lane);
     }
-    cluster_sync();
+    if (Wg) cluster_sync();   // G_0 is not an operand here: nothing went to the peer
   }
 
   // ---- end: nothing in flight, statistics of the CTA's rows, tensor memory released
@@ -876,7 +883,14 @@ Plan plan(const LossArgs& a) {
   p.stage_bytes = maxB * kKC * 4;
   p.nstages = kMaxStages;
   while (p.nstages > 2 && p.a_bytes + p.nstages * p.stage_bytes + misc > limit) --p.nstages;
-  p.smem = p.a_bytes + p.nstages * p.stage_bytes + misc;
+  // the biases of every layer follow the misc area
+  p.b_total = 0;
+  for (int l = 0; l < L; ++l) {
+    p.b_off[l] = p.b_total;
+    p.b_total += (p.N[l] + 15) / 16 * 16;
+  }
+  while (p.nstages > 2 && p.a_bytes + p.nstages * p.stage_bytes + misc + 4 * p.b_total > limit) --p.nstages;
+  p.smem = p.a_bytes + p.nstages * p.stage_bytes + misc + 4 * p.b_total;
   if (p.smem > limit) return p;
   p.tcols = pow2_cols(tneed);
   if (p.tcols > 512) return p;
