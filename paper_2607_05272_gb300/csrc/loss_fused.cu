@@ -497,35 +497,6 @@ __global__ void k_pack_loss_w(const __grid_constant__ PackArgs P) {
   }
 }
 
-__global__ void k_reduce_blocks(const float* __restrict__ part, int nb, int P, float* __restrict__ out) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= P) return;
-  float s = 0.0f;
-  for (int b = 0; b < nb; ++b) s += part[(size_t)b * P + i];
-  out[i] = s;
-}
-
-// One warp per statistic: lane l sums blocks l, l + 32, ... in order, then a fixed
-// butterfly combines the lanes (the same order on every run).
-__global__ void k_fused_stats(const double* __restrict__ sp, int nb, int64_t n, int has_value,
-                              float cv, float ce, float* __restrict__ stats) {
-  __shared__ double sh[4];
-  const int q = threadIdx.x / 32, lane = threadIdx.x % 32;
-  double acc = 0.0;
-  for (int b = lane; b < nb; b += 32) acc += sp[(size_t)b * 4 + q];
-  for (int d = 16; d > 0; d /= 2) acc += __shfl_xor_sync(0xffffffffu, acc, d);
-  if (lane == 0) sh[q] = acc;
-  __syncthreads();
-  if (threadIdx.x != 0) return;
-  const double s[4] = {sh[0], sh[1], sh[2], sh[3]};
-  const double pg = s[0] / (double)n, v = s[1] / (double)n, H = s[2] / (double)n;
-  stats[0] = (float)(pg + (has_value ? (double)cv * v : 0.0) - (double)ce * H);
-  stats[1] = (float)pg;
-  stats[2] = (float)v;
-  stats[3] = (float)H;
-  stats[4] = (float)(s[3] / (double)n);
-}
-
 namespace {
 struct FusedPlan {
   bool ok;
@@ -677,11 +648,58 @@ void launch_loss_reduce(const float* part, int nb, int n_params, const double* s
   launch_loss_reduce_n(part, nb, n_params, spart, nb, a, s);
 }
 
+// The block reduction and the statistics in one launch.  Blocks 0 .. nr - 1 sum the
+// gradient partials, element i over blocks 0, 1, ... in order.  The last block sums the
+// statistics, one warp per statistic: lane l takes blocks l, l + 32, ... in order, then a
+// fixed butterfly combines the lanes (the same order on every run).  Launched with
+// programmatic stream serialization: it waits for the kernel before it
+// (griddepcontrol.wait) before reading the partials, so its launch overlaps that kernel's
+// tail.
+__global__ void __launch_bounds__(256) k_reduce_all(const float* __restrict__ part, int nb, int P,
+                                                    float* __restrict__ out, const double* __restrict__ sp,
+                                                    int nbs, int64_t n, int has_value, float cv,
+                                                    float ce, float* __restrict__ stats) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  if ((int)blockIdx.x + 1 < (int)gridDim.x) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= P) return;
+    float s = 0.0f;
+    for (int b = 0; b < nb; ++b) s += part[(size_t)b * P + i];
+    out[i] = s;
+    return;
+  }
+  __shared__ double sh[4];
+  if (threadIdx.x >= 128) return;
+  const int q = threadIdx.x / 32, lane = threadIdx.x % 32;
+  double acc = 0.0;
+  for (int b = lane; b < nbs; b += 32) acc += sp[(size_t)b * 4 + q];
+  for (int d = 16; d > 0; d /= 2) acc += __shfl_xor_sync(0xffffffffu, acc, d);
+  if (lane == 0) sh[q] = acc;
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+  if (threadIdx.x != 0) return;
+  const double s4[4] = {sh[0], sh[1], sh[2], sh[3]};
+  const double pg = s4[0] / (double)n, v = s4[1] / (double)n, H = s4[2] / (double)n;
+  stats[0] = (float)(pg + (has_value ? (double)cv * v : 0.0) - (double)ce * H);
+  stats[1] = (float)pg;
+  stats[2] = (float)v;
+  stats[3] = (float)H;
+  stats[4] = (float)(s4[3] / (double)n);
+}
+
 void launch_loss_reduce_n(const float* part, int nb, int n_params, const double* spart, int nbs,
                           const LossArgs& a, cudaStream_t s) {
-  k_reduce_blocks<<<(n_params + 255) / 256, 256, 0, s>>>(part, nb, n_params, a.grad);
-  k_fused_stats<<<1, 128, 0, s>>>(spart, nbs, a.n, a.has_value, a.c_value, a.c_entropy, a.stats);
-  count_launches(2);
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3((unsigned)((n_params + 255) / 256 + 1));
+  lc.blockDim = dim3(256);
+  lc.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = at;
+  lc.numAttrs = 1;
+  cudaLaunchKernelEx(&lc, k_reduce_all, part, nb, n_params, a.grad, spart, nbs, a.n, a.has_value,
+                     a.c_value, a.c_entropy, a.stats);
+  count_launches(1);
 }
 
 }  // namespace simx

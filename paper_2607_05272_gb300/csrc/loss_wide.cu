@@ -158,6 +158,7 @@ __device__ __forceinline__ uint32_t chunk_off(int j, int kk) {
 // k_lw_prep: the weight operand images of every layer (TF32 rounded, zero padded).
 // ---------------------------------------------------------------------------------
 __global__ void k_lw_prep(const __grid_constant__ Args A) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const LossArgs& a = A.a;
   const Plan& P = A.p;
   int64_t total = 0;
@@ -379,6 +380,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   const int64_t grow = tile * kR + r;   // row of the padded minibatch
   const bool live = grow < a.n;
 
+  // The kernel is launched while k_lw_prep still runs (programmatic dependent launch):
+  // everything up to the first read of the weight images (barriers, tensor memory, biases,
+  // the observation gather) overlaps it; griddepcontrol.wait then waits for its images.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   // thread 0: barriers, then the first weight chunks on their way before anything else
   Sched sch;
   int issued = 0, consumed = 0;
@@ -391,6 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     mbar_init(s.accb, 1);
     mbar_fence_init();
     *s.abort_flag = 0;
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     sch = make_sched(P, A.ws, rank);
     const int upto = S - 1 < sch.total ? S - 1 : sch.total;
     for (; issued < upto; ++issued) load_chunk(s, sch, S, P.stage_bytes, issued);
@@ -444,6 +450,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     lpo = a.algo == SIMX_ALGO_PPO ? __ldg(a.logp_old + row) : 0.0f;
     ret = a.has_value ? __ldg(a.ret + row) : 0.0f;
   }
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   fence_async_smem();
   fence_before();
   __syncthreads();
@@ -714,6 +721,7 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
   const int S = P.dw_nstages, SB = P.dw_stage_bytes;
   // the first 2 KB hold the ones operand of db (feature 0 = 1, features 1..15 = 0)
   const Smem s = carve(sm, P, SB, S, 2048);
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, cq = warp >> 2;
   const int item = blockIdx.x % P.mt_total, split = blockIdx.x / P.mt_total;
@@ -739,6 +747,8 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
   for (int i = tid; i < 512; i += kDwThreads)
     reinterpret_cast<float*>(sm)[i] = (i < 256 && ((i >> 2) & 7) == 0) ? 1.0f : 0.0f;
   if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.dw_tcols);
+  // launched while k_lw_rows runs: the images it writes are read only after this wait
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   fence_async_smem();
   fence_before();
   __syncthreads();
@@ -967,17 +977,27 @@ cudaError_t launch_loss_wide(const LossArgs& a, void* ws, size_t ws_bytes, cudaS
   lc.blockDim = dim3(lw::kThreads);
   lc.dynamicSmemBytes = (size_t)p.smem;
   lc.stream = s;
-  cudaLaunchAttribute at[1];
+  // rows and dW are launched as programmatic dependents of the kernel before them: their
+  // prologues overlap its tail and griddepcontrol.wait orders the data
+  cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeClusterDimension;
   at[0].val.clusterDim.x = 2;
   at[0].val.clusterDim.y = 1;
   at[0].val.clusterDim.z = 1;
+  at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[1].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = at;
-  lc.numAttrs = 1;
+  lc.numAttrs = 2;
   cudaError_t e = cudaLaunchKernelEx(&lc, lw::k_lw_rows, A);
   if (e != cudaSuccess) return e;
   cudaFuncSetAttribute(lw::k_lw_dw, cudaFuncAttributeMaxDynamicSharedMemorySize, p.dw_smem);
-  lw::k_lw_dw<<<(unsigned)(p.mt_total * p.S), lw::kDwThreads, p.dw_smem, s>>>(A);
+  lc.gridDim = dim3((unsigned)(p.mt_total * p.S));
+  lc.blockDim = dim3(lw::kDwThreads);
+  lc.dynamicSmemBytes = (size_t)p.dw_smem;
+  lc.attrs = at + 1;
+  lc.numAttrs = 1;
+  e = cudaLaunchKernelEx(&lc, lw::k_lw_dw, A);
+  if (e != cudaSuccess) return e;
   count_launches(3);
   launch_loss_reduce_n(reinterpret_cast<const float*>(A.ws + p.part), p.S, p.n_params,
                        reinterpret_cast<const double*>(A.ws + p.spart), (int)(2 * p.ntiles), a, s);
