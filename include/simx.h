@@ -64,6 +64,7 @@ typedef enum {
 #define SIMX_DEV_EVENT_CAP 2u       /* more than 2^20 arrival candidates in one decision */
 #define SIMX_DEV_BAD_ACTION 4u      /* external action outside [0, n_actions): action 0 used */
 #define SIMX_DEV_TC_TIMEOUT 8u      /* a wait for the tensor-core policy forward timed out */
+#define SIMX_DEV_COPY_TIMEOUT 16u   /* a wait for a staged copy of the policy weights timed out */
 
 /* Simulator mode (Sec. 3.1 "Multi-GPU Support"; Sec. 4.1 action space). */
 typedef enum {
@@ -304,12 +305,14 @@ simx_status rollout_collect(simx_ctx* ctx, const simx_mlp* pol, int policy_mode,
 /*
  * The launch that rollout_collect and sim_step_batched take for this context, policy and
  * mode (host only: no device work; the lane and block choice follows the device's SM
- * count).  host_out[5] receives: [0] kernel, 0 = the fused step with the policy forward
+ * count).  host_out[6] receives: [0] kernel, 0 = the fused step with the policy forward
  * (one group of lanes per env), 1 = the thread-per-env step of the policy-free modes;
  * [1] lanes per env (1 for the thread-per-env step); [2] threads per block; [3] 1 when
  * each warp runs the policy forward for its own envs, 0 for the block-wide forward;
  * [4] 1 when a grid policy's forward runs on the tensor cores (tcgen05, bf16 operands
- * exact on the grid, FP32 accumulation: the FP32 path's bits), 0 otherwise.
+ * exact on the grid, FP32 accumulation: the FP32 path's bits), 0 otherwise; [5] 1 when
+ * the block-wide FP32 forward streams its weights through shared memory (bulk copies
+ * into two stages; the same fma chains and bits), 0 otherwise.
  * It exists so that tests and benchmarks can state which instantiation they exercise.
  * SIMX_EINVAL for a NULL argument, an unknown mode or a policy that rollout_collect
  * would refuse.

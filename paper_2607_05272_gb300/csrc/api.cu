@@ -556,13 +556,21 @@ simx_status simx_launch_shape(simx_ctx* c, const simx_mlp* pol, int policy_mode,
   host_out[2] = thread ? 128 : a.threads;
   host_out[3] = (!thread && net) ? mlp_warp_of(route, a.G, pol) : 0;
   host_out[4] = 0;
-  if (!thread && net) {  // the launch's plan for the grid forward (no repack needed)
+  host_out[5] = 0;
+  if (!thread && net) {  // the launch's forward plans (no repack needed)
     a.mlp_warp = host_out[3];
     a.mlp.n_layers = pol->n_layers;
-    for (int l = 0; l <= pol->n_layers; ++l) a.mlp.dims[l] = pol->dims[l];
+    for (int l = 0; l <= pol->n_layers; ++l) {
+      a.mlp.dims[l] = pol->dims[l];
+      a.mlp.npad[l] = l ? round_up(pol->dims[l], 4) : pol->dims[0];
+    }
     a.mlp.grid = pol->grid;
-    plan_tc_forward(a, a.threads / a.G);
+    act_layout(mlp_maxdim(pol), (int)a.n_actions, a.maxd4, a.apad);
+    a.bs_pad = a.mlp_warp ? act_stride_pad(a.mlp, 32 / a.G, 32)
+                          : act_stride_pad(a.mlp, a.threads / a.G, a.threads);
+    plan_rollout(a);
     host_out[4] = a.tc.on;
+    host_out[5] = a.stage.on;
   }
   return SIMX_OK;
 }

@@ -56,6 +56,7 @@ struct RolloutArgs {
   int bs_pad;       // activation row stride = envs per block + bs_pad (see act_stride_pad)
   int mlp_warp;     // 1: each warp runs the policy for its own envs (see mlp_forward_warp)
   TcPlan tc;        // grid policies: the tensor-core forward (tc.on = 0 otherwise)
+  StagePlan stage;  // the forward with staged weights (stage.on = 0 otherwise)
   // trace replay (arrival_kind TRACE): gaps, types (or null), costs (or null), length
   const uint32_t* tr_gap;
   const uint8_t* tr_type;
@@ -97,6 +98,9 @@ cudaError_t launch_policy_forward(const PolicyArgs& p, cudaStream_t s);
 // Sets a.tc (and the activation rows a.maxd4 it needs) when the grid forward of this
 // launch can run on the tensor cores; returns the dynamic shared memory of the launch.
 size_t plan_tc_forward(RolloutArgs& a, int B);
+// The rollout launch's forward plans (the tensor-core grid forward, else the staged
+// weights), as launch_rollout makes them; returns the dynamic shared memory.
+size_t plan_rollout(RolloutArgs& a);
 int choose_lanes(int64_t envs);
 int choose_threads(int64_t envs, int G);
 

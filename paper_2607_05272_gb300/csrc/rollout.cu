@@ -846,6 +846,16 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
   uint32_t* tc_tbase = reinterpret_cast<uint32_t*>(tsm + A.tc.bar_off + 8);
   if (tc) tcf::setup(A, tsm, tc_tbase);
   const uint32_t tc_tmem = tc ? *tc_tbase : 0u;
+  // fp32 policies with staged weights: the launch's pipeline of weight chunks (not
+  // instantiated for 32 lanes per env, whose blocks hold at most 8 envs)
+  const bool stg = G != 32 && !WARP && !tc && A.stage.on && use_mlp;
+  StagePipe sp;
+  sp.stages = reinterpret_cast<float*>(tsm + A.stage.off);
+  sp.full = reinterpret_cast<uint64_t*>(tsm + A.stage.bar_off);
+  sp.flag = reinterpret_cast<volatile int*>(tsm + A.stage.bar_off + 8u * (uint32_t)A.stage.S);
+  sp.cc = 0u;
+  sp.total = (uint32_t)A.H * (uint32_t)A.stage.n;
+  if (stg && threadIdx.x == 0) stage_start(A.mlp, A.stage, sp);
 
   for (int t = 0; t < A.H; ++t) {
     // phase 1: observation (Sec. 4.1) into column `slot` of X0
@@ -866,6 +876,9 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
       if (tc) {
         Z = tcf::forward(A, tsm, tc_tmem, X0, X1, B, Bs, tc_phase, tc_timeout);
         if (tc_timeout) s.status |= SIMX_DEV_TC_TIMEOUT;
+      } else if (stg) {
+        Z = mlp_forward_staged<GRID>(A.mlp, A.stage, sp, X0, X1, B, Bs);
+        if (*sp.flag) s.status |= SIMX_DEV_COPY_TIMEOUT;
       } else {
         Z = WARP ? mlp_forward_warp<GRID>(A.mlp, X0, X1, 32 / G, Bs, (int)(threadIdx.x / 32) * (32 / G))
                  : mlp_forward_block<GRID>(A.mlp, X0, X1, B, Bs);
@@ -1010,6 +1023,7 @@ k_rollout(const __grid_constant__ RolloutArgs A) {
     __syncwarp();
   }
   if (tc) tcf::teardown(A, tc_tmem);
+  if (stg && threadIdx.x == 0 && *sp.flag) stage_drain(A.stage, sp);
   if (!live) return;
   if (A.next_obs) {
     if (ROUTE) observe_route<G>(c, g, s, L, ocol, Bs);
@@ -1300,11 +1314,100 @@ size_t plan_tc_forward(RolloutArgs& a, int B) {
   return off;
 }
 
+// Weights of at least this many fp32 bytes are staged in shared memory by default
+// (SIMX_STAGE=0 / 1 turns staging off / on for any size); L1 holds smaller ones.
+constexpr size_t kStageMinBytes = 128 * 1024;
+
+// Register tiles of the staged forward, layer by layer: the first of 4x8, 2x8, 4x4, 2x4,
+// 1x8, 1x4 (envs x outputs) whose tiles keep at least 3/4 of the threads busy, else the
+// one that keeps the most busy; false when a layer's tiles outnumber the threads.
+static bool stage_tiles(const DevMlp& m, int B, int threads, StagePlan& P) {
+  static const int shapes[6][2] = {{4, 8}, {2, 8}, {4, 4}, {2, 4}, {1, 8}, {1, 4}};
+  for (int l = 0; l < m.n_layers; ++l) {
+    const int N = m.dims[l + 1], Np = m.npad[l + 1];
+    int best = -1, best_nt = 0;
+    for (int q = 0; q < 6; ++q) {
+      const int te = shapes[q][0], to = shapes[q][1];
+      if (B % te != 0 || Np % to != 0) continue;
+      const int nt = (B / te) * ((N + to - 1) / to);
+      if (nt > threads) continue;
+      if (4 * nt >= 3 * threads) {
+        best = q;
+        break;
+      }
+      if (nt > best_nt) {
+        best_nt = nt;
+        best = q;
+      }
+    }
+    if (best < 0) return false;
+    P.te[l] = shapes[best][0];
+    P.to[l] = shapes[best][1];
+  }
+  return true;
+}
+
+// The staged forward's plan (fp32 block-wide forwards of 8 or 16 lanes per env whose
+// weights are large): two
+// stages of the largest chunk size in 16, 12, 8, 4 KB that keeps the blocks per SM of the
+// unstaged launch of `kfn`.  Sets a.stage (and a.bs_pad = 4, so the activation rows stay
+// 16-byte aligned) and returns the dynamic shared memory; otherwise leaves a.stage off.
+static size_t plan_stage_forward(RolloutArgs& a, int B, const void* kfn) {
+  std::memset(&a.stage, 0, sizeof(a.stage));
+  const DevMlp& m = a.mlp;
+  const size_t plain = env_smem(a, B);
+  const bool net = a.policy_mode == SIMX_POLICY_SAMPLE || a.policy_mode == SIMX_POLICY_ARGMAX;
+  if (!net || a.mlp_warp || a.tc.on || a.G == 32) return plain;
+  int force = -1;
+  if (const char* f = getenv("SIMX_STAGE"))
+    if (f[0]) force = f[0] == '0' ? 0 : 1;
+  if (force == 0) return plain;
+  size_t wbytes = 0;
+  for (int l = 0; l < m.n_layers; ++l) wbytes += (size_t)m.dims[l] * m.npad[l + 1] * sizeof(float);
+  if (force < 0 && wbytes < kStageMinBytes) return plain;
+  RolloutArgs t = a;
+  t.bs_pad = 4;
+  StagePlan& P = t.stage;
+  P.S = 2;
+  if (!stage_tiles(m, B, a.threads, P)) return plain;
+  int r0 = 0;
+  cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r0, kfn, a.threads, plain) != cudaSuccess) {
+    cudaGetLastError();
+    return plain;
+  }
+  const size_t off = (env_smem(t, B) + 127) / 128 * 128;
+  for (const uint32_t cb : {16384u, 12288u, 8192u, 4096u}) {
+    const size_t total = off + (size_t)P.S * cb + 32;
+    int r = 0;
+    if (total > 227 * 1024) continue;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, kfn, a.threads, total) != cudaSuccess) {
+      cudaGetLastError();
+      return plain;
+    }
+    if (r < r0) continue;
+    P.cb = cb;
+    P.off = (uint32_t)off;
+    P.bar_off = (uint32_t)(off + (size_t)P.S * cb);
+    P.n = 0;
+    for (int l = 0; l < m.n_layers; ++l) {
+      const int K = m.dims[l];
+      int rpc = (int)(cb / (uint32_t)(m.npad[l + 1] * 4));
+      rpc = rpc < K ? rpc : K;
+      P.rpc[l] = rpc;
+      P.cnt[l] = (K + rpc - 1) / rpc;
+      P.n += P.cnt[l];
+    }
+    P.on = 1;
+    a = t;
+    return total;
+  }
+  return plain;
+}
+
+// The k_rollout instantiation a launch takes.
 template <bool ROUTE, int G>
-static cudaError_t rollout_t(const RolloutArgs& a0, cudaStream_t s) {
-  const int B = a0.threads / G;
-  RolloutArgs a = a0;
-  const size_t sh = plan_tc_forward(a, B);
+static auto pick_rollout(const RolloutArgs& a) {
   const bool tr = a.cfg.arrival_kind == SIMX_ARR_TRACE;
   // GRID: the grid policy's instantiations (a.mlp.grid is 0 without a policy)
   const bool gr = a.mlp.grid != 0;
@@ -1314,8 +1417,39 @@ static cudaError_t rollout_t(const RolloutArgs& a0, cudaStream_t s) {
     if (a.mlp_warp)
       k = tr ? (gr ? k_rollout<ROUTE, G, true, true, true> : k_rollout<ROUTE, G, true, true, false>)
              : (gr ? k_rollout<ROUTE, G, false, true, true> : k_rollout<ROUTE, G, false, true, false>);
+  return k;
+}
+
+// The launch's forward plans (tensor-core grid forward, else staged weights); returns the
+// dynamic shared memory.
+template <bool ROUTE, int G>
+static size_t plan_rollout_t(RolloutArgs& a) {
+  const int B = a.threads / G;
+  const size_t sh = plan_tc_forward(a, B);
+  if (a.tc.on) {
+    std::memset(&a.stage, 0, sizeof(a.stage));
+    return sh;
+  }
+  return plan_stage_forward(a, B, (const void*)pick_rollout<ROUTE, G>(a));
+}
+
+size_t plan_rollout(RolloutArgs& a) {
+  const bool route = a.cfg.mode == SIMX_MODE_ROUTE;
+  switch (a.G) {
+    case 8: return route ? plan_rollout_t<true, 8>(a) : plan_rollout_t<false, 8>(a);
+    case 16: return route ? plan_rollout_t<true, 16>(a) : plan_rollout_t<false, 16>(a);
+    case 32: return route ? plan_rollout_t<true, 32>(a) : plan_rollout_t<false, 32>(a);
+    default: return 0;
+  }
+}
+
+template <bool ROUTE, int G>
+static cudaError_t rollout_t(const RolloutArgs& a0, cudaStream_t s) {
+  RolloutArgs a = a0;
+  const size_t sh = plan_rollout_t<ROUTE, G>(a);
+  auto k = pick_rollout<ROUTE, G>(a);
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sh);
-  k<<<grid_for(a.st.E, B), a.threads, sh, s>>>(a);
+  k<<<grid_for(a.st.E, a.threads / G), a.threads, sh, s>>>(a);
   count_launches(1);
   return cudaGetLastError();
 }

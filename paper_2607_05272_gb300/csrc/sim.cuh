@@ -13,6 +13,7 @@
 
 #include "../../include/simx.h"
 #include "devmath.cuh"
+#include "tc_common.cuh"
 
 namespace simx {
 
@@ -45,6 +46,25 @@ struct DevMlp {
   int act[SIMX_MAX_LAYERS];  // simx_act after layer l, -1 for the output layer
   int grid;                  // grid policy: layer l's input on the grid 2^-gx[l]
   int gx[SIMX_MAX_LAYERS];
+};
+
+// The FP32 block-wide forward with its weights staged in shared memory (fp32 policies
+// whose weights L1 does not hold): one thread streams each layer's rows, in chunks of
+// rpc[l] rows, into S stages of cb bytes with bulk copies; every thread reads its
+// register tile's weights (te[l] envs x to[l] outputs) from the stage.  The chunk
+// sequence of one forward (layer 0's, then layer 1's, ...) repeats every step, so the
+// next step's first chunks load during the simulator's phases.  Byte offsets are inside
+// the kernel's dynamic shared memory.
+struct StagePlan {
+  int on;                      // 1: this launch stages the weights
+  int S;                       // stages
+  int n;                       // chunks per forward
+  uint32_t cb;                 // bytes per stage
+  uint32_t off;                // first stage
+  uint32_t bar_off;            // S mbarriers (8 B each), then the timeout flag (4 B)
+  int rpc[SIMX_MAX_LAYERS];    // weight rows per chunk
+  int cnt[SIMX_MAX_LAYERS];    // chunks of each layer
+  int te[SIMX_MAX_LAYERS], to[SIMX_MAX_LAYERS];   // register tile: envs x outputs
 };
 
 template <int G>
@@ -96,6 +116,25 @@ struct Grp {
   __device__ __forceinline__ void sync() const { __syncwarp(mask); }
 };
 
+// Two fp32 fused multiply-adds in one instruction (fma.rn.f32x2, sm_100 and later): each
+// half of the 64-bit operands is one fp32 value (the low half first) and each half of the
+// result is the IEEE fma of its own halves, rounded to nearest: the bits of two
+// __fmaf_rn.  The tiles below pair adjacent outputs of one env, whose weights arrive as
+// adjacent floats of a 16-byte load.
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
 // ---------------------------------------------------------------------------
 // Policy network (Sec. 4.2) evaluated for all envs of a block at once.
 //
@@ -103,9 +142,9 @@ struct Grp {
 // envs (row stride ld = B + 4 spreads an env's features over the banks), so one
 // layer is the small GEMM Y = X^T W^T.  Each thread owns tiles of TE
 // envs x 4 outputs; per k it loads one float4 of weights (row k of the transposed,
-// padded Wt) and TE activations and issues 4 TE fused multiply-adds.  Every output
-// is still the fp32 chain acc = fma(W[j][k], x[k], acc) over k = 0..K-1 in order
-// from acc = 0, then + bias: the same bits as evaluating one env at a time.
+// padded Wt) and TE activations and issues 2 TE paired fused multiply-adds (f2_fma).
+// Every output is still the fp32 chain acc = fma(W[j][k], x[k], acc) over k = 0..K-1 in
+// order from acc = 0, then + bias: the same bits as evaluating one env at a time.
 // ---------------------------------------------------------------------------
 // GELU over rows j0 .. min(j0 + 4, N) - 1, columns 0 .. te - 1 of Y.  Out of line: inlined,
 // its code inside the rollout kernel's loop slowed the tanh policies that never run it.
@@ -154,16 +193,14 @@ __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
   const int ntiles = neb * nob;
   for (int tile = tid; tile < ntiles; tile += nthr) {
     const int eb = tile % neb, ob = tile / neb;
-    float acc[TE][4];
+    uint64_t acc2[TE][2];   // outputs (0, 1) and (2, 3) of each env
 #pragma unroll
-    for (int e = 0; e < TE; ++e)
-#pragma unroll
-      for (int o = 0; o < 4; ++o) acc[e][o] = 0.0f;
+    for (int e = 0; e < TE; ++e) acc2[e][0] = acc2[e][1] = 0ull;
     const float* wc = Wt + 4 * ob;
     const float* xc = X + TE * eb;
 #pragma unroll 4
     for (int k = 0; k < K; ++k) {
-      const float4 w = __ldg(reinterpret_cast<const float4*>(wc + (size_t)k * Npad));
+      const ulonglong2 w = __ldg(reinterpret_cast<const ulonglong2*>(wc + (size_t)k * Npad));
       float xv[TE];
       if (TE == 4) {
         const float4 x4 = *reinterpret_cast<const float4*>(xc + k * ld);
@@ -176,11 +213,16 @@ __device__ __forceinline__ void mlp_tiles(const float* __restrict__ Wt,
       }
 #pragma unroll
       for (int e = 0; e < TE; ++e) {
-        acc[e][0] = __fmaf_rn(w.x, xv[e], acc[e][0]);
-        acc[e][1] = __fmaf_rn(w.y, xv[e], acc[e][1]);
-        acc[e][2] = __fmaf_rn(w.z, xv[e], acc[e][2]);
-        acc[e][3] = __fmaf_rn(w.w, xv[e], acc[e][3]);
+        const uint64_t xx = f2_pack(xv[e], xv[e]);
+        acc2[e][0] = f2_fma(w.x, xx, acc2[e][0]);
+        acc2[e][1] = f2_fma(w.y, xx, acc2[e][1]);
       }
+    }
+    float acc[TE][4];
+#pragma unroll
+    for (int e = 0; e < TE; ++e) {
+      f2_unpack(acc2[e][0], acc[e][0], acc[e][1]);
+      f2_unpack(acc2[e][1], acc[e][2], acc[e][3]);
     }
 #pragma unroll
     for (int o = 0; o < 4; ++o) {
@@ -263,6 +305,183 @@ __device__ __forceinline__ float* mlp_forward_warp(const DevMlp& m, float* X0, f
     else
       mlp_tiles<1, GRID>(m.Wt[l], m.bias[l], K, N, Np, in + col0, out + col0, Bw, ld, th, gq, lane, 32);
     __syncwarp();
+    float* t = in;
+    in = out;
+    out = t;
+  }
+  return in;
+}
+
+// ---------------------------------------------------------------------------
+// The block-wide forward with the weights staged in shared memory (StagePlan).  Thread 0
+// keeps S chunks of weight rows in flight (bulk copies completing on one mbarrier per
+// stage); every thread owns one register tile of TE envs x TO outputs of the layer and,
+// per chunk, waits for its stage, runs its rows k in order (paired fmas, f2_fma) and
+// meets the block at a barrier, after which thread 0 refills the stage with the chunk S
+// ahead.  Every output is the same K-ordered fma chain from 0 as in mlp_tiles, then +
+// bias, the activation and the grid rounding: the same bits.  A wait that times out sets the block's flag; from
+// then on nothing is issued or waited for and the step's outputs are garbage, which the
+// caller reports as SIMX_DEV_COPY_TIMEOUT.
+// ---------------------------------------------------------------------------
+struct StagePipe {
+  float* stages;
+  uint64_t* full;
+  volatile int* flag;
+  uint32_t cc;      // chunks consumed so far in the launch
+  uint32_t total;   // chunks the launch consumes (steps x chunks per forward)
+};
+
+// Thread 0: chunk g of the launch's sequence into stage g mod S (nothing past the last).
+__device__ __forceinline__ void stage_issue(const DevMlp& m, const StagePlan& P,
+                                            const StagePipe& p, uint32_t g) {
+  if (g >= p.total || *p.flag) return;
+  uint32_t c = g % (uint32_t)P.n;
+  int l = 0;
+  while (c >= (uint32_t)P.cnt[l]) {
+    c -= (uint32_t)P.cnt[l];
+    ++l;
+  }
+  const int Np = m.npad[l + 1];
+  const int row0 = (int)c * P.rpc[l];
+  const int rows = m.dims[l] - row0 < P.rpc[l] ? m.dims[l] - row0 : P.rpc[l];
+  const uint32_t bytes = (uint32_t)(rows * Np) * 4u;
+  const uint32_t st = g % (uint32_t)P.S;
+  tcx::mbar_arrive_expect_tx(&p.full[st], bytes);
+  tcx::bulk_g2s(p.stages + (size_t)st * (P.cb / 4u), m.Wt[l] + (size_t)row0 * Np, bytes,
+                &p.full[st]);
+}
+
+// Thread 0 at launch start: the barriers, then the first S chunks.
+__device__ __forceinline__ void stage_start(const DevMlp& m, const StagePlan& P, const StagePipe& p) {
+  for (int i = 0; i < P.S; ++i) tcx::mbar_init(&p.full[i], 1);
+  *p.flag = 0;
+  tcx::mbar_fence_init();
+  for (int i = 0; i < P.S; ++i) stage_issue(m, P, p, (uint32_t)i);
+}
+
+// Thread 0 at launch end, after a timeout only: a bounded wait for every stage's copy
+// still in flight, so that none lands after the block has exited.
+__device__ __forceinline__ void stage_drain(const StagePlan& P, const StagePipe& p) {
+  for (uint32_t g = p.cc; g < p.cc + (uint32_t)P.S && g < p.total; ++g)
+    tcx::mbar_wait(&p.full[g % (uint32_t)P.S], (g / (uint32_t)P.S) & 1u, 200000000ll);
+}
+
+// One layer of the staged forward; returns the chunks consumed so far.
+template <int TE, int TO, bool GRID>
+__device__ __forceinline__ uint32_t layer_staged(const DevMlp& m, const StagePlan& P,
+                                                     StagePipe p, int l, const float* X, float* Y,
+                                                     int B, int ld, int gq) {
+  const int K = m.dims[l], N = m.dims[l + 1], Np = m.npad[l + 1];
+  const int neb = B / TE, nob = (N + TO - 1) / TO;
+  const int tid = (int)threadIdx.x;
+  const bool active = tid < neb * nob;
+  const int eb = tid % neb, ob = tid / neb;
+  uint64_t acc2[TE][TO / 2];   // adjacent output pairs of each env
+#pragma unroll
+  for (int e = 0; e < TE; ++e)
+#pragma unroll
+    for (int o = 0; o < TO / 2; ++o) acc2[e][o] = 0ull;
+  const int rpc = P.rpc[l];
+  for (int j = 0; j < P.cnt[l]; ++j) {
+    const uint32_t st = p.cc % (uint32_t)P.S;
+    if (!*p.flag && !tcx::mbar_wait(&p.full[st], (p.cc / (uint32_t)P.S) & 1u, 2000000000ll))
+      *p.flag = 1;
+    const float* w = p.stages + (size_t)st * (P.cb / 4u) + TO * ob;
+    const float* xc = X + (size_t)(j * rpc) * ld + TE * eb;
+    const int rows = K - j * rpc < rpc ? K - j * rpc : rpc;
+    if (active) {
+#pragma unroll 4
+      for (int k = 0; k < rows; ++k) {
+        uint64_t wv[TO / 2];
+#pragma unroll
+        for (int q = 0; q < TO / 4; ++q) {
+          const ulonglong2 w4 = *reinterpret_cast<const ulonglong2*>(w + k * Np + 4 * q);
+          wv[2 * q] = w4.x;
+          wv[2 * q + 1] = w4.y;
+        }
+        float xv[TE];
+        if (TE == 4) {
+          const float4 x4 = *reinterpret_cast<const float4*>(xc + k * ld);
+          xv[0] = x4.x;
+          xv[1 % TE] = x4.y;
+          xv[2 % TE] = x4.z;
+          xv[3 % TE] = x4.w;
+        } else if (TE == 2) {
+          const float2 x2 = *reinterpret_cast<const float2*>(xc + k * ld);
+          xv[0] = x2.x;
+          xv[1 % TE] = x2.y;
+        } else {
+          xv[0] = xc[k * ld];
+        }
+#pragma unroll
+        for (int e = 0; e < TE; ++e) {
+          const uint64_t xx = f2_pack(xv[e], xv[e]);
+#pragma unroll
+          for (int o = 0; o < TO / 2; ++o) acc2[e][o] = f2_fma(wv[o], xx, acc2[e][o]);
+        }
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      tcx::fence_async_smem();
+      stage_issue(m, P, p, p.cc + (uint32_t)P.S);
+    }
+    ++p.cc;
+  }
+  if (active) {
+    float acc[TE][TO];
+#pragma unroll
+    for (int e = 0; e < TE; ++e)
+#pragma unroll
+      for (int o = 0; o < TO / 2; ++o) f2_unpack(acc2[e][o], acc[e][2 * o], acc[e][2 * o + 1]);
+    const int act = m.act[l];
+#pragma unroll
+    for (int o = 0; o < TO; ++o) {
+      const int jj = TO * ob + o;
+      if (jj < N) {
+        const float bj = __ldg(m.bias[l] + jj);
+#pragma unroll
+        for (int e = 0; e < TE; ++e) {
+          float v = __fadd_rn(acc[e][o], bj);
+          if (act == 0) v = det_tanh(v);
+          Y[jj * ld + TE * eb + e] = v;
+        }
+      }
+    }
+    if (act == 2)
+      for (int o4 = 0; o4 < TO; o4 += 4) gelu_tile(Y + TE * eb, ld, TO * ob + o4, N, TE);
+    if (GRID && gq >= 0)
+      for (int o4 = 0; o4 < TO; o4 += 4) grid_tile(Y + TE * eb, ld, TO * ob + o4, N, TE, gq);
+  }
+  return p.cc;
+}
+
+// Forward through every layer with staged weights (the same buffers and result as
+// mlp_forward_block).  Contains the block barriers.  Out of line: one copy of its six
+// tile shapes serves every rollout instantiation, and the caller's simulator state is
+// saved once per step rather than held live across the tiles.
+template <bool GRID>
+static __device__ __noinline__ float* mlp_forward_staged(const DevMlp& m, const StagePlan& P,
+                                                         StagePipe& p, float* X0, float* X1,
+                                                         int B, int ld) {
+  float* in = X0;
+  float* out = X1;
+  __syncthreads();
+  if (GRID) {
+    grid_rows(X0, m.dims[0], B, ld, m.gx[0], threadIdx.x, blockDim.x);
+    __syncthreads();
+  }
+  for (int l = 0; l < m.n_layers; ++l) {
+    const int gq = (GRID && l + 1 < m.n_layers) ? m.gx[l + 1] : -1;
+    switch (P.te[l] * 16 + P.to[l]) {
+      case 4 * 16 + 8: p.cc = layer_staged<4, 8, GRID>(m, P, p, l, in, out, B, ld, gq); break;
+      case 2 * 16 + 8: p.cc = layer_staged<2, 8, GRID>(m, P, p, l, in, out, B, ld, gq); break;
+      case 4 * 16 + 4: p.cc = layer_staged<4, 4, GRID>(m, P, p, l, in, out, B, ld, gq); break;
+      case 2 * 16 + 4: p.cc = layer_staged<2, 4, GRID>(m, P, p, l, in, out, B, ld, gq); break;
+      case 1 * 16 + 8: p.cc = layer_staged<1, 8, GRID>(m, P, p, l, in, out, B, ld, gq); break;
+      default: p.cc = layer_staged<1, 4, GRID>(m, P, p, l, in, out, B, ld, gq); break;
+    }
+    __syncthreads();
     float* t = in;
     in = out;
     out = t;

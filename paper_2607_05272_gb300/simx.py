@@ -298,13 +298,14 @@ class Sim:
 
     def launch_shape(self, policy_mode: str, policy: Policy = None) -> dict:
         """The launch rollout_collect takes (simx_launch_shape): kernel ("fused" or
-        "thread"), lanes per env, threads per block, warp-local policy forward, and
-        whether a grid policy's forward runs on the tensor cores."""
-        out = (C.c_int32 * 5)()
+        "thread"), lanes per env, threads per block, warp-local policy forward, whether
+        a grid policy's forward runs on the tensor cores, and whether the FP32 forward
+        stages its weights in shared memory."""
+        out = (C.c_int32 * 6)()
         _check(lib().simx_launch_shape(self._h, C.byref(policy.c) if policy else None,
                                        POLICY[policy_mode], out))
         return dict(kernel="thread" if out[0] else "fused", lanes=out[1], threads=out[2],
-                    mlp_warp=bool(out[3]), tensor_cores=bool(out[4]))
+                    mlp_warp=bool(out[3]), tensor_cores=bool(out[4]), staged=bool(out[5]))
 
     def stats(self) -> dict:
         c = Counters()
