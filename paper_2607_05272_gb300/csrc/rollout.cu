@@ -1316,7 +1316,7 @@ size_t plan_tc_forward(RolloutArgs& a, int B) {
 
 // Weights of at least this many fp32 bytes are staged in shared memory by default
 // (SIMX_STAGE=0 / 1 turns staging off / on for any size); L1 holds smaller ones.
-constexpr size_t kStageMinBytes = 128 * 1024;
+constexpr size_t kStageMinBytes = 64 * 1024;
 
 // Register tiles of the staged forward, layer by layer: the first of 4x8, 2x8, 4x4, 2x4,
 // 1x8, 1x4 (envs x outputs) whose tiles keep at least 3/4 of the threads busy, else the

@@ -10,8 +10,7 @@ Each case asserts the launch shape it means to cover:
 
 * c4 at 65,536 envs (4x8 tiles for the 256-wide layers, 2x4 for the 49 outputs; 256-thread
   blocks), 64 steps;
-* c3 at 16,384 envs with staging forced (its 82 KB of weights stay in L1 by default):
-  2x8 tiles, 1x4 for the 17 outputs, 128-thread blocks;
+* c3 at 16,384 envs (2x8 tiles, 1x4 for the 17 outputs; 128-thread blocks);
 * the paper's network (c1p: identity and GELU layers, five layers down to 4 wide) with
   staging forced on small weights, in 256-thread blocks;
 * a c3 grid policy with staging forced and the tensor-core forward off: the grid
@@ -81,7 +80,7 @@ def _rollout(simx, cfg, host, mode, H, seed, stage, monkeypatch):
 # name, envs, steps, mode, grid policy, SIMX_THREADS, SIMX_LANES, SIMX_STAGE, threads
 CASES = [
     ("c4", 65536, 64, "sample", False, None, None, "", 256),
-    ("c3", 16384, 96, "sample", False, None, None, "1", 128),
+    ("c3", 16384, 96, "sample", False, None, None, "", 128),
     ("c1p", 4096, 300, "sample", False, "256", None, "1", 256),
     ("c3", 16384, 64, "argmax", True, None, None, "1", 128),
     ("c4", 1003, 200, "sample", False, "128", "8", "", 128),
