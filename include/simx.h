@@ -185,7 +185,13 @@ typedef enum { SIMX_ACT_TANH = 0, SIMX_ACT_IDENTITY = 1, SIMX_ACT_GELU = 2 } sim
  * 2^16, and every fan-in is <= 256, each pre-activation is an exact fp32 value (the exact
  * dot product plus bias), identical under any summation order; the library does not read
  * the weights back to check this.  Grid policies run in rollout_collect, sim_step_batched
- * and policy_forward; the loss-gradient entry points reject them (SIMX_EINVAL).
+ * and policy_forward.  The loss-gradient entry points take them on their FP32 fused path
+ * whatever the precision asked for: the forward rounds the observation and the hidden
+ * outputs as above, the gradient passes every rounding unchanged (straight through:
+ * dQ(a)/da = 1, the activation's derivative taken at the pre-activation), and the weight
+ * gradients use the rounded layer inputs.  A grid policy too large for that path (its
+ * per-tile activations and parameters must fit one SM's shared memory: c2 and c3 / c5
+ * sizes do, c4's does not) is rejected with SIMX_EINVAL.
  */
 typedef struct simx_mlp {
   int32_t n_layers;                     /* 1 .. SIMX_MAX_LAYERS */

@@ -707,7 +707,6 @@ static simx_status loss_args(const simx_mlp* pol, const simx_rollout* buf, int64
   if (p->precision != SIMX_PREC_FP32 && p->precision != SIMX_PREC_TF32)
     return fail(SIMX_EINVAL, "precision %d", p->precision);
   if (!d_adv || !d_grad || !d_stats) return fail(SIMX_EINVAL, "adv, grad and stats are required");
-  if (pol->grid) return fail(SIMX_EINVAL, "grid policies have no loss-gradient path");
   if (pol->has_value && !d_ret) return fail(SIMX_EINVAL, "a value row needs return targets");
   if (E < 1 || buf->ld != E) return fail(SIMX_EINVAL, "n_rows_per_step %lld must equal the rollout ld %lld", (long long)E, (long long)buf->ld);
   std::memset(&a, 0, sizeof(a));
@@ -735,6 +734,10 @@ static simx_status loss_args(const simx_mlp* pol, const simx_rollout* buf, int64
   a.precision = p->precision;
   a.grad = d_grad;
   a.stats = d_stats;
+  a.grid = pol->grid ? 1 : 0;
+  for (int l = 0; l < pol->n_layers; ++l) a.gx[l] = pol->grid ? pol->gx[l] : 0;
+  if (a.grid && !loss_fused_fits(a))
+    return fail(SIMX_EINVAL, "grid policy too large for the fused FP32 loss (its only path)");
   return SIMX_OK;
 }
 
@@ -745,6 +748,7 @@ size_t ppo_loss_grad_workspace_size(const simx_mlp* pol, int64_t n) {
   a.n_layers = pol->n_layers;
   for (int l = 0; l <= pol->n_layers; ++l) a.dims[l] = pol->dims[l];
   for (int l = 0; l < pol->n_layers; ++l) a.act[l] = (l + 1 < pol->n_layers) ? pol->act[l] : -1;
+  a.grid = pol->grid ? 1 : 0;
   a.n = n;
   return loss_workspace_bytes(a);
 }

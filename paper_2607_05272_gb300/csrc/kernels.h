@@ -132,6 +132,8 @@ struct LossArgs {
   float* stats;          // [5]
   int precision;         // SIMX_PREC_FP32 (SIMT) or SIMX_PREC_TF32 (tensor cores where it fits)
   int act[SIMX_MAX_LAYERS];  // simx_act after layer l, -1 for the output layer
+  int grid;                  // grid policy (the exact forward; straight-through gradient)
+  int gx[SIMX_MAX_LAYERS];   // grid policy: input grid exponent of layer l
 };
 size_t loss_workspace_bytes(const LossArgs& a);
 // loss_fused.cu

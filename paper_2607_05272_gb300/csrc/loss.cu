@@ -377,11 +377,15 @@ size_t loss_workspace_bytes(const LossArgs& a) {
   return f > t ? f : t;
 }
 
-// TF32 requests whose policy fits the one-SM tensor-core kernel take it (loss_tc.cu), and
+// Grid policies take the fused FP32 kernel (their forward's rounding and straight-through
+// gradient live there).  TF32 requests whose policy fits the one-SM tensor-core kernel take
+// it (loss_tc.cu), and
 // wider tanh policies (layers up to 256) the streamed tensor-core kernels (loss_wide.cu);
 // otherwise policies whose parameters and per-tile activations fit in shared memory take
 // the fused FP32 one-kernel path (loss_fused.cu), and wider ones the GEMM pipeline below.
 cudaError_t launch_loss_grad(const LossArgs& a, void* ws, size_t ws_bytes, cudaStream_t s) {
+  if (a.grid)   // grid policies: the fused FP32 kernel, whatever the precision asked for
+    return loss_fused_fits(a) ? launch_loss_fused(a, ws, ws_bytes, s) : cudaErrorInvalidValue;
   if (a.precision == SIMX_PREC_TF32 && loss_tc_fits(a)) return launch_loss_tc(a, ws, ws_bytes, s);
   if (a.precision == SIMX_PREC_TF32 && loss_wide_fits(a)) return launch_loss_wide(a, ws, ws_bytes, s);
   if (loss_fused_fits(a)) return launch_loss_fused(a, ws, ws_bytes, s);

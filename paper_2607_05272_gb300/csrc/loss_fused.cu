@@ -15,6 +15,13 @@
 // fp64 loss statistics; a second kernel sums the blocks in block order, so the result
 // is deterministic for a given launch configuration.  Nothing touches HBM but the
 // gathered observations and the per-block partials.
+//
+// Grid policies (the exact policy forward) run here only: the gathered observations and
+// every hidden output are rounded to their grids exactly as the rollout rounds them, so
+// the forward reproduces the rollout's logits; the backward passes the gradient through
+// each rounding unchanged (the straight-through estimator): the activation's derivative
+// at the pre-activation is stored beside the rounded output, and dW uses the rounded
+// layer inputs.
 #include <cstdint>
 
 #include "devmath.cuh"
@@ -31,14 +38,29 @@ constexpr int kLThreads = 256;         // threads per block
 // thread owns TE rows x 4 outputs: 4-row tiles when they give every thread a tile,
 // else 1-row tiles (thin layers such as the logits).
 // epi 0: + bias, then the activation `act` (-1 none, 0 tanh, 1 identity, 2 GELU; for
-// GELU its derivative is written to D as well); epi 1: times the derivative of the
-// activation `act` of H's layer: 1 - H^2 (tanh, H = the activations), 1 (identity), or
-// H itself (GELU: H = the stored derivative).
+// GELU its derivative is written to D as well); with gq >= 0 (a grid policy's hidden
+// layer) the activation a is written to Y rounded to its grid, Q(a, gq), and its
+// derivative at the pre-activation (1 - a^2, 1 or GELU's) to D: the gradient passes the
+// rounding unchanged (straight through).  epi 1: times the derivative of the activation
+// `act` of H's layer: 1 - H^2 (tanh, H = the activations), 1 (identity), or H itself
+// (GELU and grid layers: H = the stored derivative).
+__device__ __forceinline__ void grid_act(float& y, float& d, int act, int gq) {
+  float a = y, g = 1.0f;
+  if (act == 0) {
+    a = det_tanh(y);
+    g = 1.0f - a * a;
+  } else if (act == 2) {
+    det_gelu_grad(y, a, g);
+  }
+  d = g;
+  y = grid_q(a, gq);
+}
+
 template <int R, int TE>
 __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ldw, int K, int N,
                                             const float* X, float* Y, int epi,
                                             const float* __restrict__ bias, int act,
-                                            const float* H, float* D) {
+                                            const float* H, float* D, int gq) {
   constexpr int kLld = R + 4;
   const int neb = R / TE, nob = (N + 3) / 4;
   for (int tile = threadIdx.x; tile < neb * nob; tile += blockDim.x) {
@@ -100,7 +122,13 @@ __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ld
         }
         *reinterpret_cast<float4*>(Y + j * kLld + 4 * eb) = v;
       }
-      if (epi == 0 && act == 0) {  // one det_tanh per output, four rows at a time
+      if (epi == 0 && gq >= 0) {  // grid policy: activation, derivative, rounding
+#pragma unroll 1
+        for (int q = 0; q < 16; ++q) {
+          const int j = 4 * ob + q / 4;
+          if (j < N) grid_act(Y[j * kLld + 4 * eb + q % 4], D[j * kLld + 4 * eb + q % 4], act, gq);
+        }
+      } else if (epi == 0 && act == 0) {  // one det_tanh per output, four rows at a time
 #pragma unroll 1
         for (int o = 0; o < 4; ++o) {
           const int j = 4 * ob + o;
@@ -140,7 +168,13 @@ __device__ __forceinline__ void tile_gemm_t(const float* __restrict__ Wt, int ld
         }
         Y[j * kLld + eb] = v;
       }
-      if (epi == 0 && (act == 0 || act == 2)) {
+      if (epi == 0 && gq >= 0) {
+#pragma unroll 1
+        for (int o = 0; o < 4; ++o) {
+          const int j = 4 * ob + o;
+          if (j < N) grid_act(Y[j * kLld + eb], D[j * kLld + eb], act, gq);
+        }
+      } else if (epi == 0 && (act == 0 || act == 2)) {
 #pragma unroll 1
         for (int o = 0; o < 4; ++o) {
           const int j = 4 * ob + o;
@@ -158,11 +192,11 @@ template <int R>
 __device__ __forceinline__ void tile_gemm(const float* __restrict__ Wt, int ldw, int K, int N,
                                           const float* X, float* Y, int epi,
                                           const float* __restrict__ bias, int act,
-                                          const float* H, float* D) {
+                                          const float* H, float* D, int gq = -1) {
   if ((R / 4) * ((N + 3) / 4) >= kLThreads)
-    tile_gemm_t<R, 4>(Wt, ldw, K, N, X, Y, epi, bias, act, H, D);
+    tile_gemm_t<R, 4>(Wt, ldw, K, N, X, Y, epi, bias, act, H, D, gq);
   else
-    tile_gemm_t<R, 1>(Wt, ldw, K, N, X, Y, epi, bias, act, H, D);
+    tile_gemm_t<R, 1>(Wt, ldw, K, N, X, Y, epi, bias, act, H, D, gq);
 }
 
 // Row splits for a reduction over the R rows of a tile shared by `items`
@@ -254,7 +288,8 @@ struct FusedLossArgs {
   int npad[SIMX_MAX_LAYERS + 1];     // Npad per layer output (index l + 1)
   int kpad[SIMX_MAX_LAYERS + 1];     // Kpad per layer input (index l)
   int act_off[SIMX_MAX_LAYERS + 2];  // row offset of each layer's activation buffer
-  int dact_off[SIMX_MAX_LAYERS + 1]; // row offset of the GELU derivative of layer l's input (-1: none)
+  int dact_off[SIMX_MAX_LAYERS + 1]; // row offset of the derivative of layer l's input's activation
+                                     // (GELU layers, every hidden layer of a grid policy; -1: none)
   int dz_rows;                       // rows of each dZ buffer
   int poff[SIMX_MAX_LAYERS];         // offset of layer l's dW in the flat gradient
   int n_params;
@@ -313,7 +348,10 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
         const int64_t row = a.idx ? a.idx[rr] : rr;
         const int64_t t = row / a.E, e = row % a.E;
         const float* src = a.obs + t * D * a.E + e;
-        for (int d = dq; d < D; d += kLanes) X[d * kLld + r] = src[(int64_t)d * a.E];
+        if (a.grid)   // a grid policy's input on its grid
+          for (int d = dq; d < D; d += kLanes) X[d * kLld + r] = grid_q(src[(int64_t)d * a.E], a.gx[0]);
+        else
+          for (int d = dq; d < D; d += kLanes) X[d * kLld + r] = src[(int64_t)d * a.E];
       } else {
         for (int d = dq; d < D; d += kLanes) X[d * kLld + r] = 0.0f;
       }
@@ -330,7 +368,8 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
       tile_gemm<R>(Wf, F.npad[l + 1], a.dims[l], a.dims[l + 1],
                    acts + (size_t)F.act_off[l] * kLld, acts + (size_t)F.act_off[l + 1] * kLld, 0,
                    a.b[l], a.act[l], nullptr,
-                   F.dact_off[l + 1] >= 0 ? acts + (size_t)F.dact_off[l + 1] * kLld : nullptr);
+                   F.dact_off[l + 1] >= 0 ? acts + (size_t)F.dact_off[l + 1] * kLld : nullptr,
+                   (a.grid && l + 1 < L) ? a.gx[l + 1] : -1);
       __syncthreads();
     }
     // loss head: kLanes lanes per row (R rows x kLanes = 256 threads); lane q takes
@@ -437,8 +476,9 @@ __global__ void __launch_bounds__(kLThreads) k_loss_fused(const __grid_constant_
       }
       if (l > 0) {
         float* dzn = (dz == dzA) ? dzB : dzA;
-        // dZ_{l-1}[k][r] = sum_j W_l[j][k] dZ_l[j][r] * (1 - H_l[k][r]^2)
-        const int pa = a.act[l - 1];  // activation whose derivative applies
+        // dZ_{l-1}[k][r] = sum_j W_l[j][k] dZ_l[j][r] * (1 - H_l[k][r]^2); grid policies
+        // (and GELU layers) multiply by the stored derivative instead
+        const int pa = a.grid ? 2 : a.act[l - 1];  // activation whose derivative applies
         if (WS) {
           stage_wait();
           __syncthreads();
@@ -522,9 +562,9 @@ FusedPlan plan_r(const LossArgs& a, int R) {
     rows += r4(a.dims[l]);
     if (l > 0 && a.dims[l] > maxd) maxd = a.dims[l];
   }
-  for (int l = 0; l <= L; ++l) {  // GELU derivative of layer l's input (output of l - 1)
+  for (int l = 0; l <= L; ++l) {  // derivative of layer l's input (output of l - 1)
     p.dact_off[l] = -1;
-    if (l >= 1 && l < L && a.act[l - 1] == 2) {
+    if (l >= 1 && l < L && (a.act[l - 1] == 2 || a.grid)) {
       p.dact_off[l] = rows;
       rows += r4(a.dims[l]);
     }

@@ -7,8 +7,8 @@
 * policy_forward at the premise's worst case: a hidden layer saturated at +-255 units
   feeding a fan-in-256 output layer with every mantissa at +-255 and the largest bias, so
   the kernel's fp32 FMA chains run up to 2^24 product units.
-* Validation: out-of-range grid exponents and too-wide layers are refused, and so is the
-  loss gradient of a grid policy.
+* Validation: out-of-range grid exponents and too-wide layers are refused; the loss
+  gradient takes a grid policy (its parity is test_gpu_grid_loss.py's).
 """
 import numpy as np
 import pytest
@@ -120,7 +120,8 @@ def test_grid_policy_validation():
     with pytest.raises(simx.SimxError) as e:
         simx.policy_forward(_dev(simx, wide, wb, hv, gx), obs, 4, "argmax", 1, 0)
     assert e.value.status == simx.EINVAL
-    # the loss gradient has no grid path
+    # the loss gradient takes grid policies on its fused FP32 path (checked against the
+    # oracle in test_gpu_grid_loss.py)
     pol = _dev(simx, Ws, bs, hv, gx)
     cfg = W.c2(5)
     sim = simx.Sim(cfg)
@@ -131,9 +132,8 @@ def test_grid_policy_validation():
     grad = torch.empty(pol.n_params, device="cuda")
     stats = torch.empty(5, device="cuda")
     ws = torch.empty(simx.ppo_loss_grad_workspace_size(pol, 20), dtype=torch.uint8, device="cuda")
-    with pytest.raises(simx.SimxError) as e:
-        simx.ppo_loss_grad(pol, buf, torch.zeros((4, 5), device="cuda"),
-                           torch.zeros((4, 5), device="cuda"), None, 20, "reinforce", 0.2, 0.0,
-                           0.0, grad, stats, ws)
-    assert e.value.status == simx.EINVAL
+    simx.ppo_loss_grad(pol, buf, torch.zeros((4, 5), device="cuda"),
+                       torch.ones((4, 5), device="cuda"), None, 20, "reinforce", 0.2, 0.0,
+                       0.0, grad, stats, ws)
     torch.cuda.synchronize()
+    assert torch.isfinite(grad).all() and torch.isfinite(stats).all()
