@@ -294,14 +294,17 @@ __device__ bool load_chunk(const Smem& s, const Sched& q, int S, int stage_bytes
   return true;
 }
 
-// Thread 0's side of GEMM g  D = A B^T: A resident at a_addr (row-group stride a_sbo),
-// the B chunks through the stage ring.  After the MMAs of chunk k are queued, copies are
-// issued up to chunk k + S - 1, running on into the next GEMMs' chunks, so that those
-// arrive while the other threads work on this GEMM's result.  The accumulator's
-// completion is announced on accb (one phase per GEMM), which every thread waits on.
-__device__ void gemm_issue(const Smem& s, const Sched& q, int S, int stage_bytes, int g,
-                           int& issued, int& consumed, uint32_t a_addr, uint32_t a_sbo, int Nmma,
-                           uint32_t dtm) {
+// GEMM g  D = A B^T: A resident at a_addr (row-group stride a_sbo), the B chunks through
+// the stage ring, by two threads that never wait for each other's instructions: the MMA
+// thread (warp 1) waits for each chunk to land and queues its MMAs, the load thread
+// (warp 0, which issued the first chunks before the tile's gather) refills each stage
+// once the MMAs that read it completed, up to chunk k0[g + 1] + S - 1: on into the next
+// GEMM's chunks, which arrive while the other threads work on this GEMM's result.  The
+// accumulator's completion is announced on accb (one phase per GEMM), which every thread
+// waits on.  A wait that times out sets the abort flag and returns (accb is then never
+// committed and the other threads' waits time out too).
+__device__ void gemm_mma(const Smem& s, const Sched& q, int S, int stage_bytes, int g,
+                         uint32_t a_addr, uint32_t a_sbo, int Nmma, uint32_t dtm) {
   const uint32_t id = idesc_tf32(kR, Nmma);
   for (int k = q.k0[g]; k < q.k0[g + 1]; ++k) {
     const int st = k % S, c = k - q.k0[g];
@@ -316,17 +319,32 @@ __device__ void gemm_issue(const Smem& s, const Sched& q, int S, int stage_bytes
       mma_tf32(dtm, sdesc(a_addr + (uint32_t)c * 1024u + (uint32_t)ks * 256u, 128, a_sbo),
                sdesc(bs + (uint32_t)ks * 256u, 128, 1024), id, (c | ks) ? 1u : 0u);
     commit(&s.mmab[st]);
-    consumed = k + 1;
-    const int upto = k + S < q.total ? k + S : q.total;
-    while (issued < upto) {
-      if (!load_chunk(s, q, S, stage_bytes, issued)) {
-        *s.abort_flag = 1;
-        return;
-      }
-      ++issued;
-    }
   }
   commit(s.accb);
+}
+
+__device__ void gemm_load(const Smem& s, const Sched& q, int S, int stage_bytes, int g, int& issued) {
+  const int end = q.k0[g + 1] + S - 1;
+  const int upto = end < q.total ? end : q.total;
+  while (issued < upto) {
+    if (!load_chunk(s, q, S, stage_bytes, issued)) {
+      *s.abort_flag = 1;
+      return;
+    }
+    ++issued;
+  }
+}
+
+// The end of k_lw_rows, so that nothing is in flight when the CTA's shared and tensor
+// memory are released: the load thread waits (bounded) for its last S loads to land (all
+// of them were consumed unless a wait timed out), the MMA thread for every MMA it issued.
+__device__ void drain_loads(const Smem& s, int S, int issued) {
+  for (int k = issued > S ? issued - S : 0; k < issued; ++k)
+    mbar_wait(&s.full[k % S], (uint32_t)((k / S) & 1), kWaitCycles);
+}
+__device__ void drain_mma(const Smem& s) {
+  commit(s.drain);
+  mbar_wait(s.drain, 0u, kWaitCycles);
 }
 
 // Thread 0 at the end of a kernel: waits (bounded) for loads it issued that no MMA
@@ -384,9 +402,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   // everything up to the first read of the weight images (barriers, tensor memory, biases,
   // the observation gather) overlaps it; griddepcontrol.wait then waits for its images.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  // thread 0: barriers, then the first weight chunks on their way before anything else
+  // thread 0 (the load thread): barriers, then the first weight chunks on their way
+  // before anything else; thread 32 (the MMA thread) the same chunk schedule
   Sched sch;
-  int issued = 0, consumed = 0;
+  int issued = 0;
+  if (tid == 32) sch = make_sched(P, A.ws, rank);
   if (tid == 0) {
     for (int i = 0; i < kMaxStages; ++i) {
       mbar_init(&s.full[i], 1);
@@ -469,15 +489,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     st_peer4(peer + off, v);
   };
 
-  // GEMM g: thread 0 issues it, every thread then waits for the accumulator; then both
-  // CTAs meet, so that neither writes into the other's A buffer while its products run.
+  // GEMM g: threads 0 and 32 feed and issue it, every thread then waits for the
+  // accumulator; then both CTAs meet, so that neither writes into the other's A buffer
+  // while its products run.
   // After an abort no more work is issued, but every cluster barrier is still reached.
   auto gemm = [&](int g, int a_width, int Nmma) {
     const bool go = *s.abort_flag == 0;
     if (warp == 0) {
+      if (lane == 0 && go) gemm_load(s, sch, S, P.stage_bytes, g, issued);
+      __syncwarp();
+    } else if (warp == 1) {
       if (lane == 0 && go)
-        gemm_issue(s, sch, S, P.stage_bytes, g, issued, consumed, abuf_addr,
-                   (uint32_t)(a_width / 4) * 128u, Nmma, tmem);
+        gemm_mma(s, sch, S, P.stage_bytes, g, abuf_addr, (uint32_t)(a_width / 4) * 128u, Nmma, tmem);
       __syncwarp();
     }
     if (go && !mbar_wait_idle(s.accb, (uint32_t)(ngemm & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
@@ -683,7 +706,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
   }
 
   // ---- end: nothing in flight, statistics of the CTA's rows, tensor memory released
-  if (tid == 0) drain_all(s, S, issued, consumed);
+  if (tid == 0) drain_loads(s, S, issued);
+  if (tid == 32) drain_mma(s);
   if (cq == 0) {
 #pragma unroll
     for (int d = 16; d > 0; d >>= 1) {
