@@ -335,7 +335,7 @@ __device__ void gemm_load(const Smem& s, const Sched& q, int S, int stage_bytes,
   }
 }
 
-// The end of k_lw_rows, so that nothing is in flight when the CTA's shared and tensor
+// The end of a kernel, so that nothing is in flight when the CTA's shared and tensor
 // memory are released: the load thread waits (bounded) for its last S loads to land (all
 // of them were consumed unless a wait timed out), the MMA thread for every MMA it issued.
 __device__ void drain_loads(const Smem& s, int S, int issued) {
@@ -347,14 +347,6 @@ __device__ void drain_mma(const Smem& s) {
   mbar_wait(s.drain, 0u, kWaitCycles);
 }
 
-// Thread 0 at the end of a kernel: waits (bounded) for loads it issued that no MMA
-// consumed, then for every MMA it issued, so nothing is in flight when the CTA's
-// shared and tensor memory are released.
-__device__ void drain_all(const Smem& s, int S, int issued, int consumed) {
-  for (int k = consumed; k < issued; ++k) mbar_wait(&s.full[k % S], (uint32_t)((k / S) & 1), kWaitCycles);
-  commit(s.drain);
-  mbar_wait(s.drain, 0u, kWaitCycles);
-}
 
 // The two CTAs of a cluster share one 128-row tile: each computes half of the outputs of
 // every split product (rank r: rows r * half .. of each weight chunk), and writes its half
@@ -778,28 +770,31 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
   __syncthreads();
   fence_after();
   const uint32_t tmem = *s.tbase;
-  int issued = 0, consumed = 0;
+  int issued = 0;
 
+  // thread 0 streams the row chunks of G and H through the stages, each refilled once the
+  // MMAs that read it completed; thread 32 queues each chunk's MMAs as it lands
   if (warp == 0 && lane == 0 && nc > 0) {
     const unsigned char* gsrc = A.ws + P.img_g[l];
     const unsigned char* hsrc = A.ws + P.img_h[l];
-    const uint32_t idw = idesc_tf32(kR, Fh), idb = idesc_tf32(kR, 16);
-    const uint32_t ones = su32(sm);
-    auto load = [&](int c) -> bool {
+    for (int c = 0; c < nc; ++c) {
       const int st = c % S;
-      if (c >= S && !mbar_wait(&s.mmab[st], (uint32_t)(((c - S) / S) & 1), kWaitCycles)) return false;
+      if (c >= S && !mbar_wait(&s.mmab[st], (uint32_t)(((c - S) / S) & 1), kWaitCycles)) {
+        *s.abort_flag = 1;
+        break;
+      }
       const int64_t rc = c_lo + c;
       unsigned char* dst = s.stages + (size_t)st * SB;
       mbar_arrive_expect_tx(&s.full[st], aA + bB);
       bulk_g2s(dst, gsrc + (size_t)(rc * (Fg >> 3) + 16 * mt) * 1024, aA, &s.full[st]);
       bulk_g2s(dst + 16384, hsrc + (size_t)rc * (Fh >> 3) * 1024, bB, &s.full[st]);
       issued = c + 1;
-      return true;
-    };
-    const int pre = nc < S - 1 ? nc : S - 1;
+    }
+  } else if (warp == 1 && lane == 0 && nc > 0) {
+    const uint32_t idw = idesc_tf32(kR, Fh), idb = idesc_tf32(kR, 16);
+    const uint32_t ones = su32(sm);
     bool fine = true;
-    for (int c = 0; c < pre && fine; ++c) fine = load(c);
-    for (int c = 0; c < nc && fine; ++c) {
+    for (int c = 0; c < nc; ++c) {
       const int st = c % S;
       if (!mbar_wait(&s.full[st], (uint32_t)((c / S) & 1), kWaitCycles)) {
         fine = false;
@@ -815,8 +810,6 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
         mma_tf32(tmem + (uint32_t)Fh, ad, sdesc(ones + (uint32_t)ks * 256u, 128, 1024), idb, acc);
       }
       commit(&s.mmab[st]);
-      consumed = c + 1;
-      if (c + S - 1 < nc) fine = load(c + S - 1);
     }
     if (fine) commit(s.accb);
     else *s.abort_flag = 1;
@@ -856,7 +849,8 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
     reg_fence(u);
     if (j < Nl) out[(size_t)Nl * Kl + j] = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[0]) : nanv);
   }
-  if (tid == 0) drain_all(s, S, issued, consumed);
+  if (tid == 0) drain_loads(s, S, issued);
+  if (tid == 32) drain_mma(s);
   fence_before();
   __syncthreads();
   if (warp == 0) {
