@@ -66,6 +66,11 @@ def _args():
                    help="time a grid policy's rollout with the forward on the tensor cores and on "
                         "the FP32 tiles (the exact policy forward) and exit")
     p.add_argument("--grid-envs", type=int, default=65536)
+    p.add_argument("--rollout-only", default=None, metavar="WORKLOAD",
+                   help="time rollout_collect alone (its fp32 policy) with the forward's weights "
+                        "staged in shared memory and read through L1, and exit")
+    p.add_argument("--rollout-envs", type=int, default=None)
+    p.add_argument("--rollout-steps", type=int, default=None)
     p.add_argument("--hbm-step-only", type=int, default=None, metavar="ENVS",
                    help="time only the policy-free batched step at this env count and exit")
     p.add_argument("--minibatch-loss", default=None, metavar="WORKLOAD",
@@ -526,6 +531,56 @@ def run_grid_rollout(name: str, E: int, reps: int = 3) -> None:
     print(json.dumps(line), flush=True)
 
 
+def run_rollout_only(name: str, E: int, H: int, reps: int = 3) -> None:
+    """rollout_collect of `name`'s fp32 policy over E envs x H steps, with the policy's
+    weights staged in shared memory (SIMX_STAGE=1) and read through L1 (SIMX_STAGE=0):
+    CUDA events around each launch after a warm-up; the two buffers must be equal bit for
+    bit.  One JSON line."""
+    import torch
+
+    from paper_2607_05272_gb300 import build as B
+    from paper_2607_05272_gb300 import workloads as W
+    B.build()
+    from paper_2607_05272_gb300 import simx
+    cfg = W.CONFIGS[name](E)
+    dims, hv = W.mlp_dims(name)
+    Ws, bs = W.policy_weights(name, dims, 1)
+    pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws], [torch.from_numpy(b).cuda() for b in bs],
+                      hv, W.mlp_acts(name))
+    mode = "argmax" if name == "c5" else "sample"
+    line = {"workload": name, "envs": E, "horizon": H, "mlp": dims}
+    bufs = []
+    for stage in ("1", "0"):
+        os.environ["SIMX_STAGE"] = stage
+        sim = simx.Sim(cfg)
+        shape = sim.launch_shape(mode, pol)
+        sim.reset(W.SEED[name])
+        warm = simx.alloc_rollout(E, sim.D, 4, has_value=hv)
+        sim.rollout(mode, 4, warm, pol)
+        del warm
+        buf = simx.alloc_rollout(E, sim.D, H, has_value=hv)
+        ts = []
+        for _ in range(reps):
+            sim.reset(W.SEED[name])
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            sim.rollout(mode, H, buf, pol)
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        st, _ = sim.last_status()
+        sim.close()
+        ms = statistics.median(ts)
+        key = "staged" if stage == "1" else "through_l1"
+        line[key] = {"ms": ms, "us_per_step": 1000.0 * ms / H,
+                     "decision_steps_per_s": E * H / (ms * 1e-3), "status": st, "launch": shape}
+        bufs.append(buf)
+    os.environ.pop("SIMX_STAGE", None)
+    line["bit_identical"] = all(torch.equal(bufs[0][k], bufs[1][k]) for k in bufs[0])
+    line["speedup"] = line["through_l1"]["ms"] / line["staged"]["ms"]
+    print(json.dumps(line), flush=True)
+
+
 def run_minibatch_loss(name: str, E: int = 256, steps: int = 20) -> None:
     """The PPO loss gradient (Sec. 4.3) on 8192-row minibatches drawn from a rollout of
     `name` (E envs x its horizon): median of `steps` timed calls per precision after 3
@@ -964,6 +1019,11 @@ def main():
         return
     if a.grid_rollout:
         run_grid_rollout(a.grid_rollout, a.grid_envs)
+        return
+    if a.rollout_only:
+        from paper_2607_05272_gb300 import workloads as W
+        run_rollout_only(a.rollout_only, a.rollout_envs or W.CONFIGS[a.rollout_only]()["n_envs"],
+                         a.rollout_steps or W.HORIZON[a.rollout_only])
         return
     if a.hbm_step_only:
         import torch
