@@ -820,12 +820,18 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
   __syncthreads();
   const bool ok = *s.abort_flag == 0;
 
-  // read out: lane m = output j = 128 mt + m; columns k < K_l of dW, column Fh of db
+  // read out: lane m = output j = 128 mt + m; columns k < K_l of dW, column Fh of db.
+  // dW goes through a row-major tile in the (now idle) stages, row stride = 4 words past a
+  // multiple of 32 (a warp's 16-byte row writes hit every bank once per 8 rows), and then
+  // to the partial gradient row by row, a warp writing 128 contiguous bytes at a time.
   const int Kl = P.K[l], Nl = P.N[l];
   const int j = 128 * mt + 32 * quarter + lane;
   float* out = reinterpret_cast<float*>(A.ws + P.part) + (size_t)split * P.n_params + P.poff[l];
   const uint32_t tl = tmem + ((uint32_t)(32 * quarter) << 16);
   const float nanv = __uint_as_float(0x7FC00000u);
+  float* tile = reinterpret_cast<float*>(s.stages);
+  const int ldt = (Kl + 31) / 32 * 32 + 4;
+  float* trow = tile + (size_t)(32 * quarter + lane) * ldt;
   for (int c0 = 16 * cq; c0 < Fh; c0 += 32) {
     uint32_t u[4][4];
 #pragma unroll
@@ -834,13 +840,23 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       reg_fence(u[q]);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int k = c0 + 4 * q + i;
-        if (j < Nl && k < Kl)
-          out[(size_t)j * Kl + k] = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[q][i]) : nanv);
+      const int k = c0 + 4 * q;
+      if (k < Kl) {
+        float4 v;
+        v.x = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[q][0]) : nanv);
+        v.y = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[q][1]) : nanv);
+        v.z = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[q][2]) : nanv);
+        v.w = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[q][3]) : nanv);
+        *reinterpret_cast<float4*>(trow + k) = v;
       }
     }
+  }
+  __syncthreads();
+  {
+    const int rows = Nl - 128 * mt < 128 ? Nl - 128 * mt : 128;
+    float* dst = out + (size_t)(128 * mt) * Kl;
+    for (int rr = warp; rr < rows; rr += kDwThreads / 32)
+      for (int k = lane; k < Kl; k += 32) dst[(size_t)rr * Kl + k] = tile[(size_t)rr * ldt + k];
   }
   if (cq == 0) {
     uint32_t u[4];
@@ -939,6 +955,9 @@ Plan plan(const LossArgs& a) {
   p.dw_nstages = 3;
   p.dw_smem = 2048 + p.dw_nstages * p.dw_stage_bytes + misc;
   if (p.dw_smem > limit) return p;
+  // the dW read-out tile (128 rows, row stride r32(K) + 4 floats) reuses the stages
+  for (int l = 0; l < L; ++l)
+    if ((size_t)128 * ((p.K[l] + 31) / 32 * 32 + 4) * 4 > (size_t)p.dw_nstages * p.dw_stage_bytes) return p;
   p.dw_tcols = pow2_cols(maxFh + 16);
   if (p.dw_tcols > 512) return p;
   // workspace
