@@ -12,7 +12,10 @@ namespace simx {
 namespace {
 
 constexpr int kAdamThreads = 256;
-constexpr int kNormBlocks = 304;  // fixed (two per GB300 SM): the same sum order on any device
+// Blocks of the sum of squares: fixed, so the sum order is the same on any device; few, so
+// that every block of the update finishes their partials in two loads per lane (policy
+// vectors are 10^3-10^5 parameters).
+constexpr int kNormBlocks = 64;
 
 __global__ void __launch_bounds__(kAdamThreads) k_sumsq(const float* __restrict__ g,
                                                         const uint8_t* __restrict__ mask,
