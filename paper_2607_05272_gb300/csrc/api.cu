@@ -249,7 +249,7 @@ const char* simx_strerror(simx_status s) {
     case SIMX_EINVAL: return "invalid argument";
     case SIMX_ENOMEM: return "out of memory";
     case SIMX_ECUDA: return "CUDA error";
-    case SIMX_EOVERFLOW: return "device status flag raised (time overflow, event cap or bad action)";
+    case SIMX_EOVERFLOW: return "device status flag raised (time overflow, event cap, bad action or a bounded wait timed out)";
     case SIMX_ESTATE: return "call out of order";
   }
   return "unknown status";
