@@ -16,7 +16,12 @@ Each case asserts the launch shape it means to cover:
 * a c3 grid policy with staging forced and the tensor-core forward off: the grid
   rounding in the staged epilogue;
 * c4 at 1,003 envs in 128-thread blocks (8 lanes, 4 KB stages): a last block with 11
-  envs.
+  envs;
+* c4 at 65,536 envs with 16 lanes per env (2x8 tiles, 1x4 for the 49 outputs, 16 envs per
+  256-thread block);
+* c3t, trace replay (gaps, types and costs from a trace), at 16,384 envs;
+* single steps (sim_step_batched: one launch per step, so the weight pipeline starts and
+  drains every launch) against rollout_collect, c4 at 4,096 envs in 256-thread blocks.
 """
 import numpy as np
 import pytest
@@ -84,11 +89,14 @@ CASES = [
     ("c1p", 4096, 300, "sample", False, "256", None, "1", 256),
     ("c3", 16384, 64, "argmax", True, None, None, "1", 128),
     ("c4", 1003, 200, "sample", False, "128", "8", "", 128),
+    ("c4", 65536, 32, "sample", False, None, "16", "", 256),
+    ("c3t", 16384, 64, "sample", False, None, None, "", 128),
 ]
 
 
 @pytest.mark.parametrize("name,E,H,mode,grid,threads,lanes,stage,expect", CASES,
-                         ids=["c4", "c3", "c1p-forced", "c3-grid-forced", "c4-ragged"])
+                         ids=["c4", "c3", "c1p-forced", "c3-grid-forced", "c4-ragged", "c4-16-lanes",
+                              "c3t"])
 def test_staged_forward(name, E, H, mode, grid, threads, lanes, stage, expect, monkeypatch):
     simx = _simx()
     if threads:
@@ -120,3 +128,44 @@ def test_staged_forward(name, E, H, mode, grid, threads, lanes, stage, expect, m
         assert np.array_equal(got[k].view(np.uint32), ref[k].view(np.uint32)), k
     assert np.array_equal(state[envs], ref["state"])
     assert len(np.unique(got["action"])) > 1
+
+
+def test_staged_single_steps_equal_the_rollout(monkeypatch):
+    simx = _simx()
+    monkeypatch.setenv("SIMX_LANES", "8")
+    monkeypatch.setenv("SIMX_THREADS", "256")
+    monkeypatch.delenv("SIMX_STAGE", raising=False)
+    E, H = 4096, 24
+    cfg = W.c4(E)
+    Ws, bs, hv, acts, _ = _host("c4", False)
+    pol = simx.Policy([torch.from_numpy(w).cuda() for w in Ws],
+                      [torch.from_numpy(b).cuda() for b in bs], hv, acts)
+    seed = 0x57E9
+    sim = simx.Sim(cfg)
+    shape = sim.launch_shape("sample", pol)
+    assert shape["staged"] and shape["threads"] == 256 and shape["lanes"] == 8
+    sim.reset(seed)
+    buf = simx.alloc_rollout(E, sim.D, H, has_value=hv)
+    sim.rollout("sample", H, buf, pol)
+    torch.cuda.synchronize()
+    state_r = sim.save()
+    sim.close()
+    sim = simx.Sim(cfg)
+    sim.reset(seed)
+    rew = torch.empty((H, E), device="cuda")
+    done = torch.empty((H, E), dtype=torch.uint8, device="cuda")
+    act = torch.empty((H, E), dtype=torch.uint8, device="cuda")
+    lp = torch.empty((H, E), device="cuda")
+    obs = torch.empty((H, sim.D, E), device="cuda")
+    for t in range(H):
+        sim.step("sample", pol, obs=obs[t], reward=rew[t], done=done[t], action=act[t], logp=lp[t])
+    torch.cuda.synchronize()
+    st, code = sim.last_status()
+    assert st == 0 and code == 0
+    assert torch.equal(act, buf["action"]) and torch.equal(done, buf["done"])
+    assert torch.equal(rew.view(torch.int32), buf["reward"].view(torch.int32))
+    assert torch.equal(lp.view(torch.int32), buf["logp"].view(torch.int32))
+    # a step writes the observation after it, the rollout the one before each step
+    assert torch.equal(obs[:-1].view(torch.int32), buf["obs"][1:].view(torch.int32))
+    assert np.array_equal(sim.save(), state_r)
+    sim.close()
