@@ -481,6 +481,33 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
     st_peer4(peer + off, v);
   };
 
+  // The feature-major image rows an epilogue produces (FP32 H or G for the weight-gradient
+  // kernel) wait in the second half of the tensor memory and go out while the next
+  // product runs: the stores of all CTAs at once are bound by L2 bandwidth, the product
+  // by the MMA issue, so overlapped they cost the longer of the two.  pend_*: the thread's
+  // staged block (image, its features, first column, columns) until flushed.
+  const uint32_t tstage = (uint32_t)P.tcols / 2;
+  unsigned char* pend_img = nullptr;
+  int pend_F = 0, pend_j0 = 0, pend_w = 0;
+  auto stage_img = [&](int c0, const float (&v)[16]) { tm_st16_nw(tl + tstage + (uint32_t)c0, v); };
+  auto flush = [&]() {
+    if (!pend_img) return;
+    for (int c0 = 16 * cq; c0 < pend_w; c0 += 64) {
+      const int jg = pend_j0 + c0;
+      if (jg < pend_F) {
+        uint32_t u[16];
+        tm_ld16_nw(tl + tstage + (uint32_t)c0, u);
+        tm_wait();
+        reg_fence16(u);
+        float v[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(u[i]);
+        img_store16(pend_img, jg, v, lane);
+      }
+    }
+    pend_img = nullptr;
+  };
+
   // GEMM g: threads 0 and 32 feed and issue it, every thread then waits for the
   // accumulator; then both CTAs meet, so that neither writes into the other's A buffer
   // while its products run.
@@ -495,6 +522,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
         gemm_mma(s, sch, S, P.stage_bytes, g, abuf_addr, (uint32_t)(a_width / 4) * 128u, Nmma, tmem);
       __syncwarp();
     }
+    flush();   // the previous epilogue's image rows, while the products run
     if (go && !mbar_wait_idle(s.accb, (uint32_t)(ngemm & 1), kWaitCycles)) atomicOr(s.abort_flag, 1);
     ++ngemm;
     __syncwarp();
@@ -545,7 +573,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
           put_both(rm_off(r, jg + 4 * qq, Wn),
                    make_float4(to_tf32(h[4 * qq]), to_tf32(h[4 * qq + 1]), to_tf32(h[4 * qq + 2]),
                                to_tf32(h[4 * qq + 3])));
-        if (jg < Fn) img_store16(img, jg, h, lane);
+        if (jg < Fn) stage_img(c0, h);
+      }
+      if (ok) {
+        tm_wait_st();
+        pend_img = img;
+        pend_F = Fn;
+        pend_j0 = j0h;
+        pend_w = hN;
       }
     } else {
       // loss head over the whole last layer (both CTAs hold it): rank r takes lane
@@ -654,8 +689,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
             put_both(rm_off(r, c0 + 4 * qq, Wg),
                      make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
                                  to_tf32(g[4 * qq + 3])));
-          if (c0 < Fg) img_store16(img, c0, g, lane);
+          if (c0 < Fg) stage_img(c0, g);
         }
+        tm_wait_st();
+        pend_img = img;
+        pend_F = Fg;
+        pend_j0 = 0;
+        pend_w = Wg;
       }
     }
     cluster_sync();
@@ -692,10 +732,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_lw_rows(const __grid_constant__
           put_both(rm_off(r, jg + 4 * qq, Wg),
                    make_float4(to_tf32(g[4 * qq]), to_tf32(g[4 * qq + 1]), to_tf32(g[4 * qq + 2]),
                                to_tf32(g[4 * qq + 3])));
-      if (jg < Fg) img_store16(gimg, jg, g, lane);
+      if (jg < Fg) stage_img(c0, g);
+    }
+    if (ok) {
+      tm_wait_st();
+      pend_img = gimg;
+      pend_F = Fg;
+      pend_j0 = j0h;
+      pend_w = hK;
     }
     if (Wg) cluster_sync();   // G_0 is not an operand here: nothing went to the peer
   }
+  flush();   // G_0's image rows
 
   // ---- end: nothing in flight, statistics of the CTA's rows, tensor memory released
   if (tid == 0) drain_loads(s, S, issued);
@@ -936,7 +984,7 @@ Plan plan(const LossArgs& a) {
   while (p.nstages > 2 && p.a_bytes + p.nstages * p.stage_bytes + misc + 4 * p.b_total > limit) --p.nstages;
   p.smem = p.a_bytes + p.nstages * p.stage_bytes + misc + 4 * p.b_total;
   if (p.smem > limit) return p;
-  p.tcols = pow2_cols(tneed);
+  p.tcols = pow2_cols(2 * tneed);   // accumulators, then the staged image rows
   if (p.tcols > 512) return p;
   // weight-gradient products
   p.mt_total = 0;
