@@ -783,8 +783,9 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
   extern __shared__ __align__(1024) unsigned char sm[];
   const Plan& P = A.p;
   const int S = P.dw_nstages, SB = P.dw_stage_bytes;
-  // the first 2 KB hold the ones operand of db (feature 0 = 1, features 1..15 = 0)
+  // the first 2 KB hold one mbarrier per stage on which the db warps release it
   const Smem s = carve(sm, P, SB, S, 2048);
+  uint64_t* dbe = reinterpret_cast<uint64_t*>(sm);
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int quarter = warp & 3, cq = warp >> 2;
@@ -805,11 +806,10 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
     }
     mbar_init(s.drain, 1);
     mbar_init(s.accb, 1);
+    for (int i = 0; i < kMaxStages; ++i) mbar_init(&dbe[i], kDwThreads / 32 - 4);
     mbar_fence_init();
     *s.abort_flag = 0;
   }
-  for (int i = tid; i < 512; i += kDwThreads)
-    reinterpret_cast<float*>(sm)[i] = (i < 256 && ((i >> 2) & 7) == 0) ? 1.0f : 0.0f;
   if (warp == 0) tm_alloc(s.tbase, (uint32_t)P.dw_tcols);
   // launched while k_lw_rows runs: the images it writes are read only after this wait
   asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -821,13 +821,18 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
   int issued = 0;
 
   // thread 0 streams the row chunks of G and H through the stages, each refilled once the
-  // MMAs that read it completed; thread 32 queues each chunk's MMAs as it lands
+  // MMAs that read it completed and the db warps released it; thread 32 queues each
+  // chunk's dW MMAs as it lands; warps 4 .. 7 add the chunk's G rows into db_l (one thread
+  // per output, rows in order: db = G^T 1 in FP32 on the CUDA cores, beside the MMAs)
+  float db = 0.0f;
+  const int jl = tid - 128;   // db warps: this thread's output in the block
   if (warp == 0 && lane == 0 && nc > 0) {
     const unsigned char* gsrc = A.ws + P.img_g[l];
     const unsigned char* hsrc = A.ws + P.img_h[l];
     for (int c = 0; c < nc; ++c) {
       const int st = c % S;
-      if (c >= S && !mbar_wait(&s.mmab[st], (uint32_t)(((c - S) / S) & 1), kWaitCycles)) {
+      const uint32_t par = (uint32_t)(((c - S) / S) & 1);
+      if (c >= S && (!mbar_wait(&s.mmab[st], par, kWaitCycles) || !mbar_wait(&dbe[st], par, kWaitCycles))) {
         *s.abort_flag = 1;
         break;
       }
@@ -839,8 +844,7 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
       issued = c + 1;
     }
   } else if (warp == 1 && lane == 0 && nc > 0) {
-    const uint32_t idw = idesc_tf32(kR, Fh), idb = idesc_tf32(kR, 16);
-    const uint32_t ones = su32(sm);
+    const uint32_t idw = idesc_tf32(kR, Fh);
     bool fine = true;
     for (int c = 0; c < nc; ++c) {
       const int st = c % S;
@@ -855,12 +859,31 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
         const uint64_t ad = sdesc(sa + (uint32_t)ks * 256u, 128, 1024);
         const uint32_t acc = (c | ks) ? 1u : 0u;
         mma_tf32(tmem, ad, sdesc(sb + (uint32_t)ks * 256u, 128, 1024), idw, acc);
-        mma_tf32(tmem + (uint32_t)Fh, ad, sdesc(ones + (uint32_t)ks * 256u, 128, 1024), idb, acc);
       }
       commit(&s.mmab[st]);
     }
     if (fine) commit(s.accb);
     else *s.abort_flag = 1;
+  } else if (warp >= 4 && nc > 0) {
+    // output jl's 32 rows of a chunk: 8 consecutive 16-byte core-matrix rows of its group
+    const uint32_t goff = (uint32_t)((jl >> 3) * 1024 + (jl & 7) * 16);
+    for (int c = 0; c < nc; ++c) {
+      const int st = c % S;
+      if (*s.abort_flag || !mbar_wait_idle(&s.full[st], (uint32_t)((c / S) & 1), kWaitCycles)) {
+        atomicOr(s.abort_flag, 1);
+        break;
+      }
+      if (jl < ng * 8) {
+        const unsigned char* g = s.stages + (size_t)st * SB + goff;
+#pragma unroll
+        for (int q = 0; q < kKC / 4; ++q) {
+          const float4 v = *reinterpret_cast<const float4*>(g + q * 128);
+          db = __fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(db, v.x), v.y), v.z), v.w);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&dbe[st]);
+    }
   }
   __syncwarp();
   if (nc > 0 && !mbar_wait_idle(s.accb, 0u, kWaitCycles)) atomicOr(s.abort_flag, 1);
@@ -906,13 +929,8 @@ __global__ void __launch_bounds__(kDwThreads, 1) k_lw_dw(const __grid_constant__
     for (int rr = warp; rr < rows; rr += kDwThreads / 32)
       for (int k = lane; k < Kl; k += 32) dst[(size_t)rr * Kl + k] = tile[(size_t)rr * ldt + k];
   }
-  if (cq == 0) {
-    uint32_t u[4];
-    tm_ld4_nw(tl + (uint32_t)Fh, u);
-    tm_wait();
-    reg_fence(u);
-    if (j < Nl) out[(size_t)Nl * Kl + j] = nc == 0 ? 0.0f : (ok ? __uint_as_float(u[0]) : nanv);
-  }
+  if (warp >= 4 && 128 * mt + jl < Nl)
+    out[(size_t)Nl * Kl + 128 * mt + jl] = nc == 0 ? 0.0f : (ok ? db : nanv);
   if (tid == 0) drain_loads(s, S, issued);
   if (tid == 32) drain_mma(s);
   fence_before();
@@ -1006,7 +1024,7 @@ Plan plan(const LossArgs& a) {
   // the dW read-out tile (128 rows, row stride r32(K) + 4 floats) reuses the stages
   for (int l = 0; l < L; ++l)
     if ((size_t)128 * ((p.K[l] + 31) / 32 * 32 + 4) * 4 > (size_t)p.dw_nstages * p.dw_stage_bytes) return p;
-  p.dw_tcols = pow2_cols(maxFh + 16);
+  p.dw_tcols = pow2_cols(maxFh);
   if (p.dw_tcols > 512) return p;
   // workspace
   size_t off = 0;

@@ -110,6 +110,11 @@ __device__ __forceinline__ bool mbar_wait_idle(uint64_t* mbar, uint32_t parity, 
   }
 }
 
+// One plain arrival.
+__device__ __forceinline__ void mbar_arrive(uint64_t* mbar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(mbar)) : "memory");
+}
+
 // One arrival that also announces `bytes` of transactions the phase must receive.
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* mbar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(mbar)), "r"(bytes)
