@@ -7,7 +7,8 @@
 //   forward   Z_l  = [H_l, 1] [W_l, b_l]^T          (rows x outputs; the bias rides on a
 //                                                   ones column of the activations)
 //   weights   dW_l += G_l^T H_l                      (outputs x inputs, K = the tile's rows)
-//   biases    db_l += G_l^T 1                        (an MMA against a block of ones)
+//   biases    db_l += G_l^T 1                        (FP32 sums on the CUDA cores, beside
+//                                                   the weight products)
 //   inputs    dH_l  = G_l W_l                        (rows x inputs)
 // where G_l is dL/d(pre-activation of layer l).  dW_l and db_l stay in tensor memory for
 // all of the CTA's tiles and are read out once at the end.  Threads do the elementwise
@@ -248,6 +249,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
   bool first = true;
   unsigned char* hr = sm + P.o_hr;
   unsigned char* dat = sm + P.o_dat;
+  // db_l of output tid, summed over the CTA's tiles (threads below each layer's width)
+  float dbacc[SIMX_MAX_LAYERS];
+#pragma unroll
+  for (int l = 0; l < SIMX_MAX_LAYERS; ++l) dbacc[l] = 0.0f;
 
   // One synchronisation point between a stage's shared-memory / TMEM producers and the
   // MMAs that read them; returns false when any thread saw an MMA wait time out.
@@ -480,18 +485,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
       if (tid == kThreads - 32) {
         // transposed operands advance 2 x 144 bytes (18 in the address field) per K step
         const uint32_t acc0 = first ? 0u : 1u;
-        const uint32_t idw = idesc(kR, Kp), idb = idesc(kR, 16);
+        const uint32_t idw = idesc(kR, Kp);
         uint64_t ad = sdesc(su32(dat), kRowLd, kTGroup);
         uint64_t hd = sdesc(su32(sm + P.o_ht[l]), kRowLd, kTGroup);
-        uint64_t od = sdesc(su32(sm + P.o_ones), kRowLd, kTGroup);
-        const uint32_t dw = tmem + P.t_dw[l], db = tmem + P.t_db[l];
+        const uint32_t dw = tmem + P.t_dw[l];
         for (int ks = 0; ks < kR / 8; ++ks) {
           const uint32_t acc = ks > 0 ? 1u : acc0;
           mma(dw, ad, hd, idw, acc);
-          mma(db, ad, od, idb, acc);
           ad += (2 * kRowLd) >> 4;
           hd += (2 * kRowLd) >> 4;
-          od += (2 * kRowLd) >> 4;
         }
         if (l > 0) {
           const uint32_t idh = idesc(kR, Kp);
@@ -504,6 +506,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
           }
         }
         commit(mbar);
+      }
+      if (tid < P.N[l]) {
+        // db_l of output tid over the tile's rows, from the transposed G_l the weight
+        // products read (the same TF32 values), rows in order
+        const unsigned char* col = dat + (tid >> 3) * kTGroup + (tid & 7) * 16;
+        float sacc = 0.0f;
+#pragma unroll 4
+        for (int q = 0; q < kR / 4; ++q) {
+          const float4 v = *reinterpret_cast<const float4*>(col + q * kRowLd);
+          sacc = __fadd_rn(__fadd_rn(__fadd_rn(__fadd_rn(sacc, v.x), v.y), v.z), v.w);
+        }
+        dbacc[l] = __fadd_rn(dbacc[l], sacc);
       }
       wait_mma();
       if (l > 0) {
@@ -562,10 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_loss_tc(const __grid_constant__
             if (4 * cb + i < K) gW[(size_t)r * K + 4 * cb + i] = (&v.x)[i];
         }
       }
-      if (cq == 0) {
-        const float4 v = tm_ld4(tlane + P.t_db[l]);
-        if (r < N) gW[(size_t)N * K + r] = v.x;
-      }
+      if (tid < N) gW[(size_t)N * K + tid] = dbacc[l];
     }
   } else {
     for (int i = tid; i < P.n_params; i += kThreads) out[i] = 0.0f;
