@@ -412,9 +412,9 @@ class Clocks:
 # DRAM bytes (read + write) of one k_rollout launch of the benchmark workload, from an
 # ncu capture of the current kernel; None until one is taken, and to be re-measured (or
 # set back to None) whenever the rollout kernel changes.
-ROLLOUT_DRAM_BYTES = 385558784.0 + 4579380480.0
+ROLLOUT_DRAM_BYTES = 389046528.0 + 4584373504.0
 ROLLOUT_DRAM_SOURCE = ("ncu dram__bytes_read.sum + dram__bytes_write.sum of one k_rollout launch "
-                       "of this workload (385.6 MB + 4579.4 MB; profiles/k_rollout_c4_bench.md)")
+                       "of this workload (389.0 MB + 4584.4 MB; profiles/k_rollout_c4_bench.md)")
 
 
 def _peaks():

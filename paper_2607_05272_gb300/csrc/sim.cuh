@@ -390,7 +390,7 @@ __device__ __forceinline__ uint32_t layer_staged(const DevMlp& m, const StagePla
     const float* xc = X + (size_t)(j * rpc) * ld + TE * eb;
     const int rows = K - j * rpc < rpc ? K - j * rpc : rpc;
     if (active) {
-#pragma unroll 4
+#pragma unroll 8
       for (int k = 0; k < rows; ++k) {
         uint64_t wv[TO / 2];
 #pragma unroll
