@@ -6,6 +6,9 @@
   central finite differences of the loss.
 * The PPO policy term at rho = 1 equals the REINFORCE form; loss values at uniform
   logits equal their closed forms.
+* PPO's clipping by the sign of the advantage: one row at a tabulated ratio, the gradient 0
+  exactly when the clipped branch is the minimum and rho times REINFORCE's otherwise (a max
+  for the min, the branch test reversed or a clip that ignores the sign each fail a case).
 """
 import math
 
@@ -186,6 +189,38 @@ def test_ppo_at_rho_one_equals_reinforce():
     assert np.allclose(rl.flat(g_ppo), rl.flat(g_rf), rtol=1e-12, atol=1e-14)
     assert s_ppo[1] == pytest.approx(-np.mean(adv))   # rho = 1: -mean(adv)
     assert s_ppo[4] == 0.0
+
+
+# adv, rho, whether the clipped branch is the minimum (PPO, eps = 0.2), the policy term
+CLIP_CASES = [(1.5, 1.5, True, -1.2 * 1.5), (1.5, 0.5, False, -0.5 * 1.5),
+              (-1.5, 0.5, True, 0.8 * 1.5), (-1.5, 1.5, False, 1.5 * 1.5),
+              (1.5, 1.1, False, -1.1 * 1.5), (-1.5, 0.9, False, 0.9 * 1.5)]
+
+
+@pytest.mark.parametrize("adv,rho,clipped,pg", CLIP_CASES)
+def test_ppo_clip_cases_by_advantage_sign(adv, rho, clipped, pg):
+    """One row, no entropy or value term.  The surrogate min(rho A, clip(rho, 1-eps, 1+eps) A)
+    is flat in theta exactly when its clipped branch is the smaller one: rho above 1 + eps with
+    A > 0, or below 1 - eps with A < 0.  Then the gradient is 0; otherwise the gradient is that
+    of -rho A, i.e. rho times the REINFORCE gradient -A grad log pi(a).  The policy term is the
+    tabulated value, and the clip fraction counts |rho - 1| > eps whichever branch wins."""
+    Ws, bs, X, a, _, ret, _ = _tiny(False, seed=6)
+    X, a, ret = X[:1], a[:1], ret[:1]
+    _, Z = rl.forward(Ws, bs, X)
+    m = Z.max(1, keepdims=True)
+    lpa = (Z - (m + np.log(np.exp(Z - m).sum(1, keepdims=True))))[0, a[0]]
+    lpo = np.array([lpa - math.log(rho)])
+    A = np.array([adv])
+    g_ppo, s = rl.loss_grad(Ws, bs, False, X, a, lpo, A, ret, rl.PPO, 0.2, 0.0, 0.0)
+    g_rf, _ = rl.loss_grad(Ws, bs, False, X, a, lpo, A, ret, rl.REINFORCE, 0.2, 0.0, 0.0)
+    gp, gr = rl.flat(g_ppo), rl.flat(g_rf)
+    assert np.abs(gr).max() > 1e-3
+    if clipped:
+        assert np.all(gp == 0.0)
+    else:
+        assert np.allclose(gp, rho * gr, rtol=1e-12, atol=1e-15)
+    assert s[1] == pytest.approx(pg, rel=1e-12)
+    assert s[4] == (1.0 if abs(rho - 1.0) > 0.2 else 0.0)
 
 
 def test_uniform_logits_closed_forms():
