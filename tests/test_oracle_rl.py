@@ -9,6 +9,8 @@
 * PPO's clipping by the sign of the advantage: one row at a tabulated ratio, the gradient 0
   exactly when the clipped branch is the minimum and rho times REINFORCE's otherwise (a max
   for the min, the branch test reversed or a clip that ignores the sign each fail a case).
+* The entropy bonus alone is stationary at uniform logits (its maximum); the value term alone
+  gives the value row's bias gradient 2 c_v mean(V - R) and zero on the action rows.
 """
 import math
 
@@ -221,6 +223,38 @@ def test_ppo_clip_cases_by_advantage_sign(adv, rho, clipped, pg):
         assert np.allclose(gp, rho * gr, rtol=1e-12, atol=1e-15)
     assert s[1] == pytest.approx(pg, rel=1e-12)
     assert s[4] == (1.0 if abs(rho - 1.0) > 0.2 else 0.0)
+
+
+def test_entropy_bonus_is_stationary_at_uniform_logits():
+    """The entropy of pi = softmax(z) is largest at uniform logits, so with only the entropy
+    term (A = 0, no value row) every gradient vanishes there; a sign slip in its derivative
+    (pi (log pi - H) for pi (log pi + H)) does not."""
+    Ws, bs, X, a, _, ret, lpo = _tiny(False, seed=8)
+    Ws[-1][:] = 0.0
+    bs[-1][:] = 0.0
+    g, s = rl.loss_grad(Ws, bs, False, X, a, lpo, np.zeros(len(a)), ret, rl.REINFORCE, 0.2, 0.0, 1.0)
+    assert s[3] == pytest.approx(math.log(Ws[-1].shape[0]), rel=1e-14)
+    assert np.abs(rl.flat(g)).max() < 1e-14
+    # away from uniform the same term has a gradient
+    Ws[-1][0, 0] = 1.0
+    g, _ = rl.loss_grad(Ws, bs, False, X, a, lpo, np.zeros(len(a)), ret, rl.REINFORCE, 0.2, 0.0, 1.0)
+    assert np.abs(rl.flat(g)).max() > 1e-3
+
+
+def test_value_term_bias_gradient_closed_form():
+    """Only the value term (A = 0, no entropy): L = c_v mean((V - R)^2) with V the last row of
+    the last layer, so dL/db_V = 2 c_v mean(V - R), the action rows' bias gradients are 0, and
+    the statistic is the mean squared error itself."""
+    Ws, bs, X, a, _, ret, lpo = _tiny(True, seed=12)
+    cv = 0.5
+    _, Z = rl.forward(Ws, bs, X)
+    V = Z[:, -1]
+    g, s = rl.loss_grad(Ws, bs, True, X, a, lpo, np.zeros(len(a)), ret, rl.REINFORCE, 0.2, cv, 0.0)
+    gb = g[-1][1]
+    assert gb[-1] == pytest.approx(2.0 * cv * np.mean(V - ret), rel=1e-12)
+    assert np.all(gb[:-1] == 0.0)
+    assert s[2] == pytest.approx(np.mean((V - ret) ** 2), rel=1e-12)
+    assert s[0] == pytest.approx(cv * s[2], rel=1e-12)
 
 
 def test_uniform_logits_closed_forms():
